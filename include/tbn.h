@@ -1,0 +1,223 @@
+/*
+ * tbn.h -- C ABI of the Two-Bit Networks (TBN) GPU library for GB300 (sm_103a).
+ *
+ * Two-Bit Networks (Meng, Gu, Zhang, Wu, arXiv:1701.00485) approximate each
+ * real-valued filter W of a convolutional or fully-connected layer by
+ * alpha * W~, with W~ in {-2,-1,1,2}^n stored at two bits per weight.  This
+ * library provides the data-parallel hot path of the method:
+ *
+ *   tbn_quantize_pack   discretization (Eq. 3) + optimal scaling factor
+ *                       (Eq. 5) for every filter of a layer, packed
+ *   tbn_unpack          packed codes -> int8 W~ or dequantized alpha W~
+ *   tbn_conv2d_fwd      convolution with alpha W~ (Eq. 1)
+ *   tbn_linear_fwd      fully-connected layer, treated as a convolution
+ *                       (Section 3)
+ *   tbn_maxpool2d_nhwc, tbn_nchw_to_nhwc   network glue between layers
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Pointers to tensors are DEVICE pointers, allocated and owned by the
+ *   caller.  The library allocates no device memory and keeps no state
+ *   between calls except the per-device error word (tbn_device_error) and
+ *   per-process kernel attributes.
+ * - Every compute call is asynchronous on `stream` (a cudaStream_t; NULL is
+ *   the legacy default stream).  Arguments are validated on the host before
+ *   anything is launched; an invalid call returns a status and launches
+ *   nothing.  No call aborts the process or throws.
+ * - Kernel-side waits are bounded in time.  A wait that expires sets a bit
+ *   in the per-device error word and the kernel returns early; read it with
+ *   tbn_device_error() after synchronizing.
+ * - tbn_last_error() returns a human-readable detail string for the most
+ *   recent failing call on the calling host thread.
+ *
+ * Two-bit storage format (the paper fixes only that the four values "can be
+ * encoded with two bits"; the layout below is this library's):
+ * - each code is a 2-bit field f = m + 2 s with s = 1 for a negative value and
+ *   m = 1 for magnitude two:  +1 -> 0, +2 -> 1, -1 -> 2, -2 -> 3;
+ *   W~ = (1 - 2 s)(1 + m);
+ * - a filter of n codes occupies tbn_packed_words(n) = ceil(n / 16) uint32
+ *   words; code i of filter k is in bits [2 (i mod 16), 2 (i mod 16) + 1] of
+ *   word k * ceil(n / 16) + i / 16 (little-endian: byte i/4, bits 2 (i mod 4));
+ *   unused fields of a filter's last word are zero;
+ * - codes[K][ceil(n/16)] plus alpha[K] (fp32) is the complete inference
+ *   form of a layer ("only the two-bit filters and the optimal scaling
+ *   factors are used", Section 3).
+ * - The order of the n weights of a filter is the caller's choice; the
+ *   convolution reads them in the activation layout's natural order:
+ *   NCHW -> (c, r, s), NHWC -> (r, s, c).  Discretization is elementwise and
+ *   alpha does not depend on the order, so permuting fp32 weights before
+ *   tbn_quantize_pack is how either order is produced.
+ */
+#ifndef TBN_H
+#define TBN_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TBN_ABI_VERSION 1
+
+typedef enum {
+  TBN_OK = 0,
+  TBN_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, bad enum, overflow */
+  TBN_ERR_UNSUPPORTED = 2, /* valid request that no kernel here implements       */
+  TBN_ERR_MISALIGNED = 3,  /* a pointer violates the alignment the call needs    */
+  TBN_ERR_CUDA = 4,        /* a CUDA runtime/driver call failed (see last_error) */
+  TBN_ERR_TIMEOUT = 5      /* reserved for callers mapping the device error word */
+} tbn_status;
+
+typedef enum { TBN_F32 = 0, TBN_BF16 = 1 } tbn_dtype;
+
+typedef enum { TBN_NCHW = 0, TBN_NHWC = 1 } tbn_layout;
+
+typedef enum {
+  TBN_UNPACK_I8 = 0,   /* int8 W~ in {-2,-1,1,2}                 */
+  TBN_UNPACK_F32 = 1,  /* fp32 alpha[k] * W~                      */
+  TBN_UNPACK_BF16 = 2  /* bf16 alpha[k] * W~ (round to nearest)   */
+} tbn_unpack_format;
+
+/* Convolution algorithms.  AUTO picks the fastest implemented one. */
+typedef enum {
+  TBN_CONV_AUTO = 0,
+  TBN_CONV_DIRECT = 1,        /* CUDA-core direct convolution, any layout/dtype  */
+  TBN_CONV_IMPLICIT_GEMM = 2  /* tcgen05 implicit GEMM: NHWC, bf16 x, C % 64 == 0,
+                                 stride 1 or 2                                    */
+} tbn_conv_algo;
+
+/* Fused layer epilogue (network glue, not part of the paper's method):
+ *   v = alpha[k] * acc;  if (residual) v += residual[same index];
+ *   if (relu) v = max(v, 0);  y = v rounded to y's dtype.
+ * `residual` has y's layout, shape and dtype.  Pass NULL for no epilogue. */
+typedef struct {
+  int relu;
+  const void *residual;
+} tbn_epilogue;
+
+/* A cudaStream_t, passed as an opaque pointer. */
+typedef void *tbn_stream;
+
+/* ------------------------------------------------------------------------ */
+
+/* ABI version of the loaded library (TBN_ABI_VERSION). */
+int tbn_abi_version(void);
+
+/* Words per filter for n codes: ceil(n / 16); -1 if n < 1. */
+int64_t tbn_packed_words(int64_t n);
+
+/* Static description of a status code. */
+const char *tbn_status_string(tbn_status s);
+
+/* Detail of the most recent failure on this host thread ("" if none). */
+const char *tbn_last_error(void);
+
+/* Reads and clears the error word of the current device (synchronous:
+ * waits for the device's pending work).  Bit 1: a kernel wait timed out;
+ * bit 2: a kernel saw a launch shape it could not run.  *flags = 0 when no
+ * error was recorded. */
+tbn_status tbn_device_error(uint32_t *flags);
+
+/* Quantize and pack one layer -- Algorithm 1, quantization loop; Eq. 3
+ * (discretization) and Eq. 5 (optimal scaling factor), Section 2.
+ *
+ *   W      [K][n] fp32, row k = filter k (device).  Any 4-byte alignment;
+ *          16-byte alignment with n % 4 == 0 takes the vector-load path.
+ *   codes  [K][tbn_packed_words(n)] uint32 (device, output), 4-byte aligned.
+ *   alpha  [K] fp32 (device, output):
+ *          alpha_k = (sum_{|W|<=1} |W| + 2 sum_{|W|>1} |W|) / (n + 3 |{|W|>1}|)
+ *          accumulated in fp32 per 16 weights and fp64 across them, rounded
+ *          once to fp32.  An all-zero filter gets alpha = 0.
+ *   Eq. 3 per weight: W < -1 -> -2; -1 <= W <= 0 -> -1 (including -0.0);
+ *          0 < W <= 1 -> 1; W > 1 -> 2.  NaN weights are undefined input.
+ * K >= 1, 1 <= n < 2^31, K * tbn_packed_words(n) < 2^40. */
+tbn_status tbn_quantize_pack(const float *W, int64_t K, int64_t n, uint32_t *codes,
+                             float *alpha, tbn_stream stream);
+
+/* One layer of a grouped quantization call (see tbn_quantize_pack_group). */
+typedef struct {
+  const float *W;
+  int64_t K;
+  int64_t n;
+  uint32_t *codes;
+  float *alpha;
+} tbn_quant_job;
+
+/* Up to TBN_MAX_QUANT_JOBS layers quantized by one kernel launch (used to
+ * re-quantize every layer of a network per forward pass, Algorithm 1).  Each
+ * job follows tbn_quantize_pack's contract; jobs must not overlap in memory.
+ * The job table is passed by value to the kernel; nothing is allocated. */
+#define TBN_MAX_QUANT_JOBS 16
+tbn_status tbn_quantize_pack_group(const tbn_quant_job *jobs, int njobs, tbn_stream stream);
+
+/* Unpack codes [K][tbn_packed_words(n)] into out [K][n] as int8 W~, or as
+ * fp32 / bf16 alpha[k] * W~ (alpha may be NULL only for TBN_UNPACK_I8).
+ * Padding fields are ignored. */
+tbn_status tbn_unpack(const uint32_t *codes, const float *alpha, int64_t K, int64_t n,
+                      void *out, tbn_unpack_format fmt, tbn_stream stream);
+
+/* Two-bit convolution, Eq. 1 (Section 2): cross-correlation with zero
+ * padding, no bias, groups = 1, dilation = 1 (the paper states none of
+ * these; they follow the Torch7 convention the paper's experiments used).
+ *
+ *   y[b,k,p,q] = alpha[k] * sum_{c,r,s} x[b,c,p*sh-ph+r,q*sw-pw+s] W~[k,c,r,s]
+ *
+ *   x      activations (device).  layout NCHW: [N][C][H][W];
+ *          NHWC: [N][H][W][C].  dtype fp32 or bf16.
+ *   codes  [K][tbn_packed_words(C*R*S)], filter order (c,r,s) for NCHW and
+ *          (r,s,c) for NHWC.   alpha [K] fp32.
+ *   y      [N][K][P][Q] (NCHW) or [N][P][Q][K] (NHWC), dtype fp32 or bf16,
+ *          P = (H + 2 ph - R) / sh + 1, Q = (W + 2 pw - S) / sw + 1.
+ *   epi    optional fused epilogue (NULL = none).
+ * Accumulation is fp32; x * W~ products are exact.  y must not alias x.
+ * The implicit-GEMM path needs NHWC, bf16 x, C % 64 == 0, 16-byte aligned x,
+ * stride 1 or 2, P and Q <= 256; AUTO falls back to the direct kernel
+ * otherwise. */
+tbn_status tbn_conv2d_fwd(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                          int64_t C, int64_t H, int64_t W, const uint32_t *codes,
+                          const float *alpha, int64_t K, int64_t R, int64_t S,
+                          int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
+                          void *y, tbn_dtype ydt, const tbn_epilogue *epi, tbn_stream stream);
+
+/* tbn_conv2d_fwd with an explicit algorithm.  Returns TBN_ERR_UNSUPPORTED if
+ * the requested algorithm cannot run this shape. */
+tbn_status tbn_conv2d_fwd_algo(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                               int64_t C, int64_t H, int64_t W, const uint32_t *codes,
+                               const float *alpha, int64_t K, int64_t R, int64_t S,
+                               int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                               int64_t pad_w, void *y, tbn_dtype ydt, const tbn_epilogue *epi,
+                               tbn_conv_algo algo, tbn_stream stream);
+
+/* The algorithm AUTO would choose for this shape (host-only query). */
+tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N, int64_t C,
+                                     int64_t H, int64_t W, int64_t K, int64_t R, int64_t S,
+                                     int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                                     int64_t pad_w);
+
+/* Fully-connected layer (Section 3: treated as a convolution):
+ *   y[b,k] = alpha[k] * sum_j x[b,j] W~[k,j]
+ * x [B][K_in] (fp32 or bf16), codes [K_out][tbn_packed_words(K_in)],
+ * alpha [K_out], y [B][K_out] (fp32 or bf16), optional epilogue.
+ * B <= 8 with bf16 x, K_in % 16 == 0 and 16-byte aligned x and codes runs
+ * the tensor-core GEMV; other shapes run as a 1x1 convolution. */
+tbn_status tbn_linear_fwd(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                          const uint32_t *codes, const float *alpha, int64_t K_out, void *y,
+                          tbn_dtype ydt, const tbn_epilogue *epi, tbn_stream stream);
+
+/* Max pooling over NHWC (network glue): window kh x kw, stride sh x sw, no
+ * padding; x [N][H][W][C] -> y [N][Ho][Wo][C], Ho = (H - kh)/sh + 1. */
+tbn_status tbn_maxpool2d_nhwc(const void *x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
+                              int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
+                              void *y, tbn_stream stream);
+
+/* Layout conversion NCHW -> NHWC with channel zero-padding to C_pad >= C
+ * (network glue for the first layer).  x [N][C][H][W], y [N][H][W][C_pad],
+ * same dtype. */
+tbn_status tbn_nchw_to_nhwc(const void *x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
+                            int64_t W, int64_t C_pad, void *y, tbn_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TBN_H */

@@ -1,0 +1,294 @@
+"""Two-Bit Networks (arXiv:1701.00485) on GB300: Python binding of libtbn.
+
+Thin ctypes layer over the C ABI declared in ``include/tbn.h``.  Each
+function here has the C entry point's name, checks tensor shapes/devices,
+passes raw device pointers and the current CUDA stream, and raises
+``TBNError`` on a non-OK status.  All arithmetic runs in the CUDA kernels of
+``libtbn.so``; there is no CPU path.  PyTorch supplies device memory and
+streams only.
+
+The library must have been built (``python -m paper_1701_00485_gb300.build``
+or ``__graft_entry__.build()``); importing a function that needs it raises
+``RuntimeError`` when ``libtbn.so`` is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+__all__ = [
+    "TBNError", "lib", "lib_path", "packed_words",
+    "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack", "tbn_conv2d_fwd",
+    "tbn_linear_fwd", "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_device_error",
+    "tbn_conv2d_select_algo", "conv_out_hw",
+    "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
+    "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libtbn.so")
+
+TBN_OK, TBN_ERR_INVALID_ARG, TBN_ERR_UNSUPPORTED, TBN_ERR_MISALIGNED, TBN_ERR_CUDA, \
+    TBN_ERR_TIMEOUT = range(6)
+TBN_F32, TBN_BF16 = 0, 1
+TBN_NCHW, TBN_NHWC = 0, 1
+TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
+TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM = 0, 1, 2
+TBN_MAX_QUANT_JOBS = 16
+
+# every symbol include/tbn.h declares
+EXPORTED = [
+    "tbn_abi_version", "tbn_packed_words", "tbn_status_string", "tbn_last_error",
+    "tbn_device_error", "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack",
+    "tbn_conv2d_fwd", "tbn_conv2d_fwd_algo", "tbn_conv2d_select_algo", "tbn_linear_fwd",
+    "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc",
+]
+
+
+class TBNError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        self.status = status
+        super().__init__("%s failed: status %d (%s): %s" % (
+            where, status, _status_name(status), detail))
+
+
+class QuantJob(ctypes.Structure):
+    _fields_ = [("W", ctypes.c_void_p), ("K", ctypes.c_int64), ("n", ctypes.c_int64),
+                ("codes", ctypes.c_void_p), ("alpha", ctypes.c_void_p)]
+
+
+class Epilogue(ctypes.Structure):
+    _fields_ = [("relu", ctypes.c_int), ("residual", ctypes.c_void_p)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """The loaded libtbn.so (ctypes.CDLL).  Raises if it was not built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError("libtbn.so not found at %s: build it with "
+                               "`python -m paper_1701_00485_gb300.build`" % _LIB_PATH)
+        L = ctypes.CDLL(_LIB_PATH)
+        P, I64, I32, U32P = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p
+        sig = {
+            "tbn_abi_version": ([], I32),
+            "tbn_packed_words": ([I64], I64),
+            "tbn_status_string": ([I32], ctypes.c_char_p),
+            "tbn_last_error": ([], ctypes.c_char_p),
+            "tbn_device_error": ([ctypes.POINTER(ctypes.c_uint32)], I32),
+            "tbn_quantize_pack": ([P, I64, I64, U32P, P, P], I32),
+            "tbn_quantize_pack_group": ([ctypes.POINTER(QuantJob), I32, P], I32),
+            "tbn_unpack": ([U32P, P, I64, I64, P, I32, P], I32),
+            "tbn_conv2d_fwd": ([P, I32, I32, I64, I64, I64, I64, U32P, P, I64, I64, I64,
+                                I64, I64, I64, I64, P, I32, ctypes.POINTER(Epilogue), P], I32),
+            "tbn_conv2d_fwd_algo": ([P, I32, I32, I64, I64, I64, I64, U32P, P, I64, I64, I64,
+                                     I64, I64, I64, I64, P, I32, ctypes.POINTER(Epilogue), I32,
+                                     P], I32),
+            "tbn_conv2d_select_algo": ([I32, I32, I64, I64, I64, I64, I64, I64, I64, I64, I64,
+                                        I64, I64], I32),
+            "tbn_linear_fwd": ([P, I32, I64, I64, U32P, P, I64, P, I32,
+                                ctypes.POINTER(Epilogue), P], I32),
+            "tbn_maxpool2d_nhwc": ([P, I32, I64, I64, I64, I64, I64, I64, I64, I64, P, P], I32),
+            "tbn_nchw_to_nhwc": ([P, I32, I64, I64, I64, I64, I64, P, P], I32),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        if L.tbn_abi_version() != 1:
+            raise RuntimeError("libtbn ABI version mismatch")
+        _lib = L
+        return L
+
+
+def _status_name(s: int) -> str:
+    try:
+        return lib().tbn_status_string(int(s)).decode()
+    except Exception:  # pragma: no cover - only while reporting another failure
+        return "?"
+
+
+def _check(status: int, where: str):
+    if status != TBN_OK:
+        detail = lib().tbn_last_error().decode(errors="replace")
+        raise TBNError(status, where, detail)
+
+
+def _dt(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return TBN_F32
+    if t.dtype == torch.bfloat16:
+        return TBN_BF16
+    raise TypeError("tensor dtype must be float32 or bfloat16, got %s" % t.dtype)
+
+
+def _torch_dt(code: int):
+    return torch.float32 if code == TBN_F32 else torch.bfloat16
+
+
+def _cuda(t: torch.Tensor, name: str) -> torch.Tensor:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError("%s must be a CUDA tensor" % name)
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    return t
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _epi(relu: bool, residual) -> Epilogue | None:
+    if not relu and residual is None:
+        return None
+    return Epilogue(1 if relu else 0, residual.data_ptr() if residual is not None else None)
+
+
+def packed_words(n: int) -> int:
+    """ceil(n / 16): uint32 words per filter of n two-bit codes."""
+    return int(lib().tbn_packed_words(int(n)))
+
+
+def conv_out_hw(H, W, R, S, stride=(1, 1), pad=(0, 0)):
+    return (H + 2 * pad[0] - R) // stride[0] + 1, (W + 2 * pad[1] - S) // stride[1] + 1
+
+
+def tbn_quantize_pack(W: torch.Tensor, codes: torch.Tensor | None = None,
+                      alpha: torch.Tensor | None = None, stream=None):
+    """Eq. 3 + Eq. 5 + packing for each row of W [K, n] (fp32, CUDA).
+
+    Returns (codes int32 [K, ceil(n/16)] holding the uint32 words, alpha fp32 [K])."""
+    _cuda(W, "W")
+    if W.dtype != torch.float32 or W.dim() != 2:
+        raise ValueError("W must be a 2-D float32 tensor [K, n]")
+    K, n = W.shape
+    if codes is None:
+        codes = torch.empty((K, packed_words(n)), dtype=torch.int32, device=W.device)
+    if alpha is None:
+        alpha = torch.empty((K,), dtype=torch.float32, device=W.device)
+    _cuda(codes, "codes"), _cuda(alpha, "alpha")
+    _check(lib().tbn_quantize_pack(W.data_ptr(), K, n, codes.data_ptr(), alpha.data_ptr(),
+                                   _stream(stream)), "tbn_quantize_pack")
+    return codes, alpha
+
+
+def tbn_quantize_pack_group(jobs, stream=None):
+    """One launch for up to 16 layers; jobs = [(W [K,n], codes, alpha), ...]."""
+    if not 1 <= len(jobs) <= TBN_MAX_QUANT_JOBS:
+        raise ValueError("need 1..16 jobs")
+    arr = (QuantJob * len(jobs))()
+    for i, (W, codes, alpha) in enumerate(jobs):
+        _cuda(W, "W"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
+        K, n = W.shape
+        arr[i] = QuantJob(W.data_ptr(), K, n, codes.data_ptr(), alpha.data_ptr())
+    _check(lib().tbn_quantize_pack_group(arr, len(jobs), _stream(stream)),
+           "tbn_quantize_pack_group")
+
+
+def tbn_unpack(codes: torch.Tensor, alpha: torch.Tensor | None, n: int,
+               fmt: int = TBN_UNPACK_I8, stream=None) -> torch.Tensor:
+    """codes [K, ceil(n/16)] -> int8 W~ or fp32/bf16 alpha*W~ [K, n]."""
+    _cuda(codes, "codes")
+    K = codes.shape[0]
+    dt = {TBN_UNPACK_I8: torch.int8, TBN_UNPACK_F32: torch.float32,
+          TBN_UNPACK_BF16: torch.bfloat16}[fmt]
+    out = torch.empty((K, n), dtype=dt, device=codes.device)
+    _check(lib().tbn_unpack(codes.data_ptr(), alpha.data_ptr() if alpha is not None else None,
+                            K, n, out.data_ptr(), fmt, _stream(stream)), "tbn_unpack")
+    return out
+
+
+def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K: int, R: int,
+                   S: int, stride=(1, 1), pad=(0, 0), layout: int = TBN_NHWC,
+                   out_dtype=None, relu: bool = False, residual: torch.Tensor | None = None,
+                   algo: int = TBN_CONV_AUTO, out: torch.Tensor | None = None, stream=None):
+    """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW) or [N,H,W,C] (NHWC)."""
+    _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
+    if layout == TBN_NHWC:
+        N, H, W, C = x.shape
+    else:
+        N, C, H, W = x.shape
+    P, Q = conv_out_hw(H, W, R, S, stride, pad)
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    shape = (N, P, Q, K) if layout == TBN_NHWC else (N, K, P, Q)
+    if out is None:
+        out = torch.empty(shape, dtype=_torch_dt(ydt), device=x.device)
+    elif tuple(out.shape) != shape or _dt(out) != ydt:
+        raise ValueError("out has the wrong shape or dtype")
+    if residual is not None:
+        _cuda(residual, "residual")
+        if tuple(residual.shape) != shape or _dt(residual) != ydt:
+            raise ValueError("residual must match y's shape and dtype")
+    e = _epi(relu, residual)
+    _check(lib().tbn_conv2d_fwd_algo(
+        x.data_ptr(), _dt(x), layout, N, C, H, W, codes.data_ptr(), alpha.data_ptr(), K, R, S,
+        stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,
+        ctypes.byref(e) if e is not None else None, algo, _stream(stream)), "tbn_conv2d_fwd")
+    return out
+
+
+def tbn_conv2d_select_algo(x_dtype, layout, N, C, H, W, K, R, S, stride=(1, 1), pad=(0, 0)):
+    xdt = TBN_F32 if x_dtype == torch.float32 else TBN_BF16
+    return int(lib().tbn_conv2d_select_algo(xdt, layout, N, C, H, W, K, R, S, stride[0],
+                                            stride[1], pad[0], pad[1]))
+
+
+def tbn_linear_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K_out: int,
+                   out_dtype=None, relu: bool = False, residual: torch.Tensor | None = None,
+                   out: torch.Tensor | None = None, stream=None):
+    """Fully-connected layer (Section 3): x [B, K_in] -> y [B, K_out]."""
+    _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
+    B, K_in = x.shape
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    if out is None:
+        out = torch.empty((B, K_out), dtype=_torch_dt(ydt), device=x.device)
+    e = _epi(relu, residual)
+    _check(lib().tbn_linear_fwd(x.data_ptr(), _dt(x), B, K_in, codes.data_ptr(), alpha.data_ptr(),
+                                K_out, out.data_ptr(), ydt,
+                                ctypes.byref(e) if e is not None else None, _stream(stream)),
+           "tbn_linear_fwd")
+    return out
+
+
+def tbn_maxpool2d_nhwc(x: torch.Tensor, k=(2, 2), stride=(2, 2), out=None, stream=None):
+    _cuda(x, "x")
+    N, H, W, C = x.shape
+    Ho, Wo = (H - k[0]) // stride[0] + 1, (W - k[1]) // stride[1] + 1
+    if out is None:
+        out = torch.empty((N, Ho, Wo, C), dtype=x.dtype, device=x.device)
+    _check(lib().tbn_maxpool2d_nhwc(x.data_ptr(), _dt(x), N, H, W, C, k[0], k[1], stride[0],
+                                    stride[1], out.data_ptr(), _stream(stream)),
+           "tbn_maxpool2d_nhwc")
+    return out
+
+
+def tbn_nchw_to_nhwc(x: torch.Tensor, C_pad: int | None = None, out=None, stream=None):
+    _cuda(x, "x")
+    N, C, H, W = x.shape
+    C_pad = C if C_pad is None else C_pad
+    if out is None:
+        out = torch.empty((N, H, W, C_pad), dtype=x.dtype, device=x.device)
+    _check(lib().tbn_nchw_to_nhwc(x.data_ptr(), _dt(x), N, C, H, W, C_pad, out.data_ptr(),
+                                  _stream(stream)), "tbn_nchw_to_nhwc")
+    return out
+
+
+def tbn_device_error() -> int:
+    """Read and clear the current device's error word (synchronizes)."""
+    v = ctypes.c_uint32(0)
+    _check(lib().tbn_device_error(ctypes.byref(v)), "tbn_device_error")
+    return int(v.value)

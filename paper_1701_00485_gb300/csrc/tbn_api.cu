@@ -1,0 +1,293 @@
+// tbn_api.cu -- the library's extern "C" entry points (include/tbn.h):
+// argument validation on the host, dispatch to the kernels, error reporting.
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "tbn.h"
+#include "tbn_internal.h"
+
+namespace tbn {
+
+// Per-device error word written by kernels (timeouts, bad launch shapes).
+__device__ uint32_t g_tbn_device_error;
+
+namespace {
+
+thread_local char t_last_error[512] = "";
+
+constexpr int kMaxDevices = 64;
+uint32_t* g_err_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+std::mutex g_dev_mutex;
+
+bool mul_ok(int64_t a, int64_t b, int64_t limit) {
+  return a >= 0 && b >= 0 && (a == 0 || b <= limit / a);
+}
+
+}  // namespace
+
+const char* last_error_text() { return t_last_error; }
+
+tbn_status fail(tbn_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(t_last_error, sizeof(t_last_error), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+tbn_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(TBN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+tbn_status check_launch(const char* what) {
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, what);
+  return TBN_OK;
+}
+
+uint32_t* device_error_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> g(g_dev_mutex);
+  if (g_err_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_tbn_device_error) == cudaSuccess)
+      g_err_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+int device_sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 132;
+  std::lock_guard<std::mutex> g(g_dev_mutex);
+  if (g_sm_count[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 132;
+    g_sm_count[dev] = n;
+  }
+  return g_sm_count[dev];
+}
+
+}  // namespace tbn
+
+using namespace tbn;
+
+namespace {
+
+tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N, int64_t C,
+                         int64_t H, int64_t W, const uint32_t* codes, const float* alpha,
+                         int64_t K, int64_t R, int64_t S, int64_t sh, int64_t sw, int64_t ph,
+                         int64_t pw, void* y, tbn_dtype ydt, const tbn_epilogue* epi,
+                         ConvProblem* out) {
+  if (!x || !codes || !alpha || !y) return fail(TBN_ERR_INVALID_ARG, "conv: null pointer");
+  if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad x dtype");
+  if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad y dtype");
+  if (layout != TBN_NCHW && layout != TBN_NHWC) return fail(TBN_ERR_INVALID_ARG, "conv: bad layout");
+  if (N < 1 || C < 1 || H < 1 || W < 1 || K < 1 || R < 1 || S < 1)
+    return fail(TBN_ERR_INVALID_ARG, "conv: sizes must be >= 1");
+  if (sh < 1 || sw < 1 || ph < 0 || pw < 0) return fail(TBN_ERR_INVALID_ARG, "conv: bad stride/pad");
+  if (H + 2 * ph < R || W + 2 * pw < S)
+    return fail(TBN_ERR_INVALID_ARG, "conv: kernel larger than padded input");
+  if (R > 0xFFFF || S > 0xFFFF || sh > 0xFFFF || sw > 0xFFFF || ph > 0xFFFF || pw > 0xFFFF)
+    return fail(TBN_ERR_UNSUPPORTED, "conv: kernel/stride/pad above 65535");
+  const int64_t lim = int64_t(1) << 31;
+  if (!mul_ok(C * R, S, lim) || !mul_ok(C, H * W, lim) || H * W >= lim)
+    return fail(TBN_ERR_UNSUPPORTED, "conv: C*R*S or C*H*W exceeds 2^31");
+  const int64_t P = (H + 2 * ph - R) / sh + 1, Q = (W + 2 * pw - S) / sw + 1;
+  if (!mul_ok(N, H * W * C, int64_t(1) << 46) || !mul_ok(N * P * Q, K, int64_t(1) << 46))
+    return fail(TBN_ERR_UNSUPPORTED, "conv: tensor too large");
+  const size_t xs = dtype_size(xdt), ys = dtype_size(ydt);
+  if (!is_aligned(x, xs) || !is_aligned(y, ys) || !is_aligned(codes, 4) || !is_aligned(alpha, 4))
+    return fail(TBN_ERR_MISALIGNED, "conv: pointer not aligned to its element size");
+  if (epi && epi->residual && !is_aligned(epi->residual, ys))
+    return fail(TBN_ERR_MISALIGNED, "conv: residual not aligned to its element size");
+  ConvProblem& p = *out;
+  p.N = N; p.C = C; p.H = H; p.W = W; p.K = K; p.R = R; p.S = S;
+  p.sh = sh; p.sw = sw; p.ph = ph; p.pw = pw; p.P = P; p.Q = Q;
+  p.layout = layout; p.xdt = xdt; p.ydt = ydt;
+  p.x = x; p.codes = codes; p.alpha = alpha; p.y = y;
+  p.relu = epi ? (epi->relu != 0) : 0;
+  p.residual = epi ? epi->residual : nullptr;
+  return TBN_OK;
+}
+
+tbn_status run_conv(const ConvProblem& p, tbn_conv_algo algo, cudaStream_t s) {
+  if (algo == TBN_CONV_AUTO) {
+    algo = (conv_igemm_unsupported_reason(p)[0] == '\0') ? TBN_CONV_IMPLICIT_GEMM : TBN_CONV_DIRECT;
+  }
+  if (algo == TBN_CONV_IMPLICIT_GEMM) {
+    const char* why = conv_igemm_unsupported_reason(p);
+    if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
+    return launch_conv_igemm(p, s);
+  }
+  if (algo == TBN_CONV_DIRECT) return launch_conv_direct(p, s);
+  return fail(TBN_ERR_INVALID_ARG, "conv: bad algorithm %d", (int)algo);
+}
+
+}  // namespace
+
+extern "C" {
+
+int tbn_abi_version(void) { return TBN_ABI_VERSION; }
+
+int64_t tbn_packed_words(int64_t n) { return n < 1 ? -1 : (n + 15) / 16; }
+
+const char* tbn_status_string(tbn_status s) {
+  switch (s) {
+    case TBN_OK: return "ok";
+    case TBN_ERR_INVALID_ARG: return "invalid argument";
+    case TBN_ERR_UNSUPPORTED: return "unsupported";
+    case TBN_ERR_MISALIGNED: return "misaligned pointer";
+    case TBN_ERR_CUDA: return "CUDA error";
+    case TBN_ERR_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+const char* tbn_last_error(void) { return last_error_text(); }
+
+tbn_status tbn_device_error(uint32_t* flags) {
+  if (!flags) return fail(TBN_ERR_INVALID_ARG, "device_error: null pointer");
+  *flags = 0;
+  uint32_t* p = device_error_word();
+  if (!p) return fail(TBN_ERR_CUDA, "device_error: cannot resolve the error word");
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "device_error: synchronize");
+  uint32_t v = 0;
+  e = cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "device_error: read");
+  const uint32_t zero = 0;
+  e = cudaMemcpy(p, &zero, sizeof(zero), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "device_error: clear");
+  *flags = v;
+  return TBN_OK;
+}
+
+tbn_status tbn_quantize_pack_group(const tbn_quant_job* jobs, int njobs, tbn_stream stream) {
+  if (!jobs || njobs < 1 || njobs > TBN_MAX_QUANT_JOBS)
+    return fail(TBN_ERR_INVALID_ARG, "quantize: need 1..%d jobs", TBN_MAX_QUANT_JOBS);
+  for (int i = 0; i < njobs; ++i) {
+    const tbn_quant_job& j = jobs[i];
+    if (!j.W || !j.codes || !j.alpha) return fail(TBN_ERR_INVALID_ARG, "quantize: job %d null pointer", i);
+    if (j.K < 1 || j.n < 1) return fail(TBN_ERR_INVALID_ARG, "quantize: job %d needs K, n >= 1", i);
+    if (j.n >= (int64_t(1) << 31)) return fail(TBN_ERR_UNSUPPORTED, "quantize: job %d n >= 2^31", i);
+    if (!mul_ok(j.K, (j.n + 15) / 16, int64_t(1) << 40) || !mul_ok(j.K, j.n, int64_t(1) << 44))
+      return fail(TBN_ERR_UNSUPPORTED, "quantize: job %d too large", i);
+    if (!is_aligned(j.W, 4) || !is_aligned(j.codes, 4) || !is_aligned(j.alpha, 4))
+      return fail(TBN_ERR_MISALIGNED, "quantize: job %d pointers must be 4-byte aligned", i);
+  }
+  return launch_quantize_group(jobs, njobs, as_stream(stream));
+}
+
+tbn_status tbn_quantize_pack(const float* W, int64_t K, int64_t n, uint32_t* codes, float* alpha,
+                             tbn_stream stream) {
+  tbn_quant_job j{W, K, n, codes, alpha};
+  return tbn_quantize_pack_group(&j, 1, stream);
+}
+
+tbn_status tbn_unpack(const uint32_t* codes, const float* alpha, int64_t K, int64_t n, void* out,
+                      tbn_unpack_format fmt, tbn_stream stream) {
+  if (!codes || !out) return fail(TBN_ERR_INVALID_ARG, "unpack: null pointer");
+  if (fmt != TBN_UNPACK_I8 && fmt != TBN_UNPACK_F32 && fmt != TBN_UNPACK_BF16)
+    return fail(TBN_ERR_INVALID_ARG, "unpack: bad format");
+  if (fmt != TBN_UNPACK_I8 && !alpha) return fail(TBN_ERR_INVALID_ARG, "unpack: alpha required");
+  if (K < 1 || n < 1) return fail(TBN_ERR_INVALID_ARG, "unpack: K, n must be >= 1");
+  if (!mul_ok(K, n, int64_t(1) << 44)) return fail(TBN_ERR_UNSUPPORTED, "unpack: too large");
+  const size_t es = fmt == TBN_UNPACK_I8 ? 1 : (fmt == TBN_UNPACK_F32 ? 4 : 2);
+  if (!is_aligned(codes, 4) || !is_aligned(out, es) || (alpha && !is_aligned(alpha, 4)))
+    return fail(TBN_ERR_MISALIGNED, "unpack: misaligned pointer");
+  return launch_unpack(codes, alpha, K, n, out, fmt, as_stream(stream));
+}
+
+tbn_status tbn_conv2d_fwd_algo(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                               int64_t C, int64_t H, int64_t W, const uint32_t* codes,
+                               const float* alpha, int64_t K, int64_t R, int64_t S,
+                               int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
+                               void* y, tbn_dtype ydt, const tbn_epilogue* epi,
+                               tbn_conv_algo algo, tbn_stream stream) {
+  ConvProblem p{};
+  const tbn_status st = validate_conv(x, xdt, layout, N, C, H, W, codes, alpha, K, R, S, stride_h,
+                                      stride_w, pad_h, pad_w, y, ydt, epi, &p);
+  if (st != TBN_OK) return st;
+  return run_conv(p, algo, as_stream(stream));
+}
+
+tbn_status tbn_conv2d_fwd(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N, int64_t C,
+                          int64_t H, int64_t W, const uint32_t* codes, const float* alpha,
+                          int64_t K, int64_t R, int64_t S, int64_t stride_h, int64_t stride_w,
+                          int64_t pad_h, int64_t pad_w, void* y, tbn_dtype ydt,
+                          const tbn_epilogue* epi, tbn_stream stream) {
+  return tbn_conv2d_fwd_algo(x, xdt, layout, N, C, H, W, codes, alpha, K, R, S, stride_h,
+                             stride_w, pad_h, pad_w, y, ydt, epi, TBN_CONV_AUTO, stream);
+}
+
+tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N, int64_t C,
+                                     int64_t H, int64_t W, int64_t K, int64_t R, int64_t S,
+                                     int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                                     int64_t pad_w) {
+  // Pointers only matter for alignment; use a 256-byte aligned dummy.
+  static const uint32_t dummy[64] __attribute__((aligned(256))) = {};
+  ConvProblem p{};
+  const tbn_status st =
+      validate_conv(dummy, xdt, layout, N, C, H, W, dummy, reinterpret_cast<const float*>(dummy),
+                    K, R, S, stride_h, stride_w, pad_h, pad_w, const_cast<uint32_t*>(dummy), TBN_BF16,
+                    nullptr, &p);
+  if (st != TBN_OK) return TBN_CONV_DIRECT;
+  return conv_igemm_unsupported_reason(p)[0] == '\0' ? TBN_CONV_IMPLICIT_GEMM : TBN_CONV_DIRECT;
+}
+
+tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                          const uint32_t* codes, const float* alpha, int64_t K_out, void* y,
+                          tbn_dtype ydt, const tbn_epilogue* epi, tbn_stream stream) {
+  if (!x || !codes || !alpha || !y) return fail(TBN_ERR_INVALID_ARG, "linear: null pointer");
+  if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad x dtype");
+  if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad y dtype");
+  if (B < 1 || K_in < 1 || K_out < 1) return fail(TBN_ERR_INVALID_ARG, "linear: sizes must be >= 1");
+  if (K_in >= (int64_t(1) << 31) || K_out >= (int64_t(1) << 31))
+    return fail(TBN_ERR_UNSUPPORTED, "linear: K_in / K_out >= 2^31");
+  const size_t ys = dtype_size(ydt);
+  if (!is_aligned(x, dtype_size(xdt)) || !is_aligned(y, ys) || !is_aligned(codes, 4) ||
+      !is_aligned(alpha, 4) || (epi && epi->residual && !is_aligned(epi->residual, ys)))
+    return fail(TBN_ERR_MISALIGNED, "linear: pointer not aligned to its element size");
+  if (gemv_unsupported_reason(x, xdt, B, K_in, codes)[0] == '\0') {
+    return launch_gemv(x, B, K_in, codes, alpha, K_out, y, ydt, epi ? epi->relu : 0,
+                       epi ? epi->residual : nullptr, as_stream(stream));
+  }
+  // a fully-connected layer is a 1x1 convolution over a 1x1 image (Section 3)
+  return tbn_conv2d_fwd(x, xdt, TBN_NHWC, B, K_in, 1, 1, codes, alpha, K_out, 1, 1, 1, 1, 0, 0, y,
+                        ydt, epi, stream);
+}
+
+tbn_status tbn_maxpool2d_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
+                              int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw, void* y,
+                              tbn_stream stream) {
+  if (!x || !y) return fail(TBN_ERR_INVALID_ARG, "maxpool: null pointer");
+  if (dt != TBN_F32 && dt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "maxpool: bad dtype");
+  if (N < 1 || H < 1 || W < 1 || C < 1 || kh < 1 || kw < 1 || sh < 1 || sw < 1 || kh > H || kw > W)
+    return fail(TBN_ERR_INVALID_ARG, "maxpool: bad sizes");
+  if (!mul_ok(N * H, W * C, int64_t(1) << 46)) return fail(TBN_ERR_UNSUPPORTED, "maxpool: too large");
+  if (!is_aligned(x, dtype_size(dt)) || !is_aligned(y, dtype_size(dt)))
+    return fail(TBN_ERR_MISALIGNED, "maxpool: misaligned pointer");
+  return launch_maxpool_nhwc(x, dt, N, H, W, C, kh, kw, sh, sw, y, as_stream(stream));
+}
+
+tbn_status tbn_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
+                            int64_t W, int64_t C_pad, void* y, tbn_stream stream) {
+  if (!x || !y) return fail(TBN_ERR_INVALID_ARG, "nchw_to_nhwc: null pointer");
+  if (dt != TBN_F32 && dt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "nchw_to_nhwc: bad dtype");
+  if (N < 1 || C < 1 || H < 1 || W < 1 || C_pad < C)
+    return fail(TBN_ERR_INVALID_ARG, "nchw_to_nhwc: bad sizes");
+  if (!mul_ok(N * H, W * C_pad, int64_t(1) << 46)) return fail(TBN_ERR_UNSUPPORTED, "nchw_to_nhwc: too large");
+  if (!is_aligned(x, dtype_size(dt)) || !is_aligned(y, dtype_size(dt)))
+    return fail(TBN_ERR_MISALIGNED, "nchw_to_nhwc: misaligned pointer");
+  return launch_nchw_to_nhwc(x, dt, N, C, H, W, C_pad, y, as_stream(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,297 @@
+// tbn_conv_direct.cu -- CUDA-core direct two-bit convolution (Eq. 1) for
+// every layout / dtype / stride / padding, plus the network glue kernels
+// (NHWC max pooling, NCHW -> NHWC with channel padding).
+//
+// Direct convolution: a CTA computes 128 output pixels x 32 filters.  The
+// filters' codes are decoded once per CTA into shared memory as fp32 W~ (a
+// chunk of taps at a time, tap-major so that all threads read the same
+// 32 weights -- a broadcast); each thread owns one pixel, walks the taps in
+// the codes' order, loads one activation per tap and does 32 FMAs.  This is
+// the path for small-channel layers (the first layer of a network, where
+// the implicit GEMM would pad C up to its tile) and the fallback for shapes
+// the tensor-core kernel does not take.  x * W~ is exact in fp32; the sum is
+// accumulated in fp32 in tap order.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "tbn_device.cuh"
+#include "tbn_internal.h"
+
+namespace tbn {
+namespace {
+
+constexpr int kPix = 128;    // pixels (threads) per CTA
+constexpr int kFilt = 32;    // filters per CTA
+constexpr int kTapChunk = 128;
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) {
+  return __bfloat162float(v);
+}
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float v);
+template <>
+__device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+  return __float2bfloat16_rn(v);
+}
+
+struct DirectArgs {
+  int64_t N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
+  int64_t wpf;  // words per filter
+  const void* x;
+  const uint32_t* codes;
+  const float* alpha;
+  void* y;
+  const void* residual;
+  int relu;
+};
+
+template <typename TX, typename TY, bool kNHWC>
+__global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
+  __shared__ __align__(16) float s_w[kTapChunk][kFilt];
+  __shared__ int32_t s_off[kTapChunk];
+  __shared__ int32_t s_rs[kTapChunk];
+
+  const TX* __restrict__ x = static_cast<const TX*>(a.x);
+  const int64_t npix = a.N * a.P * a.Q;
+  const int64_t pix = static_cast<int64_t>(blockIdx.x) * kPix + threadIdx.x;
+  const int64_t k0 = static_cast<int64_t>(blockIdx.y) * kFilt;
+  const bool active = pix < npix;
+  const int64_t pc = active ? pix : 0;
+  const int64_t b = pc / (a.P * a.Q);
+  const int64_t p = (pc / a.Q) % a.P;
+  const int64_t q = pc % a.Q;
+  const int64_t h0 = p * a.sh - a.ph;
+  const int64_t w0 = q * a.sw - a.pw;
+  // element offset of (b, c = 0, h0, w0)
+  const int64_t base = kNHWC ? ((b * a.H + h0) * a.W + w0) * a.C
+                             : ((b * a.C) * a.H + h0) * a.W + w0;
+
+  float acc[kFilt];
+#pragma unroll
+  for (int f = 0; f < kFilt; ++f) acc[f] = 0.0f;
+
+  const int64_t ntaps = a.C * a.R * a.S;
+  for (int64_t t0 = 0; t0 < ntaps; t0 += kTapChunk) {
+    const int tc = (ntaps - t0 < kTapChunk) ? static_cast<int>(ntaps - t0) : kTapChunk;
+    __syncthreads();
+    // decode W~ for this tap chunk: s_w[t][f]
+    for (int i = threadIdx.x; i < tc * kFilt; i += kPix) {
+      const int t = i / kFilt, f = i % kFilt;
+      const int64_t k = k0 + f;
+      float v = 0.0f;
+      if (k < a.K) {
+        const int64_t ti = t0 + t;
+        const uint32_t w = a.codes[k * a.wpf + (ti >> 4)];
+        v = code_value((w >> (2 * (ti & 15))) & 3u);
+      }
+      s_w[t][f] = v;
+    }
+    for (int t = threadIdx.x; t < tc; t += kPix) {
+      const int64_t ti = t0 + t;
+      int64_t c, r, s;
+      if (kNHWC) {
+        r = ti / (a.S * a.C);
+        s = (ti / a.C) % a.S;
+        c = ti % a.C;
+        s_off[t] = static_cast<int32_t>((r * a.W + s) * a.C + c);
+      } else {
+        c = ti / (a.R * a.S);
+        r = (ti / a.S) % a.R;
+        s = ti % a.S;
+        s_off[t] = static_cast<int32_t>((c * a.H + r) * a.W + s);
+      }
+      s_rs[t] = static_cast<int32_t>((r << 16) | s);
+    }
+    __syncthreads();
+    if (active) {
+      for (int t = 0; t < tc; ++t) {
+        const int32_t rs = s_rs[t];
+        const int64_t h = h0 + (rs >> 16), w = w0 + (rs & 0xFFFF);
+        float xv = 0.0f;
+        if (h >= 0 && h < a.H && w >= 0 && w < a.W) xv = to_f32<TX>(x[base + s_off[t]]);
+        const float4* wr = reinterpret_cast<const float4*>(&s_w[t][0]);
+#pragma unroll
+        for (int f4 = 0; f4 < kFilt / 4; ++f4) {
+          const float4 wv = wr[f4];
+          acc[4 * f4 + 0] = fmaf(xv, wv.x, acc[4 * f4 + 0]);
+          acc[4 * f4 + 1] = fmaf(xv, wv.y, acc[4 * f4 + 1]);
+          acc[4 * f4 + 2] = fmaf(xv, wv.z, acc[4 * f4 + 2]);
+          acc[4 * f4 + 3] = fmaf(xv, wv.w, acc[4 * f4 + 3]);
+        }
+      }
+    }
+  }
+  if (!active) return;
+
+  TY* __restrict__ y = static_cast<TY*>(a.y);
+  const TY* __restrict__ res = static_cast<const TY*>(a.residual);
+#pragma unroll
+  for (int f = 0; f < kFilt; ++f) {
+    const int64_t k = k0 + f;
+    if (k < a.K) {
+      const int64_t o = kNHWC ? pix * a.K + k : ((b * a.K + k) * a.P + p) * a.Q + q;
+      float v = a.alpha[k] * acc[f];
+      if (res != nullptr) v += to_f32<TY>(res[o]);
+      if (a.relu) v = fmaxf(v, 0.0f);
+      y[o] = from_f32<TY>(v);
+    }
+  }
+}
+
+template <typename TX, typename TY, bool kNHWC>
+tbn_status launch_direct_t(const DirectArgs& a, cudaStream_t s) {
+  const int64_t npix = a.N * a.P * a.Q;
+  const int64_t gx = (npix + kPix - 1) / kPix;
+  const int64_t gy = (a.K + kFilt - 1) / kFilt;
+  if (gx > 0x7fffffffLL || gy > 65535)
+    return fail(TBN_ERR_UNSUPPORTED, "conv direct: grid too large (%lld x %lld)", (long long)gx,
+                (long long)gy);
+  conv_direct_kernel<TX, TY, kNHWC><<<dim3((unsigned)gx, (unsigned)gy), kPix, 0, s>>>(a);
+  return check_launch("conv_direct_kernel");
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) maxpool_nhwc_kernel(const T* __restrict__ x, int64_t N,
+                                                           int64_t H, int64_t W, int64_t C,
+                                                           int64_t kh, int64_t kw, int64_t sh,
+                                                           int64_t sw, int64_t Ho, int64_t Wo,
+                                                           T* __restrict__ y) {
+  const int64_t total = N * Ho * Wo * C;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t c = i % C;
+    const int64_t wo = (i / C) % Wo;
+    const int64_t ho = (i / (C * Wo)) % Ho;
+    const int64_t b = i / (C * Wo * Ho);
+    float m = -INFINITY;
+    for (int64_t u = 0; u < kh; ++u)
+      for (int64_t v = 0; v < kw; ++v) {
+        const float t = to_f32<T>(x[((b * H + ho * sh + u) * W + wo * sw + v) * C + c]);
+        if (t > m) m = t;
+      }
+    y[i] = from_f32<T>(m);
+  }
+}
+
+// 8 channels (16 bytes) of bf16 per thread.
+__global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
+    const uint4* __restrict__ x, int64_t N, int64_t H, int64_t W, int64_t C8, int64_t kh,
+    int64_t kw, int64_t sh, int64_t sw, int64_t Ho, int64_t Wo, uint4* __restrict__ y) {
+  const int64_t total = N * Ho * Wo * C8;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t c = i % C8;
+    const int64_t wo = (i / C8) % Wo;
+    const int64_t ho = (i / (C8 * Wo)) % Ho;
+    const int64_t b = i / (C8 * Wo * Ho);
+    float m[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) m[e] = -INFINITY;
+    for (int64_t u = 0; u < kh; ++u)
+      for (int64_t v = 0; v < kw; ++v) {
+        const uint4 t = x[((b * H + ho * sh + u) * W + wo * sw + v) * C8 + c];
+        const __nv_bfloat16* tb = reinterpret_cast<const __nv_bfloat16*>(&t);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float f = __bfloat162float(tb[e]);
+          if (f > m[e]) m[e] = f;
+        }
+      }
+    uint4 o;
+    __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(&o);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) ob[e] = __float2bfloat16_rn(m[e]);
+    y[i] = o;
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) nchw_to_nhwc_kernel(const T* __restrict__ x, int64_t N,
+                                                           int64_t C, int64_t H, int64_t W,
+                                                           int64_t Cp, T* __restrict__ y) {
+  const int64_t total = N * H * W * Cp;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t c = i % Cp;
+    const int64_t w = (i / Cp) % W;
+    const int64_t h = (i / (Cp * W)) % H;
+    const int64_t b = i / (Cp * W * H);
+    y[i] = c < C ? x[((b * C + c) * H + h) * W + w] : from_f32<T>(0.0f);
+  }
+}
+
+int64_t grid_for(int64_t total) {
+  const int64_t cap = static_cast<int64_t>(device_sm_count()) * 16;
+  return std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, cap));
+}
+
+}  // namespace
+
+tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s) {
+  DirectArgs a{};
+  a.N = p.N; a.C = p.C; a.H = p.H; a.W = p.W; a.K = p.K; a.R = p.R; a.S = p.S;
+  a.sh = p.sh; a.sw = p.sw; a.ph = p.ph; a.pw = p.pw; a.P = p.P; a.Q = p.Q;
+  a.wpf = (p.C * p.R * p.S + 15) / 16;
+  a.x = p.x; a.codes = p.codes; a.alpha = p.alpha; a.y = p.y;
+  a.residual = p.residual; a.relu = p.relu;
+  const bool nhwc = p.layout == TBN_NHWC;
+  const bool xb = p.xdt == TBN_BF16, yb = p.ydt == TBN_BF16;
+  using bf = __nv_bfloat16;
+  if (nhwc) {
+    if (xb && yb) return launch_direct_t<bf, bf, true>(a, s);
+    if (xb && !yb) return launch_direct_t<bf, float, true>(a, s);
+    if (!xb && yb) return launch_direct_t<float, bf, true>(a, s);
+    return launch_direct_t<float, float, true>(a, s);
+  }
+  if (xb && yb) return launch_direct_t<bf, bf, false>(a, s);
+  if (xb && !yb) return launch_direct_t<bf, float, false>(a, s);
+  if (!xb && yb) return launch_direct_t<float, bf, false>(a, s);
+  return launch_direct_t<float, float, false>(a, s);
+}
+
+tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
+                               int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
+                               void* y, cudaStream_t s) {
+  const int64_t Ho = (H - kh) / sh + 1, Wo = (W - kw) / sw + 1;
+  if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16)) {
+    const int64_t total = N * Ho * Wo * (C / 8);
+    maxpool_nhwc_bf16x8_kernel<<<(unsigned)grid_for(total), 256, 0, s>>>(
+        static_cast<const uint4*>(x), N, H, W, C / 8, kh, kw, sh, sw, Ho, Wo,
+        static_cast<uint4*>(y));
+  } else if (dt == TBN_BF16) {
+    const int64_t total = N * Ho * Wo * C;
+    maxpool_nhwc_kernel<__nv_bfloat16><<<(unsigned)grid_for(total), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(x), N, H, W, C, kh, kw, sh, sw, Ho, Wo,
+        static_cast<__nv_bfloat16*>(y));
+  } else {
+    const int64_t total = N * Ho * Wo * C;
+    maxpool_nhwc_kernel<float><<<(unsigned)grid_for(total), 256, 0, s>>>(
+        static_cast<const float*>(x), N, H, W, C, kh, kw, sh, sw, Ho, Wo,
+        static_cast<float*>(y));
+  }
+  return check_launch("maxpool_nhwc_kernel");
+}
+
+tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
+                               int64_t W, int64_t C_pad, void* y, cudaStream_t s) {
+  const int64_t total = N * H * W * C_pad;
+  if (dt == TBN_BF16)
+    nchw_to_nhwc_kernel<__nv_bfloat16><<<(unsigned)grid_for(total), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(x), N, C, H, W, C_pad, static_cast<__nv_bfloat16*>(y));
+  else
+    nchw_to_nhwc_kernel<float><<<(unsigned)grid_for(total), 256, 0, s>>>(
+        static_cast<const float*>(x), N, C, H, W, C_pad, static_cast<float*>(y));
+  return check_launch("nchw_to_nhwc_kernel");
+}
+
+}  // namespace tbn

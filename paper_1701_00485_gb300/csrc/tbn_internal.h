@@ -1,0 +1,75 @@
+// tbn_internal.h -- host-side declarations shared by the library's
+// translation units: error reporting, argument helpers and the launchers
+// each kernel file provides.  Not part of the public ABI (include/tbn.h).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "tbn.h"
+
+namespace tbn {
+
+// Record a failure detail for tbn_last_error() and return `s`.
+tbn_status fail(tbn_status s, const char* fmt, ...);
+const char* last_error_text();
+
+// Map a failed CUDA call to TBN_ERR_CUDA with its message.
+tbn_status cuda_fail(cudaError_t e, const char* what);
+
+// cudaGetLastError() after a launch.
+tbn_status check_launch(const char* what);
+
+// Device address of the current device's error word (set up once per
+// device); nullptr if it could not be resolved.
+uint32_t* device_error_word();
+
+// Multiprocessor count of the current device (cached per device).
+int device_sm_count();
+
+inline bool is_aligned(const void* p, size_t a) {
+  return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+inline cudaStream_t as_stream(tbn_stream s) { return reinterpret_cast<cudaStream_t>(s); }
+
+inline size_t dtype_size(tbn_dtype d) { return d == TBN_BF16 ? 2 : 4; }
+
+// One convolution problem after validation.
+struct ConvProblem {
+  int64_t N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
+  tbn_layout layout;
+  tbn_dtype xdt, ydt;
+  const void* x;
+  const uint32_t* codes;
+  const float* alpha;
+  void* y;
+  int relu;
+  const void* residual;
+};
+
+// ---- launchers (each defined next to its kernels) ----
+tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStream_t s);
+tbn_status launch_unpack(const uint32_t* codes, const float* alpha, int64_t K, int64_t n,
+                         void* out, tbn_unpack_format fmt, cudaStream_t s);
+
+tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s);
+
+// Empty string when the implicit-GEMM kernel can run `p`, else the reason.
+const char* conv_igemm_unsupported_reason(const ConvProblem& p);
+tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s);
+
+const char* gemv_unsupported_reason(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                                    const uint32_t* codes);
+tbn_status launch_gemv(const void* x, int64_t B, int64_t K_in, const uint32_t* codes,
+                       const float* alpha, int64_t K_out, void* y, tbn_dtype ydt, int relu,
+                       const void* residual, cudaStream_t s);
+
+tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
+                               int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
+                               void* y, cudaStream_t s);
+tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
+                               int64_t W, int64_t C_pad, void* y, cudaStream_t s);
+
+}  // namespace tbn

@@ -1,0 +1,284 @@
+// tbn_quantize.cu -- per-filter discretization + optimal scaling factor +
+// two-bit packing (Algorithm 1, quantization loop; Eq. 3 and Eq. 5 of
+// Section 2), and the inverse unpack.
+//
+// One streaming pass over W: Eq. 3's thresholds are absolute (+-1, 0), so
+// the codes do not depend on alpha and Eq. 5's two sums can be accumulated
+// in the same pass that discretizes.  Each thread owns whole 32-bit output
+// words (16 consecutive weights of a filter): it loads 64 contiguous bytes,
+// forms the sixteen 2-bit fields, and accumulates |W~|*|W| (fp32 within the
+// word, fp64 across words) and the count of magnitude-two codes.  Filters
+// are reduced by a warp (short filters, 8 per CTA) or by a whole 256-thread
+// CTA (long filters).  Bytes moved per weight: 4 read + 1/4 written.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "tbn_device.cuh"
+#include "tbn_internal.h"
+
+namespace tbn {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kRowsPerNarrowCta = kThreads / 32;
+constexpr int kWideMinWords = 257;  // filters with more words use a whole CTA
+
+struct QJob {
+  const float* W;
+  uint32_t* codes;
+  float* alpha;
+  int64_t K;
+  int64_t first_task;  // index of this job's first CTA task
+  int32_t n;
+  int32_t wpf;  // words per filter
+  int32_t vec;  // 16-byte loads allowed
+  int32_t wide;
+};
+
+struct QParams {
+  QJob job[TBN_MAX_QUANT_JOBS];
+  int njobs;
+  uint32_t* err;
+};
+
+// Sixteen weights -> one packed word, the sum of |W~|*|W| over them (fp32,
+// pairwise; redone in fp64 when the fp32 sum overflows, i.e. for weights
+// near the fp32 maximum) and the number of magnitude-two codes.  Eq. 3:
+// s = [W <= 0] (so -1 <= W <= 0 and W < -1 are negative, -0.0 included),
+// m = [|W| > 1].
+__device__ __forceinline__ void encode16(const float (&v)[16], int nvalid, uint32_t& word,
+                                         double& dsum, int& cnt2) {
+  float c[16];
+  uint32_t w = 0;
+  int n2 = 0;
+#pragma unroll
+  for (int e = 0; e < 16; ++e) {
+    const float a = fabsf(v[e]);
+    const uint32_t m = a > 1.0f ? 1u : 0u;
+    const uint32_t s = v[e] <= 0.0f ? 1u : 0u;
+    const bool valid = e < nvalid;
+    w |= valid ? ((m | (s << 1)) << (2 * e)) : 0u;
+    n2 += (valid && m) ? 1 : 0;
+    c[e] = valid ? (m ? 2.0f * a : a) : 0.0f;
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) c[e] += c[e + 8];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) c[e] += c[e + 4];
+  c[0] += c[2];
+  c[1] += c[3];
+  const float sum = c[0] + c[1];
+  if (sum <= 3.4028234663852886e38f) {
+    dsum = static_cast<double>(sum);
+  } else {
+    double d = 0.0;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      const double a = fabs(static_cast<double>(v[e]));
+      d += (e < nvalid) ? (a > 1.0 ? 2.0 * a : a) : 0.0;
+    }
+    dsum = d;
+  }
+  word = w;
+  cnt2 = n2;
+}
+
+__device__ __forceinline__ void load16(const float* __restrict__ row, int n, int j, bool vec,
+                                       float (&v)[16], int& nvalid) {
+  const int base = 16 * j;
+  nvalid = min(16, n - base);
+  if (vec && nvalid == 16) {
+    const float4* p = reinterpret_cast<const float4*>(row + base);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 t = __ldcs(p + q);
+      v[4 * q + 0] = t.x;
+      v[4 * q + 1] = t.y;
+      v[4 * q + 2] = t.z;
+      v[4 * q + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 16; ++e) v[e] = (e < nvalid) ? __ldcs(row + base + e) : 0.0f;
+  }
+}
+
+// Process words j0, j0 + stride, ... of one filter; returns the partial sums.
+template <int kUnroll>
+__device__ __forceinline__ void quantize_words(const float* __restrict__ row,
+                                               uint32_t* __restrict__ out, int n, int wpf,
+                                               bool vec, int j0, int stride, double& acc,
+                                               int& cnt2) {
+  int j = j0;
+  for (; j + (kUnroll - 1) * stride < wpf; j += kUnroll * stride) {
+    float v[kUnroll][16];
+    int nv[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) load16(row, n, j + u * stride, vec, v[u], nv[u]);
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      uint32_t word;
+      double s;
+      int c;
+      encode16(v[u], nv[u], word, s, c);
+      out[j + u * stride] = word;
+      acc += s;
+      cnt2 += c;
+    }
+  }
+  for (; j < wpf; j += stride) {
+    float v[16];
+    int nv;
+    load16(row, n, j, vec, v, nv);
+    uint32_t word;
+    double s;
+    int c;
+    encode16(v, nv, word, s, c);
+    out[j] = word;
+    acc += s;
+    cnt2 += c;
+  }
+}
+
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ int warp_sum(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Eq. 5 with |B1| + 4|B2| = n + 3|B2|; one rounding to fp32 at the end.
+__device__ __forceinline__ float alpha_of(double num, int cnt2, int n) {
+  const double den = static_cast<double>(n) + 3.0 * static_cast<double>(cnt2);
+  return static_cast<float>(num / den);
+}
+
+__global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_constant__ QParams prm) {
+  __shared__ double s_acc[kThreads / 32];
+  __shared__ int s_cnt[kThreads / 32];
+
+  const int64_t task = blockIdx.x;
+  int ji = 0;
+#pragma unroll 1
+  for (int i = 1; i < prm.njobs; ++i)
+    if (task >= prm.job[i].first_task) ji = i;
+  const QJob& jb = prm.job[ji];
+  const int64_t local = task - jb.first_task;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (jb.wide) {
+    const int64_t k = local;
+    if (k >= jb.K) return;
+    const float* row = jb.W + k * static_cast<int64_t>(jb.n);
+    uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
+    double acc = 0.0;
+    int cnt2 = 0;
+    quantize_words<4>(row, out, jb.n, jb.wpf, jb.vec != 0, threadIdx.x, kThreads, acc, cnt2);
+    acc = warp_sum(acc);
+    cnt2 = warp_sum(cnt2);
+    if (lane == 0) {
+      s_acc[warp] = acc;
+      s_cnt[warp] = cnt2;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      acc = lane < kThreads / 32 ? s_acc[lane] : 0.0;
+      cnt2 = lane < kThreads / 32 ? s_cnt[lane] : 0;
+      acc = warp_sum(acc);
+      cnt2 = warp_sum(cnt2);
+      if (lane == 0) jb.alpha[k] = alpha_of(acc, cnt2, jb.n);
+    }
+  } else {
+    const int64_t k = local * kRowsPerNarrowCta + warp;
+    if (k >= jb.K) return;
+    const float* row = jb.W + k * static_cast<int64_t>(jb.n);
+    uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
+    double acc = 0.0;
+    int cnt2 = 0;
+    quantize_words<2>(row, out, jb.n, jb.wpf, jb.vec != 0, lane, 32, acc, cnt2);
+    acc = warp_sum(acc);
+    cnt2 = warp_sum(cnt2);
+    if (lane == 0) jb.alpha[k] = alpha_of(acc, cnt2, jb.n);
+  }
+}
+
+template <int kFmt>
+__global__ void __launch_bounds__(256) unpack_kernel(const uint32_t* __restrict__ codes,
+                                                     const float* __restrict__ alpha, int64_t K,
+                                                     int64_t n, int64_t wpf, void* out) {
+  const int64_t total = K * wpf;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t k = t / wpf, j = t % wpf;
+    const uint32_t w = codes[t];
+    const float a = (kFmt == TBN_UNPACK_I8) ? 1.0f : alpha[k];
+    const int64_t base = k * n + 16 * j;
+    const int64_t left = n - 16 * j;
+    const int cnt = left < 16 ? static_cast<int>(left) : 16;
+    for (int e = 0; e < cnt; ++e) {
+      const float v = code_value((w >> (2 * e)) & 3u);
+      if (kFmt == TBN_UNPACK_I8) {
+        static_cast<int8_t*>(out)[base + e] = static_cast<int8_t>(v);
+      } else if (kFmt == TBN_UNPACK_F32) {
+        static_cast<float*>(out)[base + e] = a * v;
+      } else {
+        static_cast<__nv_bfloat16*>(out)[base + e] = __float2bfloat16_rn(a * v);
+      }
+    }
+  }
+}
+
+}  // namespace
+
+tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStream_t s) {
+  QParams prm{};
+  prm.njobs = njobs;
+  prm.err = device_error_word();
+  int64_t tasks = 0;
+  for (int i = 0; i < njobs; ++i) {
+    const tbn_quant_job& j = jobs[i];
+    QJob& q = prm.job[i];
+    q.W = j.W;
+    q.codes = j.codes;
+    q.alpha = j.alpha;
+    q.K = j.K;
+    q.n = static_cast<int32_t>(j.n);
+    q.wpf = static_cast<int32_t>((j.n + 15) / 16);
+    q.vec = (is_aligned(j.W, 16) && (j.n % 4) == 0) ? 1 : 0;
+    q.wide = q.wpf >= kWideMinWords ? 1 : 0;
+    q.first_task = tasks;
+    tasks += q.wide ? j.K : (j.K + kRowsPerNarrowCta - 1) / kRowsPerNarrowCta;
+  }
+  if (tasks == 0) return TBN_OK;
+  if (tasks > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "quantize: too many filters (%lld tasks)", (long long)tasks);
+  quantize_pack_kernel<<<static_cast<unsigned>(tasks), kThreads, 0, s>>>(prm);
+  return check_launch("quantize_pack_kernel");
+}
+
+tbn_status launch_unpack(const uint32_t* codes, const float* alpha, int64_t K, int64_t n,
+                         void* out, tbn_unpack_format fmt, cudaStream_t s) {
+  const int64_t wpf = (n + 15) / 16;
+  const int64_t total = K * wpf;
+  const int64_t blocks = std::min<int64_t>((total + 255) / 256, 65536);
+  switch (fmt) {
+    case TBN_UNPACK_I8:
+      unpack_kernel<TBN_UNPACK_I8><<<blocks, 256, 0, s>>>(codes, alpha, K, n, wpf, out);
+      break;
+    case TBN_UNPACK_F32:
+      unpack_kernel<TBN_UNPACK_F32><<<blocks, 256, 0, s>>>(codes, alpha, K, n, wpf, out);
+      break;
+    case TBN_UNPACK_BF16:
+      unpack_kernel<TBN_UNPACK_BF16><<<blocks, 256, 0, s>>>(codes, alpha, K, n, wpf, out);
+      break;
+  }
+  return check_launch("unpack_kernel");
+}
+
+}  // namespace tbn

@@ -1,0 +1,114 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and
+loads, exports every function include/tbn.h declares, and rejects invalid
+arguments on the host before launching anything."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_1701_00485_gb300 as tbn
+from paper_1701_00485_gb300 import build as tbn_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "tbn.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    tbn_build.build()
+    return tbn.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"\b(tbn_[a-z0-9_]+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_header_declares_the_python_export_list():
+    assert declared_functions() == sorted(tbn.EXPORTED)
+
+
+def test_every_declared_symbol_is_exported(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+
+
+def test_abi_version_and_sizes(L):
+    assert L.tbn_abi_version() == 1
+    assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
+        [1, 1, 1, 2, 2, 72, 1024]
+    assert L.tbn_packed_words(0) == -1
+    assert L.tbn_status_string(0) == b"ok"
+    assert L.tbn_status_string(2) == b"unsupported"
+
+
+def test_quantize_rejects_bad_arguments(L):
+    dummy = ctypes.c_void_p(256)
+    assert L.tbn_quantize_pack(None, 4, 16, dummy, dummy, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_quantize_pack(dummy, 0, 16, dummy, dummy, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_quantize_pack(dummy, 4, 0, dummy, dummy, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_quantize_pack(ctypes.c_void_p(258), 4, 16, dummy, dummy, None) == \
+        tbn.TBN_ERR_MISALIGNED
+    assert L.tbn_quantize_pack(dummy, 4, 1 << 31, dummy, dummy, None) == tbn.TBN_ERR_UNSUPPORTED
+    assert b"quantize" in L.tbn_last_error()
+    jobs = (tbn.QuantJob * 17)()
+    assert L.tbn_quantize_pack_group(jobs, 17, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_quantize_pack_group(jobs, 0, None) == tbn.TBN_ERR_INVALID_ARG
+
+
+def test_unpack_rejects_bad_arguments(L):
+    d = ctypes.c_void_p(256)
+    assert L.tbn_unpack(None, d, 1, 1, d, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_unpack(d, None, 1, 1, d, tbn.TBN_UNPACK_F32, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_unpack(d, d, 1, 1, d, 7, None) == tbn.TBN_ERR_INVALID_ARG
+
+
+def _conv(L, **kw):
+    d = ctypes.c_void_p(256)
+    a = dict(x=d, xdt=1, layout=1, N=1, C=64, H=8, W=8, codes=d, alpha=d, K=64, R=3, S=3,
+             sh=1, sw=1, ph=1, pw=1, y=d, ydt=1, epi=None, algo=0)
+    a.update(kw)
+    return L.tbn_conv2d_fwd_algo(a["x"], a["xdt"], a["layout"], a["N"], a["C"], a["H"], a["W"],
+                                 a["codes"], a["alpha"], a["K"], a["R"], a["S"], a["sh"], a["sw"],
+                                 a["ph"], a["pw"], a["y"], a["ydt"], a["epi"], a["algo"], None)
+
+
+def test_conv_rejects_bad_arguments(L):
+    assert _conv(L, x=None) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, N=0) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, xdt=5) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, layout=9) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, sh=0) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, ph=-1) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, H=2, W=2, ph=0, pw=0) == tbn.TBN_ERR_INVALID_ARG   # kernel > input
+    assert _conv(L, x=ctypes.c_void_p(257)) == tbn.TBN_ERR_MISALIGNED
+    assert _conv(L, C=1 << 20, H=1 << 12, W=1) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, algo=11) == tbn.TBN_ERR_INVALID_ARG
+
+
+def test_select_algo_host_rules(L):
+    # without a GPU (or for shapes it cannot take) AUTO falls back to DIRECT;
+    # shapes the implicit GEMM never takes are DIRECT everywhere
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").float32, tbn.TBN_NHWC,
+                                      1, 64, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW,
+                                      1, 64, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NHWC,
+                                      1, 3, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+
+
+def test_linear_and_glue_reject_bad_arguments(L):
+    d = ctypes.c_void_p(256)
+    assert L.tbn_linear_fwd(None, 1, 1, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_linear_fwd(d, 1, 0, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_maxpool2d_nhwc(d, 1, 1, 4, 4, 8, 5, 5, 1, 1, d, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_nchw_to_nhwc(d, 1, 1, 4, 4, 4, 3, d, None) == tbn.TBN_ERR_INVALID_ARG
+
+
+def test_python_binding_requires_cuda_tensors():
+    import torch
+    with pytest.raises(ValueError):
+        tbn.tbn_quantize_pack(torch.zeros(2, 16))

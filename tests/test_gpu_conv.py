@@ -1,0 +1,149 @@
+"""GPU parity of tbn_conv2d_fwd (direct and tcgen05 implicit-GEMM kernels)
+against the oracle's seven-loop convolution, per output:
+|y_gpu - y_orc| <= 2e-3 * |alpha| * sum|x| (fp32 output), plus the bf16
+output rounding for bf16 output."""
+import numpy as np
+import pytest
+import torch
+
+import paper_1701_00485_gb300 as tbn
+from paper_1701_00485_gb300 import inputs
+from parity_util import ConvCase, assert_within, random_sites
+
+pytestmark = pytest.mark.gpu
+
+
+def make_case(N, C, H, W, K, R, S, stride, pad, seed, wscale=None, xdist="normal"):
+    g = inputs.generator(seed)
+    if xdist == "normal":
+        x = torch.randn(N, C, H, W, generator=g)
+    else:
+        x = torch.rand(N, C, H, W, generator=g)
+    std = wscale if wscale is not None else (2.0 / (C * R * S)) ** 0.5
+    Wt = inputs.normal((K, C, R, S), std, g)
+    return ConvCase(x, Wt, stride, pad)
+
+
+# ---------------------------------------------------------------- direct kernel
+DIRECT = [
+    # N, C, H, W, K, R, S, stride, pad
+    (2, 3, 9, 7, 5, 3, 3, (1, 1), (1, 1)),
+    (1, 1, 28, 28, 20, 5, 5, (1, 1), (0, 0)),
+    (3, 4, 11, 10, 33, 5, 5, (2, 2), (2, 2)),
+    (2, 8, 6, 6, 7, 1, 1, (1, 1), (0, 0)),
+    (1, 3, 23, 23, 40, 11, 11, (4, 4), (0, 0)),
+    (1, 5, 9, 7, 3, 3, 1, (1, 2), (0, 1)),
+    (2, 70, 5, 5, 65, 3, 3, (1, 1), (1, 1)),
+]
+
+
+@pytest.mark.parametrize("case", DIRECT)
+@pytest.mark.parametrize("layout", [tbn.TBN_NCHW, tbn.TBN_NHWC])
+@pytest.mark.parametrize("xdt", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("ydt", [torch.float32, torch.bfloat16])
+def test_direct_conv_matches_oracle(case, layout, xdt, ydt):
+    c = make_case(*case, seed=sum(case[:7]), wscale=1.3)
+    y = c.run_gpu(layout, xdt, ydt, algo=tbn.TBN_CONV_DIRECT)
+    y_orc, bound = c.oracle_full(xdt)
+    assert_within(y, y_orc, bound, out_bf16=(ydt == torch.bfloat16), what="direct %s" % (case,))
+
+
+def test_lenet_layer_full():
+    # the LeNet-like workload: fp32 input U(0,1), W ~ N(0, 0.1), quantize + conv
+    x, W = inputs.lenet_inputs(0)
+    c = ConvCase(x, W, (1, 1), (0, 0))
+    y = c.run_gpu(tbn.TBN_NCHW, torch.float32, torch.float32)
+    y_orc, bound = c.oracle_full(torch.float32)
+    assert_within(y, y_orc, bound, out_bf16=False, what="lenet")
+
+
+# ---------------------------------------------------------------- implicit GEMM
+IGEMM = [
+    # N, C, H, W, K, R, S, stride, pad    (all NHWC bf16, C % 64 == 0)
+    (1, 64, 8, 8, 128, 3, 3, (1, 1), (1, 1)),       # one tile, exact
+    (2, 64, 8, 8, 128, 1, 1, (1, 1), (0, 0)),       # 1x1
+    (3, 128, 16, 16, 256, 3, 3, (1, 1), (1, 1)),    # two filter tiles
+    (2, 64, 32, 32, 128, 3, 3, (1, 1), (1, 1)),     # 32-wide rows, 8-row tiles
+    (5, 64, 7, 7, 200, 3, 3, (1, 1), (1, 1)),       # ragged K and image packing
+    (3, 64, 13, 13, 96, 3, 3, (1, 1), (1, 1)),      # N = 176 tile, K < 128
+    (2, 128, 28, 28, 64, 3, 3, (1, 1), (1, 1)),     # balanced row tiles
+    (2, 64, 9, 11, 130, 3, 3, (1, 1), (0, 0)),      # valid conv, odd sizes
+    (2, 64, 14, 14, 128, 3, 3, (2, 2), (1, 1)),     # stride 2
+    (2, 64, 15, 15, 128, 1, 1, (2, 2), (0, 0)),     # 1x1 stride 2 projection
+    (1, 192, 6, 5, 136, 2, 3, (1, 1), (1, 0)),      # R != S, asymmetric pad
+    (1, 64, 300, 4, 128, 3, 3, (1, 1), (1, 1)),     # Q < P, tall image
+    (1, 64, 3, 300, 128, 3, 3, (1, 1), (1, 1)),     # Q > 256: several q tiles
+]
+
+
+@pytest.mark.parametrize("case", IGEMM)
+def test_igemm_conv_matches_oracle_fp32_out(case):
+    c = make_case(*case, seed=1000 + sum(case[:7]), wscale=1.2)
+    algo = tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NHWC, *case[:7], case[7], case[8])
+    assert algo == tbn.TBN_CONV_IMPLICIT_GEMM
+    y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    assert_within(y, y_orc, bound, out_bf16=False, what="igemm %s" % (case,))
+
+
+@pytest.mark.parametrize("case", IGEMM[:6])
+def test_igemm_conv_bf16_out_and_epilogue(case):
+    c = make_case(*case, seed=2000 + sum(case[:7]))
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.bfloat16, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+    assert_within(y, y_orc, bound, out_bf16=True, what="igemm bf16 %s" % (case,))
+    # fused residual + ReLU, checked against the oracle's epilogue
+    import oracle
+    g = inputs.generator(7)
+    res = torch.randn(*y_orc.shape, generator=g).to(torch.bfloat16)
+    want = oracle.epilogue(y_orc, res.float().numpy(), relu=True)
+    y2 = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.bfloat16, algo=tbn.TBN_CONV_IMPLICIT_GEMM,
+                   relu=True, residual=res)
+    assert_within(y2, want, bound, out_bf16=True, epilogue=True, what="igemm epi %s" % (case,))
+
+
+@pytest.mark.parametrize("case", IGEMM[2:5])
+def test_igemm_equals_direct_kernel(case):
+    c = make_case(*case, seed=3000 + sum(case[:7]))
+    y1 = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+    y2 = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_DIRECT)
+    _, bound = c.oracle_full(torch.bfloat16)
+    assert np.all(np.abs(y1 - y2) <= 4e-3 * bound + 1e-30)
+
+
+# ------------------------------------------------------ workload layers, full size
+def _workload_layers():
+    out = []
+    for i, s in enumerate(inputs.VGG_SMALL["convs"]):
+        hw = 32 >> (i // 2)
+        out.append(("vgg_c%d" % (i + 1), 128, s, hw))
+    a = inputs.ALEXNET["convs"]
+    out += [("alex_conv1", 256, a[0], 227), ("alex_conv2", 256, a[1], 27),
+            ("alex_conv3", 256, a[2], 13), ("alex_conv4", 256, a[3], 13),
+            ("alex_conv5", 256, a[4], 13)]
+    # input size of each ResNet-18 conv (224 -> stem /2 -> pool /2 = 56)
+    stage_hw = {"l1": 56, "l2": 28, "l3": 14, "l4": 7}
+    prev_hw = {"l1": 56, "l2": 56, "l3": 28, "l4": 14}
+    for name, s in inputs.resnet18_convs():
+        stage = name[:2]
+        h = prev_hw[stage] if (s.stride == 2) else stage_hw[stage]
+        out.append(("resnet_" + name, 128, s, h))
+    return out
+
+
+WORKLOAD = _workload_layers()
+
+
+@pytest.mark.parametrize("name,N,spec,hw", WORKLOAD, ids=[w[0] for w in WORKLOAD])
+def test_workload_layer_sampled(name, N, spec, hw):
+    """Each conv layer of the VGG-small / AlexNet / ResNet-18 workloads at its
+    full batch and size, in the launch configuration the networks use
+    (NHWC bf16 in, bf16 out, AUTO algorithm), checked at sampled outputs."""
+    g = inputs.generator(hash(name) % 100000)
+    x = torch.randn(N, spec.C, hw, hw, generator=g).to(torch.bfloat16)
+    W = inputs.he_normal(spec.K, spec.C, spec.R, spec.S, g)
+    c = ConvCase(x, W, (spec.stride, spec.stride), (spec.pad, spec.pad))
+    y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.bfloat16)
+    sites = random_sites(y.shape, 3000, seed=len(name))
+    y_orc, bound = c.oracle_sites(torch.bfloat16, sites)
+    assert_within(y[tuple(sites.T)], y_orc, bound, out_bf16=True, what=name)

@@ -1,0 +1,92 @@
+"""GPU parity of tbn_linear_fwd (tensor-core GEMV for B <= 8, 1x1
+convolution otherwise) and of the glue kernels, against the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_1701_00485_gb300 as tbn
+from paper_1701_00485_gb300 import inputs
+from parity_util import assert_within, check_quantize
+
+pytestmark = pytest.mark.gpu
+
+
+def run_linear(W, x, out_dtype, relu=False, residual=None):
+    codes, alpha = tbn.tbn_quantize_pack(W.cuda())
+    check_quantize(W, codes, alpha)
+    y = tbn.tbn_linear_fwd(x.cuda(), codes, alpha, W.shape[0], out_dtype=out_dtype, relu=relu,
+                           residual=residual.cuda() if residual is not None else None)
+    torch.cuda.synchronize()
+    wt, al = oracle.quantize(W.numpy())
+    y_orc, bound = oracle.linear(x.float().numpy(), wt, al)
+    return y.float().cpu().numpy(), y_orc, bound
+
+
+@pytest.mark.parametrize("B", [1, 2, 3, 8])
+@pytest.mark.parametrize("K_in,K_out", [(64, 16), (256, 48), (1024, 100), (4096, 4096)])
+def test_gemv_matches_oracle(B, K_in, K_out):
+    g = inputs.generator(B * 131 + K_in + K_out)
+    W = inputs.normal((K_out, K_in), 1.3, g)
+    x = torch.randn(B, K_in, generator=g).to(torch.bfloat16)
+    y, y_orc, bound = run_linear(W, x, torch.float32)
+    assert_within(y, y_orc, bound, out_bf16=False, what="gemv")
+    y, y_orc, bound = run_linear(W, x, torch.bfloat16)
+    assert_within(y, y_orc, bound, out_bf16=True, what="gemv bf16")
+
+
+@pytest.mark.parametrize("K", inputs.GEMV_SIZES)
+@pytest.mark.parametrize("B", inputs.GEMV_BATCHES)
+def test_gemv_workload_full(K, B):
+    """The GEMV workload at full size: every output compared with the oracle."""
+    W, x = inputs.gemv_inputs(K, B)
+    y, y_orc, bound = run_linear(W, x, torch.bfloat16)
+    assert_within(y, y_orc, bound, out_bf16=True, what="gemv K=%d B=%d" % (K, B))
+
+
+def test_gemv_epilogue():
+    g = inputs.generator(99)
+    W = inputs.normal((200, 512), 1.0, g)
+    x = torch.randn(3, 512, generator=g).to(torch.bfloat16)
+    res = torch.randn(3, 200, generator=g)
+    y, y_orc, bound = run_linear(W, x, torch.float32, relu=True, residual=res)
+    want = oracle.epilogue(y_orc, res.numpy(), relu=True)
+    assert_within(y, want, bound, out_bf16=False, epilogue=True, what="gemv epilogue")
+
+
+@pytest.mark.parametrize("B,K_in,K_out,xdt", [(16, 96, 40, torch.bfloat16),
+                                              (256, 1024, 1000, torch.bfloat16),
+                                              (4, 100, 30, torch.float32),
+                                              (9, 64, 64, torch.bfloat16)])
+def test_linear_as_conv_matches_oracle(B, K_in, K_out, xdt):
+    g = inputs.generator(B + K_in)
+    W = inputs.normal((K_out, K_in), 1.1, g)
+    x = torch.randn(B, K_in, generator=g).to(xdt)
+    y, y_orc, bound = run_linear(W, x, torch.float32)
+    assert_within(y, y_orc, bound, out_bf16=False, what="linear-as-conv")
+
+
+@pytest.mark.parametrize("shape,k,s", [((2, 32, 32, 128), (2, 2), (2, 2)),
+                                       ((3, 55, 55, 96), (3, 3), (2, 2)),
+                                       ((1, 9, 8, 5), (2, 2), (2, 2)),
+                                       ((2, 13, 13, 256), (3, 3), (2, 2))])
+@pytest.mark.parametrize("dt", [torch.bfloat16, torch.float32])
+def test_maxpool_matches_oracle(shape, k, s, dt):
+    g = inputs.generator(sum(shape))
+    x = torch.randn(*shape, generator=g).to(dt)
+    y = tbn.tbn_maxpool2d_nhwc(x.cuda(), k, s).float().cpu().numpy()
+    want = oracle.maxpool2d_nchw(x.float().permute(0, 3, 1, 2).numpy(), k, s)
+    assert np.array_equal(y, want.transpose(0, 2, 3, 1))
+
+
+@pytest.mark.parametrize("dt", [torch.bfloat16, torch.float32])
+def test_nchw_to_nhwc_padding(dt):
+    g = inputs.generator(5)
+    x = torch.randn(2, 3, 5, 7, generator=g).to(dt)
+    y = tbn.tbn_nchw_to_nhwc(x.cuda(), C_pad=8).cpu()
+    assert torch.equal(y[..., :3], x.permute(0, 2, 3, 1))
+    assert torch.all(y[..., 3:] == 0)
+
+
+def test_device_error_word_is_clear():
+    assert tbn.tbn_device_error() == 0
