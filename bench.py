@@ -157,10 +157,10 @@ def run_ours(args, rank, world, local_rank):
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     sampler = ClockSampler(local_rank)
     sampler.start()
-    # warm-up: W replays, and at least ~1 s of replays so clocks settle
+    # warm-up: W replays, and at least --min-warmup-s of replays so clocks settle
     t_w = time.time()
     w = 0
-    while w < args.warmup or time.time() - t_w < 1.0:
+    while w < args.warmup or time.time() - t_w < args.min_warmup_s:
         with torch.cuda.stream(stream):
             flush.zero_()
             graph.replay()
@@ -312,6 +312,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--min-warmup-s", type=float, default=1.0,
+                    help="keep replaying warm-up steps for at least this long (clock settling)")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))

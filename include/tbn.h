@@ -81,18 +81,23 @@ typedef enum {
 /* Convolution algorithms.  AUTO picks the fastest implemented one. */
 typedef enum {
   TBN_CONV_AUTO = 0,
-  TBN_CONV_DIRECT = 1,        /* CUDA-core direct convolution, any layout/dtype  */
-  TBN_CONV_IMPLICIT_GEMM = 2  /* tcgen05 implicit GEMM: NHWC, bf16 x, C % 64 == 0,
-                                 stride 1 or 2                                    */
+  TBN_CONV_DIRECT = 1,        /* CUDA-core direct convolution, any layout/dtype   */
+  TBN_CONV_IMPLICIT_GEMM = 2  /* tcgen05 implicit GEMM, NHWC bf16 x; activations
+                                 by TMA when C % 64 == 0, else gathered by threads */
 } tbn_conv_algo;
 
 /* Fused layer epilogue (network glue, not part of the paper's method):
  *   v = alpha[k] * acc;  if (residual) v += residual[same index];
- *   if (relu) v = max(v, 0);  y = v rounded to y's dtype.
- * `residual` has y's layout, shape and dtype.  Pass NULL for no epilogue. */
+ *   if (relu) v = max(v, 0);
+ *   if (pool == 2) v = max of v over a 2x2 window, stride 2 (floor sizes);
+ *   y = v rounded to y's dtype.
+ * `residual` has y's layout, shape and dtype (not combinable with pool).
+ * With pool == 2, y is [N][P/2][Q/2][K] (NHWC) / [N][K][P/2][Q/2] (NCHW).
+ * Pass NULL for no epilogue. */
 typedef struct {
   int relu;
   const void *residual;
+  int pool; /* 0: none, 2: 2x2 max pool, stride 2 */
 } tbn_epilogue;
 
 /* A cudaStream_t, passed as an opaque pointer. */
@@ -170,9 +175,9 @@ tbn_status tbn_unpack(const uint32_t *codes, const float *alpha, int64_t K, int6
  *          P = (H + 2 ph - R) / sh + 1, Q = (W + 2 pw - S) / sw + 1.
  *   epi    optional fused epilogue (NULL = none).
  * Accumulation is fp32; x * W~ products are exact.  y must not alias x.
- * The implicit-GEMM path needs NHWC, bf16 x, C % 64 == 0, 16-byte aligned x,
- * stride 1 or 2, P and Q <= 256; AUTO falls back to the direct kernel
- * otherwise. */
+ * The tensor-core implicit-GEMM path needs NHWC and bf16 x (16-byte aligned
+ * x, y and residual; stride 1 or 2 when C % 64 == 0, any stride otherwise);
+ * AUTO falls back to the CUDA-core direct kernel for every other case. */
 tbn_status tbn_conv2d_fwd(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
                           int64_t C, int64_t H, int64_t W, const uint32_t *codes,
                           const float *alpha, int64_t K, int64_t R, int64_t S,

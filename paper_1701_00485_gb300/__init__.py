@@ -61,7 +61,7 @@ class QuantJob(ctypes.Structure):
 
 
 class Epilogue(ctypes.Structure):
-    _fields_ = [("relu", ctypes.c_int), ("residual", ctypes.c_void_p)]
+    _fields_ = [("relu", ctypes.c_int), ("residual", ctypes.c_void_p), ("pool", ctypes.c_int)]
 
 
 _lock = threading.Lock()
@@ -152,10 +152,11 @@ def _stream(stream) -> ctypes.c_void_p:
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def _epi(relu: bool, residual) -> Epilogue | None:
-    if not relu and residual is None:
+def _epi(relu: bool, residual, pool: int = 0) -> Epilogue | None:
+    if not relu and residual is None and not pool:
         return None
-    return Epilogue(1 if relu else 0, residual.data_ptr() if residual is not None else None)
+    return Epilogue(1 if relu else 0, residual.data_ptr() if residual is not None else None,
+                    int(pool))
 
 
 def packed_words(n: int) -> int:
@@ -215,14 +216,18 @@ def tbn_unpack(codes: torch.Tensor, alpha: torch.Tensor | None, n: int,
 def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K: int, R: int,
                    S: int, stride=(1, 1), pad=(0, 0), layout: int = TBN_NHWC,
                    out_dtype=None, relu: bool = False, residual: torch.Tensor | None = None,
-                   algo: int = TBN_CONV_AUTO, out: torch.Tensor | None = None, stream=None):
-    """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW) or [N,H,W,C] (NHWC)."""
+                   algo: int = TBN_CONV_AUTO, out: torch.Tensor | None = None, stream=None,
+                   pool: int = 0):
+    """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW) or [N,H,W,C] (NHWC).
+    pool=2 fuses a 2x2 / stride-2 max pool (after ReLU) into the epilogue."""
     _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
     if layout == TBN_NHWC:
         N, H, W, C = x.shape
     else:
         N, C, H, W = x.shape
     P, Q = conv_out_hw(H, W, R, S, stride, pad)
+    if pool:
+        P, Q = P // 2, Q // 2
     ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
     shape = (N, P, Q, K) if layout == TBN_NHWC else (N, K, P, Q)
     if out is None:
@@ -233,7 +238,7 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
         _cuda(residual, "residual")
         if tuple(residual.shape) != shape or _dt(residual) != ydt:
             raise ValueError("residual must match y's shape and dtype")
-    e = _epi(relu, residual)
+    e = _epi(relu, residual, pool)
     _check(lib().tbn_conv2d_fwd_algo(
         x.data_ptr(), _dt(x), layout, N, C, H, W, codes.data_ptr(), alpha.data_ptr(), K, R, S,
         stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,

@@ -108,6 +108,11 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
     return fail(TBN_ERR_MISALIGNED, "conv: pointer not aligned to its element size");
   if (epi && epi->residual && !is_aligned(epi->residual, ys))
     return fail(TBN_ERR_MISALIGNED, "conv: residual not aligned to its element size");
+  const int pool = epi ? epi->pool : 0;
+  if (pool != 0 && pool != 2) return fail(TBN_ERR_INVALID_ARG, "conv: pool must be 0 or 2");
+  if (pool && (P < 2 || Q < 2)) return fail(TBN_ERR_INVALID_ARG, "conv: pool needs P, Q >= 2");
+  if (pool && epi->residual)
+    return fail(TBN_ERR_UNSUPPORTED, "conv: pool cannot be combined with a residual");
   ConvProblem& p = *out;
   p.N = N; p.C = C; p.H = H; p.W = W; p.K = K; p.R = R; p.S = S;
   p.sh = sh; p.sw = sw; p.ph = ph; p.pw = pw; p.P = P; p.Q = Q;
@@ -115,6 +120,7 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
   p.x = x; p.codes = codes; p.alpha = alpha; p.y = y;
   p.relu = epi ? (epi->relu != 0) : 0;
   p.residual = epi ? epi->residual : nullptr;
+  p.pool = pool;
   return TBN_OK;
 }
 
@@ -256,6 +262,7 @@ tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
   if (!is_aligned(x, dtype_size(xdt)) || !is_aligned(y, ys) || !is_aligned(codes, 4) ||
       !is_aligned(alpha, 4) || (epi && epi->residual && !is_aligned(epi->residual, ys)))
     return fail(TBN_ERR_MISALIGNED, "linear: pointer not aligned to its element size");
+  if (epi && epi->pool != 0) return fail(TBN_ERR_INVALID_ARG, "linear: pool is not defined");
   if (gemv_unsupported_reason(x, xdt, B, K_in, codes)[0] == '\0') {
     return launch_gemv(x, B, K_in, codes, alpha, K_out, y, ydt, epi ? epi->relu : 0,
                        epi ? epi->residual : nullptr, as_stream(stream));

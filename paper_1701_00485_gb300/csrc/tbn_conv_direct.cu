@@ -46,7 +46,8 @@ __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
 
 struct DirectArgs {
   int64_t N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
-  int64_t wpf;  // words per filter
+  int64_t Po, Qo;  // output extent (P/2, Q/2 with the fused 2x2 pool)
+  int64_t wpf;     // words per filter
   const void* x;
   const uint32_t* codes;
   const float* alpha;
@@ -55,38 +56,51 @@ struct DirectArgs {
   int relu;
 };
 
-template <typename TX, typename TY, bool kNHWC>
+// kWin = 1: one conv output per thread, 32 filters.  kWin = 4: one 2x2-pooled
+// output per thread (four conv outputs, max after ReLU), 8 filters.
+template <typename TX, typename TY, bool kNHWC, int kWin>
 __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
-  __shared__ __align__(16) float s_w[kTapChunk][kFilt];
+  constexpr int kF = kWin == 1 ? kFilt : 8;
+  __shared__ __align__(16) float s_w[kTapChunk][kF];
   __shared__ int32_t s_off[kTapChunk];
   __shared__ int32_t s_rs[kTapChunk];
 
   const TX* __restrict__ x = static_cast<const TX*>(a.x);
-  const int64_t npix = a.N * a.P * a.Q;
+  const int64_t npix = a.N * a.Po * a.Qo;
   const int64_t pix = static_cast<int64_t>(blockIdx.x) * kPix + threadIdx.x;
-  const int64_t k0 = static_cast<int64_t>(blockIdx.y) * kFilt;
+  const int64_t k0 = static_cast<int64_t>(blockIdx.y) * kF;
   const bool active = pix < npix;
   const int64_t pc = active ? pix : 0;
-  const int64_t b = pc / (a.P * a.Q);
-  const int64_t p = (pc / a.Q) % a.P;
-  const int64_t q = pc % a.Q;
-  const int64_t h0 = p * a.sh - a.ph;
-  const int64_t w0 = q * a.sw - a.pw;
-  // element offset of (b, c = 0, h0, w0)
-  const int64_t base = kNHWC ? ((b * a.H + h0) * a.W + w0) * a.C
-                             : ((b * a.C) * a.H + h0) * a.W + w0;
-
-  float acc[kFilt];
+  const int64_t b = pc / (a.Po * a.Qo);
+  const int64_t po = (pc / a.Qo) % a.Po;
+  const int64_t qo = pc % a.Qo;
+  int h0[kWin], w0[kWin];
+  int64_t base[kWin];
 #pragma unroll
-  for (int f = 0; f < kFilt; ++f) acc[f] = 0.0f;
+  for (int wdx = 0; wdx < kWin; ++wdx) {
+    const int64_t p = kWin == 1 ? po : 2 * po + wdx / 2;
+    const int64_t q = kWin == 1 ? qo : 2 * qo + wdx % 2;
+    h0[wdx] = static_cast<int>(p * a.sh - a.ph);
+    w0[wdx] = static_cast<int>(q * a.sw - a.pw);
+    // element offset of (b, c = 0, h0, w0)
+    base[wdx] = kNHWC ? ((b * a.H + h0[wdx]) * a.W + w0[wdx]) * a.C
+                      : ((b * a.C) * a.H + h0[wdx]) * a.W + w0[wdx];
+  }
+  const int H = static_cast<int>(a.H), W = static_cast<int>(a.W);
+
+  float acc[kWin][kF];
+#pragma unroll
+  for (int wdx = 0; wdx < kWin; ++wdx)
+#pragma unroll
+    for (int f = 0; f < kF; ++f) acc[wdx][f] = 0.0f;
 
   const int64_t ntaps = a.C * a.R * a.S;
   for (int64_t t0 = 0; t0 < ntaps; t0 += kTapChunk) {
     const int tc = (ntaps - t0 < kTapChunk) ? static_cast<int>(ntaps - t0) : kTapChunk;
     __syncthreads();
     // decode W~ for this tap chunk: s_w[t][f]
-    for (int i = threadIdx.x; i < tc * kFilt; i += kPix) {
-      const int t = i / kFilt, f = i % kFilt;
+    for (int i = threadIdx.x; i < tc * kF; i += kPix) {
+      const int t = i / kF, f = i % kF;
       const int64_t k = k0 + f;
       float v = 0.0f;
       if (k < a.K) {
@@ -116,17 +130,21 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
     if (active) {
       for (int t = 0; t < tc; ++t) {
         const int32_t rs = s_rs[t];
-        const int64_t h = h0 + (rs >> 16), w = w0 + (rs & 0xFFFF);
-        float xv = 0.0f;
-        if (h >= 0 && h < a.H && w >= 0 && w < a.W) xv = to_f32<TX>(x[base + s_off[t]]);
+        const int off = s_off[t];
         const float4* wr = reinterpret_cast<const float4*>(&s_w[t][0]);
 #pragma unroll
-        for (int f4 = 0; f4 < kFilt / 4; ++f4) {
-          const float4 wv = wr[f4];
-          acc[4 * f4 + 0] = fmaf(xv, wv.x, acc[4 * f4 + 0]);
-          acc[4 * f4 + 1] = fmaf(xv, wv.y, acc[4 * f4 + 1]);
-          acc[4 * f4 + 2] = fmaf(xv, wv.z, acc[4 * f4 + 2]);
-          acc[4 * f4 + 3] = fmaf(xv, wv.w, acc[4 * f4 + 3]);
+        for (int wdx = 0; wdx < kWin; ++wdx) {
+          const int h = h0[wdx] + (rs >> 16), w = w0[wdx] + (rs & 0xFFFF);
+          float xv = 0.0f;
+          if (h >= 0 && h < H && w >= 0 && w < W) xv = to_f32<TX>(x[base[wdx] + off]);
+#pragma unroll
+          for (int f4 = 0; f4 < kF / 4; ++f4) {
+            const float4 wv = wr[f4];
+            acc[wdx][4 * f4 + 0] = fmaf(xv, wv.x, acc[wdx][4 * f4 + 0]);
+            acc[wdx][4 * f4 + 1] = fmaf(xv, wv.y, acc[wdx][4 * f4 + 1]);
+            acc[wdx][4 * f4 + 2] = fmaf(xv, wv.z, acc[wdx][4 * f4 + 2]);
+            acc[wdx][4 * f4 + 3] = fmaf(xv, wv.w, acc[wdx][4 * f4 + 3]);
+          }
         }
       }
     }
@@ -136,28 +154,41 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
   TY* __restrict__ y = static_cast<TY*>(a.y);
   const TY* __restrict__ res = static_cast<const TY*>(a.residual);
 #pragma unroll
-  for (int f = 0; f < kFilt; ++f) {
+  for (int f = 0; f < kF; ++f) {
     const int64_t k = k0 + f;
     if (k < a.K) {
-      const int64_t o = kNHWC ? pix * a.K + k : ((b * a.K + k) * a.P + p) * a.Q + q;
-      float v = a.alpha[k] * acc[f];
-      if (res != nullptr) v += to_f32<TY>(res[o]);
-      if (a.relu) v = fmaxf(v, 0.0f);
-      y[o] = from_f32<TY>(v);
+      const int64_t o = kNHWC ? pix * a.K + k : ((b * a.K + k) * a.Po + po) * a.Qo + qo;
+      float best = -INFINITY;
+#pragma unroll
+      for (int wdx = 0; wdx < kWin; ++wdx) {
+        float v = a.alpha[k] * acc[wdx][f];
+        if (res != nullptr) v += to_f32<TY>(res[o]);
+        if (a.relu) v = fmaxf(v, 0.0f);
+        best = fmaxf(best, v);
+      }
+      y[o] = from_f32<TY>(best);
     }
   }
 }
 
-template <typename TX, typename TY, bool kNHWC>
+template <typename TX, typename TY, bool kNHWC, int kWin>
 tbn_status launch_direct_t(const DirectArgs& a, cudaStream_t s) {
-  const int64_t npix = a.N * a.P * a.Q;
+  constexpr int kF = kWin == 1 ? kFilt : 8;
+  const int64_t npix = a.N * a.Po * a.Qo;
   const int64_t gx = (npix + kPix - 1) / kPix;
-  const int64_t gy = (a.K + kFilt - 1) / kFilt;
+  const int64_t gy = (a.K + kF - 1) / kF;
   if (gx > 0x7fffffffLL || gy > 65535)
     return fail(TBN_ERR_UNSUPPORTED, "conv direct: grid too large (%lld x %lld)", (long long)gx,
                 (long long)gy);
-  conv_direct_kernel<TX, TY, kNHWC><<<dim3((unsigned)gx, (unsigned)gy), kPix, 0, s>>>(a);
+  if (a.H >= (1 << 30) || a.W >= (1 << 30))
+    return fail(TBN_ERR_UNSUPPORTED, "conv direct: image too large");
+  conv_direct_kernel<TX, TY, kNHWC, kWin><<<dim3((unsigned)gx, (unsigned)gy), kPix, 0, s>>>(a);
   return check_launch("conv_direct_kernel");
+}
+
+template <typename TX, typename TY, bool kNHWC>
+tbn_status launch_direct_w(const DirectArgs& a, bool pool, cudaStream_t s) {
+  return pool ? launch_direct_t<TX, TY, kNHWC, 4>(a, s) : launch_direct_t<TX, TY, kNHWC, 1>(a, s);
 }
 
 template <typename T>
@@ -241,22 +272,25 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s) {
   DirectArgs a{};
   a.N = p.N; a.C = p.C; a.H = p.H; a.W = p.W; a.K = p.K; a.R = p.R; a.S = p.S;
   a.sh = p.sh; a.sw = p.sw; a.ph = p.ph; a.pw = p.pw; a.P = p.P; a.Q = p.Q;
+  a.Po = p.pool ? p.P / 2 : p.P;
+  a.Qo = p.pool ? p.Q / 2 : p.Q;
   a.wpf = (p.C * p.R * p.S + 15) / 16;
   a.x = p.x; a.codes = p.codes; a.alpha = p.alpha; a.y = p.y;
   a.residual = p.residual; a.relu = p.relu;
+  const bool pool = p.pool != 0;
   const bool nhwc = p.layout == TBN_NHWC;
   const bool xb = p.xdt == TBN_BF16, yb = p.ydt == TBN_BF16;
   using bf = __nv_bfloat16;
   if (nhwc) {
-    if (xb && yb) return launch_direct_t<bf, bf, true>(a, s);
-    if (xb && !yb) return launch_direct_t<bf, float, true>(a, s);
-    if (!xb && yb) return launch_direct_t<float, bf, true>(a, s);
-    return launch_direct_t<float, float, true>(a, s);
+    if (xb && yb) return launch_direct_w<bf, bf, true>(a, pool, s);
+    if (xb && !yb) return launch_direct_w<bf, float, true>(a, pool, s);
+    if (!xb && yb) return launch_direct_w<float, bf, true>(a, pool, s);
+    return launch_direct_w<float, float, true>(a, pool, s);
   }
-  if (xb && yb) return launch_direct_t<bf, bf, false>(a, s);
-  if (xb && !yb) return launch_direct_t<bf, float, false>(a, s);
-  if (!xb && yb) return launch_direct_t<float, bf, false>(a, s);
-  return launch_direct_t<float, float, false>(a, s);
+  if (xb && yb) return launch_direct_w<bf, bf, false>(a, pool, s);
+  if (xb && !yb) return launch_direct_w<bf, float, false>(a, pool, s);
+  if (!xb && yb) return launch_direct_w<float, bf, false>(a, pool, s);
+  return launch_direct_w<float, float, false>(a, pool, s);
 }
 
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,

@@ -1,31 +1,54 @@
 // tbn_conv_igemm.cu -- two-bit convolution (Eq. 1, Section 2) as an
 // implicit GEMM on the sm_100-family tensor cores (tcgen05), NHWC bf16.
 //
-// GEMM view of one CTA tile:  D[128 filters x T pixels] = A[128 x K] * B[K x T]
-// with K = R*S*C walked in blocks of one filter tap (r, s) x 64 channels.
+// GEMM view of one tile:  D[128 filters x T pixels] = A[128 x n] * B[n x T]
+// with T <= 256 output pixels and n = R*S*C in the codes' (r, s, c) order,
+// 64 codes per K block (= pipeline stage: four MMAs of K = 16).
 //
 //   A (filters)     the 2-bit codes, decoded in registers to bf16 W~/2 in
 //                   {+-0.5, +-1} (exact) and written straight into tensor
-//                   memory (tcgen05.st) by four "expander" warps: thread i
-//                   owns filter row i = TMEM lane i.  The decoded weights
-//                   never touch shared memory, so shared-memory bandwidth is
-//                   left to the activation operand.
-//   B (activations) a box of NHWC pixels x 64 channels loaded by TMA with the
-//                   128-byte swizzle; the box is the tile's output pixels
-//                   shifted by the tap (zero fill supplies the padding,
-//                   element strides supply the convolution stride).
-//   D               fp32 in tensor memory; epilogue multiplies row i by
-//                   2 * alpha_i (Eq. 1 applies alpha to the whole filter, and
-//                   the factor 2 undoes the W~/2 encoding -- both exact
-//                   power-of-two / per-row scalings), adds the optional
-//                   residual, applies ReLU, and stores NHWC.
+//                   memory (tcgen05.st) by eight "expander" warps: two per
+//                   TMEM sub-partition, each decoding half of a K block's 64
+//                   codes for the 32 filter rows (= TMEM lanes) it can reach,
+//                   two K blocks per tcgen05.wait::st.  The decoded weights
+//                   never touch shared memory, which is left to the
+//                   activation operand.  Decoding costs integer-pipe issue
+//                   slots per (filter, code), so a tile spans up to 256
+//                   pixels to amortize it over as many MMA columns as the
+//                   instruction allows.
+//   B (activations) im2col rows per pixel, 128-byte rows (64 codes) with the
+//                   128-byte swizzle.  When C % 64 == 0 a K block is one tap x
+//                   64 channels and one TMA box load fetches it (the box is
+//                   the tile's output pixels shifted by the tap; zero fill
+//                   supplies the padding, element strides the conv stride).
+//                   Otherwise gather warps assemble the rows from a
+//                   per-K-block table of (tap, channel) offsets.
+//   D               fp32 in tensor memory (256 columns).  Epilogue warps read
+//                   lane = filter, column = pixel, multiply by 2 * alpha (Eq. 1
+//                   applies alpha to the whole filter; the factor 2 undoes the
+//                   W~/2 encoding -- exact scalings), add the optional
+//                   residual, apply ReLU and the optional 2x2 max pool, round
+//                   to bf16 into a shared-memory staging tile laid out as the
+//                   NHWC output box, and one TMA bulk tensor store writes the
+//                   box (clipped at the tensor's edges).  The accumulator is
+//                   released as soon as it has been read, before the staging
+//                   writes and the store complete.
 //
-// Warp roles (192 threads, one CTA per SM):
-//   warp 0     TMA producer for the activation ring (one elected lane)
-//   warp 1     TMEM allocator + MMA issuer (one elected lane)
-//   warps 2-5  expanders during the main loop, epilogue afterwards
-// All waits are bounded (see tbn_device.cuh); on a timeout the CTA records
-// the error, drains its own in-flight copies and MMAs, frees TMEM, returns.
+// The kernel is persistent: each CTA walks tiles blockIdx.x, +gridDim.x, ...
+// (filter tile fastest, so CTAs working at the same time share activation
+// tiles in L2); producers and expanders run ahead into the next tile while
+// the epilogue drains the accumulator.
+//
+// Warp roles (every role is a whole warp that waits on the barriers; where a
+// single thread must issue -- TMA copies, MMAs, commits -- one elected lane
+// does, with warp-uniform operands):
+//   warp 0        TMA producer (TMA mode)
+//   warp 1        TMEM allocator + MMA issuer
+//   warps 2-9     expanders
+//   warps 10-17   epilogue
+//   warps 18-21   gather producers (gather mode only)
+// Every wait is bounded (tbn_device.cuh); on a timeout the CTA records the
+// error, drains its own in-flight copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -41,26 +64,39 @@ namespace tbn {
 namespace {
 
 constexpr int kBM = 128;            // filters per tile = TMEM lanes
-constexpr int kBKC = 64;            // channels per K block (128-byte rows)
+constexpr int kBK = 64;             // codes per K block (128-byte rows)
 constexpr int kMaxTileN = 256;      // pixels per tile (MMA N) upper bound
-constexpr int kStagesB = 6;         // activation ring depth (shared memory)
-constexpr int kStagesA = 8;         // weight ring depth (tensor memory)
-constexpr int kAColsPerStage = kBKC / 2;   // 64 bf16 = 32 columns of 32 bits
-constexpr int kAccCols = 256;
-constexpr int kTmemCols = 512;      // accumulator [0,256) + weight ring [256,512)
-constexpr int kThreads = 192;
-constexpr int kStageBytes = kMaxTileN * kBKC * 2;   // 32 KiB
+constexpr int kStages = 5;          // pipeline depth: activation ring (shared
+                                    // memory) and weight ring (tensor memory)
+constexpr int kAColsPerStage = kBK / 2;   // 64 bf16 = 32 columns of 32 bits
+constexpr int kAccCols = kMaxTileN;       // the accumulator
+constexpr int kTmemCols = 512;      // accumulator [0,256) + weight ring [256,416)
+constexpr int kExpWarps = 8;
+constexpr int kEpiWarps = 8;
+constexpr int kGatherWarps = 4;
+constexpr int kFirstExpWarp = 2;
+constexpr int kFirstEpiWarp = kFirstExpWarp + kExpWarps;
+constexpr int kFirstGatherWarp = kFirstEpiWarp + kEpiWarps;
+constexpr int kStageBytes = kMaxTileN * kBK * 2;     // 32 KiB
+constexpr int kOutStageBytes = kMaxTileN * kBM * 2;  // 64 KiB bf16 output box
 constexpr uint64_t kWaitLimitNs = 1000000000ull;    // 1 s
 
-static_assert(kAccCols + kStagesA * kAColsPerStage <= kTmemCols, "TMEM budget");
-static_assert(kMaxTileN * kBM * 4 <= kStagesB * kStageBytes, "epilogue staging fits the ring");
+static_assert(kAccCols + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
+
+template <bool kGather>
+constexpr int threads_for() {
+  return 32 * (kFirstGatherWarp + (kGather ? kGatherWarps : 0));
+}
 
 struct IgArgs {
   int N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
   int bw, bh, bn;          // output pixels per tile along q, p, image
   int tile_n;              // MMA N: bw*bh*bn rounded up to 16
-  int tiles_q, tiles_p, tiles_k;
-  int cblocks, kblocks, wpf;
+  int tiles_q, tiles_p, tiles_k, tiles;
+  int kblocks;             // ceil(R*S*C / 64): pipeline stages per tile
+  int ncodes;              // R*S*C
+  int wpf;                 // words per filter
+  const __nv_bfloat16* x;  // gather mode
   const uint32_t* codes;
   const float* alpha;
   void* y;
@@ -70,56 +106,100 @@ struct IgArgs {
 };
 
 struct SmemCtl {
-  uint64_t b_full[kStagesB];
-  uint64_t b_empty[kStagesB];
-  uint64_t a_full[kStagesA];
-  uint64_t a_empty[kStagesA];
+  // stage s holds K block g (g % kStages == s): its activations (shared
+  // memory) and its decoded weights (tensor memory).  full: both operands
+  // written; empty: the MMAs that read them have completed.
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
   uint64_t acc_full;
+  uint64_t acc_empty;
+  uint64_t res_full;
+  uint64_t mma_drain;      // used only to drain in-flight MMAs after an abort
   uint32_t tmem_base;
   int abort;
+  int gtab_off[2][kBK];    // gather: element offset of each code of the K block
+  int gtab_rs[2][kBK];     // gather: (r << 16 | s), or -1 beyond the filter
 };
 
-constexpr size_t kSmemBytes = 1024 /*align slack*/ + kStagesB * kStageBytes + sizeof(SmemCtl);
+constexpr size_t kSmemBytes =
+    1024 /*align slack*/ + kStages * kStageBytes + kOutStageBytes + sizeof(SmemCtl);
+static_assert(kSmemBytes <= 232448, "shared memory budget");
 
 __device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-    conv_igemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ IgArgs a) {
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+struct TileCoord {
+  int ktile, q0, p0, n0;
+};
+
+__device__ __forceinline__ TileCoord tile_coord(const IgArgs& a, int t) {
+  TileCoord c;
+  c.ktile = t % a.tiles_k;
+  const int pt_lin = t / a.tiles_k;
+  const int qt = pt_lin % a.tiles_q;
+  const int pt = (pt_lin / a.tiles_q) % a.tiles_p;
+  const int nt = pt_lin / (a.tiles_q * a.tiles_p);
+  c.q0 = qt * a.bw;
+  c.p0 = pt * a.bh;
+  c.n0 = nt * a.bn;
+  return c;
+}
+
+// Direct global store of one output value (the path for fp32 output or
+// shapes the TMA store cannot take): fp32 math, residual, ReLU, rounding.
+__device__ __forceinline__ void store_out(const IgArgs& a, size_t o, float v) {
+  if (a.y_bf16) {
+    if (a.residual) v += __bfloat162float(static_cast<const __nv_bfloat16*>(a.residual)[o]);
+    if (a.relu) v = fmaxf(v, 0.0f);
+    static_cast<__nv_bfloat16*>(a.y)[o] = __float2bfloat16_rn(v);
+  } else {
+    if (a.residual) v += static_cast<const float*>(a.residual)[o];
+    if (a.relu) v = fmaxf(v, 0.0f);
+    static_cast<float*>(a.y)[o] = v;
+  }
+}
+
+// kPoolBW: 0 = no pool; 8, 16, 32 = fused 2x2/2 max pool for tiles of whole
+// output rows of that width.  kTmaStore: bf16 output through the staging
+// tile and TMA stores (else direct global stores).
+template <bool kGather, int kPoolBW, bool kTmaStore>
+__global__ void __launch_bounds__(threads_for<kGather>(), 1)
+    conv_igemm_kernel(const __grid_constant__ CUtensorMap tmap_x,
+                      const __grid_constant__ CUtensorMap tmap_y,
+                      const __grid_constant__ CUtensorMap tmap_res,
+                      const __grid_constant__ IgArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* ring = smem;  // kStagesB x 32 KiB, 1024-aligned
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(smem + kStagesB * kStageBytes);
+  uint8_t* ring = smem;                                   // kStages x 32 KiB
+  uint8_t* out_stage = smem + kStages * kStageBytes;      // 64 KiB
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(out_stage + kOutStageBytes);
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-
-  // ---- tile coordinates (filter tile fastest: neighbouring CTAs share the
-  // activation tile through L2)
-  const int lin = blockIdx.x;
-  const int ktile = lin % a.tiles_k;
-  const int ptile = lin / a.tiles_k;
-  const int qt = ptile % a.tiles_q;
-  const int pt = (ptile / a.tiles_q) % a.tiles_p;
-  const int nt = ptile / (a.tiles_q * a.tiles_p);
-  const int q0 = qt * a.bw, p0 = pt * a.bh, n0 = nt * a.bn;
+  const int KB = a.kblocks;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStagesB; ++i) {
-      mbar_init(&ctl->b_full[i], 1);
-      mbar_init(&ctl->b_empty[i], 1);
-    }
-    for (int i = 0; i < kStagesA; ++i) {
-      mbar_init(&ctl->a_full[i], 128);
-      mbar_init(&ctl->a_empty[i], 1);
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&ctl->full[i], 32 * kExpWarps + (kGather ? 32 * kGatherWarps : 1));
+      mbar_init(&ctl->empty[i], 1);
     }
     mbar_init(&ctl->acc_full, 1);
+    mbar_init(&ctl->acc_empty, 32 * kEpiWarps);
+    mbar_init(&ctl->res_full, 1);
+    mbar_init(&ctl->mma_drain, 1);
     ctl->abort = 0;
     fence_mbar_init();
-    prefetch_tmap(&tmap_x);
+    if (!kGather) prefetch_tmap(&tmap_x);
+    if (kTmaStore) prefetch_tmap(&tmap_y);
   }
   if (warp == 1) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
@@ -128,185 +208,405 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
-  const uint32_t tmem = ctl->tmem_base;
-  const uint32_t acc_tmem = tmem;                 // columns [0, tile_n)
-  const uint32_t a_tmem0 = tmem + kAccCols;       // weight ring
-  const int KB = a.kblocks;
+  // The CTA allocates all 512 columns, so the allocation can only start at
+  // lane 0, column 0: every tensor-memory address below is a compile-time
+  // constant.  Any other base is reported and the CTA does no work.
+  constexpr uint32_t tmem = 0;
+  if (ctl->tmem_base != 0u) {
+    if (threadIdx.x == 0) {
+      raise_device_error(a.err, TBN_DEVERR_BAD_LAUNCH);
+      ctl->abort = 1;
+    }
+  }
+  __syncthreads();
+  if (*abort_flag) {
+    if (warp == 1) tmem_dealloc(ctl->tmem_base, kTmemCols);
+    return;
+  }
+  const uint32_t acc_tmem = tmem;               // columns [0, 256)
+  const uint32_t a_tmem0 = tmem + kAccCols;     // weight ring
 
-  if (warp == 0) {
+  if (!kGather && warp == 0) {
     // ================= TMA producer =================
-    if (lane == 0) {
-      const uint32_t box_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBKC * 2);
-      int issued = 0;
-      for (int kb = 0; kb < KB; ++kb) {
-        const int sb = kb % kStagesB;
-        const uint32_t it = static_cast<uint32_t>(kb / kStagesB);
-        if (!mbar_wait(&ctl->b_empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs)) break;
-        const int tap = kb / a.cblocks, cb = kb % a.cblocks;
-        const int r = tap / a.S, s = tap % a.S;
-        mbar_arrive_expect_tx(&ctl->b_full[sb], box_bytes);
-        tma_load_4d(ring + sb * kStageBytes, &tmap_x, &ctl->b_full[sb], cb * kBKC,
-                    q0 * a.sw - a.pw + s, p0 * a.sh - a.ph + r, n0);
-        ++issued;
+    const uint32_t box_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBK * 2);
+    const int cblocks = a.C / kBK;
+    int g = 0;  // global K-block counter of this CTA
+    bool ok = true;
+    for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x) {
+      const TileCoord tc = tile_coord(a, t);
+      int tap = 0, cb = 0;
+      for (int kb = 0; kb < KB; ++kb, ++g) {
+        const int sb = g % kStages;
+        const uint32_t it = static_cast<uint32_t>(g / kStages);
+        ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+        const int r = tap / a.S, s = tap - r * a.S;
+        if (elect_one()) {
+          mbar_arrive_expect_tx(&ctl->full[sb], box_bytes);
+          tma_load_4d(ring + sb * kStageBytes, &tmap_x, &ctl->full[sb], cb * kBK,
+                      tc.q0 * a.sw - a.pw + s, tc.p0 * a.sh - a.ph + r, tc.n0);
+        }
+        __syncwarp();
+        if (++cb == cblocks) { cb = 0; ++tap; }
       }
-      // drain: every issued copy must land before the CTA may exit
-      for (int i = issued > kStagesB ? issued - kStagesB : 0; i < issued; ++i)
-        mbar_wait(&ctl->b_full[i % kStagesB], static_cast<uint32_t>(i / kStagesB) & 1u, nullptr,
-                  a.err, kWaitLimitNs);
+    }
+    // drain: every issued copy must land before the CTA may exit
+    for (int i = g > kStages ? g - kStages : 0; i < g; ++i)
+      mbar_wait(&ctl->full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, nullptr,
+                a.err, kWaitLimitNs);
+  } else if (kGather && warp >= kFirstGatherWarp) {
+    // ================= gather producers =================
+    // The gather warps meet at a named barrier every K block, so none of them
+    // may leave the loops early: after a failed wait a warp keeps walking the
+    // loop structure (reaching every barrier) but does no more work.
+    const int gt = threadIdx.x - 32 * kFirstGatherWarp;   // 0..127
+    const bool vec = (a.C & 7) == 0;
+    int g = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < a.tiles; t += gridDim.x) {
+      const TileCoord tc = tile_coord(a, t);
+      const int T = a.bw * a.bh * a.bn;
+      // this thread fills tile rows gt and gt + 128; offset of tap (0, 0)
+      int64_t pbase[2];
+      int rh[2], rw[2];
+      bool rv[2];
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int row = gt + 128 * i;
+        const int wi = row % a.bw, hi = (row / a.bw) % a.bh, ni = row / (a.bw * a.bh);
+        rh[i] = (tc.p0 + hi) * a.sh - a.ph;
+        rw[i] = (tc.q0 + wi) * a.sw - a.pw;
+        rv[i] = row < T && tc.n0 + ni < a.N && tc.p0 + hi < a.P && tc.q0 + wi < a.Q;
+        pbase[i] = ((static_cast<int64_t>(rv[i] ? tc.n0 + ni : 0) * a.H + rh[i]) * a.W + rw[i]) *
+                   static_cast<int64_t>(a.C);
+      }
+      for (int kb = 0; kb < KB; ++kb, ++g) {
+        // table of this K block's 64 codes: offset from the tap-(0,0) pixel
+        const int tb = g & 1;
+        if (gt < kBK) {
+          const int k = kb * kBK + gt;
+          if (k < a.ncodes) {
+            const int c = k % a.C, tap = k / a.C;
+            const int r = tap / a.S, s = tap - r * a.S;
+            ctl->gtab_off[tb][gt] = (r * a.W + s) * a.C + c;
+            ctl->gtab_rs[tb][gt] = (r << 16) | s;
+          } else {
+            ctl->gtab_off[tb][gt] = 0;
+            ctl->gtab_rs[tb][gt] = -1;
+          }
+        }
+        named_barrier_sync(2, 32 * kGatherWarps);
+        const int sb = g % kStages;
+        const uint32_t it = static_cast<uint32_t>(g / kStages);
+        if (ok) ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) continue;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+          const int row = gt + 128 * i;
+          if (row >= a.tile_n) continue;
+          const uint32_t row_addr = smem_addr(ring + sb * kStageBytes) + static_cast<uint32_t>(row) * 128u;
+          uint4 v[8];
+          if (vec) {
+#pragma unroll
+            for (int ch = 0; ch < 8; ++ch) {
+              const int rs = ctl->gtab_rs[tb][ch * 8];
+              const int h = rh[i] + (rs >> 16), w = rw[i] + (rs & 0xFFFF);
+              v[ch] = make_uint4(0u, 0u, 0u, 0u);
+              if (rv[i] && rs >= 0 && h >= 0 && h < a.H && w >= 0 && w < a.W)
+                v[ch] = __ldg(reinterpret_cast<const uint4*>(a.x + pbase[i] + ctl->gtab_off[tb][ch * 8]));
+            }
+          } else {
+            const unsigned short* xs = reinterpret_cast<const unsigned short*>(a.x);
+#pragma unroll
+            for (int ch = 0; ch < 8; ++ch) {
+              uint32_t e[8];
+#pragma unroll
+              for (int q = 0; q < 8; ++q) {
+                const int rs = ctl->gtab_rs[tb][ch * 8 + q];
+                const int h = rh[i] + (rs >> 16), w = rw[i] + (rs & 0xFFFF);
+                e[q] = 0u;
+                if (rv[i] && rs >= 0 && h >= 0 && h < a.H && w >= 0 && w < a.W)
+                  e[q] = __ldg(xs + pbase[i] + ctl->gtab_off[tb][ch * 8 + q]);
+              }
+              v[ch] = make_uint4(e[0] | (e[1] << 16), e[2] | (e[3] << 16), e[4] | (e[5] << 16),
+                                 e[6] | (e[7] << 16));
+            }
+          }
+#pragma unroll
+          for (int ch = 0; ch < 8; ++ch)  // 128-byte swizzle: chunk XOR (row mod 8)
+            st_shared_v4(row_addr + static_cast<uint32_t>(((ch ^ (row & 7)) & 7) * 16), v[ch]);
+        }
+        fence_proxy_async_smem();   // generic-proxy writes -> visible to tcgen05.mma
+        mbar_arrive(&ctl->full[sb]);
+      }
     }
   } else if (warp == 1) {
     // ================= MMA issuer =================
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, static_cast<uint32_t>(a.tile_n));
-      int issued = 0;
-      for (int kb = 0; kb < KB; ++kb) {
-        const int sb = kb % kStagesB, sa = kb % kStagesA;
-        if (!mbar_wait(&ctl->a_full[sa], static_cast<uint32_t>(kb / kStagesA) & 1u, abort_flag,
-                       a.err, kWaitLimitNs))
-          break;
-        if (!mbar_wait(&ctl->b_full[sb], static_cast<uint32_t>(kb / kStagesB) & 1u, abort_flag,
-                       a.err, kWaitLimitNs))
-          break;
+    const uint32_t idesc = idesc_bf16_f32(kBM, static_cast<uint32_t>(a.tile_n));
+    int g = 0, issued = 0;
+    uint32_t tiles_done = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x, ++tiles_done) {
+      // the epilogue must have drained the previous tile's accumulator
+      ok = mbar_wait(&ctl->acc_empty, (tiles_done & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      tc_fence_after_sync();
+      for (int kb = 0; kb < KB; ++kb, ++g) {
+        const int st = g % kStages;
+        ok = mbar_wait(&ctl->full[st], static_cast<uint32_t>(g / kStages) & 1u, abort_flag, a.err,
+                       kWaitLimitNs);
+        if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after_sync();
-        const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(ring + sb * kStageBytes));
-        const uint32_t a_col = a_tmem0 + static_cast<uint32_t>(sa * kAColsPerStage);
+        const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(ring + st * kStageBytes));
+        const uint32_t a_col = a_tmem0 + static_cast<uint32_t>(st * kAColsPerStage);
+        if (elect_one()) {
 #pragma unroll
-        for (int kk = 0; kk < kBKC / 16; ++kk) {
-          // K step kk: 16 channels = 8 TMEM columns of A, 32 bytes of B rows
-          tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
-                    (kb | kk) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            // K step kk: 16 codes = 8 TMEM columns of A, 32 bytes of B rows
+            tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
+                      (kb | kk) != 0 ? 1u : 0u);
+          }
+          tc_commit(&ctl->empty[st]);
         }
-        tc_commit(&ctl->a_empty[sa]);
-        tc_commit(&ctl->b_empty[sb]);
+        __syncwarp();
         ++issued;
       }
-      // accumulator complete (also drains in-flight MMAs after an abort)
-      tc_commit(&ctl->acc_full);
-      if (*abort_flag && issued > 0)
-        mbar_wait(&ctl->acc_full, 0u, nullptr, a.err, kWaitLimitNs);
-    }
-  } else {
-    // ================= expanders, then epilogue =================
-    const int sub = warp & 3;             // TMEM sub-partition this warp may access
-    const int m = sub * 32 + lane;        // filter row within the tile
-    const int k = ktile * kBM + m;
-    const bool kvalid = k < a.K;
-    const uint32_t lane_off = static_cast<uint32_t>(sub * 32) << 16;
-    const uint4* crow = reinterpret_cast<const uint4*>(a.codes + static_cast<size_t>(kvalid ? k : 0) * a.wpf);
-    const int cw = a.C / 64;  // uint4 (64 codes) per tap
-
-    auto load_codes = [&](int kb) -> uint4 {
-      if (!kvalid || kb >= KB) return make_uint4(0u, 0u, 0u, 0u);
-      const int tap = kb / a.cblocks, cb = kb % a.cblocks;
-      return __ldg(crow + tap * cw + cb);
-    };
-    uint4 pf0 = load_codes(0), pf1 = load_codes(1);
-    bool ok = true;
-    for (int kb = 0; kb < KB; ++kb) {
-      const uint4 cur = pf0;
-      pf0 = pf1;
-      pf1 = load_codes(kb + 2);
-      const int sa = kb % kStagesA;
-      if (!mbar_wait(&ctl->a_empty[sa], (static_cast<uint32_t>(kb / kStagesA) & 1u) ^ 1u,
-                     abort_flag, a.err, kWaitLimitNs)) {
-        ok = false;
+      if (ok) {
+        if (elect_one()) tc_commit(&ctl->acc_full);
+        __syncwarp();
       }
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
+    }
+    if (!ok && issued > 0) {
+      // drain in-flight MMAs before TMEM is freed
+      if (elect_one()) tc_commit(&ctl->mma_drain);
+      __syncwarp();
+      mbar_wait(&ctl->mma_drain, 0u, nullptr, a.err, kWaitLimitNs);
+    }
+  } else if (warp >= kFirstExpWarp && warp < kFirstExpWarp + kExpWarps) {
+    // ================= expanders =================
+    const int sub = warp & 3;                         // TMEM sub-partition
+    const int half = (warp - kFirstExpWarp) >> 2;     // which 32 codes of a K block
+    const int m = sub * 32 + lane;                    // filter row within the tile
+    const uint32_t lane_off = static_cast<uint32_t>(sub * 32) << 16;
+    const bool pair_ok = ((a.wpf & 1) == 0) && ((reinterpret_cast<uintptr_t>(a.codes) & 7) == 0);
+    // this CTA's K blocks, all tiles in sequence (g = tile_index * KB + kb)
+    const int my_tiles = (a.tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                         static_cast<int>(gridDim.x);
+    const int total = my_tiles * KB;
+    // prefetch cursor over (tile, kb): the codes of K block kb of a filter
+    // are words [4 kb, 4 kb + 4) of its row; this warp takes two of them
+    int t_ld = blockIdx.x, kb_ld = 0;
+    const uint32_t* crow_ld = nullptr;
+    auto set_row = [&]() {
+      const int k = (t_ld % a.tiles_k) * kBM + m;
+      crow_ld = (t_ld < a.tiles && k < a.K) ? a.codes + static_cast<size_t>(k) * a.wpf : nullptr;
+    };
+    set_row();
+    auto next_codes = [&]() -> uint2 {
+      uint2 r = make_uint2(0u, 0u);
+      const int w0 = kb_ld * 4 + half * 2;
+      if (crow_ld != nullptr && w0 < a.wpf) {
+        if (pair_ok) r = __ldg(reinterpret_cast<const uint2*>(crow_ld + w0));
+        else r = make_uint2(__ldg(crow_ld + w0), w0 + 1 < a.wpf ? __ldg(crow_ld + w0 + 1) : 0u);
+      }
+      if (++kb_ld == KB) {
+        kb_ld = 0;
+        t_ld += gridDim.x;
+        set_row();
+      }
+      return r;
+    };
+    uint2 q0 = next_codes(), q1 = next_codes(), q2 = next_codes(), q3 = next_codes();
+    const uint32_t col = a_tmem0 + lane_off + static_cast<uint32_t>(16 * half);
+    // two K blocks per iteration: their tensor-memory stores share one
+    // tcgen05.wait::st
+    for (int g = 0; g < total; g += 2) {
+      const bool two = g + 1 < total;   // warp-uniform
+      uint32_t v0[16], v1[16];
+      word_to_bf16x2(q0.x, v0 + 0);
+      word_to_bf16x2(q0.y, v0 + 8);
+      word_to_bf16x2(q1.x, v1 + 0);
+      word_to_bf16x2(q1.y, v1 + 8);
+      q0 = q2;
+      q1 = q3;
+      q2 = next_codes();
+      q3 = next_codes();
+      const int s0 = g % kStages, s1 = (g + 1) % kStages;
+      bool ok = mbar_wait(&ctl->empty[s0], (static_cast<uint32_t>(g / kStages) & 1u) ^ 1u,
+                          abort_flag, a.err, kWaitLimitNs);
+      if (ok && two)
+        ok = mbar_wait(&ctl->empty[s1], (static_cast<uint32_t>((g + 1) / kStages) & 1u) ^ 1u,
+                       abort_flag, a.err, kWaitLimitNs);
+      if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after_sync();
-      uint32_t v[32];
-      word_to_bf16x2(cur.x, v + 0);
-      word_to_bf16x2(cur.y, v + 8);
-      word_to_bf16x2(cur.z, v + 16);
-      word_to_bf16x2(cur.w, v + 24);
-      tmem_st_32x32b_x32(a_tmem0 + lane_off + static_cast<uint32_t>(sa * kAColsPerStage), v);
+      tmem_st_32x32b_x16(col + static_cast<uint32_t>(s0 * kAColsPerStage), v0);
+      if (two) tmem_st_32x32b_x16(col + static_cast<uint32_t>(s1 * kAColsPerStage), v1);
       tmem_wait_st();
       tc_fence_before_sync();
-      mbar_arrive(&ctl->a_full[sa]);
+      mbar_arrive(&ctl->full[s0]);
+      if (two) mbar_arrive(&ctl->full[s1]);
     }
-
-    // ---- epilogue
-    bool acc_ok = ok && mbar_wait(&ctl->acc_full, 0u, abort_flag, a.err, kWaitLimitNs);
-    acc_ok = __all_sync(0xffffffffu, acc_ok);
-    // all four epilogue warps must agree before touching the staging buffer
-    __shared__ int s_epi_ok;
-    if (threadIdx.x == 64) s_epi_ok = 1;
-    named_barrier_sync(1, 128);
-    if (!acc_ok && lane == 0) atomicAnd(&s_epi_ok, 0);
-    named_barrier_sync(1, 128);
-    if (s_epi_ok && !*abort_flag) {
-      tc_fence_after_sync();
-      float* stage = reinterpret_cast<float*>(ring);  // [tile_n][128] fp32
-      const float a2 = kvalid ? 2.0f * a.alpha[k] : 0.0f;
-      // columns beyond tile_n (up to the next multiple of 32) hold garbage
-      // and land in staging rows that the copy-out never reads
-      for (int j = 0; j < (a.tile_n + 31) / 32; ++j) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(acc_tmem + lane_off + static_cast<uint32_t>(32 * j), v);
-        tmem_wait_ld();
-#pragma unroll
-        for (int i = 0; i < 32; ++i) stage[(32 * j + i) * kBM + m] = a2 * __uint_as_float(v[i]);
+  } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
+    // ================= epilogue =================
+    // Two warps per TMEM sub-partition, each reading half of the columns.
+    const int sub = warp & 3;
+    const int half = (warp - kFirstEpiWarp) >> 2;
+    const int m = sub * 32 + lane;
+    const int et = threadIdx.x - 32 * kFirstEpiWarp;   // 0..255
+    const bool elected = et == 0;
+    const uint32_t lane_off = static_cast<uint32_t>(sub * 32) << 16;
+    const int Po = kPoolBW ? a.P / 2 : a.P;
+    const int Qo = kPoolBW ? a.Q / 2 : a.Q;
+    const uint32_t res_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBM * 2);
+    __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(out_stage);
+    uint32_t tiles_done = 0;
+    bool ok = true;
+    // The epilogue warps meet at named barriers, so after a failed wait they
+    // keep walking the tile loop (reaching every barrier) without working.
+    for (int t = blockIdx.x; t < a.tiles; t += gridDim.x, ++tiles_done) {
+      const TileCoord tc = tile_coord(a, t);
+      const uint32_t par = tiles_done & 1u;
+      const uint32_t acc = acc_tmem + lane_off;
+      const int k = tc.ktile * kBM + m;
+      const bool kvalid = k < a.K;
+      const float a2 = kvalid ? 2.0f * __ldg(a.alpha + k) : 0.0f;
+      if (kTmaStore) {
+        // the previous tile's store must have finished reading the staging tile
+        if (elected) bulk_wait_group_read<0>();
+        named_barrier_sync(1, 32 * kEpiWarps);
+        if (ok && a.residual && elected) {
+          mbar_arrive_expect_tx(&ctl->res_full, res_bytes);
+          asm volatile(
+              "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+              " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_addr(stage)),
+              "l"(&tmap_res), "r"(smem_addr(&ctl->res_full)), "r"(tc.ktile * kBM),
+              "r"(tc.q0), "r"(tc.p0), "r"(tc.n0)
+              : "memory");
+        }
       }
-      named_barrier_sync(1, 128);
-      // copy-out: 16 threads per pixel row, 8 filters (one 16-byte bf16 vector) each
-      const int e = threadIdx.x - 64;
-      const int c8 = (e & 15) * 8;
-      const int npix_tile = a.bw * a.bh * a.bn;
-      const int kbase = ktile * kBM + c8;
-      const bool vec_ok = (a.K % 8) == 0 && kbase + 8 <= a.K;
-      for (int pr = e >> 4; pr < npix_tile; pr += 8) {
-        const int wi = pr % a.bw, hi = (pr / a.bw) % a.bh, ni = pr / (a.bw * a.bh);
-        const int q = q0 + wi, p = p0 + hi, n = n0 + ni;
-        if (q >= a.Q || p >= a.P || n >= a.N || kbase >= a.K) continue;
-        const size_t o = ((static_cast<size_t>(n) * a.P + p) * a.Q + q) * a.K + kbase;
-        const float4 lo = *reinterpret_cast<const float4*>(&stage[pr * kBM + c8]);
-        const float4 hi4 = *reinterpret_cast<const float4*>(&stage[pr * kBM + c8 + 4]);
-        float v[8] = {lo.x, lo.y, lo.z, lo.w, hi4.x, hi4.y, hi4.z, hi4.w};
-        if (vec_ok) {
-          if (a.y_bf16) {
-            if (a.residual) {
-              const uint4 rr = *reinterpret_cast<const uint4*>(
-                  static_cast<const __nv_bfloat16*>(a.residual) + o);
-              const __nv_bfloat16* rb = reinterpret_cast<const __nv_bfloat16*>(&rr);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] += __bfloat162float(rb[i]);
-            }
-            uint4 out;
-            __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(&out);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) ob[i] = __float2bfloat16_rn(a.relu ? fmaxf(v[i], 0.0f) : v[i]);
-            *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.y) + o) = out;
-          } else {
-            if (a.residual) {
-              const float4* rp = reinterpret_cast<const float4*>(static_cast<const float*>(a.residual) + o);
-              const float4 r0 = rp[0], r1 = rp[1];
-              v[0] += r0.x; v[1] += r0.y; v[2] += r0.z; v[3] += r0.w;
-              v[4] += r1.x; v[5] += r1.y; v[6] += r1.z; v[7] += r1.w;
-            }
-            if (a.relu) {
-#pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] = fmaxf(v[i], 0.0f);
-            }
-            float4* yp = reinterpret_cast<float4*>(static_cast<float*>(a.y) + o);
-            yp[0] = make_float4(v[0], v[1], v[2], v[3]);
-            yp[1] = make_float4(v[4], v[5], v[6], v[7]);
+      if (ok) ok = mbar_wait(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs);
+      if (kTmaStore && a.residual && ok)
+        ok = mbar_wait(&ctl->res_full, par, abort_flag, a.err, kWaitLimitNs);
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok) tc_fence_after_sync();
+      if (!ok) {
+        // skip the work, keep the barrier schedule
+      } else if constexpr (kPoolBW == 0) {
+        const int T = a.bw * a.bh * a.bn;
+        const int nchunks = (a.tile_n + 31) / 32;
+        const int c_begin = half ? (nchunks + 1) / 2 : 0;
+        const int c_end = half ? nchunks : (nchunks + 1) / 2;
+        // direct-store path: pixel of chunk c_begin walked in column order
+        int px0 = 32 * c_begin;
+        int wi = px0 % a.bw, hi = (px0 / a.bw) % a.bh, ni = px0 / (a.bw * a.bh);
+        for (int j = c_begin; j < c_end; ++j) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(acc + static_cast<uint32_t>(32 * j), v);
+          tmem_wait_ld();
+          if (j == c_end - 1) {
+            // this warp has read its part of the accumulator
+            tc_fence_before_sync();
+            mbar_arrive(&ctl->acc_empty);
           }
-        } else {
-          for (int i = 0; i < 8 && kbase + i < a.K; ++i) {
-            float t = v[i];
-            if (a.y_bf16) {
-              if (a.residual) t += __bfloat162float(static_cast<const __nv_bfloat16*>(a.residual)[o + i]);
-              if (a.relu) t = fmaxf(t, 0.0f);
-              static_cast<__nv_bfloat16*>(a.y)[o + i] = __float2bfloat16_rn(t);
-            } else {
-              if (a.residual) t += static_cast<const float*>(a.residual)[o + i];
-              if (a.relu) t = fmaxf(t, 0.0f);
-              static_cast<float*>(a.y)[o + i] = t;
+          if (kTmaStore) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int px = 32 * j + i;
+              if (px < T) {
+                float y = a2 * __uint_as_float(v[i]);
+                __nv_bfloat16* sp = stage + px * kBM + m;
+                if (a.residual) y += __bfloat162float(*sp);
+                if (a.relu) y = fmaxf(y, 0.0f);
+                *sp = __float2bfloat16_rn(y);
+              }
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int px = 32 * j + i;
+              const int q = tc.q0 + wi, p = tc.p0 + hi, n = tc.n0 + ni;
+              if (kvalid && px < T && q < a.Q && p < a.P && n < a.N)
+                store_out(a, ((static_cast<size_t>(n) * a.P + p) * a.Q + q) * a.K + k,
+                          a2 * __uint_as_float(v[i]));
+              if (++wi == a.bw) {
+                wi = 0;
+                if (++hi == a.bh) { hi = 0; ++ni; }
+              }
             }
           }
         }
+        if (c_begin >= c_end) {
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->acc_empty);
+        }
+      } else {
+        // fused 2x2 max pool: tiles hold whole rows of width kPoolBW (q0 = 0)
+        // and an even number of rows per image; one TMEM load covers an even
+        // pair of rows or more.
+        constexpr int kCols = kPoolBW <= 16 ? 32 : 64;   // columns per load
+        constexpr int kPairs = kCols / (2 * kPoolBW);    // row pairs per load
+        const int rows_total = a.bh * a.bn;               // tile rows (all images)
+        const int bh2 = a.bh / 2;
+        const int nloads = (rows_total * kPoolBW + kCols - 1) / kCols;
+        const int l_begin = half ? (nloads + 1) / 2 : 0;
+        const int l_end = half ? nloads : (nloads + 1) / 2;
+        for (int j = l_begin; j < l_end; ++j) {
+          uint32_t v[kCols];
+          tmem_ld_32x32b_x32(acc + static_cast<uint32_t>(kCols * j),
+                             *reinterpret_cast<uint32_t(*)[32]>(v));
+          if constexpr (kCols == 64)
+            tmem_ld_32x32b_x32(acc + static_cast<uint32_t>(kCols * j + 32),
+                               *reinterpret_cast<uint32_t(*)[32]>(v + 32));
+          tmem_wait_ld();
+          if (j == l_end - 1) {
+            tc_fence_before_sync();
+            mbar_arrive(&ctl->acc_empty);
+          }
+#pragma unroll
+          for (int pp = 0; pp < kPairs; ++pp) {
+            const int pair = j * kPairs + pp;          // row pair within the tile
+            const int ni = pair / bh2;
+            const int hi2 = pair - ni * bh2;
+            const int p2 = tc.p0 / 2 + hi2, n = tc.n0 + ni;
+            const bool pv = ni < a.bn;
+#pragma unroll
+            for (int q2 = 0; q2 < kPoolBW / 2; ++q2) {
+              const int c0 = pp * 2 * kPoolBW + 2 * q2;
+              const float m0 = fmaxf(__uint_as_float(v[c0]), __uint_as_float(v[c0 + 1]));
+              const float m1 = fmaxf(__uint_as_float(v[c0 + kPoolBW]),
+                                     __uint_as_float(v[c0 + kPoolBW + 1]));
+              // alpha >= 0, so max commutes with the scaling (and with ReLU)
+              float mx = a2 * fmaxf(m0, m1);
+              if (kTmaStore) {
+                if (pv) {
+                  if (a.relu) mx = fmaxf(mx, 0.0f);
+                  stage[(pair * (kPoolBW / 2) + q2) * kBM + m] = __float2bfloat16_rn(mx);
+                }
+              } else if (kvalid && pv && p2 < Po && q2 < Qo && n < a.N) {
+                store_out(a, ((static_cast<size_t>(n) * Po + p2) * Qo + q2) * a.K + k, mx);
+              }
+            }
+          }
+        }
+        if (l_begin >= l_end) {
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->acc_empty);
+        }
+      }
+      if (kTmaStore) {
+        fence_proxy_async_smem();   // staged values -> visible to the TMA store
+        named_barrier_sync(1, 32 * kEpiWarps);
+        if (elected && ok) {
+          if (kPoolBW)
+            tma_store_4d(&tmap_y, stage, tc.ktile * kBM, 0, tc.p0 / 2, tc.n0);
+          else
+            tma_store_4d(&tmap_y, stage, tc.ktile * kBM, tc.q0, tc.p0, tc.n0);
+          bulk_commit_group();
+        }
       }
     }
+    if (kTmaStore && elected) bulk_wait_group<0>();   // all stores complete before exit
   }
 
   tc_fence_before_sync();
@@ -343,25 +643,34 @@ struct TilePlan {
 
 int ceil_div(int64_t a, int64_t b) { return static_cast<int>((a + b - 1) / b); }
 
+bool use_tma(const ConvProblem& p) { return p.C % kBK == 0 && p.sh <= 2 && p.sw <= 2; }
+
 // Output pixels per tile: whole rows of the output (so one TMA box per tap
 // covers the tile), balanced so the last tile along each axis is not a
-// sliver, at most 256 pixels.
+// sliver, at most 256 pixels.  With a fused 2x2 pool a tile holds whole
+// output rows and an even number of them per image.
 TilePlan plan_tiles(const ConvProblem& p) {
   TilePlan t{};
-  const int bw_max = std::min<int64_t>(p.Q, kMaxTileN / p.sw);
+  const int stride_w = use_tma(p) ? static_cast<int>(p.sw) : 1;
+  const int stride_h = use_tma(p) ? static_cast<int>(p.sh) : 1;
+  const int bw_max = static_cast<int>(std::min<int64_t>(p.Q, kMaxTileN / stride_w));
   t.tiles_q = ceil_div(p.Q, bw_max);
   t.bw = ceil_div(p.Q, t.tiles_q);
   if (t.tiles_q > 1) {
     t.bh = 1;
     t.bn = 1;
   } else {
-    const int bh_max = static_cast<int>(std::min<int64_t>({p.P, kMaxTileN / t.bw, kMaxTileN / p.sh}));
+    int bh_max = static_cast<int>(std::min<int64_t>({p.P, kMaxTileN / t.bw, 256 / stride_h}));
+    if (p.pool) bh_max &= ~1;
+    if (bh_max < 1) bh_max = 1;
     const int tp = ceil_div(p.P, bh_max);
     t.bh = ceil_div(p.P, tp);
-    if (tp > 1) {
+    if (p.pool && (t.bh & 1)) t.bh += 1;   // <= bh_max when bh_max is even
+    if (t.bh < p.P) {
       t.bn = 1;
     } else {
-      const int bn_max = static_cast<int>(std::min<int64_t>(p.N, kMaxTileN / (t.bw * t.bh)));
+      t.bh = static_cast<int>(p.P) + (p.pool ? static_cast<int>(p.P & 1) : 0);
+      const int bn_max = std::max(1, static_cast<int>(std::min<int64_t>(p.N, kMaxTileN / (t.bw * t.bh))));
       t.bn = ceil_div(p.N, ceil_div(p.N, bn_max));
     }
   }
@@ -372,25 +681,112 @@ TilePlan plan_tiles(const ConvProblem& p) {
   return t;
 }
 
+int pool_width(const ConvProblem& p, const TilePlan& t) {
+  if (!p.pool) return 0;
+  if (t.tiles_q != 1 || t.T > kMaxTileN || (t.bh & 1)) return -1;
+  if (t.bw == 8 || t.bw == 16 || t.bw == 32) return t.bw;
+  return -1;
+}
+
+bool use_tma_store(const ConvProblem& p) {
+  return p.ydt == TBN_BF16 && p.K % 8 == 0 && is_aligned(p.y, 16) &&
+         (!p.residual || is_aligned(p.residual, 16));
+}
+
+CUresult encode_out_map(CUtensorMap* m, const void* base, const ConvProblem& p, const TilePlan& t,
+                        int pool) {
+  const int64_t Po = pool ? p.P / 2 : p.P, Qo = pool ? p.Q / 2 : p.Q;
+  const cuuint64_t gdim[4] = {(cuuint64_t)p.K, (cuuint64_t)Qo, (cuuint64_t)Po, (cuuint64_t)p.N};
+  const cuuint64_t gstride[3] = {(cuuint64_t)(p.K * 2), (cuuint64_t)(Qo * p.K * 2),
+                                 (cuuint64_t)(Po * Qo * p.K * 2)};
+  const cuuint32_t box[4] = {(cuuint32_t)kBM, (cuuint32_t)(pool ? t.bw / 2 : t.bw),
+                             (cuuint32_t)(pool ? t.bh / 2 : t.bh), (cuuint32_t)t.bn};
+  const cuuint32_t estr[4] = {1u, 1u, 1u, 1u};
+  return get_encode_tiled()(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), gdim,
+                            gstride, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+template <bool kGather, int kPoolBW, bool kTmaStore>
+tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStream_t s) {
+  alignas(64) CUtensorMap tmap_x, tmap_y, tmap_res;
+  std::memset(&tmap_x, 0, sizeof(tmap_x));
+  std::memset(&tmap_y, 0, sizeof(tmap_y));
+  std::memset(&tmap_res, 0, sizeof(tmap_res));
+  if (!kGather) {
+    const cuuint64_t gdim[4] = {(cuuint64_t)p.C, (cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.N};
+    const cuuint64_t gstride[3] = {(cuuint64_t)(p.C * 2), (cuuint64_t)(p.W * p.C * 2),
+                                   (cuuint64_t)(p.H * p.W * p.C * 2)};
+    const cuuint32_t box[4] = {(cuuint32_t)kBK, (cuuint32_t)(t.bw * p.sw),
+                               (cuuint32_t)(t.bh * p.sh), (cuuint32_t)t.bn};
+    const cuuint32_t estr[4] = {1u, (cuuint32_t)p.sw, (cuuint32_t)p.sh, 1u};
+    if (box[1] > 256 || box[2] > 256 || box[3] > 256)
+      return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: TMA box too large");
+    const CUresult cr = get_encode_tiled()(&tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+                                           const_cast<void*>(p.x), gdim, gstride, box, estr,
+                                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed (%d)", (int)cr);
+  }
+  if (kTmaStore) {
+    CUresult cr = encode_out_map(&tmap_y, p.y, p, t, kPoolBW ? 1 : 0);
+    if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(y) failed (%d)", (int)cr);
+    if (p.residual) {
+      cr = encode_out_map(&tmap_res, p.residual, p, t, 0);
+      if (cr != CUDA_SUCCESS)
+        return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(residual) failed (%d)", (int)cr);
+    }
+  }
+  auto kern = conv_igemm_kernel<kGather, kPoolBW, kTmaStore>;
+  static bool attr_done[2][4][2][64] = {};
+  const int pidx = kPoolBW == 0 ? 0 : (kPoolBW == 8 ? 1 : (kPoolBW == 16 ? 2 : 3));
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64 || !attr_done[kGather][pidx][kTmaStore][dev]) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)kSmemBytes);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(conv_igemm_kernel)");
+    if (dev >= 0 && dev < 64) attr_done[kGather][pidx][kTmaStore][dev] = true;
+  }
+  const int grid = std::min(a.tiles, device_sm_count());
+  kern<<<grid, threads_for<kGather>(), kSmemBytes, s>>>(tmap_x, tmap_y, tmap_res, a);
+  return check_launch("conv_igemm_kernel");
+}
+
+template <bool kGather, bool kTmaStore>
+tbn_status launch_pool(const ConvProblem& p, const TilePlan& t, IgArgs& a, int pw, cudaStream_t s) {
+  switch (pw) {
+    case 8: return launch_t<kGather, 8, kTmaStore>(p, t, a, s);
+    case 16: return launch_t<kGather, 16, kTmaStore>(p, t, a, s);
+    case 32: return launch_t<kGather, 32, kTmaStore>(p, t, a, s);
+    default: return launch_t<kGather, 0, kTmaStore>(p, t, a, s);
+  }
+}
+
 }  // namespace
 
 const char* conv_igemm_unsupported_reason(const ConvProblem& p) {
   if (p.layout != TBN_NHWC) return "implicit GEMM needs NHWC";
   if (p.xdt != TBN_BF16) return "implicit GEMM needs bf16 activations";
-  if (p.C % kBKC != 0) return "implicit GEMM needs C % 64 == 0";
   if (!is_aligned(p.x, 16)) return "implicit GEMM needs 16-byte aligned x";
-  if (!is_aligned(p.codes, 16)) return "implicit GEMM needs 16-byte aligned codes";
-  if (p.sh < 1 || p.sh > 2 || p.sw < 1 || p.sw > 2) return "implicit GEMM supports stride 1 or 2";
-  if (p.residual && !is_aligned(p.residual, 16)) return "implicit GEMM needs 16-byte aligned residual";
-  if (!is_aligned(p.y, 16)) return "implicit GEMM needs 16-byte aligned y";
-  if (p.N > (1 << 30) || p.H > (1 << 30) || p.W > (1 << 30)) return "dimension too large";
-  if (p.ph > p.R || p.pw > p.S) return "implicit GEMM needs pad <= kernel extent";
+  if (p.pool && p.residual) return "pooling with a residual is not supported";
+  if (p.N > (1 << 30) || p.H > (1 << 30) || p.W > (1 << 30) || p.K > (1 << 30))
+    return "dimension too large";
+  if (p.C * p.R * p.S >= (int64_t(1) << 30)) return "filter too large";
+  if (p.H * p.W * p.C >= (int64_t(1) << 31)) return "image too large";
+  if (p.R >= (1 << 15) || p.S >= (1 << 15)) return "kernel too large";
+  if (use_tma(p) && (p.ph > p.R || p.pw > p.S)) return "implicit GEMM needs pad <= kernel extent";
+  if (p.pool && pool_width(p, plan_tiles(p)) < 0)
+    return "fused pool needs whole output rows of width 8, 16 or 32 per tile";
   int dev = 0, major = 0, minor = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return "no CUDA device";
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (major != 10 || minor != 3) return "implicit GEMM kernel is built for sm_103a only";
-  if (get_encode_tiled() == nullptr) return "cuTensorMapEncodeTiled unavailable";
+  if ((use_tma(p) || use_tma_store(p)) && get_encode_tiled() == nullptr)
+    return "cuTensorMapEncodeTiled unavailable";
   return "";
 }
 
@@ -403,44 +799,22 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
   a.bw = t.bw; a.bh = t.bh; a.bn = t.bn; a.tile_n = t.tile_n;
   a.tiles_q = t.tiles_q; a.tiles_p = t.tiles_p;
   a.tiles_k = ceil_div(p.K, kBM);
-  a.cblocks = (int)(p.C / kBKC);
-  a.kblocks = (int)(p.R * p.S) * a.cblocks;
-  a.wpf = (int)((p.C * p.R * p.S + 15) / 16);
+  const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n * a.tiles_k;
+  if (tiles > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: too many tiles");
+  a.tiles = static_cast<int>(tiles);
+  a.ncodes = (int)(p.C * p.R * p.S);
+  a.kblocks = ceil_div(a.ncodes, kBK);
+  a.wpf = (a.ncodes + 15) / 16;
+  a.x = static_cast<const __nv_bfloat16*>(p.x);
   a.codes = p.codes; a.alpha = p.alpha; a.y = p.y; a.residual = p.residual;
   a.relu = p.relu; a.y_bf16 = p.ydt == TBN_BF16 ? 1 : 0;
   a.err = device_error_word();
-
-  const int64_t grid = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n * a.tiles_k;
-  if (grid > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: grid too large");
-
-  CUtensorMap tmap;
-  std::memset(&tmap, 0, sizeof(tmap));
-  const cuuint64_t gdim[4] = {(cuuint64_t)p.C, (cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.N};
-  const cuuint64_t gstride[3] = {(cuuint64_t)(p.C * 2), (cuuint64_t)(p.W * p.C * 2),
-                                 (cuuint64_t)(p.H * p.W * p.C * 2)};
-  const cuuint32_t box[4] = {(cuuint32_t)kBKC, (cuuint32_t)(t.bw * p.sw), (cuuint32_t)(t.bh * p.sh),
-                             (cuuint32_t)t.bn};
-  const cuuint32_t estr[4] = {1u, (cuuint32_t)p.sw, (cuuint32_t)p.sh, 1u};
-  if (box[1] > 256 || box[2] > 256 || box[3] > 256)
-    return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: TMA box too large");
-  const CUresult cr = get_encode_tiled()(&tmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
-                                         const_cast<void*>(p.x), gdim, gstride, box, estr,
-                                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)cr);
-
-  static bool attr_done[64] = {};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 0 || dev >= 64 || !attr_done[dev]) {
-    const cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)kSmemBytes);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(conv_igemm_kernel)");
-    if (dev >= 0 && dev < 64) attr_done[dev] = true;
+  const int pw = pool_width(p, t);
+  const bool tst = use_tma_store(p);
+  if (use_tma(p)) {
+    return tst ? launch_pool<false, true>(p, t, a, pw, s) : launch_pool<false, false>(p, t, a, pw, s);
   }
-  conv_igemm_kernel<<<(unsigned)grid, kThreads, kSmemBytes, s>>>(tmap, a);
-  return check_launch("conv_igemm_kernel");
+  return tst ? launch_pool<true, true>(p, t, a, pw, s) : launch_pool<true, false>(p, t, a, pw, s);
 }
 
 }  // namespace tbn

@@ -47,6 +47,7 @@ struct ConvProblem {
   void* y;
   int relu;
   const void* residual;
+  int pool;  // 0 or 2 (2x2 max pool, stride 2, after ReLU)
 };
 
 // ---- launchers (each defined next to its kernels) ----

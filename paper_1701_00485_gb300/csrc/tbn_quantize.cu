@@ -7,9 +7,12 @@
 // in the same pass that discretizes.  Each thread owns whole 32-bit output
 // words (16 consecutive weights of a filter): it loads 64 contiguous bytes,
 // forms the sixteen 2-bit fields, and accumulates |W~|*|W| (fp32 within the
-// word, fp64 across words) and the count of magnitude-two codes.  Filters
-// are reduced by a warp (short filters, 8 per CTA) or by a whole 256-thread
-// CTA (long filters).  Bytes moved per weight: 4 read + 1/4 written.
+// word, fp64 across words) and the count of magnitude-two codes.  A CTA
+// covers a group of whole filters of at most 1024 words; each of its 256
+// threads issues the loads of all its (up to four) words before encoding,
+// so a whole layer's weights are in flight at once, and the filters are
+// reduced through shared memory.  Filters longer than 1024 words get a CTA
+// each.  Bytes moved per weight: 4 read + 1/4 written.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -22,8 +25,8 @@ namespace tbn {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kRowsPerNarrowCta = kThreads / 32;
-constexpr int kWideMinWords = 257;  // filters with more words use a whole CTA
+constexpr int kWordsPerThread = 4;
+constexpr int kGroupWords = kThreads * kWordsPerThread;  // words a row-group CTA covers
 
 struct QJob {
   const float* W;
@@ -32,9 +35,9 @@ struct QJob {
   int64_t K;
   int64_t first_task;  // index of this job's first CTA task
   int32_t n;
-  int32_t wpf;  // words per filter
-  int32_t vec;  // 16-byte loads allowed
-  int32_t wide;
+  int32_t wpf;   // words per filter
+  int32_t vec;   // 16-byte loads allowed
+  int32_t rows;  // filters per CTA (0: one long filter per CTA, strided words)
 };
 
 struct QParams {
@@ -42,6 +45,17 @@ struct QParams {
   int njobs;
   uint32_t* err;
 };
+
+// fp64 re-summation of one word whose fp32 sum overflowed (weights near the
+// fp32 maximum).  Kept out of line so the common path carries no fp64 work.
+__device__ __noinline__ double word_sum_fp64(const float* v, int nvalid) {
+  double d = 0.0;
+  for (int e = 0; e < nvalid; ++e) {
+    const double a = fabs(static_cast<double>(v[e]));
+    d += a > 1.0 ? 2.0 * a : a;
+  }
+  return d;
+}
 
 // Sixteen weights -> one packed word, the sum of |W~|*|W| over them (fp32,
 // pairwise; redone in fp64 when the fp32 sum overflows, i.e. for weights
@@ -70,16 +84,13 @@ __device__ __forceinline__ void encode16(const float (&v)[16], int nvalid, uint3
   c[0] += c[2];
   c[1] += c[3];
   const float sum = c[0] + c[1];
-  if (sum <= 3.4028234663852886e38f) {
+  if (__builtin_expect(sum <= 3.4028234663852886e38f, 1)) {
     dsum = static_cast<double>(sum);
   } else {
-    double d = 0.0;
+    float tmp[16];
 #pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      const double a = fabs(static_cast<double>(v[e]));
-      d += (e < nvalid) ? (a > 1.0 ? 2.0 * a : a) : 0.0;
-    }
-    dsum = d;
+    for (int e = 0; e < 16; ++e) tmp[e] = v[e];
+    dsum = word_sum_fp64(tmp, nvalid);
   }
   word = w;
   cnt2 = n2;
@@ -161,8 +172,8 @@ __device__ __forceinline__ float alpha_of(double num, int cnt2, int n) {
 }
 
 __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_constant__ QParams prm) {
-  __shared__ double s_acc[kThreads / 32];
-  __shared__ int s_cnt[kThreads / 32];
+  __shared__ double s_num[kGroupWords];
+  __shared__ int s_cnt[kGroupWords];
 
   const int64_t task = blockIdx.x;
   int ji = 0;
@@ -173,9 +184,9 @@ __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_co
   const int64_t local = task - jb.first_task;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (jb.wide) {
+  if (jb.rows == 0) {
+    // one long filter per CTA: words strided over the threads, block reduction
     const int64_t k = local;
-    if (k >= jb.K) return;
     const float* row = jb.W + k * static_cast<int64_t>(jb.n);
     uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
     double acc = 0.0;
@@ -184,28 +195,64 @@ __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_co
     acc = warp_sum(acc);
     cnt2 = warp_sum(cnt2);
     if (lane == 0) {
-      s_acc[warp] = acc;
+      s_num[warp] = acc;
       s_cnt[warp] = cnt2;
     }
     __syncthreads();
     if (warp == 0) {
-      acc = lane < kThreads / 32 ? s_acc[lane] : 0.0;
+      acc = lane < kThreads / 32 ? s_num[lane] : 0.0;
       cnt2 = lane < kThreads / 32 ? s_cnt[lane] : 0;
       acc = warp_sum(acc);
       cnt2 = warp_sum(cnt2);
       if (lane == 0) jb.alpha[k] = alpha_of(acc, cnt2, jb.n);
     }
-  } else {
-    const int64_t k = local * kRowsPerNarrowCta + warp;
-    if (k >= jb.K) return;
-    const float* row = jb.W + k * static_cast<int64_t>(jb.n);
-    uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
+    return;
+  }
+
+  // a group of whole filters, at most kGroupWords words: every thread issues
+  // the loads of all its words (up to 4 x 64 bytes) before encoding any
+  const int64_t k0 = local * jb.rows;
+  const int nrows = static_cast<int>(jb.K - k0 < jb.rows ? jb.K - k0 : jb.rows);
+  const int nwords = nrows * jb.wpf;
+  const float* base = jb.W + k0 * static_cast<int64_t>(jb.n);
+  uint32_t* out = jb.codes + k0 * static_cast<int64_t>(jb.wpf);
+  float v[kWordsPerThread][16];
+  int nv[kWordsPerThread];
+#pragma unroll
+  for (int u = 0; u < kWordsPerThread; ++u) {
+    const int j = threadIdx.x + u * kThreads;
+    if (j < nwords) {
+      const int r = j / jb.wpf, c = j - r * jb.wpf;
+      load16(base + static_cast<int64_t>(r) * jb.n, jb.n, c, jb.vec != 0, v[u], nv[u]);
+    } else {
+      nv[u] = 0;
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kWordsPerThread; ++u) {
+    const int j = threadIdx.x + u * kThreads;
+    if (j < nwords) {
+      uint32_t word;
+      double sum;
+      int c2;
+      encode16(v[u], nv[u], word, sum, c2);
+      out[j] = word;   // the group's words are contiguous in the codes array
+      s_num[j] = sum;
+      s_cnt[j] = c2;
+    }
+  }
+  __syncthreads();
+  // one warp per filter of the group: sum its words in index order per lane
+  for (int r = warp; r < nrows; r += kThreads / 32) {
     double acc = 0.0;
     int cnt2 = 0;
-    quantize_words<2>(row, out, jb.n, jb.wpf, jb.vec != 0, lane, 32, acc, cnt2);
+    for (int c = lane; c < jb.wpf; c += 32) {
+      acc += s_num[r * jb.wpf + c];
+      cnt2 += s_cnt[r * jb.wpf + c];
+    }
     acc = warp_sum(acc);
     cnt2 = warp_sum(cnt2);
-    if (lane == 0) jb.alpha[k] = alpha_of(acc, cnt2, jb.n);
+    if (lane == 0) jb.alpha[k0 + r] = alpha_of(acc, cnt2, jb.n);
   }
 }
 
@@ -252,9 +299,9 @@ tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStrea
     q.n = static_cast<int32_t>(j.n);
     q.wpf = static_cast<int32_t>((j.n + 15) / 16);
     q.vec = (is_aligned(j.W, 16) && (j.n % 4) == 0) ? 1 : 0;
-    q.wide = q.wpf >= kWideMinWords ? 1 : 0;
+    q.rows = q.wpf <= kGroupWords ? static_cast<int32_t>(std::min<int64_t>(j.K, kGroupWords / q.wpf)) : 0;
     q.first_task = tasks;
-    tasks += q.wide ? j.K : (j.K + kRowsPerNarrowCta - 1) / kRowsPerNarrowCta;
+    tasks += q.rows == 0 ? j.K : (j.K + q.rows - 1) / q.rows;
   }
   if (tasks == 0) return TBN_OK;
   if (tasks > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "quantize: too many filters (%lld tasks)", (long long)tasks);

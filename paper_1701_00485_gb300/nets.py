@@ -61,18 +61,24 @@ class ConvStack:
             codes = torch.empty((K, packed_words(n)), dtype=torch.int32, device=self.device)
             alpha = torch.empty((K,), dtype=torch.float32, device=self.device)
             ohw = conv_out_hw(hw[0], hw[1], R, S, (spec.stride, spec.stride), (spec.pad, spec.pad))
-            y = torch.empty((N, ohw[0], ohw[1], K), dtype=torch.bfloat16, device=self.device)
             pooled = None
             nhw = ohw
+            fused = spec.pool == (2, 2)
             if spec.pool is not None:
                 k, st = spec.pool
                 nhw = ((ohw[0] - k) // st + 1, (ohw[1] - k) // st + 1)
-                pooled = torch.empty((N, nhw[0], nhw[1], K), dtype=torch.bfloat16,
-                                     device=self.device)
+            if fused:
+                # 2x2/2 max pool fused into the convolution's epilogue
+                y = torch.empty((N, nhw[0], nhw[1], K), dtype=torch.bfloat16, device=self.device)
+            else:
+                y = torch.empty((N, ohw[0], ohw[1], K), dtype=torch.bfloat16, device=self.device)
+                if spec.pool is not None:
+                    pooled = torch.empty((N, nhw[0], nhw[1], K), dtype=torch.bfloat16,
+                                         device=self.device)
             self.layers.append(ConvLayer(spec, Wl, codes, alpha, hw, ohw, y, pooled))
             hw = nhw
-        self.out = self.layers[-1].pooled if self.layers[-1].pooled is not None else \
-            self.layers[-1].y
+        last = self.layers[-1]
+        self.out = last.pooled if last.pooled is not None else last.y
 
     @property
     def flops(self) -> int:
@@ -97,7 +103,8 @@ class ConvStack:
             if conv_hook:
                 conv_hook(i, l, "before")
             tbn_conv2d_fwd(h, l.codes, l.alpha, s.K, s.R, s.S, (s.stride, s.stride),
-                           (s.pad, s.pad), layout=TBN_NHWC, relu=s.relu, out=l.y)
+                           (s.pad, s.pad), layout=TBN_NHWC, relu=s.relu, out=l.y,
+                           pool=2 if s.pool == (2, 2) else 0)
             if conv_hook:
                 conv_hook(i, l, "after")
             h = l.y
@@ -108,6 +115,7 @@ class ConvStack:
         return h
 
     def launches_per_forward(self, requantize: bool = True) -> int:
+        # NCHW->NHWC, one launch per conv, one per pool that is not fused
         n = 1 + len(self.layers) + sum(1 for l in self.layers if l.pooled is not None)
         if requantize:
             n += (len(self.layers) + 15) // 16

@@ -86,6 +86,108 @@ def test_igemm_conv_matches_oracle_fp32_out(case):
     assert_within(y, y_orc, bound, out_bf16=False, what="igemm %s" % (case,))
 
 
+GATHER = [
+    # C % 64 != 0 (activations gathered by threads) or stride > 2
+    (2, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)),      # VGG first layer shape (C=3)
+    (1, 1, 28, 28, 20, 5, 5, (1, 1), (0, 0)),       # C=1
+    (1, 3, 35, 35, 96, 11, 11, (4, 4), (0, 0)),     # AlexNet conv1 geometry
+    (2, 96, 13, 13, 128, 5, 5, (1, 1), (2, 2)),     # C % 8 == 0, not % 64 (vector gather)
+    (2, 5, 9, 7, 70, 3, 3, (1, 1), (1, 1)),         # odd C, ragged K
+    (1, 16, 12, 12, 64, 3, 3, (2, 2), (1, 1)),      # stride 2 gathered
+    (1, 64, 20, 20, 128, 3, 3, (3, 3), (1, 1)),     # C % 64 == 0 but stride 3
+    (3, 24, 6, 6, 40, 1, 1, (1, 1), (0, 0)),        # 1x1, C=24
+]
+
+
+@pytest.mark.parametrize("case", GATHER)
+def test_igemm_gather_conv_matches_oracle(case):
+    c = make_case(*case, seed=4000 + sum(case[:7]), wscale=1.2)
+    algo = tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NHWC, *case[:7], case[7], case[8])
+    assert algo == tbn.TBN_CONV_IMPLICIT_GEMM
+    y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    assert_within(y, y_orc, bound, out_bf16=False, what="gather %s" % (case,))
+
+
+POOL = [
+    # N, C, H, W, K, R, S, stride, pad  -> conv + ReLU + 2x2/2 max pool fused
+    (2, 64, 32, 32, 128, 3, 3, (1, 1), (1, 1)),     # VGG c2 geometry (8-row tiles)
+    (4, 128, 8, 8, 256, 3, 3, (1, 1), (1, 1)),      # several images per tile
+    (3, 128, 16, 16, 200, 3, 3, (1, 1), (1, 1)),    # 16-wide rows, ragged K
+    (2, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)),      # gathered activations
+    (5, 64, 9, 8, 64, 3, 3, (1, 1), (1, 1)),        # odd P (floor), images per tile
+]
+POOL_OTHER = [
+    (1, 64, 13, 11, 72, 3, 3, (1, 1), (1, 1)),      # odd P, Q: direct kernel
+    (1, 64, 60, 60, 128, 3, 3, (1, 1), (1, 1)),     # 60-wide rows: direct kernel
+]
+
+
+def _pooled_oracle(c, x_dtype):
+    import oracle
+    y, bound = c.oracle_full(x_dtype)
+    y = oracle.epilogue(y, None, relu=True)
+    P2, Q2 = y.shape[2] // 2, y.shape[3] // 2
+    yp = oracle.maxpool2d_nchw(y, (2, 2), (2, 2))
+    # the tolerance of a pooled output: the largest bound in its window
+    bw = bound[:, :, :2 * P2, :2 * Q2].reshape(bound.shape[0], bound.shape[1], P2, 2, Q2, 2)
+    return yp, bw.max(axis=(3, 5))
+
+
+def _run_pooled(c, layout, x_dtype, y_dtype, algo):
+    Wl, codes, alpha = c.quantize_gpu(layout)
+    x = c.x.to(x_dtype)
+    if layout == tbn.TBN_NHWC:
+        x = x.permute(0, 2, 3, 1).contiguous()
+    y = tbn.tbn_conv2d_fwd(x.cuda(), codes, alpha, c.K, c.R, c.S, c.stride, c.pad, layout=layout,
+                           out_dtype=y_dtype, relu=True, pool=2, algo=algo)
+    y = y.float().cpu()
+    if layout == tbn.TBN_NHWC:
+        y = y.permute(0, 3, 1, 2)
+    return y.numpy()
+
+
+@pytest.mark.parametrize("case", POOL)
+@pytest.mark.parametrize("algo", [tbn.TBN_CONV_IMPLICIT_GEMM, tbn.TBN_CONV_DIRECT])
+def test_fused_relu_pool_matches_oracle(case, algo):
+    c = make_case(*case, seed=5000 + sum(case[:7]))
+    want, bound = _pooled_oracle(c, torch.bfloat16)
+    y = _run_pooled(c, tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo)
+    assert y.shape == want.shape
+    assert_within(y, want, bound, out_bf16=False, epilogue=True, what="pool %s" % (case,))
+    yb = _run_pooled(c, tbn.TBN_NHWC, torch.bfloat16, torch.bfloat16, algo)
+    assert_within(yb, want, bound, out_bf16=True, epilogue=True, what="pool bf16 %s" % (case,))
+
+
+@pytest.mark.parametrize("case", POOL_OTHER)
+def test_fused_pool_other_widths_auto(case):
+    c = make_case(*case, seed=5100 + sum(case[:7]))
+    want, bound = _pooled_oracle(c, torch.bfloat16)
+    y = _run_pooled(c, tbn.TBN_NHWC, torch.bfloat16, torch.float32, tbn.TBN_CONV_AUTO)
+    assert_within(y, want, bound, out_bf16=False, epilogue=True, what="pool auto %s" % (case,))
+    with pytest.raises(tbn.TBNError):
+        _run_pooled(c, tbn.TBN_NHWC, torch.bfloat16, torch.float32, tbn.TBN_CONV_IMPLICIT_GEMM)
+
+
+@pytest.mark.parametrize("case", IGEMM[3:6] + GATHER[:2])
+def test_igemm_persistent_many_tiles_per_cta(case):
+    """Batches large enough that every CTA of the persistent kernel walks
+    several tiles (accumulator reuse across tiles)."""
+    N = case[0] * 40
+    c = make_case(N, *case[1:], seed=6000 + sum(case[:7]))
+    y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.bfloat16, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+    sites = random_sites(y.shape, 4000, seed=N)
+    y_orc, bound = c.oracle_sites(torch.bfloat16, sites)
+    assert_within(y[tuple(sites.T)], y_orc, bound, out_bf16=True, what="persistent %s" % (case,))
+
+
+def test_fused_pool_nchw_direct():
+    c = make_case(2, 3, 10, 12, 9, 3, 3, (1, 1), (1, 1), seed=77)
+    want, bound = _pooled_oracle(c, torch.float32)
+    y = _run_pooled(c, tbn.TBN_NCHW, torch.float32, torch.float32, tbn.TBN_CONV_DIRECT)
+    assert_within(y, want, bound, out_bf16=False, epilogue=True, what="pool nchw")
+
+
 @pytest.mark.parametrize("case", IGEMM[:6])
 def test_igemm_conv_bf16_out_and_epilogue(case):
     c = make_case(*case, seed=2000 + sum(case[:7]))
