@@ -1,34 +1,41 @@
 """Benchmark of the TBN hot path on GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload vgg_small|gemv|quantize]
 
-Workload (default): the VGG-small TBN conv stack at batch 128 on CIFAR-sized
+Default workload: the VGG-small TBN conv stack at batch 128 on CIFAR-sized
 input (3x32x32 bf16 ~ N(0,1), six 3x3/p1 layers 128-128-256-256-512-512,
 ReLU, 2x2 max pool after every second layer, He-normal weights), seed 1.
 One step = one pass of the whole hot path over the batch: re-quantize every
 layer's real-valued weights (Eq. 3 + Eq. 5 + packing, one grouped launch),
-NCHW -> NHWC, six two-bit convolutions (Eq. 1) with fused ReLU, three max
-pools.  The metric is TBN-conv TFLOP/s: the algorithmic 2*N*K*P*Q*C*R*S
-flops of the six convolutions per step over the step's device time (every
-launch of the step included); images/s is reported beside it.
+NCHW -> NHWC, six two-bit convolutions (Eq. 1) with fused ReLU and, after
+every second layer, the fused 2x2 max pool.  The metric is TBN-conv TFLOP/s:
+the algorithmic 2*N*K*P*Q*C*R*S flops of the six convolutions per step over
+the step's device time (every launch of the step included); images/s is
+reported beside it.
 
-Timing: the step is captured once in a CUDA graph; W warm-up replays, then
-K timed replays, each timed with CUDA events recorded inside the graph
-(start/end of the step and around every tensor-core convolution), a 512 MiB
-L2 flush between replays (outside the timed events).  nvidia-smi samples the
-SM clock from the last second of warm-up to the end of the timed region.
-
-The e2e figure replays a second graph that adds, each step, the copy of the
-input batch from pinned host memory and the copy of the output feature map
-back to pinned host memory.
+Timing: the step is captured in a CUDA graph; W warm-up replays (and at
+least --min-warmup-s seconds of them, so the clocks settle), then K timed
+replays, each bracketed by CUDA events recorded inside the graph, with a
+512 MiB write between replays that flushes L2 (outside the timed events).
+nvidia-smi samples the SM clock through the timed regions.  A second timed
+region replays an instrumented copy of the graph with events around every
+tensor-core convolution: the roofline entry (the tcgen05 conv kernel) is
+its flops over those durations.  The e2e figure replays a third graph that
+adds, each step, the copy of the input batch from pinned host memory and the
+copy of the output feature map back to pinned host memory.
 
 Under torchrun (N > 1) every rank runs its own batch on its own GPU (data
-parallel replicas, no collective on the data path): value = the images of all
+parallel replicas, no collective on the data path): value = the work of all
 ranks over the slowest rank's time.
 
---impl reference times the CPU oracle (plain C, fp64) on the same workload:
-a bounded sample of images through re-quantization + the six convolutions +
-glue, reported in the same unit.
+--workload gemv       batch-1/8 fully-connected layers, K_out = K_in in
+                      {4096, 8192, 16384}: HBM GB/s on the 2-bit stream
+--workload quantize   tbn_quantize_pack on 8192^2 and 16384^2 fp32 matrices:
+                      HBM GB/s at 4.25 bytes per weight
+--impl reference      the CPU oracle (plain C, fp64) on the VGG-small
+                      workload: one image of the batch per step through
+                      re-quantization + the six convolutions + glue.
 """
 from __future__ import annotations
 
@@ -49,6 +56,7 @@ import torch  # noqa: E402
 WORKLOAD = "vgg_small_b128_cifar"
 METRIC = "TBN conv TFLOP/s (VGG-small b128 forward incl. per-step re-quantization)"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FLUSH_BYTES = 512 * 1024 * 1024
 
 
 def load_peaks():
@@ -113,8 +121,47 @@ class ClockSampler:
                 "samples": len(sel)}
 
 
-# ------------------------------------------------------------------ our arm
-def run_ours(args, rank, world, local_rank):
+def timed_replays(graph, stream, flush, ev, steps, dev):
+    """Replay `graph` `steps` times, flushing L2 before each replay; returns
+    the per-replay device times (ms) between the graph's own events ev."""
+    out = []
+    for _ in range(steps):
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            graph.replay()
+        stream.synchronize()
+        out.append(ev[0].elapsed_time(ev[1]))
+    return out
+
+
+def warm(graph, stream, flush, steps, min_s, dev):
+    t = time.time()
+    w = 0
+    while w < steps or time.time() - t < min_s:
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            graph.replay()
+        w += 1
+        if w % 50 == 0:
+            torch.cuda.synchronize(dev)
+    torch.cuda.synchronize(dev)
+
+
+def max_over_ranks(x: float, world: int, dev) -> float:
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+# ------------------------------------------------------------------ VGG-small
+def run_vgg(args, rank, world, local_rank):
     import paper_1701_00485_gb300 as tbn
     from paper_1701_00485_gb300 import nets
 
@@ -138,7 +185,20 @@ def run_ours(args, rank, world, local_rank):
     if tbn.tbn_device_error() != 0:
         raise RuntimeError("device error word set after warm-up")
 
-    ev_step = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+    def capture(body):
+        ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(g, stream=stream):
+                ev[0].record()
+                body()
+                ev[1].record()
+        torch.cuda.synchronize(dev)
+        return g, ev
+
+    # plain step: the timed graph
+    graph, ev_step = capture(lambda: net.forward(requantize=True))
+    # instrumented step: events around every tensor-core convolution
     ev_conv = {i: [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
                for i in tc_layers}
 
@@ -146,98 +206,62 @@ def run_ours(args, rank, world, local_rank):
         if i in ev_conv:
             ev_conv[i][0 if when == "before" else 1].record()
 
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(stream):
-        with torch.cuda.graph(graph, stream=stream):
-            ev_step[0].record()
-            net.forward(requantize=True, conv_hook=hook)
-            ev_step[1].record()
-    torch.cuda.synchronize(dev)
+    graph_i, ev_i = capture(lambda: net.forward(requantize=True, conv_hook=hook))
+    # e2e step: host input in, output feature map out
+    x_host = net.x_in.cpu().pin_memory()
+    out_host = torch.empty(net.out.shape, dtype=net.out.dtype).pin_memory()
 
-    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    def e2e_body():
+        net.x_in.copy_(x_host, non_blocking=True)
+        net.forward(requantize=True)
+        out_host.copy_(net.out, non_blocking=True)
+
+    graph_e, ev_e = capture(e2e_body)
+
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
     sampler = ClockSampler(local_rank)
     sampler.start()
-    # warm-up: W replays, and at least --min-warmup-s of replays so clocks settle
-    t_w = time.time()
-    w = 0
-    while w < args.warmup or time.time() - t_w < args.min_warmup_s:
-        with torch.cuda.stream(stream):
-            flush.zero_()
-            graph.replay()
-        w += 1
-        if w % 50 == 0:
-            torch.cuda.synchronize(dev)
-    torch.cuda.synchronize(dev)
+    warm(graph, stream, flush, args.warmup, args.min_warmup_s, dev)
 
-    if world > 1:
-        torch.distributed.barrier()
+    barrier(world)
     torch.cuda.synchronize(dev)
     t0 = time.time()
-    step_ms, conv_ms = [], []
+    step_ms = timed_replays(graph, stream, flush, ev_step, args.steps, dev)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    # roofline region: the instrumented graph, same number of steps
+    conv_ms = []
     for _ in range(args.steps):
         with torch.cuda.stream(stream):
             flush.zero_()
-            graph.replay()
+            graph_i.replay()
         stream.synchronize()
-        step_ms.append(ev_step[0].elapsed_time(ev_step[1]))
         conv_ms.append(sum(ev_conv[i][0].elapsed_time(ev_conv[i][1]) for i in tc_layers))
-    torch.cuda.synchronize(dev)
     t1 = time.time()
-    if world > 1:
-        torch.distributed.barrier()
     clocks = sampler.stop(t0, t1)
 
-    total_ms = float(np.sum(step_ms))
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(float(np.sum(step_ms)), world, dev)
     ms_per_step = total_ms / args.steps
     value = world * flops * args.steps / (total_ms * 1e-3) / 1e12
     images_per_s = world * N * args.steps / (total_ms * 1e-3)
 
-    # e2e: pinned host input -> device, step, output -> pinned host
-    x_host = net.x_in.cpu().pin_memory()
-    out_host = torch.empty(net.out.shape, dtype=net.out.dtype).pin_memory()
-    g2 = torch.cuda.CUDAGraph()
-    ev_e = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-    with torch.cuda.stream(stream):
-        with torch.cuda.graph(g2, stream=stream):
-            ev_e[0].record()
-            net.x_in.copy_(x_host, non_blocking=True)
-            net.forward(requantize=True)
-            out_host.copy_(net.out, non_blocking=True)
-            ev_e[1].record()
-    for _ in range(3):
-        with torch.cuda.stream(stream):
-            g2.replay()
-    torch.cuda.synchronize(dev)
-    e2e_ms = []
-    for _ in range(args.steps):
-        with torch.cuda.stream(stream):
-            flush.zero_()
-            g2.replay()
-        stream.synchronize()
-        e2e_ms.append(ev_e[0].elapsed_time(ev_e[1]))
-    e2e_total = float(np.sum(e2e_ms))
-    if world > 1:
-        t = torch.tensor([e2e_total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_total = float(t.item())
+    warm(graph_e, stream, flush, 3, 0.0, dev)
+    e2e_ms = timed_replays(graph_e, stream, flush, ev_e, args.steps, dev)
+    e2e_total = max_over_ranks(float(np.sum(e2e_ms)), world, dev)
     e2e_value = world * flops * args.steps / (e2e_total * 1e-3) / 1e12
 
     err = tbn.tbn_device_error()
     peaks, peak_kind = load_peaks()
-    tc_ms = float(np.mean(conv_ms)) / max(1, len(tc_layers))  # mean per launch
-    achieved = (tc_flops / max(1, len(tc_layers))) / (tc_ms * 1e-3) / 1e12
+    tc_launch_ms = float(np.mean(conv_ms)) / max(1, len(tc_layers))  # mean per launch
+    achieved = (tc_flops / max(1, len(tc_layers))) / (tc_launch_ms * 1e-3) / 1e12
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
     roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
                 "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
-                "kernel": "conv_igemm_kernel (tcgen05 implicit GEMM), layers %s" %
-                          ",".join("c%d" % (i + 1) for i in tc_layers),
+                "kernel": "conv_igemm_kernel (tcgen05 implicit GEMM), %d launches per step "
+                          "(layers %s)" % (len(tc_layers),
+                                           ",".join("c%d" % (i + 1) for i in tc_layers)),
                 "peak_kind": "%s bf16 dense, sustained" % peak_kind}
-
-    result = {
+    return {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
@@ -257,7 +281,127 @@ def run_ours(args, rank, world, local_rank):
         "clocks": clocks,
         "device_error_word": err,
     }
-    return result
+
+
+# ------------------------------------------------------------------ HBM-bound paths
+def _rotating_graph(fn_list, stream, dev):
+    """One graph that calls each fn once (launches rotate over buffers that
+    together exceed L2), bracketed by events."""
+    ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(g, stream=stream):
+            ev[0].record()
+            for fn in fn_list:
+                fn()
+            ev[1].record()
+    torch.cuda.synchronize(dev)
+    return g, ev
+
+
+def run_gemv(args, rank, world, local_rank):
+    import paper_1701_00485_gb300 as tbn
+    from paper_1701_00485_gb300 import inputs
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    stream = torch.cuda.Stream(device=dev)
+    sweep = []
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    t0 = time.time()
+    for K in inputs.GEMV_SIZES:
+        W, _ = inputs.gemv_inputs(K, 1)
+        codes, alpha = tbn.tbn_quantize_pack(W.to(dev))
+        del W
+        code_bytes = codes.numel() * 4
+        copies = max(2, int(np.ceil(3 * l2 / code_bytes)))
+        bufs = [codes] + [codes.clone() for _ in range(copies - 1)]
+        for B in inputs.GEMV_BATCHES:
+            gx = torch.Generator(device=dev)
+            gx.manual_seed(1000 * K + B)
+            x = torch.randn((B, K), generator=gx, device=dev).to(torch.bfloat16)
+            y = torch.empty((B, K), dtype=torch.bfloat16, device=dev)
+            reps = max(copies, 64)
+            fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x, c, alpha, K, out=y))
+                   for r in range(reps)]
+            with torch.cuda.stream(stream):
+                fns[0]()
+            torch.cuda.synchronize(dev)
+            g, ev = _rotating_graph(fns, stream, dev)
+            for _ in range(max(3, args.warmup)):
+                g.replay()
+            torch.cuda.synchronize(dev)
+            ms = []
+            for _ in range(max(3, args.steps // 20)):
+                with torch.cuda.stream(stream):
+                    g.replay()
+                stream.synchronize()
+                ms.append(ev[0].elapsed_time(ev[1]) / reps)
+            t = float(np.median(ms)) * 1e-3
+            byts = code_bytes + 4 * K + 2 * B * K * 2
+            sweep.append({"K": K, "B": B, "us_per_call": round(t * 1e6, 3),
+                          "gbs": round(byts / t / 1e9, 1), "frac_hbm": round(byts / t / 1e9 / hbm, 4),
+                          "tflops": round(2 * B * K * K / t / 1e12, 3)})
+        del bufs
+        torch.cuda.empty_cache()
+    clocks = sampler.stop(t0, time.time())
+    head = [s for s in sweep if s["K"] == 16384 and s["B"] == 1][0]
+    return {"metric": "TBN GEMV HBM GB/s (B=1, K_out=K_in=16384, 2-bit weight stream)",
+            "value": head["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (He-normal weights, N(0,1) activations)",
+            "config": {"workload": "gemv_sweep", "l2": "rotating weight copies > 3x L2"},
+            "roofline": {"bound": "hbm", "achieved": head["gbs"], "peak": hbm, "unit": "GB/s",
+                         "frac": round(head["gbs"] / hbm, 4), "traffic": None,
+                         "kernel": "gemv_kernel", "peak_kind": peak_kind},
+            "sweep": sweep, "clocks": clocks}
+
+
+def run_quantize(args, rank, world, local_rank):
+    import paper_1701_00485_gb300 as tbn
+    from paper_1701_00485_gb300 import inputs
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    sweep = []
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    t0 = time.time()
+    for K in (8192, 16384):
+        W, _ = inputs.gemv_inputs(K, 1)
+        W = W.to(dev)
+        codes = torch.empty((K, K // 16), dtype=torch.int32, device=dev)
+        alpha = torch.empty((K,), dtype=torch.float32, device=dev)
+        g, ev = _rotating_graph([lambda: tbn.tbn_quantize_pack(W, codes, alpha)], stream, dev)
+        for _ in range(max(3, args.warmup)):
+            g.replay()
+        torch.cuda.synchronize(dev)
+        ms = timed_replays(g, stream, flush, ev, max(5, args.steps // 10), dev)
+        t = float(np.median(ms)) * 1e-3
+        byts = K * K * 4.25 + 4 * K
+        sweep.append({"K": K, "n": K, "us": round(t * 1e6, 2), "gbs": round(byts / t / 1e9, 1),
+                      "frac_hbm": round(byts / t / 1e9 / hbm, 4)})
+        del W, codes, alpha
+        torch.cuda.empty_cache()
+    clocks = sampler.stop(t0, time.time())
+    head = sweep[-1]
+    return {"metric": "TBN quantize+pack HBM GB/s (16384 x 16384 fp32, 4.25 B/weight)",
+            "value": head["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (He-normal weights)",
+            "config": {"workload": "quantize_16384", "l2": "512 MiB flush between timed steps"},
+            "roofline": {"bound": "hbm", "achieved": head["gbs"], "peak": hbm, "unit": "GB/s",
+                         "frac": head["frac_hbm"], "traffic": None,
+                         "kernel": "quantize_pack_kernel", "peak_kind": peak_kind},
+            "sweep": sweep, "clocks": clocks}
 
 
 # ------------------------------------------------------------------ CPU oracle
@@ -311,6 +455,7 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize"], default="vgg_small")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--min-warmup-s", type=float, default=1.0,
                     help="keep replaying warm-up steps for at least this long (clock settling)")
@@ -354,9 +499,10 @@ def main():
         torch.distributed.init_process_group("nccl")
     # the CPU baseline forks no workers after CUDA init: run it first
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "vgg_small":
         cpu = run_cpu_oracle()
-    res = run_ours(args, rank, world, local_rank)
+    runner = {"vgg_small": run_vgg, "gemv": run_gemv, "quantize": run_quantize}[args.workload]
+    res = runner(args, rank, world, local_rank)
     if rank == 0:
         if cpu is not None:
             res["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")}

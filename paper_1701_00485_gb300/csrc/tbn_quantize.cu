@@ -6,13 +6,19 @@
 // the codes do not depend on alpha and Eq. 5's two sums can be accumulated
 // in the same pass that discretizes.  Each thread owns whole 32-bit output
 // words (16 consecutive weights of a filter): it loads 64 contiguous bytes,
-// forms the sixteen 2-bit fields, and accumulates |W~|*|W| (fp32 within the
-// word, fp64 across words) and the count of magnitude-two codes.  A CTA
-// covers a group of whole filters of at most 1024 words; each of its 256
-// threads issues the loads of all its (up to four) words before encoding,
-// so a whole layer's weights are in flight at once, and the filters are
-// reduced through shared memory.  Filters longer than 1024 words get a CTA
-// each.  Bytes moved per weight: 4 read + 1/4 written.
+// forms the sixteen 2-bit fields, sums |W~|*|W| over the word in fp32
+// (pairwise), and counts the magnitude-two codes.  A CTA covers a group of
+// whole filters of at most 1024 words; each of its 256 threads issues the
+// loads of all its (up to four) words before encoding, so a whole layer's
+// weights are in flight at once, and the filters are reduced through shared
+// memory.  Filters longer than 1024 words get a CTA each.
+//
+// The word sums are accumulated exactly as a two-float (hi, lo) pair
+// (TwoSum, fp32 adds only: GB300's fp64 rate is a small fraction of its fp32
+// rate) and alpha = num / (n + 3 |B2|) is formed as hi / den plus the
+// remainder correction, one fp32 rounding, well inside 1e-6 relative.  A
+// word whose fp32 sum overflows (weights near the fp32 maximum) sends its
+// filter down an fp64 path.  Bytes moved per weight: 4 read + 1/4 written.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -46,24 +52,77 @@ struct QParams {
   uint32_t* err;
 };
 
-// fp64 re-summation of one word whose fp32 sum overflowed (weights near the
-// fp32 maximum).  Kept out of line so the common path carries no fp64 work.
-__device__ __noinline__ double word_sum_fp64(const float* v, int nvalid) {
-  double d = 0.0;
-  for (int e = 0; e < nvalid; ++e) {
-    const double a = fabs(static_cast<double>(v[e]));
-    d += a > 1.0 ? 2.0 * a : a;
-  }
-  return d;
+// ---- exact two-float accumulation (fp32 adds only) -----------------------
+struct Sum2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ void add2(Sum2& s, float x) {
+  // TwoSum: hi + lo gains x with the rounding error of the add kept in lo
+  const float t = __fadd_rn(s.hi, x);
+  const float bp = __fsub_rn(t, s.hi);
+  const float e = __fadd_rn(__fsub_rn(s.hi, __fsub_rn(t, bp)), __fsub_rn(x, bp));
+  s.hi = t;
+  s.lo = __fadd_rn(s.lo, e);
 }
 
-// Sixteen weights -> one packed word, the sum of |W~|*|W| over them (fp32,
-// pairwise; redone in fp64 when the fp32 sum overflows, i.e. for weights
-// near the fp32 maximum) and the number of magnitude-two codes.  Eq. 3:
-// s = [W <= 0] (so -1 <= W <= 0 and W < -1 are negative, -0.0 included),
-// m = [|W| > 1].
+__device__ __forceinline__ void merge2(Sum2& s, const Sum2& o) {
+  add2(s, o.hi);
+  s.lo = __fadd_rn(s.lo, o.lo);
+}
+
+__device__ __forceinline__ Sum2 warp_sum2(Sum2 s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    Sum2 t;
+    t.hi = __shfl_xor_sync(0xffffffffu, s.hi, o);
+    t.lo = __shfl_xor_sync(0xffffffffu, s.lo, o);
+    merge2(s, t);
+  }
+  return s;
+}
+
+__device__ __forceinline__ int warp_sum(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Eq. 5 with |B1| + 4|B2| = n + 3|B2|: (hi + lo) / den with one final
+// rounding, from an fp32 quotient and its exact remainder (den < 2^24 is
+// exact in fp32; longer filters take the fp64 division).
+__device__ __forceinline__ float alpha_of(const Sum2& s, int cnt2, int n) {
+  const int64_t den_i = static_cast<int64_t>(n) + 3 * static_cast<int64_t>(cnt2);
+  if (den_i >= (int64_t(1) << 24))
+    return static_cast<float>((static_cast<double>(s.hi) + static_cast<double>(s.lo)) /
+                              static_cast<double>(den_i));
+  const float den = static_cast<float>(den_i);
+  const float q = __fdiv_rn(s.hi, den);
+  const float r = __fadd_rn(__fmaf_rn(-q, den, s.hi), s.lo);   // exact remainder + lo
+  return __fadd_rn(q, __fdiv_rn(r, den));
+}
+
+// fp64 alpha of one filter, used only when a word sum overflowed fp32.
+__device__ __noinline__ float alpha_fp64_row(const float* __restrict__ row, int n) {
+  double num = 0.0;
+  int64_t cnt2 = 0;
+  for (int i = 0; i < n; ++i) {
+    const double a = fabs(static_cast<double>(row[i]));
+    if (a > 1.0) {
+      num += 2.0 * a;
+      ++cnt2;
+    } else {
+      num += a;
+    }
+  }
+  return static_cast<float>(num / (static_cast<double>(n) + 3.0 * static_cast<double>(cnt2)));
+}
+
+// Sixteen weights -> one packed word, the fp32 pairwise sum of |W~|*|W| over
+// them and the number of magnitude-two codes.  Eq. 3: s = [W <= 0] (so
+// -1 <= W <= 0 and W < -1 are negative, -0.0 included), m = [|W| > 1].
 __device__ __forceinline__ void encode16(const float (&v)[16], int nvalid, uint32_t& word,
-                                         double& dsum, int& cnt2) {
+                                         float& sum, int& cnt2) {
   float c[16];
   uint32_t w = 0;
   int n2 = 0;
@@ -83,18 +142,12 @@ __device__ __forceinline__ void encode16(const float (&v)[16], int nvalid, uint3
   for (int e = 0; e < 4; ++e) c[e] += c[e + 4];
   c[0] += c[2];
   c[1] += c[3];
-  const float sum = c[0] + c[1];
-  if (__builtin_expect(sum <= 3.4028234663852886e38f, 1)) {
-    dsum = static_cast<double>(sum);
-  } else {
-    float tmp[16];
-#pragma unroll
-    for (int e = 0; e < 16; ++e) tmp[e] = v[e];
-    dsum = word_sum_fp64(tmp, nvalid);
-  }
+  sum = c[0] + c[1];
   word = w;
   cnt2 = n2;
 }
+
+__device__ __forceinline__ bool finite_sum(float s) { return s <= 3.4028234663852886e38f; }
 
 __device__ __forceinline__ void load16(const float* __restrict__ row, int n, int j, bool vec,
                                        float (&v)[16], int& nvalid) {
@@ -116,26 +169,27 @@ __device__ __forceinline__ void load16(const float* __restrict__ row, int n, int
   }
 }
 
-// Process words j0, j0 + stride, ... of one filter; returns the partial sums.
-template <int kUnroll>
-__device__ __forceinline__ void quantize_words(const float* __restrict__ row,
-                                               uint32_t* __restrict__ out, int n, int wpf,
-                                               bool vec, int j0, int stride, double& acc,
-                                               int& cnt2) {
+// Words j0, j0 + stride, ... of one long filter; accumulates the partials.
+__device__ __forceinline__ void quantize_words_strided(const float* __restrict__ row,
+                                                       uint32_t* __restrict__ out, int n, int wpf,
+                                                       bool vec, int j0, int stride, Sum2& acc,
+                                                       int& cnt2, bool& huge) {
+  constexpr int kU = 4;
   int j = j0;
-  for (; j + (kUnroll - 1) * stride < wpf; j += kUnroll * stride) {
-    float v[kUnroll][16];
-    int nv[kUnroll];
+  for (; j + (kU - 1) * stride < wpf; j += kU * stride) {
+    float v[kU][16];
+    int nv[kU];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) load16(row, n, j + u * stride, vec, v[u], nv[u]);
+    for (int u = 0; u < kU; ++u) load16(row, n, j + u * stride, vec, v[u], nv[u]);
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
+    for (int u = 0; u < kU; ++u) {
       uint32_t word;
-      double s;
+      float s;
       int c;
       encode16(v[u], nv[u], word, s, c);
       out[j + u * stride] = word;
-      acc += s;
+      huge |= !finite_sum(s);
+      add2(acc, s);
       cnt2 += c;
     }
   }
@@ -144,36 +198,22 @@ __device__ __forceinline__ void quantize_words(const float* __restrict__ row,
     int nv;
     load16(row, n, j, vec, v, nv);
     uint32_t word;
-    double s;
+    float s;
     int c;
     encode16(v, nv, word, s, c);
     out[j] = word;
-    acc += s;
+    huge |= !finite_sum(s);
+    add2(acc, s);
     cnt2 += c;
   }
 }
 
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
-__device__ __forceinline__ int warp_sum(int v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
-// Eq. 5 with |B1| + 4|B2| = n + 3|B2|; one rounding to fp32 at the end.
-__device__ __forceinline__ float alpha_of(double num, int cnt2, int n) {
-  const double den = static_cast<double>(n) + 3.0 * static_cast<double>(cnt2);
-  return static_cast<float>(num / den);
-}
-
 __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_constant__ QParams prm) {
-  __shared__ double s_num[kGroupWords];
+  __shared__ float s_sum[kGroupWords];
   __shared__ int s_cnt[kGroupWords];
+  __shared__ Sum2 s_part[kThreads / 32];
+  __shared__ int s_pcnt[kThreads / 32];
+  __shared__ int s_huge;
 
   const int64_t task = blockIdx.x;
   int ji = 0;
@@ -189,22 +229,28 @@ __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_co
     const int64_t k = local;
     const float* row = jb.W + k * static_cast<int64_t>(jb.n);
     uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
-    double acc = 0.0;
+    Sum2 acc{0.0f, 0.0f};
     int cnt2 = 0;
-    quantize_words<4>(row, out, jb.n, jb.wpf, jb.vec != 0, threadIdx.x, kThreads, acc, cnt2);
-    acc = warp_sum(acc);
+    bool huge = false;
+    if (threadIdx.x == 0) s_huge = 0;
+    quantize_words_strided(row, out, jb.n, jb.wpf, jb.vec != 0, threadIdx.x, kThreads, acc, cnt2,
+                           huge);
+    acc = warp_sum2(acc);
     cnt2 = warp_sum(cnt2);
+    __syncthreads();
+    if (huge) s_huge = 1;
     if (lane == 0) {
-      s_num[warp] = acc;
-      s_cnt[warp] = cnt2;
+      s_part[warp] = acc;
+      s_pcnt[warp] = cnt2;
     }
     __syncthreads();
     if (warp == 0) {
-      acc = lane < kThreads / 32 ? s_num[lane] : 0.0;
-      cnt2 = lane < kThreads / 32 ? s_cnt[lane] : 0;
-      acc = warp_sum(acc);
-      cnt2 = warp_sum(cnt2);
-      if (lane == 0) jb.alpha[k] = alpha_of(acc, cnt2, jb.n);
+      Sum2 t = lane < kThreads / 32 ? s_part[lane] : Sum2{0.0f, 0.0f};
+      int c = lane < kThreads / 32 ? s_pcnt[lane] : 0;
+      t = warp_sum2(t);
+      c = warp_sum(c);
+      if (lane == 0)
+        jb.alpha[k] = s_huge ? alpha_fp64_row(row, jb.n) : alpha_of(t, c, jb.n);
     }
     return;
   }
@@ -233,26 +279,32 @@ __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_co
     const int j = threadIdx.x + u * kThreads;
     if (j < nwords) {
       uint32_t word;
-      double sum;
+      float sum;
       int c2;
       encode16(v[u], nv[u], word, sum, c2);
       out[j] = word;   // the group's words are contiguous in the codes array
-      s_num[j] = sum;
+      s_sum[j] = sum;
       s_cnt[j] = c2;
     }
   }
   __syncthreads();
-  // one warp per filter of the group: sum its words in index order per lane
+  // one warp per filter of the group: two-float sum of its word sums
   for (int r = warp; r < nrows; r += kThreads / 32) {
-    double acc = 0.0;
+    Sum2 acc{0.0f, 0.0f};
     int cnt2 = 0;
+    bool huge = false;
     for (int c = lane; c < jb.wpf; c += 32) {
-      acc += s_num[r * jb.wpf + c];
+      const float s = s_sum[r * jb.wpf + c];
+      huge |= !finite_sum(s);
+      add2(acc, s);
       cnt2 += s_cnt[r * jb.wpf + c];
     }
-    acc = warp_sum(acc);
+    acc = warp_sum2(acc);
     cnt2 = warp_sum(cnt2);
-    if (lane == 0) jb.alpha[k0 + r] = alpha_of(acc, cnt2, jb.n);
+    huge = __any_sync(0xffffffffu, huge);
+    if (lane == 0)
+      jb.alpha[k0 + r] = huge ? alpha_fp64_row(base + static_cast<int64_t>(r) * jb.n, jb.n)
+                              : alpha_of(acc, cnt2, jb.n);
   }
 }
 
