@@ -30,18 +30,23 @@
  * - tbn_last_error() returns a human-readable detail string for the most
  *   recent failing call on the calling host thread.
  *
- * Two-bit storage format (the paper fixes only that the four values "can be
- * encoded with two bits"; the layout below is this library's):
+ * Two-bit storage format (the paper fixes only that each of the four values
+ * takes two bits, Section 1; the layout below is this library's):
  * - each code is a 2-bit field f = m + 2 s with s = 1 for a negative value and
  *   m = 1 for magnitude two:  +1 -> 0, +2 -> 1, -1 -> 2, -2 -> 3;
  *   W~ = (1 - 2 s)(1 + m);
  * - a filter of n codes occupies tbn_packed_words(n) = ceil(n / 16) uint32
- *   words; code i of filter k is in bits [2 (i mod 16), 2 (i mod 16) + 1] of
- *   word k * ceil(n / 16) + i / 16 (little-endian: byte i/4, bits 2 (i mod 4));
- *   unused fields of a filter's last word are zero;
+ *   words; code i of filter k is in word k * ceil(n / 16) + i / 16;
+ * - inside a word ("byte-planar"), code l = i mod 16 = 2p + h (pair p in
+ *   0..7, half h in {0, 1}) has its m bit at bit 16h + p and its s bit at
+ *   bit 16h + 8 + p: byte 0 = m of the even codes, byte 1 = s of the even
+ *   codes, byte 2 = m of the odd codes, byte 3 = s of the odd codes.  A pair
+ *   of codes then decodes to two bf16 values with one mask, one shift and one
+ *   OR, which is what the kernels do;
+ * - unused codes of a filter's last word have m = s = 0;
  * - codes[K][ceil(n/16)] plus alpha[K] (fp32) is the complete inference
- *   form of a layer ("only the two-bit filters and the optimal scaling
- *   factors are used", Section 3).
+ *   form of a layer (at inference only the two-bit filters and their
+ *   scaling factors are needed, Section 3).
  * - The order of the n weights of a filter is the caller's choice; the
  *   convolution reads them in the activation layout's natural order:
  *   NCHW -> (c, r, s), NHWC -> (r, s, c).  Discretization is elementwise and
@@ -57,7 +62,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 1
+#define TBN_ABI_VERSION 2
 
 typedef enum {
   TBN_OK = 0,

@@ -65,9 +65,26 @@ void orc_quantize(const float *W, int64_t K, int64_t n, int8_t *wt, double *alph
 }
 
 /* ---- two-bit storage ---------------------------------------------------- */
+/* Layout (build-defined; the paper fixes only that a weight takes two bits):
+ * code i of a filter lives in word i / 16 of that filter.  Inside the word,
+ * with l = i % 16, pair p = l / 2 and half h = l % 2, the code's magnitude
+ * bit m sits at bit 16 h + p and its sign bit s at bit 16 h + 8 + p.  So byte
+ * 0 holds the magnitude bits of the even codes, byte 1 their sign bits,
+ * byte 2 the magnitude bits of the odd codes and byte 3 their sign bits. */
 int64_t orc_words_per_filter(int64_t n)
 {
     return (n + 15) / 16;
+}
+
+static int magnitude_bit(int64_t i)
+{
+    int64_t l = i % 16;
+    return (int)(16 * (l % 2) + l / 2);
+}
+
+static int sign_bit(int64_t i)
+{
+    return magnitude_bit(i) + 8;
 }
 
 /* field value for a code: m + 2 s  (s = negative, m = magnitude two) */
@@ -89,6 +106,14 @@ static int value_of(uint32_t field)
     return (1 - 2 * (int)s) * (1 + (int)m);
 }
 
+static uint32_t field_at(const uint32_t *words, int64_t wpf, int64_t k, int64_t i)
+{
+    uint32_t w = words[k * wpf + i / 16];
+    uint32_t m = (w >> magnitude_bit(i)) & 1u;
+    uint32_t s = (w >> sign_bit(i)) & 1u;
+    return m + 2u * s;
+}
+
 int orc_pack(const int8_t *wt, int64_t K, int64_t n, uint32_t *words)
 {
     int64_t wpf = orc_words_per_filter(n);
@@ -99,7 +124,8 @@ int orc_pack(const int8_t *wt, int64_t K, int64_t n, uint32_t *words)
             uint32_t f;
             if (field_of(wt[k * n + i], &f) != 0)
                 return -1;
-            words[k * wpf + i / 16] |= f << (2 * (i % 16));
+            uint32_t m = f & 1u, s = f >> 1;
+            words[k * wpf + i / 16] |= (m << magnitude_bit(i)) | (s << sign_bit(i));
         }
     }
     return 0;
@@ -110,15 +136,11 @@ int orc_unpack(const uint32_t *words, int64_t K, int64_t n, int8_t *wt)
     int64_t wpf = orc_words_per_filter(n);
     int bad_padding = 0;
     for (int64_t k = 0; k < K; ++k) {
-        for (int64_t i = 0; i < n; ++i) {
-            uint32_t f = (words[k * wpf + i / 16] >> (2 * (i % 16))) & 3u;
-            wt[k * n + i] = (int8_t)value_of(f);
-        }
-        for (int64_t i = n; i < wpf * 16; ++i) {
-            uint32_t f = (words[k * wpf + i / 16] >> (2 * (i % 16))) & 3u;
-            if (f != 0u)
+        for (int64_t i = 0; i < n; ++i)
+            wt[k * n + i] = (int8_t)value_of(field_at(words, wpf, k, i));
+        for (int64_t i = n; i < wpf * 16; ++i)
+            if (field_at(words, wpf, k, i) != 0u)
                 bad_padding = 1;
-        }
     }
     return bad_padding ? -1 : 0;
 }

@@ -14,8 +14,8 @@
  *   Eq. 2  (Section 2)  quantization error ||W - alpha W~||^2
  *   Eq. 1  (Section 2)  convolution with the approximated filter alpha W~
  *   Section 3           fully-connected layers treated as convolutions
- * plus the two-bit storage format (the paper says only that the four values
- * "can be encoded with two bits"; the bit layout is this library's own and
+ * plus the two-bit storage format (the paper fixes only that each of the four
+ * values takes two bits, Section 1; the bit layout is this library's own and
  * is spelled out at orc_pack below).
  *
  * All arrays are caller-owned host memory; nothing is allocated that
@@ -52,9 +52,12 @@ int64_t orc_words_per_filter(int64_t n);
 /* Two-bit storage format.  Each code is a 2-bit field (s, m):
  *   s = 1 when W~ < 0 (sign), m = 1 when |W~| = 2 (magnitude),
  *   field value = m + 2 s, i.e.  +1 -> 0, +2 -> 1, -1 -> 2, -2 -> 3,
- * and W~ = (1 - 2 s)(1 + m).  Code i of filter k occupies bits
- * [2 (i mod 16), 2 (i mod 16) + 1] of word k * words_per_filter + i / 16;
- * unused fields of the last word of a filter are zero.
+ * and W~ = (1 - 2 s)(1 + m).  Code i of filter k lives in word
+ * k * words_per_filter + i / 16.  With l = i mod 16, pair p = l / 2 and half
+ * h = l mod 2, its m bit is bit 16 h + p of that word and its s bit is bit
+ * 16 h + 8 + p ("byte-planar": byte 0 = m of the even codes, byte 1 = s of
+ * the even codes, byte 2 = m of the odd codes, byte 3 = s of the odd codes).
+ * Unused codes of the last word of a filter have m = s = 0.
  * words is [K][orc_words_per_filter(n)].  Returns 0, or -1 if some wt value
  * is not in {-2,-1,1,2}. */
 int orc_pack(const int8_t *wt, int64_t K, int64_t n, uint32_t *words);

@@ -68,6 +68,9 @@ _lock = threading.Lock()
 _lib = None
 
 
+ABI_VERSION = 2  # must match TBN_ABI_VERSION in include/tbn.h
+
+
 def lib_path() -> str:
     return _LIB_PATH
 
@@ -108,7 +111,7 @@ def lib():
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = res
-        if L.tbn_abi_version() != 1:
+        if L.tbn_abi_version() != ABI_VERSION:
             raise RuntimeError("libtbn ABI version mismatch")
         _lib = L
         return L

@@ -106,7 +106,7 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
       if (k < a.K) {
         const int64_t ti = t0 + t;
         const uint32_t w = a.codes[k * a.wpf + (ti >> 4)];
-        v = code_value((w >> (2 * (ti & 15))) & 3u);
+        v = code_value(code_field(w, static_cast<int>(ti & 15)));
       }
       s_w[t][f] = v;
     }

@@ -125,9 +125,6 @@ constexpr size_t kSmemBytes =
     1024 /*align slack*/ + kStages * kStageBytes + kOutStageBytes + sizeof(SmemCtl);
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 
-__device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
@@ -417,6 +414,7 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       }
       return r;
     };
+    const PairMultipliers pm;
     uint2 q0 = next_codes(), q1 = next_codes(), q2 = next_codes(), q3 = next_codes();
     const uint32_t col = a_tmem0 + lane_off + static_cast<uint32_t>(16 * half);
     // two K blocks per iteration: their tensor-memory stores share one
@@ -424,10 +422,10 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
     for (int g = 0; g < total; g += 2) {
       const bool two = g + 1 < total;   // warp-uniform
       uint32_t v0[16], v1[16];
-      word_to_bf16x2(q0.x, v0 + 0);
-      word_to_bf16x2(q0.y, v0 + 8);
-      word_to_bf16x2(q1.x, v1 + 0);
-      word_to_bf16x2(q1.y, v1 + 8);
+      word_to_bf16x2(q0.x, v0 + 0, pm);
+      word_to_bf16x2(q0.y, v0 + 8, pm);
+      word_to_bf16x2(q1.x, v1 + 0, pm);
+      word_to_bf16x2(q1.y, v1 + 8, pm);
       q0 = q2;
       q1 = q3;
       q2 = next_codes();
@@ -618,25 +616,6 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
 }
 
 // ---------------------------------------------------------------- host side
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn get_encode_tiled() {
-  static EncodeTiledFn fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(p);
-  });
-  return fn;
-}
-
 struct TilePlan {
   int bw, bh, bn, T, tile_n, tiles_q, tiles_p, tiles_n;
 };

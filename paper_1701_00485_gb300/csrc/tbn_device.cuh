@@ -81,6 +81,40 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return done != 0;
 }
 
+// try_wait with a suspend-time hint: the waiting thread may be parked (not
+// issuing) for up to `hint_ns` until the phase completes.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity,
+                                                    uint32_t hint_ns) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return done != 0;
+}
+
+// Bounded wait like mbar_wait below, parking the thread between polls
+// instead of spinning (for roles whose spinning would steal issue slots
+// from compute warps on the same SM sub-partition).
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity,
+                                                volatile int* abort, uint32_t* err,
+                                                uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (abort != nullptr && *abort) return false;
+    if (global_timer_ns() - t0 > limit_ns) {
+      raise_device_error(err, TBN_DEVERR_TIMEOUT);
+      if (abort != nullptr) *abort = 1;
+      return false;
+    }
+  }
+}
+
 // Wait until the phase with the given parity has completed, for at most
 // `limit_ns` nanoseconds.  Returns false (and records a timeout) on expiry,
 // or immediately when *abort is already set by another role.
@@ -103,7 +137,32 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
   }
 }
 
+// Named barrier over `nthreads` threads (a multiple of 32) of the CTA.
+__device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 // ---------------------------------------------------------------- TMA
+// 2-D and 3-D tiled bulk tensor loads global -> shared, completion on an
+// mbarrier (coordinates innermost first, in elements).
+__device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                            int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(tmap), "r"(smem_addr(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                            int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(tmap), "r"(smem_addr(bar)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
 // 4-D tiled bulk tensor load global -> shared, completion on an mbarrier.
 __device__ __forceinline__ void tma_load_4d(void* dst, const void* tmap, uint64_t* bar, int c0,
                                             int c1, int c2, int c3) {
@@ -267,20 +326,63 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N) {
 }
 
 // ---------------------------------------------------------------- codes
-// Two codes (one nibble: m_lo, s_lo, m_hi, s_hi) -> a pair of bf16 values
-// W~/2 in {+-0.5, +-1}.  bf16(+-0.5) = 0x3F00 | s<<15 and the magnitude-two
-// bit m is the exponent's low bit (1 << 7), so each half is
-// 0x3F00 | m << 7 | s << 15.  The multiply spreads the four nibble bits to
-// bits 7, 15, 23, 31 (the shifts 7, 14, 21, 28 put all sixteen partial
-// products at distinct positions, so no carries occur).
-__device__ __forceinline__ uint32_t nibble_to_bf16x2(uint32_t nib) {
-  return ((nib * 0x10204080u) & 0x80808080u) | 0x3F003F00u;
+// Packed word layout ("byte-planar"): code l = 2p + h of a word (pair p in
+// 0..7, half h in {0, 1}) keeps its magnitude-two bit m at bit 16h + p and
+// its sign bit s at bit 16h + 8 + p.  Byte 0 = m of the even codes, byte 1 =
+// s of the even codes, byte 2 = m of the odd codes, byte 3 = s of the odd
+// codes.  Field f = m + 2 s; W~ = (1 - 2 s)(1 + m).
+
+// Bit position of code l's magnitude bit (its sign bit is 8 above).
+__host__ __device__ constexpr int code_mag_bit(int l) { return 16 * (l & 1) + (l >> 1); }
+
+// Field (m + 2 s) of code l (0..15) of word w.
+__device__ __forceinline__ uint32_t code_field(uint32_t w, int l) {
+  const int b = code_mag_bit(l);
+  return ((w >> b) & 1u) | (((w >> (b + 8)) & 1u) << 1);
+}
+
+// Pair p (codes 2p, 2p+1) of word w as two bf16 values W~/2 in {+-0.5, +-1}.
+// bf16(+-0.5) = 0x3F00 | s << 15 and m is the exponent's low bit (1 << 7),
+// so each half is 0x3F00 | m << 7 | s << 15.  The pair's four bits sit at
+// p, 8 + p, 16 + p, 24 + p; isolating them and scaling by 2^(7-p) lands them
+// on 7, 15, 23, 31 without carries, and the constant fills the rest.
+template <int p>
+__device__ __forceinline__ uint32_t pair_to_bf16x2(uint32_t w) {
+  return (w & (0x01010101u << p)) * (1u << (7 - p)) + 0x3F003F00u;
 }
 
 // All 16 codes of one word as 8 bf16 pairs (pair p = codes 2p, 2p+1).
 __device__ __forceinline__ void word_to_bf16x2(uint32_t w, uint32_t* out8) {
+  out8[0] = pair_to_bf16x2<0>(w);
+  out8[1] = pair_to_bf16x2<1>(w);
+  out8[2] = pair_to_bf16x2<2>(w);
+  out8[3] = pair_to_bf16x2<3>(w);
+  out8[4] = pair_to_bf16x2<4>(w);
+  out8[5] = pair_to_bf16x2<5>(w);
+  out8[6] = pair_to_bf16x2<6>(w);
+  out8[7] = pair_to_bf16x2<7>(w);
+}
+
+// The multipliers 2^(7-p), p = 0..6, of pair_to_bf16x2 held in registers
+// the compiler cannot see through.  With a literal power of two the
+// compiler rewrites the multiply-add as shift + OR, putting both operations
+// of every pair on the integer ALU pipe; an opaque multiplier keeps one on
+// the ALU (the mask) and one on the FMA pipe (the multiply-add).
+struct PairMultipliers {
+  uint32_t m[7];
+  __device__ __forceinline__ PairMultipliers() {
 #pragma unroll
-  for (int p = 0; p < 8; ++p) out8[p] = nibble_to_bf16x2((w >> (4 * p)) & 0xFu);
+    for (int p = 0; p < 7; ++p) asm("mov.b32 %0, %1;" : "=r"(m[p]) : "r"(1u << (7 - p)));
+  }
+};
+
+// word_to_bf16x2 with opaque multipliers (pair 7 needs no shift: one
+// mask-and-OR).
+__device__ __forceinline__ void word_to_bf16x2(uint32_t w, uint32_t* out8,
+                                               const PairMultipliers& pm) {
+#pragma unroll
+  for (int p = 0; p < 7; ++p) out8[p] = (w & (0x01010101u << p)) * pm.m[p] + 0x3F003F00u;
+  out8[7] = (w & 0x80808080u) | 0x3F003F00u;
 }
 
 // Value W~ of code field f (m + 2 s) as float: (1 - 2 s)(1 + m).

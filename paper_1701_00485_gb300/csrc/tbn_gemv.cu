@@ -1,19 +1,38 @@
-// tbn_gemv.cu -- small-batch two-bit fully-connected layer (Section 3:
-// fully-connected layers treated as convolutions), y[b,k] = alpha_k *
-// sum_j x[b,j] W~[k,j] for B <= 8, bandwidth-bound on the 2-bit weight stream.
+// tbn_gemv.cu -- small-batch two-bit fully-connected layer (Section 3: a
+// fully-connected layer is a convolution whose filters span the whole
+// input), y[b, k] = alpha_k * sum_j x[b, j] W~[k, j] for 1 <= B <= 8.
 //
-// Tensor-core formulation per warp: mma.m16n8k16 with A = 16 weight rows x 16
-// codes decoded in registers to bf16 W~/2 (exact), B = 16 inputs x 8 batch
-// columns (batch padded with zeros), fp32 accumulation; 2 * alpha in the
-// epilogue.  The A fragment of lane (g = lane/4, t = lane%4) needs codes
-// 2t, 2t+1 and 2t+8, 2t+9 of rows g and g+8 -- nibbles t and t+4 of each
-// row's word for the K step -- so every lane of a quad reads the same
-// 16-byte group of four words (one transaction, broadcast) and decodes its
-// own nibbles.  A CTA is 8 warps: 2 row tiles x 4 K quarters (interleaved
-// 64-code chunks), reduced through shared memory.
+// The packed weight stream (K_in / 4 bytes per output) dominates the
+// traffic, so the kernel is organised to keep HBM busy and to spend as few
+// issue slots as possible per weight:
+//
+// * Persistent CTAs, at most one per SM.  The K_out / 16 row tiles are cut
+//   into bands of n_t consecutive tiles (n_t <= 16, balanced to within one
+//   tile across the grid); a CTA processes `rounds` bands.
+// * One producer warp streams a band through an mbarrier ring with TMA.  A
+//   stage holds 512 input positions: a [16 n_t rows x 32 words] box of
+//   packed codes with the 128-byte swizzle, and the matching inputs of all
+//   B batch rows laid out [64 chunks][B][8 bf16], so the eight batch rows
+//   of one 8-wide chunk are one contiguous 128-byte ldmatrix read.
+// * Sixteen consumer warps: P = 16 / n_t warps per tile split the tile's
+//   stages (stage ks goes to warp ks % P of the tile) and their partial sums
+//   are added in a fixed order.  Per K step of 16 a warp runs
+//   one mma.m16n8k16: A = 16 rows x 16 codes decoded in registers to bf16
+//   W~/2, B = 16 inputs x 8 batch columns (rows past B read a zero chunk),
+//   fp32 accumulation.  Lane (g, t) of the A fragment holds pairs t and
+//   t + 4 of the K step's word of rows g and g + 8; with the byte-planar
+//   packing a pair is one mask and one multiply-add.  2 alpha is applied
+//   in the epilogue (W~/2 is exact in bf16).
+//
+// Every mbarrier wait is bounded; on expiry the kernel records a timeout in
+// the device error word, stops issuing, drains the copies it started and
+// returns.
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <cstdint>
+#include <mutex>
+#include <utility>
 
 #include "tbn_device.cuh"
 #include "tbn_internal.h"
@@ -21,99 +40,351 @@
 namespace tbn {
 namespace {
 
-constexpr int kRowTiles = 2;   // 16-row tiles per CTA
-constexpr int kKSplit = 4;     // warps along K per row tile
-constexpr int kThreads = 32 * kRowTiles * kKSplit;
+constexpr int kConsumerWarps = 16;
+constexpr int kThreads = 32 * (kConsumerWarps + 1);
+constexpr int kProducerWarp = kConsumerWarps;
+constexpr int kCodesPerStage = 512;           // 32 packed words per row
+constexpr int kWordsPerStage = kCodesPerStage / 16;
+constexpr int kMaxTilesPerBand = 16;          // TMA box height 256 rows
+constexpr int kMaxStages = 16;
+constexpr int kSmemBudget = 200 * 1024;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4],
-                                               uint32_t b0, uint32_t b1) {
-  asm volatile(
+struct GemvArgs {
+  const float* alpha;
+  void* y;
+  const void* residual;
+  uint32_t* err;
+  int K_out, K_in, B;
+  int T;           // row tiles = ceil(K_out / 16)
+  int n_t;         // tiles per band
+  int rounds;      // bands per CTA
+  int nks;         // stages per band = ceil(K_in / 512)
+  int P;           // consumer warps per tile (K split), n_t * P <= 16
+  int stages;      // ring depth
+  uint32_t w_bytes;      // packed-code bytes per stage = n_t * 2048
+  uint32_t stage_bytes;  // w_bytes + B * 1024
+  int y_bf16, relu;
+};
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
+                                               uint32_t a2, uint32_t a3, uint32_t b0,
+                                               uint32_t b1) {
+  // no side effects beyond its registers: the compiler may schedule it freely
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
       "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// ldmatrix.x4 at addr + kOff (kOff folded into the instruction).
+template <int kOff>
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4+%5];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr), "n"(kOff)
+               : "memory");
+}
+
+template <int kOff>
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4+%5];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr), "n"(kOff)
+               : "memory");
+  return v;
+}
+
+// Per-lane decode constants for pairs t and t + 4 (t = lane % 4): the
+// pair's bits (at p, 8+p, 16+p, 24+p) are masked and moved to 7, 15, 23,
+// 31 by a power-of-two multiply; adding 0x3F003F00 sets the remaining bf16
+// bits of +-0.5 / +-1 (no carries: the bit sets are disjoint).
+struct PairDecode {
+  uint32_t mask_lo, mul_lo, mask_hi, mul_hi;
+  __device__ __forceinline__ explicit PairDecode(int t)
+      : mask_lo(0x01010101u << t), mask_hi(0x10101010u << t) {
+    // The multipliers pass through an opaque move so the compiler keeps the
+    // multiply-add (FMA pipe) instead of rewriting it as shift + OR on the
+    // integer ALU pipe, which the masks already load.
+    asm("mov.b32 %0, %1;" : "=r"(mul_lo) : "r"(1u << (7 - t)));
+    asm("mov.b32 %0, %1;" : "=r"(mul_hi) : "r"(1u << (3 - t)));
+  }
+  __device__ __forceinline__ uint32_t lo(uint32_t w) const {
+    return (w & mask_lo) * mul_lo + 0x3F003F00u;
+  }
+  __device__ __forceinline__ uint32_t hi(uint32_t w) const {
+    return (w & mask_hi) * mul_hi + 0x3F003F00u;
+  }
+};
+
+// One stage of one 16-row tile: 32 K steps of 16, accumulated into two
+// independent chains (K step i goes to chain i % 2) so consecutive mma
+// instructions do not wait on each other.
+//   w_lane: shared address of the tile's row g with this lane's swizzle
+//   phase folded in, (row address) | (g << 4).  Rows are 128-byte swizzled
+//   (chunk j of row r stored at j ^ (r & 7)), so chunk j of row g is at
+//   w_lane ^ (j << 4) and row g + 8 is 1024 bytes further.
+//   x_lane: this lane's ldmatrix row address for chunk 0: matrix m =
+//   lane / 8 (chunk offset), batch row n = lane % 8.  Lanes with n >= B
+//   read row n % B; that only fills mma columns n >= B, which are dropped.
+// Operands of one 4-K-step chunk: words 4J .. 4J + 3 of rows g and g + 8
+// and the x fragments of chunks 8J .. 8J + 7.
+struct ChunkRegs {
+  uint4 wa, wb;
+  uint32_t b0[4], b1[4];
+};
+
+template <int kB, int J>
+__device__ __forceinline__ void load_chunk(ChunkRegs& r, uint32_t w_lane, uint32_t x_lane) {
+  const uint32_t aw = w_lane ^ static_cast<uint32_t>(J << 4);
+  r.wa = lds128<0>(aw);
+  r.wb = lds128<1024>(aw);
+  ldmatrix_x4<(8 * J) * kB * 16>(r.b0, x_lane);
+  ldmatrix_x4<(8 * J + 4) * kB * 16>(r.b1, x_lane);
+}
+
+__device__ __forceinline__ void mma_chunk(float (&d)[2][4], const ChunkRegs& r,
+                                          const PairDecode& dec) {
+  const uint4& wa = r.wa;
+  const uint4& wb = r.wb;
+  mma_bf16_16816(d[0], dec.lo(wa.x), dec.lo(wb.x), dec.hi(wa.x), dec.hi(wb.x), r.b0[0], r.b0[1]);
+  mma_bf16_16816(d[1], dec.lo(wa.y), dec.lo(wb.y), dec.hi(wa.y), dec.hi(wb.y), r.b0[2], r.b0[3]);
+  mma_bf16_16816(d[0], dec.lo(wa.z), dec.lo(wb.z), dec.hi(wa.z), dec.hi(wb.z), r.b1[0], r.b1[1]);
+  mma_bf16_16816(d[1], dec.lo(wa.w), dec.lo(wb.w), dec.hi(wa.w), dec.hi(wb.w), r.b1[2], r.b1[3]);
+}
+
+// Chunk J: issue the loads of chunk J + 1, then the four mma of chunk J
+// (the shared-memory loads keep program order, so this is the prefetch).
+template <int kB, int J>
+__device__ __forceinline__ void tile_chunk(float (&d)[2][4], uint32_t w_lane, uint32_t x_lane,
+                                           const PairDecode& dec, ChunkRegs& cur) {
+  if constexpr (J + 1 < 8) {
+    ChunkRegs nxt;
+    load_chunk<kB, J + 1>(nxt, w_lane, x_lane);
+    mma_chunk(d, cur, dec);
+    cur = nxt;
+  } else {
+    mma_chunk(d, cur, dec);
+  }
+}
+
+template <int kB, int... J>
+__device__ __forceinline__ void tile_stage_chunks(float (&d)[2][4], uint32_t w_lane,
+                                                  uint32_t x_lane, const PairDecode& dec,
+                                                  std::integer_sequence<int, J...>) {
+  ChunkRegs cur;
+  load_chunk<kB, 0>(cur, w_lane, x_lane);
+  (tile_chunk<kB, J>(d, w_lane, x_lane, dec, cur), ...);
 }
 
 template <int kB>
-__global__ void __launch_bounds__(kThreads) gemv_kernel(const __nv_bfloat16* __restrict__ x,
-                                                        int K_in, const uint32_t* __restrict__ codes,
-                                                        const float* __restrict__ alpha, int K_out,
-                                                        void* __restrict__ y, int y_bf16, int relu,
-                                                        const void* __restrict__ residual) {
-  __shared__ float s_part[kRowTiles][kKSplit][32][4];
+__device__ __forceinline__ void tile_stage(float (&d)[2][4], uint32_t w_lane, uint32_t x_lane,
+                                           const PairDecode& dec) {
+  tile_stage_chunks<kB>(d, w_lane, x_lane, dec, std::make_integer_sequence<int, 8>{});
+}
+
+template <int kB>
+__device__ __forceinline__ void store_out(const GemvArgs& a, int row, int n, float acc) {
+  if (row >= a.K_out || n >= kB) return;
+  float v = 2.0f * a.alpha[row] * acc;
+  const size_t o = static_cast<size_t>(n) * a.K_out + row;
+  if (a.y_bf16) {
+    if (a.residual) v += __bfloat162float(static_cast<const __nv_bfloat16*>(a.residual)[o]);
+    if (a.relu) v = fmaxf(v, 0.0f);
+    static_cast<__nv_bfloat16*>(a.y)[o] = __float2bfloat16_rn(v);
+  } else {
+    if (a.residual) v += static_cast<const float*>(a.residual)[o];
+    if (a.relu) v = fmaxf(v, 0.0f);
+    static_cast<float*>(a.y)[o] = v;
+  }
+}
+
+template <int kB>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemv_tma_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                    const __grid_constant__ CUtensorMap tmap_x, const GemvArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t full_bar[kMaxStages], empty_bar[kMaxStages];
+  __shared__ float partial[kConsumerWarps][32][4];
+  __shared__ volatile int abort_flag;
+
+  // stage s at ring + s * stage_bytes; 1024-byte aligned for the swizzle
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t ring = (raw + 1023u) & ~1023u;
+  uint8_t* ring_ptr = smem_raw + (ring - raw);
+
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rt = warp / kKSplit, ks = warp % kKSplit;
-  const int g = lane >> 2, t = lane & 3;
-  const int row0 = (blockIdx.x * kRowTiles + rt) * 16;
-  const int wpf = K_in / 16;
-  const int rA = row0 + g, rB = row0 + g + 8;
-  const uint4* wa = reinterpret_cast<const uint4*>(codes + static_cast<size_t>(rA < K_out ? rA : 0) * wpf);
-  const uint4* wb = reinterpret_cast<const uint4*>(codes + static_cast<size_t>(rB < K_out ? rB : 0) * wpf);
-  const bool va = rA < K_out, vb = rB < K_out;
-  // batch column n = g of the B fragment
-  const bool xb = g < kB;
-  const uint32_t* xrow = reinterpret_cast<const uint32_t*>(x + static_cast<size_t>(xb ? g : 0) * K_in);
-
-  float d[4] = {0.f, 0.f, 0.f, 0.f};
-  const int nchunks = K_in / 64;  // 64 codes = 4 words = one uint4 per row
-  for (int c = ks; c < nchunks; c += kKSplit) {
-    const uint4 A4 = va ? __ldg(wa + c) : make_uint4(0u, 0u, 0u, 0u);
-    const uint4 B4 = vb ? __ldg(wb + c) : make_uint4(0u, 0u, 0u, 0u);
-    const uint32_t wA[4] = {A4.x, A4.y, A4.z, A4.w};
-    const uint32_t wB[4] = {B4.x, B4.y, B4.z, B4.w};
-#pragma unroll
-    for (int s = 0; s < 4; ++s) {
-      const int k0 = c * 64 + s * 16;
-      uint32_t a[4];
-      a[0] = nibble_to_bf16x2((wA[s] >> (4 * t)) & 0xFu);        // row g,   k 2t..2t+1
-      a[1] = nibble_to_bf16x2((wB[s] >> (4 * t)) & 0xFu);        // row g+8, k 2t..2t+1
-      a[2] = nibble_to_bf16x2((wA[s] >> (4 * t + 16)) & 0xFu);   // row g,   k 2t+8..
-      a[3] = nibble_to_bf16x2((wB[s] >> (4 * t + 16)) & 0xFu);   // row g+8, k 2t+8..
-      const uint32_t b0 = xb ? __ldg(xrow + (k0 >> 1) + t) : 0u;
-      const uint32_t b1 = xb ? __ldg(xrow + (k0 >> 1) + t + 4) : 0u;
-      mma_bf16_16816(d, a, b0, b1);
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < a.stages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], static_cast<uint32_t>(a.n_t));   // one warp per tile per stage
     }
+    fence_mbar_init();
   }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) s_part[rt][ks][lane][i] = d[i];
   __syncthreads();
-  if (ks != 0) return;
-  float sum[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    sum[i] = s_part[rt][0][lane][i];
-#pragma unroll
-    for (int w = 1; w < kKSplit; ++w) sum[i] += s_part[rt][w][lane][i];
+
+  if (warp == kProducerWarp) {
+    // ---------------------------------------------------------- producer
+    const bool elected = elect_one();
+    if (elected) {
+      prefetch_tmap(&tmap_w);
+      prefetch_tmap(&tmap_x);
+    }
+    // CTAs start their sweep over K at evenly spread offsets, so at any
+    // moment the grid reads many different column ranges of the (row-pitch
+    // strided) code matrix instead of one.  Consumers do not depend on the
+    // order: a stage's data position only enters through these coordinates.
+    const int k_start = static_cast<int>((static_cast<int64_t>(blockIdx.x) * a.nks) / gridDim.x);
+    int it = 0;                      // stages issued so far
+    int slot = 0;                    // it % stages
+    uint32_t empty_parity = 1;       // parity of the release before use it / stages
+    for (int r = 0; r < a.rounds; ++r) {
+      const int band = blockIdx.x + r * gridDim.x;
+      if (band * a.n_t >= a.T) break;
+      int kc = k_start;
+      for (int ks = 0; ks < a.nks; ++ks) {
+        bool ok = true;
+        if (it >= a.stages)
+          ok = mbar_wait_sleep(&empty_bar[slot], empty_parity, &abort_flag, a.err, kWaitLimitNs);
+        // one decision for the whole warp (lane 0's)
+        if (!__shfl_sync(0xffffffffu, ok && !abort_flag, 0)) break;
+        if (elected) {
+          uint8_t* st = ring_ptr + static_cast<size_t>(slot) * a.stage_bytes;
+          mbar_arrive_expect_tx(&full_bar[slot], a.stage_bytes);
+          tma_load_2d(st, &tmap_w, &full_bar[slot], kc * kWordsPerStage, band * a.n_t * 16);
+          if (kB == 1) {
+            // one batch row: the stage's inputs are 1 KB contiguous
+            tma_load_2d(st + a.w_bytes, &tmap_x, &full_bar[slot], kc * kCodesPerStage, 0);
+            tma_load_2d(st + a.w_bytes + 512, &tmap_x, &full_bar[slot],
+                        kc * kCodesPerStage + 256, 0);
+          } else {
+            tma_load_3d(st + a.w_bytes, &tmap_x, &full_bar[slot], 0, 0,
+                        kc * (kCodesPerStage / 8));
+          }
+        }
+        __syncwarp();
+        ++it;
+        if (++kc == a.nks) kc = 0;
+        if (++slot == a.stages) {
+          slot = 0;
+          empty_parity ^= 1u;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, abort_flag, 0)) break;
+    }
+    // On abort, wait (bounded) for the last copy issued into each slot so
+    // no TMA write lands after the CTA has exited.
+    if (elected && abort_flag) {
+      for (int s = 0; s < a.stages && s < it; ++s) {
+        const int last_use = (it - 1 - s) / a.stages;
+        mbar_wait(&full_bar[s], static_cast<uint32_t>(last_use & 1), nullptr, a.err,
+                  kWaitLimitNs);
+      }
+    }
+    return;
   }
-  // d[0]: (row g, batch 2t)  d[1]: (row g, batch 2t+1)  d[2], d[3]: row g+8
+
+  // ------------------------------------------------------------ consumers
+  const int g = lane >> 2, t = lane & 3;
+  const PairDecode dec(t);
+  // warp w works on tile w / P of the band, stages ks with ks % P == w % P
+  const int P = a.P;
+  const int tau = warp / P, pi = warp % P;
+  const bool active = tau < a.n_t;
+  // per-lane shared-memory offsets inside a stage
+  const uint32_t w_lane_off = static_cast<uint32_t>((tau * 16 + g) * 128 + (g << 4));
+  const uint32_t x_lane_off =
+      static_cast<uint32_t>(((lane >> 3) * kB + (lane & 7) % kB) * 16);
+
+  int it_slot = 0;            // ring slot of the band's first stage
+  uint32_t it_parity = 0;     // full-barrier parity of that stage
+  for (int r = 0; r < a.rounds; ++r) {
+    const int band = blockIdx.x + r * gridDim.x;
+    if (band * a.n_t >= a.T) break;
+    float c[2][4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int row = (i < 2) ? rA : rB;
-    const int b = 2 * t + (i & 1);
-    if (row >= K_out || b >= kB) continue;
-    float v = 2.0f * alpha[row] * sum[i];
-    const size_t o = static_cast<size_t>(b) * K_out + row;
-    if (y_bf16) {
-      if (residual) v += __bfloat162float(static_cast<const __nv_bfloat16*>(residual)[o]);
-      if (relu) v = fmaxf(v, 0.0f);
-      static_cast<__nv_bfloat16*>(y)[o] = __float2bfloat16_rn(v);
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[q][i] = 0.0f;
+    // this warp takes stages pi, pi + P, ...; slot / parity of stage `it`
+    // advance incrementally (P may exceed the ring depth)
+    int slot = it_slot, ks = pi;
+    uint32_t parity = it_parity;
+    for (int q = 0; q < pi; ++q)
+      if (++slot == a.stages) { slot = 0; parity ^= 1u; }
+    for (; active && ks < a.nks; ks += P) {
+      const bool ok_lane = mbar_wait_sleep(&full_bar[slot], parity, &abort_flag, a.err,
+                                           kWaitLimitNs);
+      // ldmatrix / mma need the whole warp: follow lane 0's outcome
+      if (__shfl_sync(0xffffffffu, ok_lane, 0)) {
+        const uint32_t st = ring + static_cast<uint32_t>(slot) * a.stage_bytes;
+        tile_stage<kB>(c, st + w_lane_off, st + a.w_bytes + x_lane_off, dec);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty_bar[slot]);
+      for (int q = 0; q < P; ++q)
+        if (++slot == a.stages) { slot = 0; parity ^= 1u; }
+    }
+    // the band consumed nks stages of the ring
+    for (int q = 0; q < a.nks; ++q)
+      if (++it_slot == a.stages) { it_slot = 0; it_parity ^= 1u; }
+    float d[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) d[i] = c[0][i] + c[1][i];
+    const int ra = band * a.n_t * 16 + tau * 16 + g;
+    if (P == 1) {
+      if (active && !abort_flag) {
+        store_out<kB>(a, ra, 2 * t, d[0]);
+        store_out<kB>(a, ra, 2 * t + 1, d[1]);
+        store_out<kB>(a, ra + 8, 2 * t, d[2]);
+        store_out<kB>(a, ra + 8, 2 * t + 1, d[3]);
+      }
     } else {
-      if (residual) v += static_cast<const float*>(residual)[o];
-      if (relu) v = fmaxf(v, 0.0f);
-      static_cast<float*>(y)[o] = v;
+      // fixed-order sum of the P partial tiles
+#pragma unroll
+      for (int i = 0; i < 4; ++i) partial[warp][lane][i] = d[i];
+      named_barrier_sync(1, 32 * kConsumerWarps);
+      if (active && pi == 0 && !abort_flag) {
+        float sum[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          sum[i] = partial[warp][lane][i];
+          for (int q = 1; q < P; ++q) sum[i] += partial[warp + q][lane][i];
+        }
+        store_out<kB>(a, ra, 2 * t, sum[0]);
+        store_out<kB>(a, ra, 2 * t + 1, sum[1]);
+        store_out<kB>(a, ra + 8, 2 * t, sum[2]);
+        store_out<kB>(a, ra + 8, 2 * t + 1, sum[3]);
+      }
+      named_barrier_sync(1, 32 * kConsumerWarps);
     }
   }
 }
 
-template <int kB>
-tbn_status launch_b(const void* x, int64_t K_in, const uint32_t* codes, const float* alpha,
-                    int64_t K_out, void* y, tbn_dtype ydt, int relu, const void* residual,
-                    cudaStream_t s) {
-  const int64_t blocks = (K_out + 16 * kRowTiles - 1) / (16 * kRowTiles);
-  gemv_kernel<kB><<<(unsigned)blocks, kThreads, 0, s>>>(
-      static_cast<const __nv_bfloat16*>(x), (int)K_in, codes, alpha, (int)K_out, y,
-      ydt == TBN_BF16 ? 1 : 0, relu, residual);
-  return check_launch("gemv_kernel");
+struct GemvPlan {
+  int T, n_t, rounds, grid, nks, P, stages;
+  uint32_t w_bytes, stage_bytes;
+  size_t smem;
+};
+
+GemvPlan plan_gemv(int64_t B, int64_t K_in, int64_t K_out, int sms) {
+  GemvPlan p{};
+  p.T = static_cast<int>((K_out + 15) / 16);
+  p.rounds = (p.T + kMaxTilesPerBand * sms - 1) / (kMaxTilesPerBand * sms);
+  p.n_t = (p.T + sms * p.rounds - 1) / (sms * p.rounds);
+  p.grid = (p.T + p.n_t * p.rounds - 1) / (p.n_t * p.rounds);
+  p.nks = static_cast<int>((K_in + kCodesPerStage - 1) / kCodesPerStage);
+  p.P = kConsumerWarps / p.n_t;   // n_t <= 16
+  if (p.P > p.nks) p.P = p.nks;
+  p.w_bytes = static_cast<uint32_t>(p.n_t) * 16u * 128u;
+  p.stage_bytes = p.w_bytes + static_cast<uint32_t>(B) * 1024u;
+  p.stages = static_cast<int>(kSmemBudget / p.stage_bytes);
+  if (p.stages > kMaxStages) p.stages = kMaxStages;
+  p.smem = static_cast<size_t>(p.stages) * p.stage_bytes + 1024;
+  return p;
 }
 
 }  // namespace
@@ -125,22 +396,100 @@ const char* gemv_unsupported_reason(const void* x, tbn_dtype xdt, int64_t B, int
   if (K_in % 64 != 0) return "GEMV needs K_in % 64 == 0";
   if (K_in >= (1ll << 30)) return "GEMV: K_in too large";
   if (!is_aligned(x, 16) || !is_aligned(codes, 16)) return "GEMV needs 16-byte aligned x and codes";
+  if (get_encode_tiled() == nullptr) return "cuTensorMapEncodeTiled unavailable";
   return "";
 }
 
 tbn_status launch_gemv(const void* x, int64_t B, int64_t K_in, const uint32_t* codes,
                        const float* alpha, int64_t K_out, void* y, tbn_dtype ydt, int relu,
                        const void* residual, cudaStream_t s) {
-  switch (B) {
-    case 1: return launch_b<1>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 2: return launch_b<2>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 3: return launch_b<3>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 4: return launch_b<4>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 5: return launch_b<5>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 6: return launch_b<6>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    case 7: return launch_b<7>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
-    default: return launch_b<8>(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, s);
+  if (K_out >= (1ll << 31) - 16) return fail(TBN_ERR_INVALID_ARG, "GEMV: K_out too large");
+  const GemvPlan p = plan_gemv(B, K_in, K_out, device_sm_count());
+  if (p.stages < 2) return fail(TBN_ERR_UNSUPPORTED, "GEMV: stage does not fit shared memory");
+
+  alignas(64) CUtensorMap tmap_w, tmap_x;
+  {
+    const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(K_in / 16), static_cast<cuuint64_t>(K_out)};
+    const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(K_in / 4)};
+    const cuuint32_t box[2] = {kWordsPerStage, static_cast<cuuint32_t>(p.n_t * 16)};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult cr = get_encode_tiled()(
+        &tmap_w, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint32_t*>(codes), gdim, gstride,
+        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS)
+      return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(codes) failed (%d)", (int)cr);
   }
+  if (B == 1) {
+    const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(K_in), 1};
+    const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(K_in * 2)};
+    const cuuint32_t box[2] = {256, 1};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult cr = get_encode_tiled()(
+        &tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), gdim, gstride, box,
+        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS)
+      return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed (%d)", (int)cr);
+  } else {
+    // x [B][K_in] viewed as (8 elements, B rows, K_in / 8 chunks) so a box
+    // lands in shared memory as [chunk][batch row][8 elements]
+    const cuuint64_t gdim[3] = {8, static_cast<cuuint64_t>(B), static_cast<cuuint64_t>(K_in / 8)};
+    const cuuint64_t gstride[2] = {static_cast<cuuint64_t>(K_in * 2), 16};
+    const cuuint32_t box[3] = {8, static_cast<cuuint32_t>(B), kCodesPerStage / 8};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult cr = get_encode_tiled()(
+        &tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(x), gdim, gstride, box,
+        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (cr != CUDA_SUCCESS)
+      return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed (%d)", (int)cr);
+  }
+
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    const void* fns[8] = {(const void*)gemv_tma_kernel<1>, (const void*)gemv_tma_kernel<2>,
+                          (const void*)gemv_tma_kernel<3>, (const void*)gemv_tma_kernel<4>,
+                          (const void*)gemv_tma_kernel<5>, (const void*)gemv_tma_kernel<6>,
+                          (const void*)gemv_tma_kernel<7>, (const void*)gemv_tma_kernel<8>};
+    for (const void* f : fns) {
+      const cudaError_t e =
+          cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget + 1024);
+      if (e != cudaSuccess && attr_err == cudaSuccess) attr_err = e;
+    }
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(gemv)");
+
+  GemvArgs a{};
+  a.alpha = alpha;
+  a.y = y;
+  a.residual = residual;
+  a.err = device_error_word();
+  a.K_out = static_cast<int>(K_out);
+  a.K_in = static_cast<int>(K_in);
+  a.B = static_cast<int>(B);
+  a.T = p.T;
+  a.n_t = p.n_t;
+  a.rounds = p.rounds;
+  a.nks = p.nks;
+  a.P = p.P;
+  a.stages = p.stages;
+  a.w_bytes = p.w_bytes;
+  a.stage_bytes = p.stage_bytes;
+  a.y_bf16 = ydt == TBN_BF16 ? 1 : 0;
+  a.relu = relu;
+  switch (B) {
+    case 1: gemv_tma_kernel<1><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 2: gemv_tma_kernel<2><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 3: gemv_tma_kernel<3><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 4: gemv_tma_kernel<4><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 5: gemv_tma_kernel<5><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 6: gemv_tma_kernel<6><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 7: gemv_tma_kernel<7><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    default: gemv_tma_kernel<8><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+  }
+  return check_launch("gemv_tma_kernel");
 }
 
 }  // namespace tbn

@@ -132,7 +132,7 @@ __device__ __forceinline__ void encode16(const float (&v)[16], int nvalid, uint3
     const uint32_t m = a > 1.0f ? 1u : 0u;
     const uint32_t s = v[e] <= 0.0f ? 1u : 0u;
     const bool valid = e < nvalid;
-    w |= valid ? ((m | (s << 1)) << (2 * e)) : 0u;
+    w |= valid ? ((m << code_mag_bit(e)) | (s << (code_mag_bit(e) + 8))) : 0u;
     n2 += (valid && m) ? 1 : 0;
     c[e] = valid ? (m ? 2.0f * a : a) : 0.0f;
   }
@@ -322,7 +322,7 @@ __global__ void __launch_bounds__(256) unpack_kernel(const uint32_t* __restrict_
     const int64_t left = n - 16 * j;
     const int cnt = left < 16 ? static_cast<int>(left) : 16;
     for (int e = 0; e < cnt; ++e) {
-      const float v = code_value((w >> (2 * e)) & 3u);
+      const float v = code_value(code_field(w, e));
       if (kFmt == TBN_UNPACK_I8) {
         static_cast<int8_t*>(out)[base + e] = static_cast<int8_t>(v);
       } else if (kFmt == TBN_UNPACK_F32) {

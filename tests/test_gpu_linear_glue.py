@@ -35,6 +35,24 @@ def test_gemv_matches_oracle(B, K_in, K_out):
     assert_within(y, y_orc, bound, out_bf16=True, what="gemv bf16")
 
 
+@pytest.mark.parametrize("B,K_in,K_out", [
+    (7, 64, 16),        # one stage, one tile
+    (4, 3072, 33),      # one tile per band: six warps split K, fixed-order sum
+    (5, 4160, 20000),   # nine tiles per band, ragged last stage
+    (3, 1024, 38912),   # sixteen tiles per band
+    (2, 576, 40000),    # two bands per CTA
+    (1, 8192, 1000),    # K split over sixteen warps
+    (8, 2048, 8192),    # four tiles per band, four warps per tile
+])
+def test_gemv_launch_shapes(B, K_in, K_out):
+    """Shapes that exercise every branch of the GEMV work split."""
+    g = inputs.generator(B * 7 + K_in * 3 + K_out)
+    W = inputs.normal((K_out, K_in), 1.1, g)
+    x = torch.randn(B, K_in, generator=g).to(torch.bfloat16)
+    y, y_orc, bound = run_linear(W, x, torch.float32)
+    assert_within(y, y_orc, bound, out_bf16=False, what="gemv shapes")
+
+
 @pytest.mark.parametrize("K", inputs.GEMV_SIZES)
 @pytest.mark.parametrize("B", inputs.GEMV_BATCHES)
 def test_gemv_workload_full(K, B):

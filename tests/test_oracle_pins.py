@@ -174,22 +174,39 @@ def pin_exact_special_case(orc):
     assert _bruteforce_min(W)[0] == 0
 
 
+def _planar_bits(i, field):
+    """Bit mask of code i's field in its word, written out per bit position:
+    magnitude at 16 (l % 2) + l // 2, sign 8 above it, l = i % 16."""
+    l = i % 16
+    mb = 16 * (l % 2) + l // 2
+    return ((field & 1) << mb) | ((field >> 1) << (mb + 8))
+
+
 def pin_pack_bit_layout(orc):
-    # codes 1, 2, -1, -2 -> fields 0, 1, 2, 3 at bits 0-1, 2-3, 4-5, 6-7
+    # codes 1, 2, -1, -2 (fields 0, 1, 2, 3): code 1 = pair 0 odd half ->
+    # magnitude at bit 16; code 2 = pair 1 even half -> sign at bit 9;
+    # code 3 = pair 1 odd half -> magnitude at bit 17 and sign at bit 25
     words = orc.pack(np.array([[1, 2, -1, -2]], dtype=np.int8))
-    assert int(words[0, 0]) == 0 + (1 << 2) + (2 << 4) + (3 << 6)
-    # code 15 lands in the top field, code 16 starts the next word
+    assert int(words[0, 0]) == (1 << 16) | (1 << 9) | (1 << 17) | (1 << 25)
+    # code 15 is the odd half of pair 7 (bits 23 and 31); code 16 starts the next word
     c = np.ones((1, 17), dtype=np.int8)
     c[0, 15] = -2
     c[0, 16] = 2
     words = orc.pack(c)
     assert words.shape == (1, 2)
-    assert int(words[0, 0]) == 3 << 30 and int(words[0, 1]) == 1
-    # every filter starts on a fresh word
+    assert int(words[0, 0]) == (1 << 23) | (1 << 31) and int(words[0, 1]) == 1
+    # every filter starts on a fresh word; all -2 fills bytes 0,1 (pairs 0..2)
+    # and bytes 2,3 (pairs 0..2) for six codes
     c2 = np.array([[1] * 5 + [-1], [-2] * 6], dtype=np.int8)
     w2 = orc.pack(c2)
     assert w2.shape == (2, 1)
-    assert int(w2[0, 0]) == 2 << 10 and int(w2[1, 0]) == 0xFFF
+    assert int(w2[0, 0]) == 1 << 26 and int(w2[1, 0]) == 0x07070707
+    # each single code in each position, against the per-bit formula
+    for i in range(16):
+        for v, f in ((1, 0), (2, 1), (-1, 2), (-2, 3)):
+            c = np.ones((1, 16), dtype=np.int8)
+            c[0, i] = v
+            assert int(orc.pack(c)[0, 0]) == _planar_bits(i, f), (i, v)
 
 
 def pin_pack_roundtrip(orc):
@@ -202,11 +219,14 @@ def pin_pack_roundtrip(orc):
         assert np.array_equal(orc.unpack(words, n), codes)
         rnd = rng.integers(0, 2**32, size=words.shape, dtype=np.uint64).astype(np.uint32)
         if n % 16:
-            rnd[:, -1] &= np.uint32((1 << (2 * (n % 16))) - 1)
+            keep = 0
+            for i in range(n % 16):
+                keep |= _planar_bits(i, 3)
+            rnd[:, -1] &= np.uint32(keep)
         assert np.array_equal(orc.pack(orc.unpack(rnd, n)), rnd)
         if n % 16:
             bad = rnd.copy()
-            bad[0, -1] |= np.uint32(1 << 31)
+            bad[0, -1] |= np.uint32(_planar_bits(15, 2))
             with pytest.raises(ValueError):
                 orc.unpack(bad, n)
 
@@ -391,8 +411,10 @@ MUTANTS = [
      "(double)size_b1 + 2.0 * (double)size_b2"),
     ("sign/magnitude bits swapped", "case 2:  *field = 1u; return 0;\n    case -1: *field = 2u;",
      "case 2:  *field = 2u; return 0;\n    case -1: *field = 1u;"),
-    ("codes packed from the top of the word", "words[k * wpf + i / 16] |= f << (2 * (i % 16));",
-     "words[k * wpf + i / 16] |= f << (30 - 2 * (i % 16));"),
+    ("codes 0-7 in the low half-word instead of even/odd halves",
+     "return (int)(16 * (l % 2) + l / 2);", "return (int)(16 * (l / 8) + l % 8);"),
+    ("sign bit next to the magnitude bit", "return magnitude_bit(i) + 8;",
+     "return magnitude_bit(i) + 1;"),
     ("padding ignored in the row index", "int64_t h = p * sh - ph + r;", "int64_t h = p * sh + r;"),
     ("convolution instead of cross-correlation",
      "double wv = (double)wt[((k * C + c) * R + r) * S + s];",
