@@ -58,6 +58,23 @@ METRIC = "TBN conv TFLOP/s (VGG-small b128 forward incl. per-step re-quantizatio
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FLUSH_BYTES = 512 * 1024 * 1024
 
+# DRAM bytes (read + write) per convolution launch, mean over the six launches of
+# one step, from the ncu capture summarised in profiles/vgg_small_b128_launches.md.
+# Valid only for the kernel sources it was measured on (hash below); otherwise the
+# roofline entry reports null.
+CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
+                            "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
+                "sha256_16": "fc952fb0541013c3", "bytes_per_launch": 12.26e6}
+
+
+def measured_traffic(rec):
+    import hashlib
+    h = hashlib.sha256()
+    for f in rec["sources"]:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return rec["bytes_per_launch"] if h.hexdigest()[:16] == rec["sha256_16"] else None
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -256,7 +273,8 @@ def run_vgg(args, rank, world, local_rank):
     achieved = (tc_flops / max(1, len(tc_layers))) / (tc_launch_ms * 1e-3) / 1e12
     peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
     roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
-                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": None,
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+                "traffic": measured_traffic(CONV_TRAFFIC),
                 "kernel": "conv_igemm_kernel (tcgen05 implicit GEMM), %d launches per step "
                           "(layers %s)" % (len(tc_layers),
                                            ",".join("c%d" % (i + 1) for i in tc_layers)),

@@ -45,8 +45,7 @@
  *   OR, which is what the kernels do;
  * - unused codes of a filter's last word have m = s = 0;
  * - codes[K][ceil(n/16)] plus alpha[K] (fp32) is the complete inference
- *   form of a layer (at inference only the two-bit filters and their
- *   scaling factors are needed, Section 3).
+ *   form of a layer: inference reads nothing else of the layer (Section 3).
  * - The order of the n weights of a filter is the caller's choice; the
  *   convolution reads them in the activation layout's natural order:
  *   NCHW -> (c, r, s), NHWC -> (r, s, c).  Discretization is elementwise and
