@@ -217,10 +217,14 @@ def run_vgg(args, rank, world, local_rank):
     graph, ev_step = capture(lambda: net.forward(requantize=True))
     # instrumented step: events around every tensor-core convolution
     ev_conv = {i: [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-               for i in tc_layers}
+               for i in range(len(net.layers))}
+
+    ev_quant = torch.cuda.Event(enable_timing=True, external=True)
 
     def hook(i, layer, when):
-        if i in ev_conv:
+        if i < 0:
+            ev_quant.record()
+        elif i in ev_conv:
             ev_conv[i][0 if when == "before" else 1].record()
 
     graph_i, ev_i = capture(lambda: net.forward(requantize=True, conv_hook=hook))
@@ -248,12 +252,18 @@ def run_vgg(args, rank, world, local_rank):
     barrier(world)
     # roofline region: the instrumented graph, same number of steps
     conv_ms = []
+    layer_ms = np.zeros(len(net.layers))
+    quant_ms = 0.0
+    prefix_ms = 0.0
     for _ in range(args.steps):
         with torch.cuda.stream(stream):
             flush.zero_()
             graph_i.replay()
         stream.synchronize()
         conv_ms.append(sum(ev_conv[i][0].elapsed_time(ev_conv[i][1]) for i in tc_layers))
+        layer_ms += [ev_conv[i][0].elapsed_time(ev_conv[i][1]) for i in range(len(net.layers))]
+        quant_ms += ev_i[0].elapsed_time(ev_quant)
+        prefix_ms += ev_quant.elapsed_time(ev_conv[0][0])
     t1 = time.time()
     clocks = sampler.stop(t0, t1)
 
@@ -289,6 +299,10 @@ def run_vgg(args, rank, world, local_rank):
                    "requantize_per_step": True, "parallelism": "replicas x%d" % world,
                    "l2": "512 MiB flush between timed steps"},
         "images_per_s": round(images_per_s, 1),
+        "breakdown_us": dict([("quantize", round(1e3 * quant_ms / args.steps, 2)),
+                              ("nchw_to_nhwc", round(1e3 * prefix_ms / args.steps, 2))] +
+                             [("c%d" % (i + 1), round(1e3 * layer_ms[i] / args.steps, 2))
+                              for i in range(len(net.layers))]),
         "tbn_conv_gflop_per_step": round(flops * world / 1e9, 3),
         "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": int(x_host.numel() * x_host.element_size()),

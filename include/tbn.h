@@ -86,8 +86,12 @@ typedef enum {
 typedef enum {
   TBN_CONV_AUTO = 0,
   TBN_CONV_DIRECT = 1,        /* CUDA-core direct convolution, any layout/dtype   */
-  TBN_CONV_IMPLICIT_GEMM = 2  /* tcgen05 implicit GEMM, NHWC bf16 x; activations
+  TBN_CONV_IMPLICIT_GEMM = 2, /* tcgen05 implicit GEMM, NHWC bf16 x; activations
                                  by TMA when C % 64 == 0, else gathered by threads */
+  TBN_CONV_SMALL_TAPS = 3     /* tensor-core (mma.sync) convolution for short
+                                 filters, C*R*S <= 64, bf16 x in NCHW or NHWC,
+                                 no fused pool: the input patch and its im2col
+                                 expansion are staged in shared memory        */
 } tbn_conv_algo;
 
 /* Fused layer epilogue (network glue, not part of the paper's method):

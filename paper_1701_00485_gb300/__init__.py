@@ -26,6 +26,7 @@ __all__ = [
     "tbn_conv2d_select_algo", "conv_out_hw",
     "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
+    "TBN_CONV_SMALL_TAPS",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -36,7 +37,7 @@ TBN_OK, TBN_ERR_INVALID_ARG, TBN_ERR_UNSUPPORTED, TBN_ERR_MISALIGNED, TBN_ERR_CU
 TBN_F32, TBN_BF16 = 0, 1
 TBN_NCHW, TBN_NHWC = 0, 1
 TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
-TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM = 0, 1, 2
+TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM, TBN_CONV_SMALL_TAPS = 0, 1, 2, 3
 TBN_MAX_QUANT_JOBS = 16
 
 # every symbol include/tbn.h declares

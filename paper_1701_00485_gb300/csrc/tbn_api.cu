@@ -138,9 +138,23 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
   return TBN_OK;
 }
 
+// AUTO: the implicit GEMM when it can feed activations by TMA, else the
+// small-tap kernel for short filters, else the implicit GEMM with gathered
+// activations, else the CUDA-core direct kernel.
+tbn_conv_algo pick_algo(const ConvProblem& p) {
+  const bool igemm = conv_igemm_unsupported_reason(p)[0] == '\0';
+  if (igemm && conv_igemm_uses_tma(p)) return TBN_CONV_IMPLICIT_GEMM;
+  if (conv_smalltap_unsupported_reason(p)[0] == '\0') return TBN_CONV_SMALL_TAPS;
+  if (igemm) return TBN_CONV_IMPLICIT_GEMM;
+  return TBN_CONV_DIRECT;
+}
+
 tbn_status run_conv(const ConvProblem& p, tbn_conv_algo algo, cudaStream_t s) {
-  if (algo == TBN_CONV_AUTO) {
-    algo = (conv_igemm_unsupported_reason(p)[0] == '\0') ? TBN_CONV_IMPLICIT_GEMM : TBN_CONV_DIRECT;
+  if (algo == TBN_CONV_AUTO) algo = pick_algo(p);
+  if (algo == TBN_CONV_SMALL_TAPS) {
+    const char* why = conv_smalltap_unsupported_reason(p);
+    if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
+    return launch_conv_smalltap(p, s);
   }
   if (algo == TBN_CONV_IMPLICIT_GEMM) {
     const char* why = conv_igemm_unsupported_reason(p);
@@ -260,7 +274,7 @@ tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N
                     K, R, S, stride_h, stride_w, pad_h, pad_w, const_cast<uint32_t*>(dummy), TBN_BF16,
                     nullptr, &p);
   if (st != TBN_OK) return TBN_CONV_DIRECT;
-  return conv_igemm_unsupported_reason(p)[0] == '\0' ? TBN_CONV_IMPLICIT_GEMM : TBN_CONV_DIRECT;
+  return pick_algo(p);
 }
 
 tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,

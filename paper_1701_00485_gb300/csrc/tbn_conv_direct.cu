@@ -246,19 +246,19 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
   }
 }
 
+// One thread per pixel of one image (blockIdx.y): reads the pixel's C
+// values from the C planes (coalesced across the warp's consecutive pixels)
+// and writes its Cp channels contiguously; no index divisions.
 template <typename T>
-__global__ void __launch_bounds__(256) nchw_to_nhwc_kernel(const T* __restrict__ x, int64_t N,
-                                                           int64_t C, int64_t H, int64_t W,
-                                                           int64_t Cp, T* __restrict__ y) {
-  const int64_t total = N * H * W * Cp;
-  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t c = i % Cp;
-    const int64_t w = (i / Cp) % W;
-    const int64_t h = (i / (Cp * W)) % H;
-    const int64_t b = i / (Cp * W * H);
-    y[i] = c < C ? x[((b * C + c) * H + h) * W + w] : from_f32<T>(0.0f);
-  }
+__global__ void __launch_bounds__(256) nchw_to_nhwc_kernel(const T* __restrict__ x, int C, int HW,
+                                                           int Cp, T* __restrict__ y) {
+  const int hw = blockIdx.x * 256 + threadIdx.x;
+  if (hw >= HW) return;
+  const int64_t b = blockIdx.y;
+  const T* src = x + b * C * static_cast<int64_t>(HW) + hw;
+  T* dst = y + (b * HW + hw) * static_cast<int64_t>(Cp);
+  for (int c = 0; c < Cp; ++c)
+    dst[c] = c < C ? src[static_cast<int64_t>(c) * HW] : from_f32<T>(0.0f);
 }
 
 int64_t grid_for(int64_t total) {
@@ -318,13 +318,16 @@ tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H
 
 tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
                                int64_t W, int64_t C_pad, void* y, cudaStream_t s) {
-  const int64_t total = N * H * W * C_pad;
+  if (N > 65535 || H * W >= (int64_t(1) << 31) - 256 || C_pad >= (int64_t(1) << 31))
+    return fail(TBN_ERR_UNSUPPORTED, "nchw_to_nhwc: N > 65535 or H*W too large");
+  const dim3 grid(static_cast<unsigned>((H * W + 255) / 256), static_cast<unsigned>(N));
   if (dt == TBN_BF16)
-    nchw_to_nhwc_kernel<__nv_bfloat16><<<(unsigned)grid_for(total), 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(x), N, C, H, W, C_pad, static_cast<__nv_bfloat16*>(y));
+    nchw_to_nhwc_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(x), (int)C, (int)(H * W), (int)C_pad,
+        static_cast<__nv_bfloat16*>(y));
   else
-    nchw_to_nhwc_kernel<float><<<(unsigned)grid_for(total), 256, 0, s>>>(
-        static_cast<const float*>(x), N, C, H, W, C_pad, static_cast<float*>(y));
+    nchw_to_nhwc_kernel<float><<<grid, 256, 0, s>>>(
+        static_cast<const float*>(x), (int)C, (int)(H * W), (int)C_pad, static_cast<float*>(y));
   return check_launch("nchw_to_nhwc_kernel");
 }
 

@@ -746,6 +746,8 @@ tbn_status launch_pool(const ConvProblem& p, const TilePlan& t, IgArgs& a, int p
 
 }  // namespace
 
+bool conv_igemm_uses_tma(const ConvProblem& p) { return use_tma(p); }
+
 const char* conv_igemm_unsupported_reason(const ConvProblem& p) {
   if (p.layout != TBN_NHWC) return "implicit GEMM needs NHWC";
   if (p.xdt != TBN_BF16) return "implicit GEMM needs bf16 activations";

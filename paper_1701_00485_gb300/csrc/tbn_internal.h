@@ -69,6 +69,11 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s);
 // Empty string when the implicit-GEMM kernel can run `p`, else the reason.
 const char* conv_igemm_unsupported_reason(const ConvProblem& p);
 tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s);
+// True when the implicit-GEMM kernel would feed activations by TMA (its fast mode).
+bool conv_igemm_uses_tma(const ConvProblem& p);
+
+const char* conv_smalltap_unsupported_reason(const ConvProblem& p);
+tbn_status launch_conv_smalltap(const ConvProblem& p, cudaStream_t s);
 
 const char* gemv_unsupported_reason(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
                                     const uint32_t* codes);

@@ -4,14 +4,21 @@
 //
 // One streaming pass over W: Eq. 3's thresholds are absolute (+-1, 0), so
 // the codes do not depend on alpha and Eq. 5's two sums can be accumulated
-// in the same pass that discretizes.  Each thread owns whole 32-bit output
-// words (16 consecutive weights of a filter): it loads 64 contiguous bytes,
-// forms the sixteen 2-bit fields, sums |W~|*|W| over the word in fp32
-// (pairwise), and counts the magnitude-two codes.  A CTA covers a group of
-// whole filters of at most 1024 words; each of its 256 threads issues the
-// loads of all its (up to four) words before encoding, so a whole layer's
-// weights are in flight at once, and the filters are reduced through shared
-// memory.  Filters longer than 1024 words get a CTA each.
+// in the same pass that discretizes.  Each thread encodes whole 32-bit
+// output words (16 consecutive weights of a filter): it forms the sixteen
+// 2-bit fields, sums |W~|*|W| over the word in fp32 (pairwise) and counts
+// the magnitude-two codes; per-word results go to shared memory and one
+// warp per filter reduces them in word order.
+//
+// The kernel is persistent (two CTAs per SM).  A launch's filters (all jobs
+// of a group: one network's layers) are cut into tasks of whole filters
+// carrying about equal bytes, one task per CTA when they fit.  A task whose
+// rows are 16-byte aligned with n % 16 == 0 streams its weights (contiguous
+// in W, at most 2048 words = 128 KB) through a ring of three 32 KB shared-
+// memory stages filled by 1-D TMA bulk copies (thread 0 keeps three in
+// flight, every wait bounded); other tasks load through registers, and a
+// filter longer than 2048 words is a task of its own with its words strided
+// over the threads.
 //
 // The word sums are accumulated exactly as a two-float (hi, lo) pair
 // (TwoSum, fp32 adds only: GB300's fp64 rate is a small fraction of its fp32
@@ -23,6 +30,7 @@
 
 #include <algorithm>
 #include <cstdint>
+#include <mutex>
 
 #include "tbn_device.cuh"
 #include "tbn_internal.h"
@@ -31,8 +39,14 @@ namespace tbn {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kWordsPerThread = 4;
-constexpr int kGroupWords = kThreads * kWordsPerThread;  // words a row-group CTA covers
+constexpr int kGroupWords = 1024;                        // words of a register-loaded task
+constexpr int kItemWords = 2048;                         // words of a streamed item, at most
+constexpr int kChunkBytes = 32768;                       // one ring stage: 512 words
+constexpr int kChunkWords = kChunkBytes / 64;
+constexpr int kStages = 3;
+constexpr int kRingBytes = kStages * kChunkBytes;
+constexpr int kCtasPerSm = 2;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
 struct QJob {
   const float* W;
@@ -43,8 +57,11 @@ struct QJob {
   int32_t n;
   int32_t wpf;   // words per filter
   int32_t vec;   // 16-byte loads allowed
-  int32_t rows;  // filters per CTA (0: one long filter per CTA, strided words)
+  int32_t rows;  // filters per task (0: one long filter per task, strided words)
+  int32_t mode;  // kModeStream, kModeRegs or kModeLong
 };
+
+enum : int32_t { kModeStream = 0, kModeRegs = 1, kModeLong = 2 };
 
 struct QParams {
   QJob job[TBN_MAX_QUANT_JOBS];
@@ -174,7 +191,7 @@ __device__ __forceinline__ void quantize_words_strided(const float* __restrict__
                                                        uint32_t* __restrict__ out, int n, int wpf,
                                                        bool vec, int j0, int stride, Sum2& acc,
                                                        int& cnt2, bool& huge) {
-  constexpr int kU = 4;
+  constexpr int kU = 2;
   int j = j0;
   for (; j + (kU - 1) * stride < wpf; j += kU * stride) {
     float v[kU][16];
@@ -208,96 +225,44 @@ __device__ __forceinline__ void quantize_words_strided(const float* __restrict__
   }
 }
 
-__global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_constant__ QParams prm) {
-  __shared__ float s_sum[kGroupWords];
-  __shared__ int s_cnt[kGroupWords];
-  __shared__ Sum2 s_part[kThreads / 32];
-  __shared__ int s_pcnt[kThreads / 32];
-  __shared__ int s_huge;
+struct QShared {
+  float sum[kItemWords];
+  int cnt[kItemWords];
+  Sum2 part[kThreads / 32];
+  int pcnt[kThreads / 32];
+  int huge;
+};
 
-  const int64_t task = blockIdx.x;
-  int ji = 0;
-#pragma unroll 1
-  for (int i = 1; i < prm.njobs; ++i)
-    if (task >= prm.job[i].first_task) ji = i;
-  const QJob& jb = prm.job[ji];
-  const int64_t local = task - jb.first_task;
+// One warp per filter of a task: two-float sum of its word sums (word order).
+__device__ __forceinline__ void reduce_rows(const QJob& jb, int64_t k0, int nrows,
+                                            const float* base, QShared& sh) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (jb.rows == 0) {
-    // one long filter per CTA: words strided over the threads, block reduction
-    const int64_t k = local;
-    const float* row = jb.W + k * static_cast<int64_t>(jb.n);
-    uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
-    Sum2 acc{0.0f, 0.0f};
-    int cnt2 = 0;
-    bool huge = false;
-    if (threadIdx.x == 0) s_huge = 0;
-    quantize_words_strided(row, out, jb.n, jb.wpf, jb.vec != 0, threadIdx.x, kThreads, acc, cnt2,
-                           huge);
-    acc = warp_sum2(acc);
-    cnt2 = warp_sum(cnt2);
-    __syncthreads();
-    if (huge) s_huge = 1;
-    if (lane == 0) {
-      s_part[warp] = acc;
-      s_pcnt[warp] = cnt2;
-    }
-    __syncthreads();
-    if (warp == 0) {
-      Sum2 t = lane < kThreads / 32 ? s_part[lane] : Sum2{0.0f, 0.0f};
-      int c = lane < kThreads / 32 ? s_pcnt[lane] : 0;
-      t = warp_sum2(t);
-      c = warp_sum(c);
-      if (lane == 0)
-        jb.alpha[k] = s_huge ? alpha_fp64_row(row, jb.n) : alpha_of(t, c, jb.n);
+  if (jb.wpf <= 16) {
+    // short filters: one thread per filter, its words in order
+    for (int r = threadIdx.x; r < nrows; r += kThreads) {
+      Sum2 acc{0.0f, 0.0f};
+      int cnt2 = 0;
+      bool huge = false;
+      for (int c = 0; c < jb.wpf; ++c) {
+        const float sv = sh.sum[r * jb.wpf + c];
+        huge |= !finite_sum(sv);
+        add2(acc, sv);
+        cnt2 += sh.cnt[r * jb.wpf + c];
+      }
+      jb.alpha[k0 + r] = huge ? alpha_fp64_row(base + static_cast<int64_t>(r) * jb.n, jb.n)
+                              : alpha_of(acc, cnt2, jb.n);
     }
     return;
   }
-
-  // a group of whole filters, at most kGroupWords words: every thread issues
-  // the loads of all its words (up to 4 x 64 bytes) before encoding any
-  const int64_t k0 = local * jb.rows;
-  const int nrows = static_cast<int>(jb.K - k0 < jb.rows ? jb.K - k0 : jb.rows);
-  const int nwords = nrows * jb.wpf;
-  const float* base = jb.W + k0 * static_cast<int64_t>(jb.n);
-  uint32_t* out = jb.codes + k0 * static_cast<int64_t>(jb.wpf);
-  float v[kWordsPerThread][16];
-  int nv[kWordsPerThread];
-#pragma unroll
-  for (int u = 0; u < kWordsPerThread; ++u) {
-    const int j = threadIdx.x + u * kThreads;
-    if (j < nwords) {
-      const int r = j / jb.wpf, c = j - r * jb.wpf;
-      load16(base + static_cast<int64_t>(r) * jb.n, jb.n, c, jb.vec != 0, v[u], nv[u]);
-    } else {
-      nv[u] = 0;
-    }
-  }
-#pragma unroll
-  for (int u = 0; u < kWordsPerThread; ++u) {
-    const int j = threadIdx.x + u * kThreads;
-    if (j < nwords) {
-      uint32_t word;
-      float sum;
-      int c2;
-      encode16(v[u], nv[u], word, sum, c2);
-      out[j] = word;   // the group's words are contiguous in the codes array
-      s_sum[j] = sum;
-      s_cnt[j] = c2;
-    }
-  }
-  __syncthreads();
-  // one warp per filter of the group: two-float sum of its word sums
   for (int r = warp; r < nrows; r += kThreads / 32) {
     Sum2 acc{0.0f, 0.0f};
     int cnt2 = 0;
     bool huge = false;
     for (int c = lane; c < jb.wpf; c += 32) {
-      const float s = s_sum[r * jb.wpf + c];
-      huge |= !finite_sum(s);
-      add2(acc, s);
-      cnt2 += s_cnt[r * jb.wpf + c];
+      const float sv = sh.sum[r * jb.wpf + c];
+      huge |= !finite_sum(sv);
+      add2(acc, sv);
+      cnt2 += sh.cnt[r * jb.wpf + c];
     }
     acc = warp_sum2(acc);
     cnt2 = warp_sum(cnt2);
@@ -305,6 +270,167 @@ __global__ void __launch_bounds__(kThreads) quantize_pack_kernel(const __grid_co
     if (lane == 0)
       jb.alpha[k0 + r] = huge ? alpha_fp64_row(base + static_cast<int64_t>(r) * jb.n, jb.n)
                               : alpha_of(acc, cnt2, jb.n);
+  }
+}
+
+// Streamed task: nrows whole filters (n % 16 == 0, 16-byte aligned rows,
+// nrows * wpf <= kItemWords words) flow through the ring of kStages 32 KB
+// chunks; thread 0 keeps up to kStages bulk copies in flight.  `seq` counts
+// the chunks this CTA has pushed through the ring (slot and phase).
+// Returns false if a wait timed out (after draining its copies).
+__device__ bool task_stream(const QJob& jb, int64_t k0, int nrows, QShared& sh, uint8_t* ring,
+                            uint64_t* full, uint32_t& seq, uint32_t* err) {
+  const int words = nrows * jb.wpf;
+  const float* base = jb.W + k0 * static_cast<int64_t>(jb.n);
+  const uint8_t* src = reinterpret_cast<const uint8_t*>(base);
+  uint32_t* out = jb.codes + k0 * static_cast<int64_t>(jb.wpf);
+  const uint32_t bytes = static_cast<uint32_t>(words) * 64u;
+  const int nch = (words + kChunkWords - 1) / kChunkWords;
+  auto issue = [&](int i) {
+    const uint32_t g = seq + static_cast<uint32_t>(i);
+    const uint32_t off = static_cast<uint32_t>(i) * kChunkBytes;
+    const uint32_t len = bytes - off < static_cast<uint32_t>(kChunkBytes) ? bytes - off
+                                                                          : static_cast<uint32_t>(kChunkBytes);
+    mbar_arrive_expect_tx(&full[g % kStages], len);
+    bulk_load_1d(ring + (g % kStages) * kChunkBytes, src + off, len, &full[g % kStages]);
+  };
+  if (threadIdx.x == 0)
+    for (int i = 0; i < nch && i < kStages; ++i) issue(i);
+  for (int i = 0; i < nch; ++i) {
+    const uint32_t g = seq + static_cast<uint32_t>(i);
+    const bool ok = mbar_wait(&full[g % kStages], (g / kStages) & 1u, nullptr, err, kWaitLimitNs);
+    if (ok) {
+      const float* chunk = reinterpret_cast<const float*>(ring + (g % kStages) * kChunkBytes);
+      const int w0 = i * kChunkWords;
+      const int wn = words - w0 < kChunkWords ? words - w0 : kChunkWords;
+#pragma unroll
+      for (int u = 0; u < kChunkWords / kThreads; ++u) {
+        const int w = threadIdx.x + u * kThreads;
+        if (w >= wn) break;
+        float v[16];
+        const float4* q4 = reinterpret_cast<const float4*>(chunk + 16 * w);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 t4 = q4[q];
+          v[4 * q + 0] = t4.x;
+          v[4 * q + 1] = t4.y;
+          v[4 * q + 2] = t4.z;
+          v[4 * q + 3] = t4.w;
+        }
+        uint32_t word;
+        float sum;
+        int c2;
+        encode16(v, 16, word, sum, c2);
+        out[w0 + w] = word;   // the task's words are contiguous in the codes array
+        sh.sum[w0 + w] = sum;
+        sh.cnt[w0 + w] = c2;
+      }
+    }
+    // everyone is done with this slot (or something timed out)
+    if (__syncthreads_or(!ok)) {
+      if (threadIdx.x == 0) {
+        // copies issued but not consumed: chunks i .. min(nch, i + kStages) - 1
+        for (int j = i; j < nch && j < i + kStages; ++j) {
+          const uint32_t gj = seq + static_cast<uint32_t>(j);
+          mbar_wait(&full[gj % kStages], (gj / kStages) & 1u, nullptr, err, kWaitLimitNs);
+        }
+      }
+      return false;
+    }
+    if (threadIdx.x == 0 && i + kStages < nch) issue(i + kStages);
+  }
+  seq += static_cast<uint32_t>(nch);
+  reduce_rows(jb, k0, nrows, base, sh);
+  __syncthreads();   // sums consumed before the next task overwrites them
+  return true;
+}
+
+// Register-loaded task (rows not 16-byte aligned or n % 16 != 0; small
+// layers such as a network's first): one word per thread per round.
+__device__ void task_regs(const QJob& jb, int64_t k0, int nrows, QShared& sh) {
+  const int nwords = nrows * jb.wpf;
+  const float* base = jb.W + k0 * static_cast<int64_t>(jb.n);
+  uint32_t* out = jb.codes + k0 * static_cast<int64_t>(jb.wpf);
+  for (int j = threadIdx.x; j < nwords; j += kThreads) {
+    const int r = j / jb.wpf, c = j - r * jb.wpf;
+    float v[16];
+    int nv;
+    load16(base + static_cast<int64_t>(r) * jb.n, jb.n, c, jb.vec != 0, v, nv);
+    uint32_t word;
+    float sum;
+    int c2;
+    encode16(v, nv, word, sum, c2);
+    out[j] = word;
+    sh.sum[j] = sum;
+    sh.cnt[j] = c2;
+  }
+  __syncthreads();
+  reduce_rows(jb, k0, nrows, base, sh);
+  __syncthreads();
+}
+
+// One long filter (more than kItemWords words): words strided over the
+// threads, block reduction.
+__device__ void task_long(const QJob& jb, int64_t k, QShared& sh) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* row = jb.W + k * static_cast<int64_t>(jb.n);
+  uint32_t* out = jb.codes + k * static_cast<int64_t>(jb.wpf);
+  Sum2 acc{0.0f, 0.0f};
+  int cnt2 = 0;
+  bool huge = false;
+  if (threadIdx.x == 0) sh.huge = 0;
+  quantize_words_strided(row, out, jb.n, jb.wpf, jb.vec != 0, threadIdx.x, kThreads, acc, cnt2,
+                         huge);
+  acc = warp_sum2(acc);
+  cnt2 = warp_sum(cnt2);
+  __syncthreads();
+  if (huge) sh.huge = 1;
+  if (lane == 0) {
+    sh.part[warp] = acc;
+    sh.pcnt[warp] = cnt2;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    Sum2 t = lane < kThreads / 32 ? sh.part[lane] : Sum2{0.0f, 0.0f};
+    int c = lane < kThreads / 32 ? sh.pcnt[lane] : 0;
+    t = warp_sum2(t);
+    c = warp_sum(c);
+    if (lane == 0) jb.alpha[k] = sh.huge ? alpha_fp64_row(row, jb.n) : alpha_of(t, c, jb.n);
+  }
+  __syncthreads();
+}
+
+// Persistent: CTA b takes tasks b, b + grid, ...; a task is a run of whole
+// filters of one job (sized so that tasks carry about equal bytes).
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) quantize_pack_kernel(const __grid_constant__ QParams prm,
+                                                                    int64_t ntasks) {
+  extern __shared__ __align__(128) uint8_t q_ring[];   // kRingBytes when any job streams
+  __shared__ QShared sh;
+  __shared__ uint64_t full[kStages];
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) mbar_init(&full[i], 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  uint32_t seq = 0;
+  for (int64_t task = blockIdx.x; task < ntasks; task += gridDim.x) {
+    int ji = 0;
+#pragma unroll 1
+    for (int i = 1; i < prm.njobs; ++i)
+      if (task >= prm.job[i].first_task) ji = i;
+    const QJob& jb = prm.job[ji];
+    const int64_t local = task - jb.first_task;
+    if (jb.mode == kModeLong) {
+      task_long(jb, local, sh);
+    } else {
+      const int64_t k0 = local * jb.rows;
+      const int nrows = static_cast<int>(jb.K - k0 < jb.rows ? jb.K - k0 : jb.rows);
+      if (jb.mode == kModeStream) {
+        if (!task_stream(jb, k0, nrows, sh, q_ring, full, seq, prm.err)) return;
+      } else {
+        task_regs(jb, k0, nrows, sh);
+      }
+    }
   }
 }
 
@@ -340,7 +466,13 @@ tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStrea
   QParams prm{};
   prm.njobs = njobs;
   prm.err = device_error_word();
+  const int slots = device_sm_count() * kCtasPerSm;
+  // tasks of about equal bytes: the group's words spread over one task per CTA slot
+  int64_t total_words = 0;
+  for (int i = 0; i < njobs; ++i) total_words += jobs[i].K * ((jobs[i].n + 15) / 16);
+  const int64_t target = std::max<int64_t>(1, (total_words + slots - 1) / std::max(1, slots));
   int64_t tasks = 0;
+  bool any_stream = false;
   for (int i = 0; i < njobs; ++i) {
     const tbn_quant_job& j = jobs[i];
     QJob& q = prm.job[i];
@@ -351,13 +483,35 @@ tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStrea
     q.n = static_cast<int32_t>(j.n);
     q.wpf = static_cast<int32_t>((j.n + 15) / 16);
     q.vec = (is_aligned(j.W, 16) && (j.n % 4) == 0) ? 1 : 0;
-    q.rows = q.wpf <= kGroupWords ? static_cast<int32_t>(std::min<int64_t>(j.K, kGroupWords / q.wpf)) : 0;
+    if (q.vec && j.n % 16 == 0 && q.wpf <= kItemWords) {
+      q.mode = kModeStream;
+      const int64_t want = (std::min<int64_t>(target, kItemWords) + q.wpf - 1) / q.wpf;
+      q.rows = static_cast<int32_t>(std::max<int64_t>(1, std::min<int64_t>({want, j.K, kItemWords / q.wpf})));
+      any_stream = true;
+    } else if (q.wpf <= kGroupWords) {
+      q.mode = kModeRegs;
+      q.rows = static_cast<int32_t>(std::min<int64_t>(j.K, kGroupWords / q.wpf));
+    } else {
+      q.mode = kModeLong;
+      q.rows = 0;
+    }
     q.first_task = tasks;
     tasks += q.rows == 0 ? j.K : (j.K + q.rows - 1) / q.rows;
   }
   if (tasks == 0) return TBN_OK;
   if (tasks > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "quantize: too many filters (%lld tasks)", (long long)tasks);
-  quantize_pack_kernel<<<static_cast<unsigned>(tasks), kThreads, 0, s>>>(prm);
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    attr_err = cudaFuncSetAttribute(quantize_pack_kernel,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+    if (attr_err == cudaSuccess)   // two ring-holding CTAs per SM
+      attr_err = cudaFuncSetAttribute(quantize_pack_kernel,
+                                      cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(quantize)");
+  const unsigned grid = static_cast<unsigned>(std::min<int64_t>(tasks, slots));
+  quantize_pack_kernel<<<grid, kThreads, any_stream ? kRingBytes : 0, s>>>(prm, tasks);
   return check_launch("quantize_pack_kernel");
 }
 

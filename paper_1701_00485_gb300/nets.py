@@ -92,10 +92,13 @@ class ConvStack:
 
     def forward(self, requantize: bool = True, conv_hook=None):
         """One forward pass on the current stream; returns the output tensor.
-        conv_hook(i, layer, when) is called before/after each conv launch
+        conv_hook(i, layer, when) is called before/after each conv launch, and
+        once as conv_hook(-1, None, "quantized") after the re-quantization
         (used by the benchmark to record timing events)."""
         if requantize:
             self.quantize()
+        if conv_hook:
+            conv_hook(-1, None, "quantized")
         tbn_nchw_to_nhwc(self.x_in, out=self.x_nhwc)
         h = self.x_nhwc
         for i, l in enumerate(self.layers):

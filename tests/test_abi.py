@@ -96,8 +96,13 @@ def test_select_algo_host_rules(L):
                                       1, 64, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
     assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW,
                                       1, 64, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+    # short bf16 filters (C*R*S <= 64) go to the small-tap kernel in either layout
     assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NHWC,
-                                      1, 3, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+                                      1, 3, 8, 8, 64, 3, 3) == tbn.TBN_CONV_SMALL_TAPS
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW,
+                                      1, 7, 8, 8, 64, 3, 3) == tbn.TBN_CONV_SMALL_TAPS
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW,
+                                      1, 8, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
 
 
 def test_linear_and_glue_reject_bad_arguments(L):

@@ -103,10 +103,62 @@ GATHER = [
 def test_igemm_gather_conv_matches_oracle(case):
     c = make_case(*case, seed=4000 + sum(case[:7]), wscale=1.2)
     algo = tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NHWC, *case[:7], case[7], case[8])
-    assert algo == tbn.TBN_CONV_IMPLICIT_GEMM
+    short = case[1] * case[5] * case[6] <= 64
+    assert algo == (tbn.TBN_CONV_SMALL_TAPS if short else tbn.TBN_CONV_IMPLICIT_GEMM)
     y = c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_IMPLICIT_GEMM)
     y_orc, bound = c.oracle_full(torch.bfloat16)
     assert_within(y, y_orc, bound, out_bf16=False, what="gather %s" % (case,))
+
+
+# ---------------------------------------------------------------- small-tap kernel
+SMALLTAP = [
+    # N, C, H, W, K, R, S, stride, pad    (bf16 x, C*R*S <= 64)
+    (2, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)),      # VGG first layer geometry, n = 27
+    (1, 1, 28, 28, 20, 5, 5, (1, 1), (0, 0)),       # C = 1, 5x5, K < 128
+    (2, 7, 10, 9, 200, 3, 3, (1, 1), (1, 1)),       # n = 63 (64-code rows), two filter tiles
+    (1, 2, 17, 300, 24, 3, 3, (1, 1), (1, 1)),      # Q > 256: column tiles
+    (3, 4, 15, 13, 37, 3, 3, (2, 2), (1, 1)),       # stride 2, odd K
+    (1, 16, 9, 9, 64, 2, 2, (1, 1), (0, 0)),        # n = 64 exactly
+    (2, 3, 20, 20, 16, 1, 1, (1, 1), (0, 0)),       # 1x1
+    (1, 5, 12, 7, 130, 3, 1, (1, 2), (0, 1)),       # R != S, mixed stride / pad
+]
+
+
+@pytest.mark.parametrize("case", SMALLTAP)
+@pytest.mark.parametrize("layout", [tbn.TBN_NCHW, tbn.TBN_NHWC])
+def test_smalltap_conv_matches_oracle(case, layout):
+    c = make_case(*case, seed=6000 + sum(case[:7]), wscale=1.2)
+    algo = tbn.tbn_conv2d_select_algo(torch.bfloat16, layout, *case[:7], case[7], case[8])
+    assert algo == tbn.TBN_CONV_SMALL_TAPS
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    y = c.run_gpu(layout, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_SMALL_TAPS)
+    assert_within(y, y_orc, bound, out_bf16=False, what="smalltap %s" % (case,))
+    yb = c.run_gpu(layout, torch.bfloat16, torch.bfloat16, algo=tbn.TBN_CONV_SMALL_TAPS)
+    assert_within(yb, y_orc, bound, out_bf16=True, what="smalltap bf16 %s" % (case,))
+
+
+@pytest.mark.parametrize("case", SMALLTAP[:3])
+@pytest.mark.parametrize("layout", [tbn.TBN_NCHW, tbn.TBN_NHWC])
+@pytest.mark.parametrize("ydt", [torch.float32, torch.bfloat16])
+def test_smalltap_conv_epilogue(case, layout, ydt):
+    import oracle
+    c = make_case(*case, seed=6500 + sum(case[:7]))
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    g = inputs.generator(17)
+    res = torch.randn(*y_orc.shape, generator=g).to(ydt)
+    want = oracle.epilogue(y_orc, res.float().numpy(), relu=True)
+    y = c.run_gpu(layout, torch.bfloat16, ydt, algo=tbn.TBN_CONV_SMALL_TAPS, relu=True,
+                  residual=res)
+    assert_within(y, want, bound, out_bf16=(ydt == torch.bfloat16), epilogue=True,
+                  what="smalltap epi %s" % (case,))
+
+
+def test_smalltap_rejects_long_filters_and_pool():
+    c = make_case(1, 8, 6, 6, 16, 3, 3, (1, 1), (1, 1), seed=5)   # n = 72
+    with pytest.raises(tbn.TBNError):
+        c.run_gpu(tbn.TBN_NHWC, torch.bfloat16, torch.float32, algo=tbn.TBN_CONV_SMALL_TAPS)
+    assert tbn.tbn_conv2d_select_algo(torch.float32, tbn.TBN_NHWC, 1, 3, 8, 8, 16, 3, 3) != \
+        tbn.TBN_CONV_SMALL_TAPS
 
 
 POOL = [
