@@ -149,6 +149,34 @@ __device__ __forceinline__ TileCoord tile_coord(const IgArgs& a, int t) {
   return c;
 }
 
+// D block of 16 TMEM lanes x 32 columns, four 16x256b fragments: register
+// 4b + 0/1 = lane i/4, columns 8b + 2(i%4) + 0/1; 4b + 2/3 = lane i/4 + 8.
+__device__ __forceinline__ void tmem_ld_16x256b_x4(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+        "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr)
+      : "memory");
+}
+
+// Four 8x8 bf16 matrices, each stored transposed: row i of the shared
+// destination (address from lane 8m + i for matrix m) receives column i.
+__device__ __forceinline__ void stmatrix_x4_trans(uint32_t addr, uint32_t r0, uint32_t r1,
+                                                  uint32_t r2, uint32_t r3) {
+  asm volatile("stmatrix.sync.aligned.m8n8.x4.trans.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(
+                   addr),
+               "r"(r0), "r"(r1), "r"(r2), "r"(r3)
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&b);
+}
+
 // Direct global store of one output value (the path for fp32 output or
 // shapes the TMA store cannot take): fp32 math, residual, ReLU, rounding.
 __device__ __forceinline__ void store_out(const IgArgs& a, size_t o, float v) {
@@ -490,6 +518,73 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       if (ok) tc_fence_after_sync();
       if (!ok) {
         // skip the work, keep the barrier schedule
+      } else if (kPoolBW == 0 && kTmaStore && a.residual == nullptr) {
+        // Fragment epilogue: 16x256b loads (lane = filter, column = pixel),
+        // scale / ReLU / bf16 pairs, transposed 8x8 stores into the staging
+        // tile [pixel][filter] as two 128-byte-swizzled halves of 64
+        // filters (chunk c of pixel row px at c ^ (px & 7)).
+        const int nchunks = (a.tile_n + 31) / 32;
+        const int c_begin = half ? (nchunks + 1) / 2 : 0;
+        const int c_end = half ? nchunks : (nchunks + 1) / 2;
+        const int fr = lane >> 2;                       // fragment row within 8
+        float a2f[2][2];
+#pragma unroll
+        for (int lg = 0; lg < 2; ++lg) {
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int kk = tc.ktile * kBM + sub * 32 + lg * 16 + u * 8 + fr;
+            a2f[lg][u] = kk < a.K ? 2.0f * __ldg(a.alpha + kk) : 0.0f;
+          }
+        }
+        // this lane's stmatrix row address pieces: matrix mi = lane / 8, row = lane % 8
+        const int mi = lane >> 3, mrow = lane & 7;
+        const uint32_t stage_s = smem_addr(stage);
+        for (int j = c_begin; j < c_end; ++j) {
+          uint32_t v[2][16];
+#pragma unroll
+          for (int lg = 0; lg < 2; ++lg)
+            tmem_ld_16x256b_x4(acc_tmem + (static_cast<uint32_t>(sub * 32 + lg * 16) << 16) +
+                                   static_cast<uint32_t>(32 * j),
+                               v[lg]);
+          tmem_wait_ld();
+          if (j == c_end - 1) {
+            tc_fence_before_sync();
+            mbar_arrive(&ctl->acc_empty);
+          }
+#pragma unroll
+          for (int lg = 0; lg < 2; ++lg) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+              float y0 = a2f[lg][0] * __uint_as_float(v[lg][4 * b + 0]);
+              float y1 = a2f[lg][0] * __uint_as_float(v[lg][4 * b + 1]);
+              float y2 = a2f[lg][1] * __uint_as_float(v[lg][4 * b + 2]);
+              float y3 = a2f[lg][1] * __uint_as_float(v[lg][4 * b + 3]);
+              if (a.relu) {
+                y0 = fmaxf(y0, 0.0f);
+                y1 = fmaxf(y1, 0.0f);
+                y2 = fmaxf(y2, 0.0f);
+                y3 = fmaxf(y3, 0.0f);
+              }
+              pk[2 * b] = pack_bf16x2(y0, y1);       // filters fr, pixels 2(i%4) + 0/1
+              pk[2 * b + 1] = pack_bf16x2(y2, y3);   // filters fr + 8
+            }
+#pragma unroll
+            for (int bp = 0; bp < 2; ++bp) {
+              // matrices: (filters +0, block 2bp), (+8, 2bp), (+0, 2bp+1), (+8, 2bp+1)
+              const int px = 32 * j + 8 * (2 * bp + (mi >> 1)) + mrow;
+              const int chunk = 4 * sub + 2 * lg + (mi & 1);           // 8-filter chunk 0..15
+              const uint32_t addr = stage_s + static_cast<uint32_t>((chunk >> 3) * 32768 + px * 128 +
+                                                                    (((chunk & 7) ^ (px & 7)) << 4));
+              stmatrix_x4_trans(addr, pk[4 * bp + 0], pk[4 * bp + 1], pk[4 * bp + 2],
+                                pk[4 * bp + 3]);
+            }
+          }
+        }
+        if (c_begin >= c_end) {
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->acc_empty);
+        }
       } else if constexpr (kPoolBW == 0) {
         const int T = a.bw * a.bh * a.bn;
         const int nchunks = (a.tile_n + 31) / 32;
@@ -596,10 +691,16 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
         fence_proxy_async_smem();   // staged values -> visible to the TMA store
         named_barrier_sync(1, 32 * kEpiWarps);
         if (elected && ok) {
-          if (kPoolBW)
+          if (kPoolBW) {
             tma_store_4d(&tmap_y, stage, tc.ktile * kBM, 0, tc.p0 / 2, tc.n0);
-          else
+          } else if (a.residual == nullptr) {
             tma_store_4d(&tmap_y, stage, tc.ktile * kBM, tc.q0, tc.p0, tc.n0);
+            if (tc.ktile * kBM + kBM / 2 < a.K)
+              tma_store_4d(&tmap_y, reinterpret_cast<uint8_t*>(stage) + 32768,
+                           tc.ktile * kBM + kBM / 2, tc.q0, tc.p0, tc.n0);
+          } else {
+            tma_store_4d(&tmap_y, stage, tc.ktile * kBM, tc.q0, tc.p0, tc.n0);
+          }
           bulk_commit_group();
         }
       }
@@ -672,19 +773,22 @@ bool use_tma_store(const ConvProblem& p) {
          (!p.residual || is_aligned(p.residual, 16));
 }
 
+// Output map: box = 128 filters x the tile's pixels (no swizzle), or with
+// `halves`, 64 filters (128 bytes) per box with the 128-byte swizzle (the
+// staging layout of the fragment epilogue, two stores per tile).
 CUresult encode_out_map(CUtensorMap* m, const void* base, const ConvProblem& p, const TilePlan& t,
-                        int pool) {
+                        int pool, bool halves = false) {
   const int64_t Po = pool ? p.P / 2 : p.P, Qo = pool ? p.Q / 2 : p.Q;
   const cuuint64_t gdim[4] = {(cuuint64_t)p.K, (cuuint64_t)Qo, (cuuint64_t)Po, (cuuint64_t)p.N};
   const cuuint64_t gstride[3] = {(cuuint64_t)(p.K * 2), (cuuint64_t)(Qo * p.K * 2),
                                  (cuuint64_t)(Po * Qo * p.K * 2)};
-  const cuuint32_t box[4] = {(cuuint32_t)kBM, (cuuint32_t)(pool ? t.bw / 2 : t.bw),
+  const cuuint32_t box[4] = {(cuuint32_t)(halves ? kBM / 2 : kBM), (cuuint32_t)(pool ? t.bw / 2 : t.bw),
                              (cuuint32_t)(pool ? t.bh / 2 : t.bh), (cuuint32_t)t.bn};
   const cuuint32_t estr[4] = {1u, 1u, 1u, 1u};
   return get_encode_tiled()(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), gdim,
                             gstride, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                            halves ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
 template <bool kGather, int kPoolBW, bool kTmaStore>
@@ -710,7 +814,9 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
     if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed (%d)", (int)cr);
   }
   if (kTmaStore) {
-    CUresult cr = encode_out_map(&tmap_y, p.y, p, t, kPoolBW ? 1 : 0);
+    // the fragment epilogue (no pool, no residual) stages two swizzled halves
+    const bool halves = kPoolBW == 0 && p.residual == nullptr;
+    CUresult cr = encode_out_map(&tmap_y, p.y, p, t, kPoolBW ? 1 : 0, halves);
     if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(y) failed (%d)", (int)cr);
     if (p.residual) {
       cr = encode_out_map(&tmap_res, p.residual, p, t, 0);

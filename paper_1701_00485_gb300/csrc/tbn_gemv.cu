@@ -18,8 +18,9 @@
 //   stages (stage ks goes to warp ks % P of the tile) and their partial sums
 //   are added in a fixed order.  Per K step of 16 a warp runs
 //   one mma.m16n8k16: A = 16 rows x 16 codes decoded in registers to bf16
-//   W~/2, B = 16 inputs x 8 batch columns (rows past B read a zero chunk),
-//   fp32 accumulation.  Lane (g, t) of the A fragment holds pairs t and
+//   W~/2, B = 16 inputs x 8 batch columns (lanes past B read batch row
+//   n mod B, which only fills mma columns that are dropped), fp32
+//   accumulation.  Lane (g, t) of the A fragment holds pairs t and
 //   t + 4 of the K step's word of rows g and g + 8; with the byte-planar
 //   packing a pair is one mask and one multiply-add.  2 alpha is applied
 //   in the epilogue (W~/2 is exact in bf16).
@@ -119,7 +120,7 @@ struct PairDecode {
   }
 };
 
-// One stage of one 16-row tile: 32 K steps of 16, accumulated into two
+// A stage of a 16-row tile is 32 K steps of 16, accumulated into two
 // independent chains (K step i goes to chain i % 2) so consecutive mma
 // instructions do not wait on each other.
 //   w_lane: shared address of the tile's row g with this lane's swizzle
