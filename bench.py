@@ -138,6 +138,25 @@ class ClockSampler:
                 "samples": len(sel)}
 
 
+class L2Flush:
+    """Evicts the step's data from L2 between timed replays: writes a 512 MiB
+    buffer (larger than the 129 MB L2) and, in "write+read" mode, then reads
+    another 512 MiB buffer, so the write's dirty lines are written back
+    before the timed region instead of during it (L2 ends up holding clean,
+    unrelated lines)."""
+
+    def __init__(self, dev, mode):
+        self.mode = mode
+        self.w = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+        self.r = torch.ones(FLUSH_BYTES // 4, dtype=torch.int32, device=dev) if mode == "write+read" else None
+        self.acc = torch.empty((), dtype=torch.int32, device=dev)
+
+    def zero_(self):
+        self.w.zero_()
+        if self.r is not None:
+            torch.sum(self.r, dim=0, dtype=torch.int32, out=self.acc)
+
+
 def timed_replays(graph, stream, flush, ev, steps, dev):
     """Replay `graph` `steps` times, flushing L2 before each replay; returns
     the per-replay device times (ms) between the graph's own events ev."""
@@ -239,7 +258,7 @@ def run_vgg(args, rank, world, local_rank):
 
     graph_e, ev_e = capture(e2e_body)
 
-    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush = L2Flush(dev, args.l2_flush)
     sampler = ClockSampler(local_rank)
     sampler.start()
     warm(graph, stream, flush, args.warmup, args.min_warmup_s, dev)
@@ -297,7 +316,7 @@ def run_vgg(args, rank, world, local_rank):
         "config": {"workload": WORKLOAD, "global_batch": N * world, "image": [3, 32, 32],
                    "layers": "3x3/p1 128-128-256-256-512-512, 2x2 pool every 2nd",
                    "requantize_per_step": True, "parallelism": "replicas x%d" % world,
-                   "l2": "512 MiB flush between timed steps"},
+                   "l2": "512 MiB %s between timed steps" % args.l2_flush},
         "images_per_s": round(images_per_s, 1),
         "breakdown_us": dict([("quantize", round(1e3 * quant_ms / args.steps, 2)),
                               ("nchw_to_nhwc", round(1e3 * prefix_ms / args.steps, 2))] +
@@ -489,6 +508,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize"], default="vgg_small")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--l2-flush", choices=["write", "write+read"], default="write",
+                    help="L2 eviction between timed steps (write+read also drains the dirty lines)")
     ap.add_argument("--min-warmup-s", type=float, default=1.0,
                     help="keep replaying warm-up steps for at least this long (clock settling)")
     args = ap.parse_args()
