@@ -58,13 +58,13 @@ METRIC = "TBN conv TFLOP/s (VGG-small b128 forward incl. per-step re-quantizatio
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FLUSH_BYTES = 512 * 1024 * 1024
 
-# DRAM bytes (read + write) per convolution launch, mean over the six launches of
-# one step, from the ncu capture summarised in profiles/vgg_small_b128_launches.md.
+# DRAM bytes (read + write) per convolution launch, mean over the five
+# implicit-GEMM launches of one step (c2..c6), from the ncu capture summarised in profiles/vgg_small_b128_launches.md.
 # Valid only for the kernel sources it was measured on (hash below); otherwise the
 # roofline entry reports null.
 CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
                             "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
-                "sha256_16": "fc952fb0541013c3", "bytes_per_launch": 12.26e6}
+                "sha256_16": "0ad18e6e5c94b6f0", "bytes_per_launch": 14.53e6}
 
 
 def measured_traffic(rec):
@@ -363,14 +363,14 @@ def run_gemv(args, rank, world, local_rank):
     sampler = ClockSampler(local_rank)
     sampler.start()
     t0 = time.time()
-    for K in inputs.GEMV_SIZES:
+    for K in args.gemv_sizes:
         W, _ = inputs.gemv_inputs(K, 1)
         codes, alpha = tbn.tbn_quantize_pack(W.to(dev))
         del W
         code_bytes = codes.numel() * 4
         copies = max(2, int(np.ceil(3 * l2 / code_bytes)))
         bufs = [codes] + [codes.clone() for _ in range(copies - 1)]
-        for B in inputs.GEMV_BATCHES:
+        for B in args.gemv_batches:
             gx = torch.Generator(device=dev)
             gx.manual_seed(1000 * K + B)
             x = torch.randn((B, K), generator=gx, device=dev).to(torch.bfloat16)
@@ -399,7 +399,7 @@ def run_gemv(args, rank, world, local_rank):
         del bufs
         torch.cuda.empty_cache()
     clocks = sampler.stop(t0, time.time())
-    head = [s for s in sweep if s["K"] == 16384 and s["B"] == 1][0]
+    head = ([s for s in sweep if s["K"] == 16384 and s["B"] == 1] or sweep)[0]
     return {"metric": "TBN GEMV HBM GB/s (B=1, K_out=K_in=16384, 2-bit weight stream)",
             "value": head["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
@@ -425,7 +425,7 @@ def run_quantize(args, rank, world, local_rank):
     sampler = ClockSampler(local_rank)
     sampler.start()
     t0 = time.time()
-    for K in (8192, 16384):
+    for K in args.quant_sizes:
         W, _ = inputs.gemv_inputs(K, 1)
         W = W.to(dev)
         codes = torch.empty((K, K // 16), dtype=torch.int32, device=dev)
@@ -508,6 +508,11 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize"], default="vgg_small")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--gemv-sizes", type=int, nargs="+", default=[4096, 8192, 16384],
+                    help="K_out = K_in of the GEMV workload")
+    ap.add_argument("--gemv-batches", type=int, nargs="+", default=[1, 8])
+    ap.add_argument("--quant-sizes", type=int, nargs="+", default=[8192, 16384],
+                    help="square fp32 matrices of the quantize workload")
     ap.add_argument("--l2-flush", choices=["write", "write+read"], default="write",
                     help="L2 eviction between timed steps (write+read also drains the dirty lines)")
     ap.add_argument("--min-warmup-s", type=float, default=1.0,
