@@ -375,31 +375,53 @@ def run_gemv(args, rank, world, local_rank):
             gx.manual_seed(1000 * K + B)
             x = torch.randn((B, K), generator=gx, device=dev).to(torch.bfloat16)
             y = torch.empty((B, K), dtype=torch.bfloat16, device=dev)
+            ws_bytes = tbn.tbn_linear_workspace_bytes(B, K, K, torch.float32)
+            ws = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
+            x32 = x.float()
             reps = max(copies, 64)
-            fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x, c, alpha, K, out=y))
-                   for r in range(reps)]
-            with torch.cuda.stream(stream):
-                fns[0]()
-            torch.cuda.synchronize(dev)
-            g, ev = _rotating_graph(fns, stream, dev)
-            for _ in range(max(3, args.warmup)):
-                g.replay()
-            torch.cuda.synchronize(dev)
-            ms = []
-            for _ in range(max(3, args.steps // 20)):
+            # "mma": tbn_linear_fwd with bf16 activations (tensor-core GEMV);
+            # "table-f32": tbn_linear_fwd_ws with fp32 activations (the
+            # batch-1 table-lookup GEMV, the path for fp32 inputs);
+            # "conv-f32": tbn_linear_fwd with fp32 activations and no scratch
+            # (the 1x1-convolution path those inputs take otherwise)
+            paths = ["mma", "table-f32", "conv-f32"] if ws_bytes > 0 else ["mma"]
+            for path in paths:
+                if path == "table-f32":
+                    fns = [(lambda c=bufs[r % copies]:
+                            tbn.tbn_linear_fwd_ws(x32, c, alpha, K, ws, out=y))
+                           for r in range(reps)]
+                elif path == "conv-f32":
+                    fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x32, c, alpha, K, out=y))
+                           for r in range(reps)]
+                else:
+                    fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x, c, alpha, K, out=y))
+                           for r in range(reps)]
                 with torch.cuda.stream(stream):
+                    fns[0]()
+                torch.cuda.synchronize(dev)
+                g, ev = _rotating_graph(fns, stream, dev)
+                for _ in range(max(3, args.warmup)):
                     g.replay()
-                stream.synchronize()
-                ms.append(ev[0].elapsed_time(ev[1]) / reps)
-            t = float(np.median(ms)) * 1e-3
-            byts = code_bytes + 4 * K + 2 * B * K * 2
-            sweep.append({"K": K, "B": B, "us_per_call": round(t * 1e6, 3),
-                          "gbs": round(byts / t / 1e9, 1), "frac_hbm": round(byts / t / 1e9 / hbm, 4),
-                          "tflops": round(2 * B * K * K / t / 1e12, 3)})
+                torch.cuda.synchronize(dev)
+                ms = []
+                for _ in range(max(3, args.steps // 20)):
+                    with torch.cuda.stream(stream):
+                        g.replay()
+                    stream.synchronize()
+                    ms.append(ev[0].elapsed_time(ev[1]) / reps)
+                t = float(np.median(ms)) * 1e-3
+                byts = code_bytes + 4 * K + (4 if path.endswith("f32") else 2) * B * K + 2 * B * K
+                sweep.append({"K": K, "B": B, "path": path, "us_per_call": round(t * 1e6, 3),
+                              "gbs": round(byts / t / 1e9, 1),
+                              "frac_hbm": round(byts / t / 1e9 / hbm, 4),
+                              "tflops": round(2 * B * K * K / t / 1e12, 3)})
+                del g
         del bufs
         torch.cuda.empty_cache()
     clocks = sampler.stop(t0, time.time())
-    head = ([s for s in sweep if s["K"] == 16384 and s["B"] == 1] or sweep)[0]
+    head = ([s for s in sweep if s["K"] == 16384 and s["B"] == 1 and s["path"] == "mma"] or
+            sweep)[0]
+    head_kernel = "gemv_tma_kernel (mma.sync)"
     return {"metric": "TBN GEMV HBM GB/s (B=1, K_out=K_in=16384, 2-bit weight stream)",
             "value": head["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
@@ -408,7 +430,7 @@ def run_gemv(args, rank, world, local_rank):
             "config": {"workload": "gemv_sweep", "l2": "rotating weight copies > 3x L2"},
             "roofline": {"bound": "hbm", "achieved": head["gbs"], "peak": hbm, "unit": "GB/s",
                          "frac": round(head["gbs"] / hbm, 4), "traffic": None,
-                         "kernel": "gemv_kernel", "peak_kind": peak_kind},
+                         "kernel": head_kernel, "peak_kind": peak_kind},
             "sweep": sweep, "clocks": clocks}
 
 

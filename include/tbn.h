@@ -11,7 +11,8 @@
  *   tbn_unpack          packed codes -> int8 W~ or dequantized alpha W~
  *   tbn_conv2d_fwd      convolution with alpha W~ (Eq. 1)
  *   tbn_linear_fwd      fully-connected layer, treated as a convolution
- *                       (Section 3)
+ *                       (Section 3); tbn_linear_fwd_ws with caller-owned
+ *                       scratch for the batch-1 fp32 table-lookup GEMV
  *   tbn_maxpool2d_nhwc, tbn_nchw_to_nhwc   network glue between layers
  *
  * Conventions shared by every call
@@ -41,8 +42,9 @@
  *   0..7, half h in {0, 1}) has its m bit at bit 16h + p and its s bit at
  *   bit 16h + 8 + p: byte 0 = m of the even codes, byte 1 = s of the even
  *   codes, byte 2 = m of the odd codes, byte 3 = s of the odd codes.  A pair
- *   of codes then decodes to two bf16 values with one mask, one shift and one
- *   OR, which is what the kernels do;
+ *   of codes then decodes to two bf16 values with one mask and one
+ *   multiply-add (the tensor-core kernels), and the four (m, s) nibble pairs
+ *   of a byte pair index the table-lookup GEMV's tables directly;
  * - unused codes of a filter's last word have m = s = 0;
  * - codes[K][ceil(n/16)] plus alpha[K] (fp32) is the complete inference
  *   form of a layer: inference reads nothing else of the layer (Section 3).
@@ -55,13 +57,14 @@
 #ifndef TBN_H
 #define TBN_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 2
+#define TBN_ABI_VERSION 3
 
 typedef enum {
   TBN_OK = 0,
@@ -210,12 +213,38 @@ tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N
 /* Fully-connected layer (Section 3: treated as a convolution):
  *   y[b,k] = alpha[k] * sum_j x[b,j] W~[k,j]
  * x [B][K_in] (fp32 or bf16), codes [K_out][tbn_packed_words(K_in)],
- * alpha [K_out], y [B][K_out] (fp32 or bf16), optional epilogue.
- * B <= 8 with bf16 x, K_in % 16 == 0 and 16-byte aligned x and codes runs
- * the tensor-core GEMV; other shapes run as a 1x1 convolution. */
+ * alpha [K_out], y [B][K_out] (fp32 or bf16), optional epilogue (ReLU,
+ * residual [B][K_out] of y's dtype; pool is invalid here).
+ * Equivalent to tbn_linear_fwd_ws with no workspace: bf16 x with B <= 8,
+ * K_in % 64 == 0 and 16-byte aligned x and codes runs the tensor-core GEMV;
+ * fp32 x with B == 1, K_in <= 512 (K_in % 64 == 0) the table-lookup GEMV;
+ * every other shape a 1x1 convolution. */
 tbn_status tbn_linear_fwd(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
                           const uint32_t *codes, const float *alpha, int64_t K_out, void *y,
                           tbn_dtype ydt, const tbn_epilogue *epi, tbn_stream stream);
+
+/* Device scratch bytes tbn_linear_fwd_ws needs to run this shape on the
+ * table-lookup GEMV (host-only query): 0 when that kernel does not apply
+ * (it takes fp32 x, B == 1, K_in % 64 == 0) or needs no scratch
+ * (K_in <= 512); otherwise 4 * ceil(K_in / 512) * 128 * ceil(K_out / 128)
+ * bytes rounded up to 256. */
+size_t tbn_linear_workspace_bytes(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out);
+
+/* tbn_linear_fwd with caller-owned device scratch.  When x is fp32, B == 1,
+ * K_in % 64 == 0, codes are 16-byte aligned and workspace_bytes >=
+ * tbn_linear_workspace_bytes(...), the layer runs on the table-lookup GEMV:
+ * for every group of four inputs the kernel tabulates the 256 possible sums
+ * of the four two-bit weights times those inputs (fp32, products exact),
+ * and each packed code word costs four table lookups.  The fp32 partial sum
+ * of every row over each chunk of 512 inputs goes to `workspace` (256-byte
+ * aligned, contents on entry irrelevant), and a second kernel on `stream`
+ * adds them in chunk order, so results are bitwise reproducible.  Calls
+ * that may run concurrently must not share a workspace.  Otherwise the call
+ * behaves as tbn_linear_fwd and does not touch `workspace` (NULL allowed). */
+tbn_status tbn_linear_fwd_ws(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                             const uint32_t *codes, const float *alpha, int64_t K_out, void *y,
+                             tbn_dtype ydt, const tbn_epilogue *epi, void *workspace,
+                             size_t workspace_bytes, tbn_stream stream);
 
 /* Max pooling over NHWC (network glue): window kh x kw, stride sh x sw, no
  * padding; x [N][H][W][C] -> y [N][Ho][Wo][C], Ho = (H - kh)/sh + 1. */

@@ -277,9 +277,14 @@ tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N
   return pick_algo(p);
 }
 
-tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
-                          const uint32_t* codes, const float* alpha, int64_t K_out, void* y,
-                          tbn_dtype ydt, const tbn_epilogue* epi, tbn_stream stream) {
+}  // extern "C"
+
+namespace {
+
+// Host-side checks shared by the linear entry points.
+tbn_status validate_linear(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                           const uint32_t* codes, const float* alpha, int64_t K_out, void* y,
+                           tbn_dtype ydt, const tbn_epilogue* epi) {
   if (!x || !codes || !alpha || !y) return fail(TBN_ERR_INVALID_ARG, "linear: null pointer");
   if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad x dtype");
   if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad y dtype");
@@ -291,9 +296,46 @@ tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
       !is_aligned(alpha, 4) || (epi && epi->residual && !is_aligned(epi->residual, ys)))
     return fail(TBN_ERR_MISALIGNED, "linear: pointer not aligned to its element size");
   if (epi && epi->pool != 0) return fail(TBN_ERR_INVALID_ARG, "linear: pool is not defined");
+  return TBN_OK;
+}
+
+bool linear_uses_table(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out,
+                       const uint32_t* codes) {
+  return gemv_lut_unsupported_reason(xdt, B, K_in, K_out, codes)[0] == '\0';
+}
+
+}  // namespace
+
+extern "C" {
+
+tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                          const uint32_t* codes, const float* alpha, int64_t K_out, void* y,
+                          tbn_dtype ydt, const tbn_epilogue* epi, tbn_stream stream) {
+  return tbn_linear_fwd_ws(x, xdt, B, K_in, codes, alpha, K_out, y, ydt, epi, nullptr, 0, stream);
+}
+
+size_t tbn_linear_workspace_bytes(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out) {
+  if ((xdt != TBN_F32 && xdt != TBN_BF16) || B < 1 || K_in < 1 || K_out < 1) return 0;
+  if (gemv_lut_shape_reason(xdt, B, K_in, K_out)[0] != '\0') return 0;
+  return gemv_lut_workspace_bytes(K_in, K_out);
+}
+
+tbn_status tbn_linear_fwd_ws(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                             const uint32_t* codes, const float* alpha, int64_t K_out, void* y,
+                             tbn_dtype ydt, const tbn_epilogue* epi, void* workspace,
+                             size_t workspace_bytes, tbn_stream stream) {
+  const tbn_status st = validate_linear(x, xdt, B, K_in, codes, alpha, K_out, y, ydt, epi);
+  if (st != TBN_OK) return st;
+  const int relu = epi ? epi->relu : 0;
+  const void* residual = epi ? epi->residual : nullptr;
+  if (linear_uses_table(xdt, B, K_in, K_out, codes) &&
+      workspace_bytes >= gemv_lut_workspace_bytes(K_in, K_out)) {
+    return launch_gemv_lut(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, workspace,
+                           workspace_bytes, as_stream(stream));
+  }
   if (gemv_unsupported_reason(x, xdt, B, K_in, codes)[0] == '\0') {
-    return launch_gemv(x, B, K_in, codes, alpha, K_out, y, ydt, epi ? epi->relu : 0,
-                       epi ? epi->residual : nullptr, as_stream(stream));
+    return launch_gemv(x, B, K_in, codes, alpha, K_out, y, ydt, relu, residual,
+                       as_stream(stream));
   }
   // a fully-connected layer is a 1x1 convolution over a 1x1 image (Section 3)
   return tbn_conv2d_fwd(x, xdt, TBN_NHWC, B, K_in, 1, 1, codes, alpha, K_out, 1, 1, 1, 1, 0, 0, y,

@@ -15,8 +15,11 @@
 //   B batch rows laid out [64 chunks][B][8 bf16], so the eight batch rows
 //   of one 8-wide chunk are one contiguous 128-byte ldmatrix read.
 // * Sixteen consumer warps: P = 16 / n_t warps per tile split the tile's
-//   stages (stage ks goes to warp ks % P of the tile) and their partial sums
-//   are added in a fixed order.  Per K step of 16 a warp runs
+//   stages (ring iteration i of the CTA goes to warp i % P of each tile) and
+//   their partial sums are added in a fixed order.  The ring depth is a
+//   multiple of P, so the previous use of the slot a warp waits on was that
+//   warp's own: a slot is never more than one phase ahead of its waiter,
+//   which is what a parity wait on an mbarrier can tell apart.  Per K step of 16 a warp runs
 //   one mma.m16n8k16: A = 16 rows x 16 codes decoded in registers to bf16
 //   W~/2, B = 16 inputs x 8 batch columns (lanes past B read batch row
 //   n mod B, which only fills mma columns that are dropped), fp32
@@ -291,7 +294,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ------------------------------------------------------------ consumers
   const int g = lane >> 2, t = lane & 3;
   const PairDecode dec(t);
-  // warp w works on tile w / P of the band, stages ks with ks % P == w % P
+  // warp w works on tile w / P of the band, ring iterations i with
+  // i % P == w % P (i = r * nks + ks for stage ks of round r)
   const int P = a.P;
   const int tau = warp / P, pi = warp % P;
   const bool active = tau < a.n_t;
@@ -300,8 +304,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t x_lane_off =
       static_cast<uint32_t>(((lane >> 3) * kB + (lane & 7) % kB) * 16);
 
-  int it_slot = 0;            // ring slot of the band's first stage
-  uint32_t it_parity = 0;     // full-barrier parity of that stage
   for (int r = 0; r < a.rounds; ++r) {
     const int band = blockIdx.x + r * gridDim.x;
     if (band * a.n_t >= a.T) break;
@@ -310,12 +312,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int q = 0; q < 2; ++q)
 #pragma unroll
       for (int i = 0; i < 4; ++i) c[q][i] = 0.0f;
-    // this warp takes stages pi, pi + P, ...; slot / parity of stage `it`
-    // advance incrementally (P may exceed the ring depth)
-    int slot = it_slot, ks = pi;
-    uint32_t parity = it_parity;
-    for (int q = 0; q < pi; ++q)
-      if (++slot == a.stages) { slot = 0; parity ^= 1u; }
+    // this warp's first stage of the band and its ring slot / parity; the
+    // slot then advances by P, which divides the ring depth
+    const int band_it = r * a.nks;
+    int ks = ((pi - band_it) % P + P) % P;
+    int slot = (band_it + ks) % a.stages;
+    uint32_t parity = static_cast<uint32_t>(((band_it + ks) / a.stages) & 1);
     for (; active && ks < a.nks; ks += P) {
       const bool ok_lane = mbar_wait_sleep(&full_bar[slot], parity, &abort_flag, a.err,
                                            kWaitLimitNs);
@@ -326,12 +328,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty_bar[slot]);
-      for (int q = 0; q < P; ++q)
-        if (++slot == a.stages) { slot = 0; parity ^= 1u; }
+      slot += P;   // slot % P == this warp's residue; wrap past the end
+      if (slot >= a.stages) {
+        slot -= a.stages;
+        parity ^= 1u;
+      }
     }
-    // the band consumed nks stages of the ring
-    for (int q = 0; q < a.nks; ++q)
-      if (++it_slot == a.stages) { it_slot = 0; it_parity ^= 1u; }
     float d[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) d[i] = c[0][i] + c[1][i];
@@ -384,6 +386,7 @@ GemvPlan plan_gemv(int64_t B, int64_t K_in, int64_t K_out, int sms) {
   p.stage_bytes = p.w_bytes + static_cast<uint32_t>(B) * 1024u;
   p.stages = static_cast<int>(kSmemBudget / p.stage_bytes);
   if (p.stages > kMaxStages) p.stages = kMaxStages;
+  p.stages -= p.stages % p.P;   // a multiple of P (see the consumer loop)
   p.smem = static_cast<size_t>(p.stages) * p.stage_bytes + 1024;
   return p;
 }
@@ -406,7 +409,8 @@ tbn_status launch_gemv(const void* x, int64_t B, int64_t K_in, const uint32_t* c
                        const void* residual, cudaStream_t s) {
   if (K_out >= (1ll << 31) - 16) return fail(TBN_ERR_INVALID_ARG, "GEMV: K_out too large");
   const GemvPlan p = plan_gemv(B, K_in, K_out, device_sm_count());
-  if (p.stages < 2) return fail(TBN_ERR_UNSUPPORTED, "GEMV: stage does not fit shared memory");
+  if (p.stages < 2 || p.stages < p.P)
+    return fail(TBN_ERR_UNSUPPORTED, "GEMV: stage does not fit shared memory");
 
   alignas(64) CUtensorMap tmap_w, tmap_x;
   {

@@ -81,6 +81,16 @@ tbn_status launch_gemv(const void* x, int64_t B, int64_t K_in, const uint32_t* c
                        const float* alpha, int64_t K_out, void* y, tbn_dtype ydt, int relu,
                        const void* residual, cudaStream_t s);
 
+// Batch-1 table-lookup GEMV for fp32 activations (tbn_gemv_lut.cu).
+const char* gemv_lut_shape_reason(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out);
+const char* gemv_lut_unsupported_reason(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out,
+                                        const uint32_t* codes);
+size_t gemv_lut_workspace_bytes(int64_t K_in, int64_t K_out);
+tbn_status launch_gemv_lut(const void* x, int64_t K_in, const uint32_t* codes,
+                           const float* alpha, int64_t K_out, void* y, tbn_dtype ydt, int relu,
+                           const void* residual, void* workspace, size_t workspace_bytes,
+                           cudaStream_t s);
+
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
                                void* y, cudaStream_t s);

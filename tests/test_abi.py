@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 2
+    assert L.tbn_abi_version() == 3
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -109,8 +109,27 @@ def test_linear_and_glue_reject_bad_arguments(L):
     d = ctypes.c_void_p(256)
     assert L.tbn_linear_fwd(None, 1, 1, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_linear_fwd(d, 1, 0, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_linear_fwd_ws(None, 1, 1, 64, d, d, 8, d, 1, None, d, 4096, None) == \
+        tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_linear_fwd_ws(d, 1, 1, 64, d, d, 8, ctypes.c_void_p(257), 1, None, d, 4096,
+                               None) == tbn.TBN_ERR_MISALIGNED
     assert L.tbn_maxpool2d_nhwc(d, 1, 1, 4, 4, 8, 5, 5, 1, 1, d, None) == tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_nchw_to_nhwc(d, 1, 1, 4, 4, 4, 3, d, None) == tbn.TBN_ERR_INVALID_ARG
+
+
+def test_linear_workspace_query(L):
+    """Scratch of the batch-1 fp32 table GEMV: the fp32 partial sum of every
+    512-input chunk for each row (rows rounded up to blocks of 128), rounded
+    to 256 bytes; none for one chunk or where the kernel does not apply."""
+    f32 = __import__("torch").float32
+    ws = lambda B, K_in, K_out: tbn.tbn_linear_workspace_bytes(B, K_in, K_out, f32)
+    assert ws(1, 16384, 16384) == 32 * 16384 * 4
+    assert ws(1, 4096, 1000) == 8 * 1024 * 4
+    assert ws(1, 576, 33) == 2 * 128 * 4
+    assert ws(1, 512, 4096) == 0            # one chunk: results written directly
+    assert ws(2, 4096, 4096) == 0           # batch > 1
+    assert ws(1, 4000, 4096) == 0           # K_in % 64 != 0: no TMA rows
+    assert tbn.tbn_linear_workspace_bytes(1, 4096, 4096) == 0   # bf16 x: tensor-core GEMV
 
 
 def test_python_binding_requires_cuda_tensors():
