@@ -246,6 +246,25 @@ tbn_status tbn_linear_fwd_ws(const void *x, tbn_dtype xdt, int64_t B, int64_t K_
                              tbn_dtype ydt, const tbn_epilogue *epi, void *workspace,
                              size_t workspace_bytes, tbn_stream stream);
 
+/* tbn_linear_fwd_ws for callers that cannot allocate device memory (the
+ * paper has no counterpart; this is a deployment variant of the same
+ * computation).  It runs only the table-lookup GEMV (fp32 x, B == 1,
+ * K_in % 64 == 0, 16-byte aligned codes; otherwise TBN_ERR_UNSUPPORTED) and
+ * keeps its chunk partial sums in a 4 MiB array inside the library's own
+ * device module instead of a caller's workspace: layers needing more,
+ * tbn_linear_workspace_bytes(...) > 4 MiB (e.g. more than 32768 outputs at
+ * 16384 inputs), return TBN_ERR_UNSUPPORTED before launching.  Nothing in
+ * the array needs clearing between calls.  There is one array per device
+ * and process: calls that could run concurrently (other streams, other
+ * host threads) race on it and must be serialized by the caller.  The
+ * first call on each device resolves the array's address
+ * (cudaGetSymbolAddress); make it before any stream capture.  Results are
+ * bitwise equal to tbn_linear_fwd_ws's. */
+tbn_status tbn_linear_fwd_noalloc(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                                  const uint32_t *codes, const float *alpha, int64_t K_out,
+                                  void *y, tbn_dtype ydt, const tbn_epilogue *epi,
+                                  tbn_stream stream);
+
 /* Max pooling over NHWC (network glue): window kh x kw, stride sh x sw, no
  * padding; x [N][H][W][C] -> y [N][Ho][Wo][C], Ho = (H - kh)/sh + 1. */
 tbn_status tbn_maxpool2d_nhwc(const void *x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,

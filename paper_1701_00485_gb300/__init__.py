@@ -22,8 +22,8 @@ import torch
 __all__ = [
     "TBNError", "lib", "lib_path", "packed_words",
     "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack", "tbn_conv2d_fwd",
-    "tbn_linear_fwd", "tbn_linear_fwd_ws", "tbn_linear_workspace_bytes", "tbn_maxpool2d_nhwc",
-    "tbn_nchw_to_nhwc", "tbn_device_error",
+    "tbn_linear_fwd", "tbn_linear_fwd_ws", "tbn_linear_workspace_bytes",
+    "tbn_linear_fwd_noalloc", "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_device_error",
     "tbn_conv2d_select_algo", "conv_out_hw",
     "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
@@ -46,7 +46,8 @@ EXPORTED = [
     "tbn_abi_version", "tbn_packed_words", "tbn_status_string", "tbn_last_error",
     "tbn_device_error", "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack",
     "tbn_conv2d_fwd", "tbn_conv2d_fwd_algo", "tbn_conv2d_select_algo", "tbn_linear_fwd",
-    "tbn_linear_workspace_bytes", "tbn_linear_fwd_ws", "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc",
+    "tbn_linear_workspace_bytes", "tbn_linear_fwd_ws", "tbn_linear_fwd_noalloc",
+    "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc",
 ]
 
 
@@ -109,6 +110,8 @@ def lib():
             "tbn_linear_workspace_bytes": ([I32, I64, I64, I64], ctypes.c_size_t),
             "tbn_linear_fwd_ws": ([P, I32, I64, I64, U32P, P, I64, P, I32,
                                    ctypes.POINTER(Epilogue), P, ctypes.c_size_t, P], I32),
+            "tbn_linear_fwd_noalloc": ([P, I32, I64, I64, U32P, P, I64, P, I32,
+                                        ctypes.POINTER(Epilogue), P], I32),
             "tbn_maxpool2d_nhwc": ([P, I32, I64, I64, I64, I64, I64, I64, I64, I64, P, P], I32),
             "tbn_nchw_to_nhwc": ([P, I32, I64, I64, I64, I64, I64, P, P], I32),
         }
@@ -305,6 +308,26 @@ def tbn_linear_fwd_ws(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor,
                                    ctypes.byref(e) if e is not None else None, ws_ptr, ws_bytes,
                                    _stream(stream)),
            "tbn_linear_fwd_ws")
+    return out
+
+
+def tbn_linear_fwd_noalloc(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor,
+                           K_out: int, out_dtype=None, relu: bool = False,
+                           residual: torch.Tensor | None = None, out: torch.Tensor | None = None,
+                           stream=None):
+    """The batch-1 fp32 table GEMV with its scratch inside the library (the C
+    call allocates nothing; `out` is allocated here only when not given)."""
+    _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
+    B, K_in = x.shape
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    if out is None:
+        out = torch.empty((B, K_out), dtype=_torch_dt(ydt), device=x.device)
+    e = _epi(relu, residual)
+    _check(lib().tbn_linear_fwd_noalloc(x.data_ptr(), _dt(x), B, K_in, codes.data_ptr(),
+                                        alpha.data_ptr(), K_out, out.data_ptr(), ydt,
+                                        ctypes.byref(e) if e is not None else None,
+                                        _stream(stream)),
+           "tbn_linear_fwd_noalloc")
     return out
 
 

@@ -342,6 +342,18 @@ tbn_status tbn_linear_fwd_ws(const void* x, tbn_dtype xdt, int64_t B, int64_t K_
                         ydt, epi, stream);
 }
 
+tbn_status tbn_linear_fwd_noalloc(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                                  const uint32_t* codes, const float* alpha, int64_t K_out,
+                                  void* y, tbn_dtype ydt, const tbn_epilogue* epi,
+                                  tbn_stream stream) {
+  const tbn_status st = validate_linear(x, xdt, B, K_in, codes, alpha, K_out, y, ydt, epi);
+  if (st != TBN_OK) return st;
+  const char* why = gemv_lut_unsupported_reason(xdt, B, K_in, K_out, codes);
+  if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "linear (no-alloc): %s", why);
+  return launch_gemv_lut_static(x, K_in, codes, alpha, K_out, y, ydt, epi ? epi->relu : 0,
+                                epi ? epi->residual : nullptr, as_stream(stream));
+}
+
 tbn_status tbn_maxpool2d_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                               int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw, void* y,
                               tbn_stream stream) {

@@ -472,4 +472,50 @@ tbn_status launch_gemv_lut(const void* x, int64_t K_in, const uint32_t* codes,
   return check_launch("gemv_lut_reduce_kernel");
 }
 
+// ---- the same kernel with file-scope scratch (tbn_linear_fwd_noalloc) ----
+// Chunk partial sums for callers that cannot allocate device memory: a
+// fixed array in the library's own module, enough for any layer whose
+// table-GEMV scratch is at most 4 MiB (e.g. 16384 inputs x 32768 outputs).
+// One array per device and process, so calls that could overlap race.
+constexpr size_t kStaticScratchBytes = size_t(4) << 20;
+static __device__ __align__(256) uint8_t g_lut_scratch[kStaticScratchBytes];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+}  // namespace
+
+size_t gemv_lut_static_scratch_bytes() { return kStaticScratchBytes; }
+
+tbn_status launch_gemv_lut_static(const void* x, int64_t K_in, const uint32_t* codes,
+                                  const float* alpha, int64_t K_out, void* y, tbn_dtype ydt,
+                                  int relu, const void* residual, cudaStream_t s) {
+  const size_t need = gemv_lut_workspace_bytes(K_in, K_out);
+  if (need > kStaticScratchBytes)
+    return fail(TBN_ERR_UNSUPPORTED,
+                "linear (no-alloc): %zu bytes of scratch needed, the static scratch has %zu",
+                need, kStaticScratchBytes);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices)
+    return fail(TBN_ERR_UNSUPPORTED, "linear (no-alloc): device ordinal %d out of range", dev);
+  void* ptr = nullptr;
+  {
+    // set-up once per device, with that device current
+    std::lock_guard<std::mutex> lock(g_scratch_mutex);
+    if (g_scratch_ptr[dev] == nullptr) {
+      e = cudaGetSymbolAddress(&g_scratch_ptr[dev], g_lut_scratch);
+      if (e != cudaSuccess) {
+        g_scratch_ptr[dev] = nullptr;
+        return cuda_fail(e, "cudaGetSymbolAddress(table GEMV scratch)");
+      }
+    }
+    ptr = g_scratch_ptr[dev];
+  }
+  return launch_gemv_lut(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, ptr,
+                         kStaticScratchBytes, s);
+}
+
 }  // namespace tbn

@@ -91,6 +91,12 @@ tbn_status launch_gemv_lut(const void* x, int64_t K_in, const uint32_t* codes,
                            const void* residual, void* workspace, size_t workspace_bytes,
                            cudaStream_t s);
 
+// The table GEMV with its scratch in a file-scope device array.
+size_t gemv_lut_static_scratch_bytes();
+tbn_status launch_gemv_lut_static(const void* x, int64_t K_in, const uint32_t* codes,
+                                  const float* alpha, int64_t K_out, void* y, tbn_dtype ydt,
+                                  int relu, const void* residual, cudaStream_t s);
+
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
                                void* y, cudaStream_t s);
