@@ -42,7 +42,9 @@
 // Warp roles (every role is a whole warp that waits on the barriers; where a
 // single thread must issue -- TMA copies, MMAs, commits -- one elected lane
 // does, with warp-uniform operands):
-//   warp 0        TMA producer (TMA mode)
+//   warps 0, 18.. TMA producers (TMA mode), taking K blocks in turn: one
+//                 issuing thread delivers tiled boxes at a limited rate, so
+//                 several keep the activation ring fuller
 //   warp 1        TMEM allocator + MMA issuer
 //   warps 2-9     expanders
 //   warps 10-17   epilogue
@@ -74,6 +76,8 @@ constexpr int kTmemCols = 512;      // accumulator [0,256) + weight ring [256,41
 constexpr int kExpWarps = 8;
 constexpr int kEpiWarps = 8;
 constexpr int kGatherWarps = 4;
+constexpr int kTmaProducers = 2;    // TMA mode: warp 0 and warps 18 .. 18 + kTmaProducers - 2
+static_assert(kTmaProducers <= kStages, "a producer's parity wait needs kStages >= producers");
 constexpr int kFirstExpWarp = 2;
 constexpr int kFirstEpiWarp = kFirstExpWarp + kExpWarps;
 constexpr int kFirstGatherWarp = kFirstEpiWarp + kEpiWarps;
@@ -85,7 +89,7 @@ static_assert(kAccCols + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
 template <bool kGather>
 constexpr int threads_for() {
-  return 32 * (kFirstGatherWarp + (kGather ? kGatherWarps : 0));
+  return 32 * (kFirstGatherWarp + (kGather ? kGatherWarps : kTmaProducers - 1));
 }
 
 struct IgArgs {
@@ -251,8 +255,14 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
   const uint32_t acc_tmem = tmem;               // columns [0, 256)
   const uint32_t a_tmem0 = tmem + kAccCols;     // weight ring
 
-  if (!kGather && warp == 0) {
-    // ================= TMA producer =================
+  if (!kGather && (warp == 0 || warp >= kFirstGatherWarp)) {
+    // ================= TMA producers =================
+    // producer pid issues the K blocks g with g % kTmaProducers == pid; the
+    // ring has at least as many stages as producers, so the release a
+    // producer waits for always follows the previous release of that slot
+    // (the MMA warp releases in order) and its parity wait cannot alias
+    const int pid = warp == 0 ? 0 : warp - kFirstGatherWarp + 1;
+    int turn = 0;   // g % kTmaProducers
     const uint32_t box_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBK * 2);
     const int cblocks = a.C / kBK;
     int g = 0;  // global K-block counter of this CTA
@@ -261,6 +271,12 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       const TileCoord tc = tile_coord(a, t);
       int tap = 0, cb = 0;
       for (int kb = 0; kb < KB; ++kb, ++g) {
+        const bool mine = turn == pid;
+        if (++turn == kTmaProducers) turn = 0;
+        if (!mine) {
+          if (++cb == cblocks) { cb = 0; ++tap; }
+          continue;
+        }
         const int sb = g % kStages;
         const uint32_t it = static_cast<uint32_t>(g / kStages);
         ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
@@ -275,10 +291,11 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
         if (++cb == cblocks) { cb = 0; ++tap; }
       }
     }
-    // drain: every issued copy must land before the CTA may exit
+    // drain: every copy this warp issued must land before the CTA may exit
     for (int i = g > kStages ? g - kStages : 0; i < g; ++i)
-      mbar_wait(&ctl->full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, nullptr,
-                a.err, kWaitLimitNs);
+      if (i % kTmaProducers == pid)
+        mbar_wait(&ctl->full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, nullptr,
+                  a.err, kWaitLimitNs);
   } else if (kGather && warp >= kFirstGatherWarp) {
     // ================= gather producers =================
     // The gather warps meet at a named barrier every K block, so none of them
