@@ -14,6 +14,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <mutex>
 #include <cstdint>
 
 #include "tbn_device.cuh"
@@ -261,6 +262,43 @@ __global__ void __launch_bounds__(256) nchw_to_nhwc_kernel(const T* __restrict__
     dst[c] = c < C ? src[static_cast<int64_t>(c) * HW] : from_f32<T>(0.0f);
 }
 
+// bf16 with H*W % 8 == 0 and 16-byte aligned tensors, Cp <= 8: one thread
+// per 8 consecutive pixels of one image reads one 16-byte vector from each of
+// the C planes and writes the 8 pixels' Cp channels as Cp 16-byte vectors.
+template <int kCp>
+__global__ void __launch_bounds__(256) nchw_to_nhwc_bf16x8_kernel(const uint4* __restrict__ x,
+                                                                  int C, int HW8, int64_t total,
+                                                                  uint4* __restrict__ y) {
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
+  if (t >= total) return;
+  const int64_t b = t / HW8;
+  const int hw8 = static_cast<int>(t - b * HW8);
+  uint32_t in[kCp][4];
+#pragma unroll
+  for (int c = 0; c < kCp; ++c) {
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (c < C) v = x[(b * C + c) * HW8 + hw8];
+    in[c][0] = v.x;
+    in[c][1] = v.y;
+    in[c][2] = v.z;
+    in[c][3] = v.w;
+  }
+  uint4* dst = y + t * kCp;
+#pragma unroll
+  for (int o = 0; o < kCp; ++o) {
+    uint32_t w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      // output elements e = 8 o + 2 k, 8 o + 2 k + 1 -> (pixel e / kCp, channel e % kCp)
+      const int e0 = 8 * o + 2 * k, e1 = e0 + 1;
+      const uint32_t lo = (in[e0 % kCp][(e0 / kCp) >> 1] >> (16 * ((e0 / kCp) & 1))) & 0xFFFFu;
+      const uint32_t hi = (in[e1 % kCp][(e1 / kCp) >> 1] >> (16 * ((e1 / kCp) & 1))) & 0xFFFFu;
+      w[k] = lo | (hi << 16);
+    }
+    dst[o] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 int64_t grid_for(int64_t total) {
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 16;
   return std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, cap));
@@ -320,6 +358,46 @@ tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C
                                int64_t W, int64_t C_pad, void* y, cudaStream_t s) {
   if (N > 65535 || H * W >= (int64_t(1) << 31) - 256 || C_pad >= (int64_t(1) << 31))
     return fail(TBN_ERR_UNSUPPORTED, "nchw_to_nhwc: N > 65535 or H*W too large");
+  // the shared-memory split of the kernels around it in a network (which
+  // need nearly all of it): no SM reconfiguration between launches
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    const void* fns[10] = {(const void*)nchw_to_nhwc_bf16x8_kernel<1>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<2>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<3>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<4>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<5>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<6>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<7>,
+                           (const void*)nchw_to_nhwc_bf16x8_kernel<8>,
+                           (const void*)nchw_to_nhwc_kernel<__nv_bfloat16>,
+                           (const void*)nchw_to_nhwc_kernel<float>};
+    for (const void* f : fns) {
+      const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+      if (e != cudaSuccess && attr_err == cudaSuccess) attr_err = e;
+    }
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(nchw_to_nhwc)");
+  if (dt == TBN_BF16 && (H * W) % 8 == 0 && C_pad <= 8 && is_aligned(x, 16) && is_aligned(y, 16)) {
+    const int HW8 = static_cast<int>(H * W / 8);
+    const int64_t total = N * HW8;
+    const unsigned blocks = static_cast<unsigned>((total + 255) / 256);
+    const uint4* xv = static_cast<const uint4*>(x);
+    uint4* yv = static_cast<uint4*>(y);
+    const int c = static_cast<int>(C);
+    switch (C_pad) {
+      case 1: nchw_to_nhwc_bf16x8_kernel<1><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 2: nchw_to_nhwc_bf16x8_kernel<2><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 3: nchw_to_nhwc_bf16x8_kernel<3><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 4: nchw_to_nhwc_bf16x8_kernel<4><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 5: nchw_to_nhwc_bf16x8_kernel<5><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 6: nchw_to_nhwc_bf16x8_kernel<6><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      case 7: nchw_to_nhwc_bf16x8_kernel<7><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+      default: nchw_to_nhwc_bf16x8_kernel<8><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
+    }
+    return check_launch("nchw_to_nhwc_bf16x8_kernel");
+  }
   const dim3 grid(static_cast<unsigned>((H * W + 255) / 256), static_cast<unsigned>(N));
   if (dt == TBN_BF16)
     nchw_to_nhwc_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(

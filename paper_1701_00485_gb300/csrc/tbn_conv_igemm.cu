@@ -847,8 +847,10 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64 || !attr_done[kGather][pidx][kTmaStore][dev]) {
-    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(conv_igemm_kernel)");
     if (dev >= 0 && dev < 64) attr_done[kGather][pidx][kTmaStore][dev] = true;
   }

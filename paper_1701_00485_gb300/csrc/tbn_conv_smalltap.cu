@@ -458,9 +458,14 @@ tbn_status launch_conv_smalltap(const ConvProblem& p, cudaStream_t s) {
                           (const void*)conv_smalltap_kernel<64, true>};
     const int kps[4] = {32, 32, 64, 64};
     const bool st[4] = {false, true, false, true};
-    for (int i = 0; i < 4 && attr_err == cudaSuccess; ++i)
+    for (int i = 0; i < 4 && attr_err == cudaSuccess; ++i) {
       attr_err = cudaFuncSetAttribute(fns[i], cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       (int)smalltap_smem(kps[i], st[i], kMaxPatchBytes));
+      // the same shared-memory split as the network's other kernels: no
+      // reconfiguration of the SMs between consecutive launches
+      if (attr_err == cudaSuccess)
+        attr_err = cudaFuncSetAttribute(fns[i], cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    }
   });
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(smalltap)");
 

@@ -106,5 +106,20 @@ def test_nchw_to_nhwc_padding(dt):
     assert torch.all(y[..., 3:] == 0)
 
 
+@pytest.mark.parametrize("N,C,H,W,C_pad", [(3, 1, 8, 16, 1), (3, 3, 8, 16, 3), (2, 3, 4, 6, 4),
+                                           (2, 2, 8, 8, 5), (3, 3, 8, 16, 8), (1, 7, 16, 8, 7),
+                                           (2, 8, 8, 8, 8), (128, 3, 32, 32, 3),
+                                           (2, 3, 5, 8, 3)])
+def test_nchw_to_nhwc_vector_path(N, C, H, W, C_pad):
+    """bf16 with H*W % 8 == 0 takes the 8-pixel vector kernel (C_pad <= 8):
+    every element and the zero padding, exactly."""
+    g = inputs.generator(N * 100 + C * 10 + C_pad)
+    x = torch.randn(N, C, H, W, generator=g).to(torch.bfloat16)
+    y = tbn.tbn_nchw_to_nhwc(x.cuda(), C_pad=C_pad).cpu()
+    want = torch.zeros(N, H, W, C_pad, dtype=torch.bfloat16)
+    want[..., :C] = x.permute(0, 2, 3, 1)
+    assert torch.equal(y, want)
+
+
 def test_device_error_word_is_clear():
     assert tbn.tbn_device_error() == 0
