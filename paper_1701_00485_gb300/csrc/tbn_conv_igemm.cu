@@ -51,6 +51,17 @@
 //   warps 18-21   gather producers (gather mode only)
 // Every wait is bounded (tbn_device.cuh); on a timeout the CTA records the
 // error, drains its own in-flight copies and MMAs, frees TMEM and returns.
+//
+// The kernel is launched as a programmatic dependent of the previous kernel
+// on the stream: its start-up (TMEM allocation, barrier set-up, loading and
+// decoding the first blocks of codes) may overlap the previous kernel's last
+// wave, and only the reads of activations and of the residual wait for that
+// kernel to complete (grid_dependency_wait).  Codes and alpha are read
+// before that wait, so they must not be written by the immediately
+// preceding kernel when that kernel is one of this library's convolutions
+// (which let their dependents start early); no convolution writes anything
+// but its output.  Each CTA lets its own dependents start once it has passed
+// its wait, so everything older than the previous kernel is complete by then.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -257,6 +268,8 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
 
   if (!kGather && (warp == 0 || warp >= kFirstGatherWarp)) {
     // ================= TMA producers =================
+    grid_dependency_wait();   // activations may come from the previous kernel
+    grid_dependents_launch();
     // producer pid issues the K blocks g with g % kTmaProducers == pid; the
     // ring has at least as many stages as producers, so the release a
     // producer waits for always follows the previous release of that slot
@@ -303,6 +316,8 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
     // loop structure (reaching every barrier) but does no more work.
     const int gt = threadIdx.x - 32 * kFirstGatherWarp;   // 0..127
     const bool vec = (a.C & 7) == 0;
+    grid_dependency_wait();   // activations may come from the previous kernel
+    grid_dependents_launch();
     int g = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < a.tiles; t += gridDim.x) {
@@ -503,6 +518,7 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
     const int Qo = kPoolBW ? a.Q / 2 : a.Q;
     const uint32_t res_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBM * 2);
     __nv_bfloat16* stage = reinterpret_cast<__nv_bfloat16*>(out_stage);
+    grid_dependency_wait();   // the residual may come from the previous kernel
     uint32_t tiles_done = 0;
     bool ok = true;
     // The epilogue warps meet at named barriers, so after a failed wait they
@@ -855,7 +871,18 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
     if (dev >= 0 && dev < 64) attr_done[kGather][pidx][kTmaStore][dev] = true;
   }
   const int grid = std::min(a.tiles, device_sm_count());
-  kern<<<grid, threads_for<kGather>(), kSmemBytes, s>>>(tmap_x, tmap_y, tmap_res, a);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(threads_for<kGather>());
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, tmap_x, tmap_y, tmap_res, a);
+  if (le != cudaSuccess) return cuda_fail(le, "cudaLaunchKernelEx(conv_igemm_kernel)");
   return check_launch("conv_igemm_kernel");
 }
 

@@ -20,6 +20,9 @@
 //      fragments straight to global memory (each pixel's 8 consecutive
 //      filters of an n-tile are 16 contiguous bytes in NHWC).
 // CTAs are persistent (a few per SM) and walk the tiles with a grid stride.
+// Launched as a programmatic dependent of the previous kernel: the set-up
+// before the tile loop may overlap that kernel's end; activations are read
+// only after it has completed (grid_dependency_wait).
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -214,6 +217,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) conv_smalltap_kernel(Sma
   const int m_pad = (tile_px + 15) & ~15;
   const int row_elems = a.PW * a.C;
 
+  grid_dependency_wait();   // activations may come from the previous kernel
+  grid_dependents_launch();
   for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x) {
     // tile order: k-tile slowest so a CTA keeps its decoded filters
     const int kt = tile / (a.N * a.tiles_p * a.tiles_q);
@@ -472,13 +477,22 @@ tbn_status launch_conv_smalltap(const ConvProblem& p, cudaStream_t s) {
   const int64_t slots = static_cast<int64_t>(device_sm_count()) * kCtasPerSm;
   const int grid = static_cast<int>(std::min<int64_t>(tiles, slots));
   const bool staged = smalltap_staged(p);
-  if (t.KP == 32) {
-    if (staged) conv_smalltap_kernel<32, true><<<grid, kThreads, t.smem, s>>>(a);
-    else conv_smalltap_kernel<32, false><<<grid, kThreads, t.smem, s>>>(a);
-  } else {
-    if (staged) conv_smalltap_kernel<64, true><<<grid, kThreads, t.smem, s>>>(a);
-    else conv_smalltap_kernel<64, false><<<grid, kThreads, t.smem, s>>>(a);
-  }
+  void (*kern)(SmallTapArgs) = t.KP == 32 ? (staged ? conv_smalltap_kernel<32, true>
+                                                    : conv_smalltap_kernel<32, false>)
+                                          : (staged ? conv_smalltap_kernel<64, true>
+                                                    : conv_smalltap_kernel<64, false>);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = t.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, a);
+  if (le != cudaSuccess) return cuda_fail(le, "cudaLaunchKernelEx(conv_smalltap_kernel)");
   return check_launch("conv_smalltap_kernel");
 }
 

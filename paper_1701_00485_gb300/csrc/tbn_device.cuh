@@ -142,6 +142,20 @@ __device__ __forceinline__ void named_barrier_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// ------------------------------------------- programmatic dependent launch
+// Block until the grid this one depends on (the previous kernel of the
+// stream, when this grid was launched as a programmatic dependent) has
+// completed and its memory is visible; returns at once otherwise.
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Allow this grid's programmatic dependents to launch once every CTA of it
+// has called this or exited.
+__device__ __forceinline__ void grid_dependents_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 // 2-D and 3-D tiled bulk tensor loads global -> shared, completion on an
 // mbarrier (coordinates innermost first, in elements).
