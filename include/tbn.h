@@ -30,6 +30,13 @@
  *   tbn_device_error() after synchronizing.
  * - tbn_last_error() returns a human-readable detail string for the most
  *   recent failing call on the calling host thread.
+ * - The convolutions are launched as programmatic dependents of the previous
+ *   kernel on `stream`: their start-up may overlap that kernel's end, and
+ *   they read activations and residuals only after it has completed.  Codes
+ *   and alpha may be read earlier, while a previous convolution of this
+ *   library (or tbn_nchw_to_nhwc) is still finishing, so they must not be
+ *   the output of the immediately preceding call.  Everything older, and
+ *   every other kind of preceding kernel, is complete before they start.
  *
  * Two-bit storage format (the paper fixes only that each of the four values
  * takes two bits, Section 1; the layout below is this library's):

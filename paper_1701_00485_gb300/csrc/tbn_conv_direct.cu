@@ -269,6 +269,10 @@ template <int kCp>
 __global__ void __launch_bounds__(256) nchw_to_nhwc_bf16x8_kernel(const uint4* __restrict__ x,
                                                                   int C, int HW8, int64_t total,
                                                                   uint4* __restrict__ y) {
+  // the next kernel (a convolution launched as a programmatic dependent)
+  // may start its set-up now; it reads this kernel's output only after
+  // this grid has completed
+  grid_dependents_launch();
   const int64_t t = static_cast<int64_t>(blockIdx.x) * 256 + threadIdx.x;
   if (t >= total) return;
   const int64_t b = t / HW8;

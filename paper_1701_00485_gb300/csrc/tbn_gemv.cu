@@ -31,6 +31,14 @@
 // Every mbarrier wait is bounded; on expiry the kernel records a timeout in
 // the device error word, stops issuing, drains the copies it started and
 // returns.
+//
+// The kernel is launched as a programmatic dependent of the previous kernel
+// on the stream: the first ring's worth of code boxes is requested before
+// griddepcontrol.wait, the inputs (and the residual) only after it, so in a
+// chain of layers the weight stream of one starts while the previous one
+// finishes.  Codes and alpha must therefore not be the output of the
+// immediately preceding call when that call is one of this library's
+// kernels that let their dependents start early.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -245,11 +253,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     int it = 0;                      // stages issued so far
     int slot = 0;                    // it % stages
     uint32_t empty_parity = 1;       // parity of the release before use it / stages
+    auto load_x = [&](int sl, int kc) {
+      uint8_t* st = ring_ptr + static_cast<size_t>(sl) * a.stage_bytes;
+      if (kB == 1) {
+        // one batch row: the stage's inputs are 1 KB contiguous
+        tma_load_2d(st + a.w_bytes, &tmap_x, &full_bar[sl], kc * kCodesPerStage, 0);
+        tma_load_2d(st + a.w_bytes + 512, &tmap_x, &full_bar[sl], kc * kCodesPerStage + 256, 0);
+      } else {
+        tma_load_3d(st + a.w_bytes, &tmap_x, &full_bar[sl], 0, 0, kc * (kCodesPerStage / 8));
+      }
+    };
+    // The first band's first stages: codes now, inputs after the wait.
+    int deferred = 0;
+    bool waited = false;
+    auto finish_wait = [&]() {
+      grid_dependency_wait();   // the inputs may come from the previous kernel
+      grid_dependents_launch();
+      if (elected)
+        for (int i = 0; i < deferred; ++i) load_x(i, (k_start + i) % a.nks);
+      __syncwarp();
+      waited = true;
+    };
     for (int r = 0; r < a.rounds; ++r) {
       const int band = blockIdx.x + r * gridDim.x;
       if (band * a.n_t >= a.T) break;
       int kc = k_start;
       for (int ks = 0; ks < a.nks; ++ks) {
+        if (!waited && (r > 0 || it >= a.stages)) finish_wait();
         bool ok = true;
         if (it >= a.stages)
           ok = mbar_wait_sleep(&empty_bar[slot], empty_parity, &abort_flag, a.err, kWaitLimitNs);
@@ -259,16 +289,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* st = ring_ptr + static_cast<size_t>(slot) * a.stage_bytes;
           mbar_arrive_expect_tx(&full_bar[slot], a.stage_bytes);
           tma_load_2d(st, &tmap_w, &full_bar[slot], kc * kWordsPerStage, band * a.n_t * 16);
-          if (kB == 1) {
-            // one batch row: the stage's inputs are 1 KB contiguous
-            tma_load_2d(st + a.w_bytes, &tmap_x, &full_bar[slot], kc * kCodesPerStage, 0);
-            tma_load_2d(st + a.w_bytes + 512, &tmap_x, &full_bar[slot],
-                        kc * kCodesPerStage + 256, 0);
-          } else {
-            tma_load_3d(st + a.w_bytes, &tmap_x, &full_bar[slot], 0, 0,
-                        kc * (kCodesPerStage / 8));
-          }
+          if (waited) load_x(slot, kc);
         }
+        if (!waited) ++deferred;
         __syncwarp();
         ++it;
         if (++kc == a.nks) kc = 0;
@@ -279,6 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (__shfl_sync(0xffffffffu, abort_flag, 0)) break;
     }
+    if (!waited) finish_wait();
     // On abort, wait (bounded) for the last copy issued into each slot so
     // no TMA write lands after the CTA has exited.
     if (elected && abort_flag) {
@@ -292,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ------------------------------------------------------------ consumers
+  grid_dependency_wait();   // the residual may come from the previous kernel
   const int g = lane >> 2, t = lane & 3;
   const PairDecode dec(t);
   // warp w works on tile w / P of the band, ring iterations i with
@@ -484,16 +509,29 @@ tbn_status launch_gemv(const void* x, int64_t B, int64_t K_in, const uint32_t* c
   a.stage_bytes = p.stage_bytes;
   a.y_bf16 = ydt == TBN_BF16 ? 1 : 0;
   a.relu = relu;
+  void (*kern)(CUtensorMap, CUtensorMap, GemvArgs) = nullptr;
   switch (B) {
-    case 1: gemv_tma_kernel<1><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 2: gemv_tma_kernel<2><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 3: gemv_tma_kernel<3><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 4: gemv_tma_kernel<4><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 5: gemv_tma_kernel<5><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 6: gemv_tma_kernel<6><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    case 7: gemv_tma_kernel<7><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
-    default: gemv_tma_kernel<8><<<p.grid, kThreads, p.smem, s>>>(tmap_w, tmap_x, a); break;
+    case 1: kern = gemv_tma_kernel<1>; break;
+    case 2: kern = gemv_tma_kernel<2>; break;
+    case 3: kern = gemv_tma_kernel<3>; break;
+    case 4: kern = gemv_tma_kernel<4>; break;
+    case 5: kern = gemv_tma_kernel<5>; break;
+    case 6: kern = gemv_tma_kernel<6>; break;
+    case 7: kern = gemv_tma_kernel<7>; break;
+    default: kern = gemv_tma_kernel<8>; break;
   }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(p.grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = p.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, tmap_w, tmap_x, a);
+  if (le != cudaSuccess) return cuda_fail(le, "cudaLaunchKernelEx(gemv_tma_kernel)");
   return check_launch("gemv_tma_kernel");
 }
 
