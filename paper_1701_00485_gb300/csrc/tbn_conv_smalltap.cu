@@ -27,6 +27,7 @@
 
 #include <algorithm>
 #include <cstdint>
+#include <cstring>
 #include <mutex>
 
 #include "tbn_device.cuh"
@@ -56,6 +57,10 @@ struct SmallTapArgs {
   const float* alpha;
   void* y;
   const void* residual;
+  // tensor-core variant
+  int mma_n;        // MMA N: tile pixels rounded up to 16
+  int patch_bytes;  // patch buffer size (multiple of 16)
+  uint32_t* err;    // device error word
 };
 
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
@@ -381,6 +386,297 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) conv_smalltap_kernel(Sma
   }
 }
 
+
+// ------------------------------------------------------ tensor-core variant
+// NHWC bf16 activations and NHWC bf16 output without a residual (K % 8 == 0,
+// 16-byte aligned y): the configuration the image networks launch.  The
+// mma.sync loop above issues one m16n8k16 per ~30 cycles per SM
+// sub-partition on this GPU.  Here a CTA takes a tile of up to 128 output
+// pixels and 128 filters:
+//   1. the patch goes to shared memory; its first batch of elements was
+//      loaded into registers while the previous tile computed;
+//   2. the threads build the im2col rows [pixel][64 codes] in the K-major,
+//      128-byte-swizzled layout of a tcgen05 operand (codes past n zero);
+//   3. one thread issues KP/16 tcgen05.mma, M = 128 filters (decoded codes
+//      W~/2, same layout, built once per filter tile), N = the tile's pixels
+//      rounded up to 16, fp32 accumulators in tensor memory, while the
+//      others load the next tile's first patch batch;
+//   4. eight warps read the accumulators as 16x256b fragments, apply
+//      2 alpha and ReLU (in the bf16 conversion) and store them transposed
+//      (stmatrix) into a staging tile [pixel][filter] (two halves of 64
+//      filters, 16-byte chunks XOR-swizzled by the pixel);
+//   5. two threads of different warps write the halves with TMA stores
+//      (asynchronous: the copy-out overlaps the next tile; a cooperative
+//      copy with 16-byte stores from every thread measured slower, and one
+//      thread issuing both boxes waited about 0.5 us per tile).
+// Three CTAs share an SM, so one CTA's loads overlap another's MMA and
+// stores.
+constexpr int kTcPixels = 128;
+constexpr int kTcCtasPerSm = 3;
+constexpr int kTcMaxPatchBytes = 8 * 1024;
+constexpr int kTcTmemCols = 128;
+constexpr int kTcOperandBytes = 128 * 128;   // 128 rows x 64 bf16 codes
+constexpr uint64_t kTcWaitLimitNs = 1000000000ull;
+
+size_t smalltap_tc_smem(size_t patch_bytes) {
+  return 1024 /*alignment slack*/ + 4 * static_cast<size_t>(kTcOperandBytes) +
+         ((patch_bytes + 15) & ~static_cast<size_t>(15)) + (kTcPixels + kMaxCodes) * sizeof(int) + 64;
+}
+
+// Tile t: filter tile slowest (a CTA keeps its decoded filters), then
+// image, row block, column block.
+struct TcTile {
+  int kt, img, p0, q0;
+};
+
+__device__ __forceinline__ TcTile tc_tile(const SmallTapArgs& a, int tile) {
+  TcTile c;
+  const int per_k = a.N * a.tiles_p * a.tiles_q;
+  c.kt = tile / per_k;
+  int rest = tile - c.kt * per_k;
+  c.img = rest / (a.tiles_p * a.tiles_q);
+  rest -= c.img * (a.tiles_p * a.tiles_q);
+  const int pt = rest / a.tiles_q;
+  c.p0 = pt * a.TP;
+  c.q0 = (rest - pt * a.tiles_q) * a.TQ;
+  return c;
+}
+
+template <int KP>
+__global__ void __launch_bounds__(kThreads, kTcCtasPerSm)
+    conv_smalltap_tc_kernel(const __grid_constant__ CUtensorMap tmap_y, SmallTapArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* opA = smem;                                  // [128 filters][128 B]
+  uint8_t* opB = smem + kTcOperandBytes;                // [128 pixels][128 B]
+  uint8_t* stage = smem + 2 * kTcOperandBytes;          // 2 x [128 pixels][64 filters]
+  __nv_bfloat16* patch = reinterpret_cast<__nv_bfloat16*>(smem + 4 * kTcOperandBytes);
+  int* pxbase = reinterpret_cast<int*>(smem + 4 * kTcOperandBytes + a.patch_bytes);
+  int* koff_tab = pxbase + kTcPixels;                   // patch offset of code k, -1 past n
+  uint64_t* bar = reinterpret_cast<uint64_t*>(koff_tab + kMaxCodes);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 1);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  constexpr int kChunks = KP / 8;   // 16-byte chunks of an im2col row that hold codes
+
+  if (tid < kTcPixels) {
+    const int pp = tid / a.TQ, qq = tid % a.TQ;
+    pxbase[tid] = (pp * a.sh * a.PW + qq * a.sw) * a.C;
+  }
+  if (tid < kMaxCodes) {
+    int off = -1;
+    if (tid < a.n) {
+      const int c = tid % a.C, s = (tid / a.C) % a.S, r = tid / (a.C * a.S);
+      off = (r * a.PW + s) * a.C + c;
+    }
+    koff_tab[tid] = off;
+  }
+  const int my_ch = tid % kChunks;
+  if (warp == 0) {
+    tmem_alloc(tmem_slot, kTcTmemCols);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tmap_y);
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t acc = *tmem_slot;
+  int koff[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) koff[j] = koff_tab[my_ch * 8 + j];
+
+  const int tile_px = a.TP * a.TQ;
+  const int row_elems = a.PW * a.C, patch_elems = a.PH * row_elems;
+  const int row_len = a.W * a.C;
+  const int r_first = tid / row_elems, e_first = tid % row_elems;
+  const int dr = kThreads / row_elems, de = kThreads % row_elems;
+  const uint32_t idesc = idesc_bf16_f32(128, static_cast<uint32_t>(a.mma_n));
+  const uint64_t adesc = smem_desc_sw128_kmajor(smem_addr(opA));
+  const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(opB));
+  const uint32_t stage_s = smem_addr(stage);
+  // epilogue role: TMEM lane quarter `sub` (filters 32 sub ..), pixel half
+  const int sub = warp & 3, half = warp >> 2;
+  const int fr = lane >> 2;
+  const int mi = lane >> 3, mrow = lane & 7;
+  const int nchunks = (a.mma_n + 31) / 32;
+  const int c_begin = half ? (nchunks + 1) / 2 : 0;
+  const int c_end = half ? nchunks : (nchunks + 1) / 2;
+  float a2f[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+  const bool relu = a.relu != 0;
+
+  // The patch of a tile: element idx = r * row_elems + e (patch row r,
+  // element e of that row) is image row ih0 + r, element e0 + e of the row.
+  // A thread holds elements idx = tid + kThreads j; its (r, e) advance by the
+  // constant (dr, de) per j.  The first eight (j < 8) of the next tile are
+  // loaded into registers while the current tile computes.
+  const uint16_t* xbase = reinterpret_cast<const uint16_t*>(a.x);
+  auto load_batch = [&](int tile, int idx0, uint16_t (&v)[8]) {
+    const TcTile c = tc_tile(a, tile);
+    const int ih0 = c.p0 * a.sh - a.ph, e0 = (c.q0 * a.sw - a.pw) * a.C;
+    const uint16_t* img_x = xbase + static_cast<size_t>(c.img) * a.H * row_len;
+    int r = r_first, e = e_first;
+    if (idx0 != tid) {
+      r = idx0 / row_elems;
+      e = idx0 - r * row_elems;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int gh = ih0 + r, ge = e0 + e;
+      const bool ok = idx0 + j * kThreads < patch_elems &&
+                      static_cast<unsigned>(gh) < static_cast<unsigned>(a.H) &&
+                      static_cast<unsigned>(ge) < static_cast<unsigned>(row_len);
+      v[j] = ok ? __ldg(img_x + gh * row_len + ge) : uint16_t(0);
+      r += dr;
+      e += de;
+      if (e >= row_elems) {
+        e -= row_elems;
+        ++r;
+      }
+    }
+  };
+  uint16_t* patch_u = reinterpret_cast<uint16_t*>(patch);
+
+  grid_dependency_wait();   // activations may come from the previous kernel
+  grid_dependents_launch();
+  uint16_t pre[8];
+  if (static_cast<int>(blockIdx.x) < a.tiles) load_batch(blockIdx.x, tid, pre);
+  int cur_ktile = -1;
+  uint32_t tiles_done = 0;
+  for (int tile = blockIdx.x; tile < a.tiles; tile += gridDim.x, ++tiles_done) {
+    const TcTile tc = tc_tile(a, tile);
+    const int kt = tc.kt;
+    if (kt != cur_ktile) {
+      cur_ktile = kt;
+      // operand A: filter f's codes as bf16 W~/2, chunk c of row f at c ^ (f & 7)
+      const int f = tid & 127;
+      const int fg = kt * kFiltersPerCta + f;
+      for (int ks = tid >> 7; ks < KP / 16; ks += 2) {
+        const uint32_t w =
+            (fg < a.K && ks < a.wpf) ? __ldg(a.codes + static_cast<size_t>(fg) * a.wpf + ks) : 0u;
+        uint32_t o[8];
+        word_to_bf16x2(w, o);
+        uint8_t* row = opA + f * 128;
+        *reinterpret_cast<uint4*>(row + (((2 * ks) ^ (f & 7)) << 4)) =
+            make_uint4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(row + (((2 * ks + 1) ^ (f & 7)) << 4)) =
+            make_uint4(o[4], o[5], o[6], o[7]);
+      }
+#pragma unroll
+      for (int lg = 0; lg < 2; ++lg) {
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int kk = kt * kFiltersPerCta + sub * 32 + lg * 16 + u * 8 + fr;
+          a2f[lg][u] = kk < a.K ? 2.0f * __ldg(a.alpha + kk) : 0.0f;
+        }
+      }
+    }
+    // 1. input patch (zero outside the image): the prefetched first batch,
+    //    then any further batches of a large patch
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (tid + j * kThreads < patch_elems) patch_u[tid + j * kThreads] = pre[j];
+    for (int idx0 = tid + 8 * kThreads; idx0 - tid < patch_elems; idx0 += 8 * kThreads) {
+      uint16_t v[8];
+      load_batch(tile, idx0, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (idx0 + j * kThreads < patch_elems) patch_u[idx0 + j * kThreads] = v[j];
+    }
+    __syncthreads();
+    // 2. operand B: im2col rows, chunk c of pixel row px at c ^ (px & 7)
+    for (int px = tid / kChunks; px < a.mma_n; px += kThreads / kChunks) {
+      uint32_t v[4] = {0u, 0u, 0u, 0u};
+      if (px < tile_px) {
+        const uint16_t* src = patch_u + pxbase[px];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const uint32_t lo = koff[2 * i] >= 0 ? src[koff[2 * i]] : 0u;
+          const uint32_t hi = koff[2 * i + 1] >= 0 ? src[koff[2 * i + 1]] : 0u;
+          v[i] = lo | (hi << 16);
+        }
+      }
+      *reinterpret_cast<uint4*>(opB + px * 128 + ((my_ch ^ (px & 7)) << 4)) =
+          make_uint4(v[0], v[1], v[2], v[3]);
+    }
+    fence_proxy_async_smem();   // operands written here are read by the tensor core
+    __syncthreads();
+    if (tile + static_cast<int>(gridDim.x) < a.tiles) load_batch(tile + gridDim.x, tid, pre);
+    // 3. MMA
+    if (tid == 0) {
+      tc_fence_after_sync();
+#pragma unroll
+      for (int kk = 0; kk < KP / 16; ++kk)
+        tc_mma_ss(acc, adesc + static_cast<uint64_t>(2 * kk), bdesc + static_cast<uint64_t>(2 * kk),
+                  idesc, kk > 0 ? 1u : 0u);
+      tc_commit(bar);
+    }
+    // one thread waits for the accumulators, the two storing threads for
+    // their previous stores to finish reading the staging tile; the others
+    // park at the barrier
+    if (tid == 0 || tid == 32) bulk_wait_group_read<0>();
+    const bool ok = tid != 0 || mbar_wait(bar, tiles_done & 1u, nullptr, a.err, kTcWaitLimitNs);
+    if (!__syncthreads_and(ok)) break;
+    tc_fence_after_sync();
+    // 4. epilogue: fragments (lane = filter, column = pixel) -> 2 alpha,
+    //    ReLU, bf16 pairs -> transposed 8x8 stores into the staging tile
+    for (int j = c_begin; j < c_end; ++j) {
+      uint32_t v[2][16];
+#pragma unroll
+      for (int lg = 0; lg < 2; ++lg)
+        tmem_ld_16x256b_x4(acc + (static_cast<uint32_t>(sub * 32 + lg * 16) << 16) +
+                               static_cast<uint32_t>(32 * j),
+                           v[lg]);
+      tmem_wait_ld();
+#pragma unroll
+      for (int lg = 0; lg < 2; ++lg) {
+        uint32_t pk[8];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          const float y0 = a2f[lg][0] * __uint_as_float(v[lg][4 * b + 0]);
+          const float y1 = a2f[lg][0] * __uint_as_float(v[lg][4 * b + 1]);
+          const float y2 = a2f[lg][1] * __uint_as_float(v[lg][4 * b + 2]);
+          const float y3 = a2f[lg][1] * __uint_as_float(v[lg][4 * b + 3]);
+          // filter fr, pixels 8b + 2(lane % 4) + 0/1; then filter fr + 8
+          pk[2 * b] = relu ? pack_bf16x2_relu(y0, y1) : pack_bf16x2(y0, y1);
+          pk[2 * b + 1] = relu ? pack_bf16x2_relu(y2, y3) : pack_bf16x2(y2, y3);
+        }
+#pragma unroll
+        for (int bp = 0; bp < 2; ++bp) {
+          const int px = 32 * j + 8 * (2 * bp + (mi >> 1)) + mrow;
+          const int chunk = 4 * sub + 2 * lg + (mi & 1);   // 8-filter chunk 0..15
+          const uint32_t addr = stage_s + static_cast<uint32_t>((chunk >> 3) * kTcOperandBytes +
+                                                                px * 128 +
+                                                                (((chunk & 7) ^ (px & 7)) << 4));
+          stmatrix_x4_trans(addr, pk[4 * bp + 0], pk[4 * bp + 1], pk[4 * bp + 2], pk[4 * bp + 3]);
+        }
+      }
+    }
+    tc_fence_before_sync();
+    fence_proxy_async_smem();   // staged values -> visible to the TMA stores
+    __syncthreads();
+    // 5. two TMA stores from threads of different warps (filters 0-63 from
+    //    thread 0, 64-127 from thread 32): one issuing thread per box keeps
+    //    the two boxes in flight together
+    if (tid == 0 || (tid == 32 && kt * kFiltersPerCta + kFiltersPerCta / 2 < a.K)) {
+      const int h = tid >> 5;
+      tma_store_4d(&tmap_y, stage + h * kTcOperandBytes, kt * kFiltersPerCta + h * 64, tc.q0,
+                   tc.p0, tc.img);
+      bulk_commit_group();
+    }
+  }
+  if (tid == 0 || tid == 32) bulk_wait_group<0>();   // stores complete before the CTA exits
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after_sync();
+    tmem_dealloc(acc, kTcTmemCols);
+  }
+}
+
 struct SmallTapPlan {
   int TP, TQ, PH, PW, KP;
   size_t smem;
@@ -414,6 +710,104 @@ SmallTapPlan plan_smalltap(const ConvProblem& p) {
   return t;
 }
 
+
+// Tile plan of the tensor-core variant: up to 128 pixels (whole rows when
+// they fit), fewer rows while the patch exceeds its 8 KB budget.
+struct SmallTapTcPlan {
+  int TP, TQ, PH, PW, KP, mma_n;
+  int patch_bytes;
+  size_t smem;
+  bool fits;
+};
+
+SmallTapTcPlan plan_smalltap_tc(const ConvProblem& p) {
+  SmallTapTcPlan t{};
+  t.TQ = static_cast<int>(std::min<int64_t>(p.Q, kTcPixels));
+  t.TP = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(p.P, kTcPixels / t.TQ)));
+  t.KP = p.C * p.R * p.S <= 32 ? 32 : 64;
+  int64_t bytes = 0;
+  for (;;) {
+    t.PH = static_cast<int>((t.TP - 1) * p.sh + p.R);
+    t.PW = static_cast<int>((t.TQ - 1) * p.sw + p.S);
+    bytes = static_cast<int64_t>(t.PH) * t.PW * p.C * 2;
+    if (t.TP == 1 || bytes <= kTcMaxPatchBytes) break;
+    --t.TP;
+  }
+  t.fits = bytes <= kTcMaxPatchBytes;
+  t.patch_bytes = static_cast<int>((bytes + 15) & ~int64_t(15));
+  t.mma_n = (t.TP * t.TQ + 15) & ~15;
+  t.smem = smalltap_tc_smem(static_cast<size_t>(t.patch_bytes));
+  return t;
+}
+
+// The tensor-core variant takes NHWC bf16 output without a residual, stored
+// by TMA (K % 8 == 0 for the 16-byte row pitch, 16-byte aligned y).
+bool smalltap_tc_eligible(const ConvProblem& p) {
+  return p.layout == TBN_NHWC && p.ydt == TBN_BF16 && p.residual == nullptr && p.K % 8 == 0 &&
+         is_aligned(p.y, 16) && get_encode_tiled() != nullptr && plan_smalltap_tc(p).fits;
+}
+
+tbn_status launch_smalltap_tc(const ConvProblem& p, SmallTapArgs a, cudaStream_t s) {
+  const SmallTapTcPlan t = plan_smalltap_tc(p);
+  a.TP = t.TP; a.TQ = t.TQ; a.PH = t.PH; a.PW = t.PW;
+  a.tiles_p = (a.P + a.TP - 1) / a.TP;
+  a.tiles_q = (a.Q + a.TQ - 1) / a.TQ;
+  const int64_t tiles = static_cast<int64_t>(a.N) * a.tiles_p * a.tiles_q * a.tiles_k;
+  if (tiles >= (1ll << 31)) return fail(TBN_ERR_UNSUPPORTED, "small-tap conv: too many tiles");
+  a.tiles = static_cast<int>(tiles);
+  a.mma_n = t.mma_n;
+  a.patch_bytes = t.patch_bytes;
+  a.err = device_error_word();
+
+  // output map: box = 64 filters (128 bytes, 128-byte swizzle) x TQ x TP x 1,
+  // the layout of a staging half
+  alignas(64) CUtensorMap tmap_y;
+  std::memset(&tmap_y, 0, sizeof(tmap_y));
+  const cuuint64_t gdim[4] = {(cuuint64_t)p.K, (cuuint64_t)p.Q, (cuuint64_t)p.P, (cuuint64_t)p.N};
+  const cuuint64_t gstride[3] = {(cuuint64_t)(p.K * 2), (cuuint64_t)(p.Q * p.K * 2),
+                                 (cuuint64_t)(p.P * p.Q * p.K * 2)};
+  const cuuint32_t box[4] = {(cuuint32_t)(kFiltersPerCta / 2), (cuuint32_t)t.TQ,
+                             (cuuint32_t)t.TP, 1u};
+  const cuuint32_t estr[4] = {1u, 1u, 1u, 1u};
+  const CUresult cr = get_encode_tiled()(
+      &tmap_y, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, p.y, gdim, gstride, box, estr,
+      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS)
+    return fail(TBN_ERR_CUDA, "small-tap conv: cuTensorMapEncodeTiled(y) failed (%d)", (int)cr);
+
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    const void* fns[2] = {(const void*)conv_smalltap_tc_kernel<32>,
+                          (const void*)conv_smalltap_tc_kernel<64>};
+    for (int i = 0; i < 2 && attr_err == cudaSuccess; ++i) {
+      attr_err = cudaFuncSetAttribute(fns[i], cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)smalltap_tc_smem(kTcMaxPatchBytes));
+      if (attr_err == cudaSuccess)
+        attr_err = cudaFuncSetAttribute(fns[i], cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    }
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(smalltap tc)");
+
+  const int64_t slots = static_cast<int64_t>(device_sm_count()) * kTcCtasPerSm;
+  const int grid = static_cast<int>(std::min<int64_t>(tiles, slots));
+  void (*kern)(const CUtensorMap, SmallTapArgs) =
+      t.KP == 32 ? conv_smalltap_tc_kernel<32> : conv_smalltap_tc_kernel<64>;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = t.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, tmap_y, a);
+  if (le != cudaSuccess) return cuda_fail(le, "cudaLaunchKernelEx(conv_smalltap_tc_kernel)");
+  return check_launch("conv_smalltap_tc_kernel");
+}
 }  // namespace
 
 const char* conv_smalltap_unsupported_reason(const ConvProblem& p) {
@@ -453,6 +847,7 @@ tbn_status launch_conv_smalltap(const ConvProblem& p, cudaStream_t s) {
   a.alpha = p.alpha;
   a.y = p.y;
   a.residual = p.residual;
+  if (smalltap_tc_eligible(p)) return launch_smalltap_tc(p, a, s);
 
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
