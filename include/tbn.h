@@ -57,7 +57,7 @@
  *   form of a layer: inference reads nothing else of the layer (Section 3).
  * - The order of the n weights of a filter is the caller's choice; the
  *   convolution reads them in the activation layout's natural order:
- *   NCHW -> (c, r, s), NHWC -> (r, s, c).  Discretization is elementwise and
+ *   NCHW -> (c, r, s), NHWC and NCHW_NHWC -> (r, s, c).  Discretization is elementwise and
  *   alpha does not depend on the order, so permuting fp32 weights before
  *   tbn_quantize_pack is how either order is produced.
  */
@@ -71,7 +71,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 3
+#define TBN_ABI_VERSION 4
 
 typedef enum {
   TBN_OK = 0,
@@ -84,7 +84,11 @@ typedef enum {
 
 typedef enum { TBN_F32 = 0, TBN_BF16 = 1 } tbn_dtype;
 
-typedef enum { TBN_NCHW = 0, TBN_NHWC = 1 } tbn_layout;
+/* Activation layouts.  TBN_NCHW_NHWC (convolutions only) reads an NCHW x
+ * and writes an NHWC y (and residual), with codes in the NHWC order
+ * (r, s, c): the first layer of an NHWC network can read its NCHW input
+ * batch without a converted copy (small-tap and direct kernels). */
+typedef enum { TBN_NCHW = 0, TBN_NHWC = 1, TBN_NCHW_NHWC = 2 } tbn_layout;
 
 typedef enum {
   TBN_UNPACK_I8 = 0,   /* int8 W~ in {-2,-1,1,2}                 */
@@ -98,10 +102,12 @@ typedef enum {
   TBN_CONV_DIRECT = 1,        /* CUDA-core direct convolution, any layout/dtype   */
   TBN_CONV_IMPLICIT_GEMM = 2, /* tcgen05 implicit GEMM, NHWC bf16 x; activations
                                  by TMA when C % 64 == 0, else gathered by threads */
-  TBN_CONV_SMALL_TAPS = 3     /* tensor-core (mma.sync) convolution for short
-                                 filters, C*R*S <= 64, bf16 x in NCHW or NHWC,
-                                 no fused pool: the input patch and its im2col
-                                 expansion are staged in shared memory        */
+  TBN_CONV_SMALL_TAPS = 3     /* tensor-core convolution for short filters,
+                                 C*R*S <= 64, bf16 x in any layout, no fused
+                                 pool: the input patch and its im2col
+                                 expansion are staged in shared memory
+                                 (tcgen05 for NHWC x and bf16 NHWC y without
+                                 residual, K % 8 == 0; mma.sync otherwise)   */
 } tbn_conv_algo;
 
 /* Fused layer epilogue (network glue, not part of the paper's method):
@@ -110,7 +116,8 @@ typedef enum {
  *   if (pool == 2) v = max of v over a 2x2 window, stride 2 (floor sizes);
  *   y = v rounded to y's dtype.
  * `residual` has y's layout, shape and dtype (not combinable with pool).
- * With pool == 2, y is [N][P/2][Q/2][K] (NHWC) / [N][K][P/2][Q/2] (NCHW).
+ * With pool == 2, y is [N][P/2][Q/2][K] (NHWC, NCHW_NHWC) / [N][K][P/2][Q/2]
+ * (NCHW).
  * Pass NULL for no epilogue. */
 typedef struct {
   int relu;
@@ -185,17 +192,18 @@ tbn_status tbn_unpack(const uint32_t *codes, const float *alpha, int64_t K, int6
  *
  *   y[b,k,p,q] = alpha[k] * sum_{c,r,s} x[b,c,p*sh-ph+r,q*sw-pw+s] W~[k,c,r,s]
  *
- *   x      activations (device).  layout NCHW: [N][C][H][W];
+ *   x      activations (device).  layout NCHW and NCHW_NHWC: [N][C][H][W];
  *          NHWC: [N][H][W][C].  dtype fp32 or bf16.
  *   codes  [K][tbn_packed_words(C*R*S)], filter order (c,r,s) for NCHW and
- *          (r,s,c) for NHWC.   alpha [K] fp32.
- *   y      [N][K][P][Q] (NCHW) or [N][P][Q][K] (NHWC), dtype fp32 or bf16,
- *          P = (H + 2 ph - R) / sh + 1, Q = (W + 2 pw - S) / sw + 1.
+ *          (r,s,c) for NHWC and NCHW_NHWC.   alpha [K] fp32.
+ *   y      [N][K][P][Q] (NCHW) or [N][P][Q][K] (NHWC, NCHW_NHWC), dtype
+ *          fp32 or bf16, P = (H + 2 ph - R) / sh + 1, Q = (W + 2 pw - S) / sw + 1.
  *   epi    optional fused epilogue (NULL = none).
  * Accumulation is fp32; x * W~ products are exact.  y must not alias x.
  * The tensor-core implicit-GEMM path needs NHWC and bf16 x (16-byte aligned
  * x, y and residual; stride 1 or 2 when C % 64 == 0, any stride otherwise);
- * AUTO falls back to the CUDA-core direct kernel for every other case. */
+ * the small-tap path takes bf16 x with C*R*S <= 64 in any layout; AUTO falls
+ * back to the CUDA-core direct kernel for every other case. */
 tbn_status tbn_conv2d_fwd(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
                           int64_t C, int64_t H, int64_t W, const uint32_t *codes,
                           const float *alpha, int64_t K, int64_t R, int64_t S,

@@ -25,7 +25,7 @@ __all__ = [
     "tbn_linear_fwd", "tbn_linear_fwd_ws", "tbn_linear_workspace_bytes",
     "tbn_linear_fwd_noalloc", "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_device_error",
     "tbn_conv2d_select_algo", "conv_out_hw",
-    "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
+    "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_NCHW_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
     "TBN_CONV_SMALL_TAPS",
 ]
@@ -36,7 +36,7 @@ _LIB_PATH = os.path.join(_HERE, "libtbn.so")
 TBN_OK, TBN_ERR_INVALID_ARG, TBN_ERR_UNSUPPORTED, TBN_ERR_MISALIGNED, TBN_ERR_CUDA, \
     TBN_ERR_TIMEOUT = range(6)
 TBN_F32, TBN_BF16 = 0, 1
-TBN_NCHW, TBN_NHWC = 0, 1
+TBN_NCHW, TBN_NHWC, TBN_NCHW_NHWC = 0, 1, 2
 TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
 TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM, TBN_CONV_SMALL_TAPS = 0, 1, 2, 3
 TBN_MAX_QUANT_JOBS = 16
@@ -71,7 +71,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 3  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 4  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -229,7 +229,8 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
                    out_dtype=None, relu: bool = False, residual: torch.Tensor | None = None,
                    algo: int = TBN_CONV_AUTO, out: torch.Tensor | None = None, stream=None,
                    pool: int = 0):
-    """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW) or [N,H,W,C] (NHWC).
+    """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW, NCHW_NHWC) or
+    [N,H,W,C] (NHWC); y is NCHW for NCHW, else NHWC.
     pool=2 fuses a 2x2 / stride-2 max pool (after ReLU) into the epilogue."""
     _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
     if layout == TBN_NHWC:
@@ -240,7 +241,7 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
     if pool:
         P, Q = P // 2, Q // 2
     ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
-    shape = (N, P, Q, K) if layout == TBN_NHWC else (N, K, P, Q)
+    shape = (N, K, P, Q) if layout == TBN_NCHW else (N, P, Q, K)
     if out is None:
         out = torch.empty(shape, dtype=_torch_dt(ydt), device=x.device)
     elif tuple(out.shape) != shape or _dt(out) != ydt:

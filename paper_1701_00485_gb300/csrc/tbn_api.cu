@@ -103,7 +103,8 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
   if (!x || !codes || !alpha || !y) return fail(TBN_ERR_INVALID_ARG, "conv: null pointer");
   if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad x dtype");
   if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad y dtype");
-  if (layout != TBN_NCHW && layout != TBN_NHWC) return fail(TBN_ERR_INVALID_ARG, "conv: bad layout");
+  if (layout != TBN_NCHW && layout != TBN_NHWC && layout != TBN_NCHW_NHWC)
+    return fail(TBN_ERR_INVALID_ARG, "conv: bad layout");
   if (N < 1 || C < 1 || H < 1 || W < 1 || K < 1 || R < 1 || S < 1)
     return fail(TBN_ERR_INVALID_ARG, "conv: sizes must be >= 1");
   if (sh < 1 || sw < 1 || ph < 0 || pw < 0) return fail(TBN_ERR_INVALID_ARG, "conv: bad stride/pad");

@@ -59,9 +59,13 @@ struct DirectArgs {
 
 // kWin = 1: one conv output per thread, 32 filters.  kWin = 4: one 2x2-pooled
 // output per thread (four conv outputs, max after ReLU), 8 filters.
-template <typename TX, typename TY, bool kNHWC, int kWin>
+// kLayout (tbn_layout): x is NHWC only for TBN_NHWC; the codes are in
+// (r, s, c) order and y is NHWC for TBN_NHWC and TBN_NCHW_NHWC.
+template <typename TX, typename TY, int kLayout, int kWin>
 __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
   constexpr int kF = kWin == 1 ? kFilt : 8;
+  constexpr bool kXNhwc = kLayout == TBN_NHWC, kRsc = kLayout != TBN_NCHW;
+  constexpr bool kYNhwc = kLayout != TBN_NCHW;
   __shared__ __align__(16) float s_w[kTapChunk][kF];
   __shared__ int32_t s_off[kTapChunk];
   __shared__ int32_t s_rs[kTapChunk];
@@ -84,7 +88,7 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
     h0[wdx] = static_cast<int>(p * a.sh - a.ph);
     w0[wdx] = static_cast<int>(q * a.sw - a.pw);
     // element offset of (b, c = 0, h0, w0)
-    base[wdx] = kNHWC ? ((b * a.H + h0[wdx]) * a.W + w0[wdx]) * a.C
+    base[wdx] = kXNhwc ? ((b * a.H + h0[wdx]) * a.W + w0[wdx]) * a.C
                       : ((b * a.C) * a.H + h0[wdx]) * a.W + w0[wdx];
   }
   const int H = static_cast<int>(a.H), W = static_cast<int>(a.W);
@@ -114,17 +118,16 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
     for (int t = threadIdx.x; t < tc; t += kPix) {
       const int64_t ti = t0 + t;
       int64_t c, r, s;
-      if (kNHWC) {
+      if (kRsc) {
         r = ti / (a.S * a.C);
         s = (ti / a.C) % a.S;
         c = ti % a.C;
-        s_off[t] = static_cast<int32_t>((r * a.W + s) * a.C + c);
       } else {
         c = ti / (a.R * a.S);
         r = (ti / a.S) % a.R;
         s = ti % a.S;
-        s_off[t] = static_cast<int32_t>((c * a.H + r) * a.W + s);
       }
+      s_off[t] = static_cast<int32_t>(kXNhwc ? (r * a.W + s) * a.C + c : (c * a.H + r) * a.W + s);
       s_rs[t] = static_cast<int32_t>((r << 16) | s);
     }
     __syncthreads();
@@ -158,7 +161,7 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
   for (int f = 0; f < kF; ++f) {
     const int64_t k = k0 + f;
     if (k < a.K) {
-      const int64_t o = kNHWC ? pix * a.K + k : ((b * a.K + k) * a.Po + po) * a.Qo + qo;
+      const int64_t o = kYNhwc ? pix * a.K + k : ((b * a.K + k) * a.Po + po) * a.Qo + qo;
       float best = -INFINITY;
 #pragma unroll
       for (int wdx = 0; wdx < kWin; ++wdx) {
@@ -172,7 +175,7 @@ __global__ void __launch_bounds__(kPix) conv_direct_kernel(const DirectArgs a) {
   }
 }
 
-template <typename TX, typename TY, bool kNHWC, int kWin>
+template <typename TX, typename TY, int kLayout, int kWin>
 tbn_status launch_direct_t(const DirectArgs& a, cudaStream_t s) {
   constexpr int kF = kWin == 1 ? kFilt : 8;
   const int64_t npix = a.N * a.Po * a.Qo;
@@ -183,13 +186,22 @@ tbn_status launch_direct_t(const DirectArgs& a, cudaStream_t s) {
                 (long long)gy);
   if (a.H >= (1 << 30) || a.W >= (1 << 30))
     return fail(TBN_ERR_UNSUPPORTED, "conv direct: image too large");
-  conv_direct_kernel<TX, TY, kNHWC, kWin><<<dim3((unsigned)gx, (unsigned)gy), kPix, 0, s>>>(a);
+  conv_direct_kernel<TX, TY, kLayout, kWin><<<dim3((unsigned)gx, (unsigned)gy), kPix, 0, s>>>(a);
   return check_launch("conv_direct_kernel");
 }
 
-template <typename TX, typename TY, bool kNHWC>
+template <typename TX, typename TY, int kLayout>
 tbn_status launch_direct_w(const DirectArgs& a, bool pool, cudaStream_t s) {
-  return pool ? launch_direct_t<TX, TY, kNHWC, 4>(a, s) : launch_direct_t<TX, TY, kNHWC, 1>(a, s);
+  return pool ? launch_direct_t<TX, TY, kLayout, 4>(a, s) : launch_direct_t<TX, TY, kLayout, 1>(a, s);
+}
+
+template <int kLayout>
+tbn_status launch_direct_l(const DirectArgs& a, bool xb, bool yb, bool pool, cudaStream_t s) {
+  using bf = __nv_bfloat16;
+  if (xb && yb) return launch_direct_w<bf, bf, kLayout>(a, pool, s);
+  if (xb && !yb) return launch_direct_w<bf, float, kLayout>(a, pool, s);
+  if (!xb && yb) return launch_direct_w<float, bf, kLayout>(a, pool, s);
+  return launch_direct_w<float, float, kLayout>(a, pool, s);
 }
 
 template <typename T>
@@ -320,19 +332,10 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s) {
   a.x = p.x; a.codes = p.codes; a.alpha = p.alpha; a.y = p.y;
   a.residual = p.residual; a.relu = p.relu;
   const bool pool = p.pool != 0;
-  const bool nhwc = p.layout == TBN_NHWC;
   const bool xb = p.xdt == TBN_BF16, yb = p.ydt == TBN_BF16;
-  using bf = __nv_bfloat16;
-  if (nhwc) {
-    if (xb && yb) return launch_direct_w<bf, bf, true>(a, pool, s);
-    if (xb && !yb) return launch_direct_w<bf, float, true>(a, pool, s);
-    if (!xb && yb) return launch_direct_w<float, bf, true>(a, pool, s);
-    return launch_direct_w<float, float, true>(a, pool, s);
-  }
-  if (xb && yb) return launch_direct_w<bf, bf, false>(a, pool, s);
-  if (xb && !yb) return launch_direct_w<bf, float, false>(a, pool, s);
-  if (!xb && yb) return launch_direct_w<float, bf, false>(a, pool, s);
-  return launch_direct_w<float, float, false>(a, pool, s);
+  if (p.layout == TBN_NHWC) return launch_direct_l<TBN_NHWC>(a, xb, yb, pool, s);
+  if (p.layout == TBN_NCHW_NHWC) return launch_direct_l<TBN_NCHW_NHWC>(a, xb, yb, pool, s);
+  return launch_direct_l<TBN_NCHW>(a, xb, yb, pool, s);
 }
 
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,

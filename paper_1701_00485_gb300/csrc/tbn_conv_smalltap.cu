@@ -50,7 +50,9 @@ struct SmallTapArgs {
   int TP, TQ;       // tile rows / columns of output
   int tiles_p, tiles_q, tiles_k, tiles;
   int PH, PW;       // patch rows / columns
-  int nhwc;
+  int x_nhwc;       // x is [N][H][W][C] (else [N][C][H][W])
+  int rsc;          // codes in (r, s, c) order (else (c, r, s))
+  int y_nhwc;       // y and residual are [N][P][Q][K] (else [N][K][P][Q])
   int y_bf16, relu;
   const __nv_bfloat16* x;
   const uint32_t* codes;
@@ -99,7 +101,7 @@ __device__ __forceinline__ uint32_t decode_pair(uint32_t w, int p) {
 __device__ __forceinline__ void store_pair(const SmallTapArgs& a, int img, int p, int q, int f,
                                            float v0, float v1) {
   const bool has1 = f + 1 < a.K;
-  if (a.nhwc) {
+  if (a.y_nhwc) {
     const size_t o = ((static_cast<size_t>(img) * a.P + p) * a.Q + q) * a.K + f;
     if (a.residual) {
       if (a.y_bf16) {
@@ -200,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) conv_smalltap_kernel(Sma
     int off = -1;
     if (k < a.n) {
       int c, r, s;
-      if (a.nhwc) {
+      if (a.rsc) {
         c = k % a.C;
         s = (k / a.C) % a.S;
         r = k / (a.C * a.S);
@@ -257,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) conv_smalltap_kernel(Sma
     // 1. input patch, zero outside the image: NHWC rows are contiguous runs
     //    of W*C elements, NCHW rows runs of W elements per channel
     const int ih0 = p0 * a.sh - a.ph, iw0 = q0 * a.sw - a.pw;
-    if (a.nhwc) {
+    if (a.x_nhwc) {
       // thread owns row offsets e = tid, tid + 256, ...; all its loads of a
       // batch of rows are issued before any is stored
       const int e0 = iw0 * a.C, row_len = a.W * a.C;
@@ -514,7 +516,7 @@ __global__ void __launch_bounds__(kThreads, kTcCtasPerSm)
   // constant (dr, de) per j.  The first eight (j < 8) of the next tile are
   // loaded into registers while the current tile computes.
   const uint16_t* xbase = reinterpret_cast<const uint16_t*>(a.x);
-  auto load_batch = [&](int tile, int idx0, uint16_t (&v)[8]) {
+  auto load_batch = [&](int tile, int idx0, uint32_t (&v)[4]) {
     const TcTile c = tc_tile(a, tile);
     const int ih0 = c.p0 * a.sh - a.ph, e0 = (c.q0 * a.sw - a.pw) * a.C;
     const uint16_t* img_x = xbase + static_cast<size_t>(c.img) * a.H * row_len;
@@ -529,7 +531,8 @@ __global__ void __launch_bounds__(kThreads, kTcCtasPerSm)
       const bool ok = idx0 + j * kThreads < patch_elems &&
                       static_cast<unsigned>(gh) < static_cast<unsigned>(a.H) &&
                       static_cast<unsigned>(ge) < static_cast<unsigned>(row_len);
-      v[j] = ok ? __ldg(img_x + gh * row_len + ge) : uint16_t(0);
+      const uint32_t el = ok ? __ldg(img_x + gh * row_len + ge) : 0u;
+      v[j >> 1] = (j & 1) ? (v[j >> 1] | (el << 16)) : el;
       r += dr;
       e += de;
       if (e >= row_elems) {
@@ -542,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, kTcCtasPerSm)
 
   grid_dependency_wait();   // activations may come from the previous kernel
   grid_dependents_launch();
-  uint16_t pre[8];
+  uint32_t pre[4];   // next tile's first eight patch elements, two per word
   if (static_cast<int>(blockIdx.x) < a.tiles) load_batch(blockIdx.x, tid, pre);
   int cur_ktile = -1;
   uint32_t tiles_done = 0;
@@ -576,15 +579,17 @@ __global__ void __launch_bounds__(kThreads, kTcCtasPerSm)
     }
     // 1. input patch (zero outside the image): the prefetched first batch,
     //    then any further batches of a large patch
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      if (tid + j * kThreads < patch_elems) patch_u[tid + j * kThreads] = pre[j];
-    for (int idx0 = tid + 8 * kThreads; idx0 - tid < patch_elems; idx0 += 8 * kThreads) {
-      uint16_t v[8];
-      load_batch(tile, idx0, v);
+    auto store_batch = [&](int idx0, const uint32_t (&v)[4]) {
 #pragma unroll
       for (int j = 0; j < 8; ++j)
-        if (idx0 + j * kThreads < patch_elems) patch_u[idx0 + j * kThreads] = v[j];
+        if (idx0 + j * kThreads < patch_elems)
+          patch_u[idx0 + j * kThreads] = static_cast<uint16_t>(v[j >> 1] >> (16 * (j & 1)));
+    };
+    store_batch(tid, pre);
+    for (int idx0 = tid + 8 * kThreads; idx0 - tid < patch_elems; idx0 += 8 * kThreads) {
+      uint32_t v[4];
+      load_batch(tile, idx0, v);
+      store_batch(idx0, v);
     }
     __syncthreads();
     // 2. operand B: im2col rows, chunk c of pixel row px at c ^ (px & 7)
@@ -683,7 +688,7 @@ struct SmallTapPlan {
 };
 
 bool smalltap_staged(const ConvProblem& p) {
-  return p.layout == TBN_NHWC && p.ydt == TBN_BF16 && p.residual == nullptr && p.K % 8 == 0 &&
+  return p.layout != TBN_NCHW && p.ydt == TBN_BF16 && p.residual == nullptr && p.K % 8 == 0 &&
          is_aligned(p.y, 16);
 }
 
@@ -839,7 +844,9 @@ tbn_status launch_conv_smalltap(const ConvProblem& p, cudaStream_t s) {
   const int64_t tiles = static_cast<int64_t>(a.N) * a.tiles_p * a.tiles_q * a.tiles_k;
   if (tiles >= (1ll << 31)) return fail(TBN_ERR_UNSUPPORTED, "small-tap conv: too many tiles");
   a.tiles = static_cast<int>(tiles);
-  a.nhwc = p.layout == TBN_NHWC ? 1 : 0;
+  a.x_nhwc = p.layout == TBN_NHWC ? 1 : 0;
+  a.rsc = p.layout != TBN_NCHW ? 1 : 0;
+  a.y_nhwc = p.layout != TBN_NCHW ? 1 : 0;
   a.y_bf16 = p.ydt == TBN_BF16 ? 1 : 0;
   a.relu = p.relu;
   a.x = static_cast<const __nv_bfloat16*>(p.x);

@@ -75,7 +75,8 @@ class ConvCase:
         self.K, self.C, self.R, self.S = W.shape
 
     def quantize_gpu(self, layout):
-        if layout == tbn.TBN_NHWC:
+        # codes in (r, s, c) order for NHWC and NCHW_NHWC, (c, r, s) for NCHW
+        if layout != tbn.TBN_NCHW:
             Wl = self.W.permute(0, 2, 3, 1).reshape(self.K, -1).contiguous()
         else:
             Wl = self.W.reshape(self.K, -1).contiguous()
@@ -90,9 +91,10 @@ class ConvCase:
         if layout == tbn.TBN_NHWC:
             x = x.permute(0, 2, 3, 1).contiguous()
         res = None
+        y_nhwc = layout != tbn.TBN_NCHW
         if residual is not None:
             res = residual.to(out_dtype)
-            if layout == tbn.TBN_NHWC:
+            if y_nhwc:
                 res = res.permute(0, 2, 3, 1).contiguous()
             res = res.cuda()
         y = tbn.tbn_conv2d_fwd(x.cuda(), codes, alpha, self.K, self.R, self.S, self.stride,
@@ -100,7 +102,7 @@ class ConvCase:
                                residual=res, algo=algo)
         torch.cuda.synchronize()
         y = y.float().cpu()
-        if layout == tbn.TBN_NHWC:
+        if y_nhwc:
             y = y.permute(0, 3, 1, 2).contiguous()
         return y.numpy()
 

@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 3
+    assert L.tbn_abi_version() == 4
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -81,6 +81,7 @@ def test_conv_rejects_bad_arguments(L):
     assert _conv(L, N=0) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, xdt=5) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, layout=9) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, layout=3) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, sh=0) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, ph=-1) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, H=2, W=2, ph=0, pw=0) == tbn.TBN_ERR_INVALID_ARG   # kernel > input
@@ -103,6 +104,14 @@ def test_select_algo_host_rules(L):
                                       1, 7, 8, 8, 64, 3, 3) == tbn.TBN_CONV_SMALL_TAPS
     assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW,
                                       1, 8, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+    # NCHW in, NHWC out: small-tap for short bf16 filters, else the direct kernel
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW_NHWC,
+                                      128, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)) == \
+        tbn.TBN_CONV_SMALL_TAPS
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").bfloat16, tbn.TBN_NCHW_NHWC,
+                                      1, 64, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
+    assert tbn.tbn_conv2d_select_algo(__import__("torch").float32, tbn.TBN_NCHW_NHWC,
+                                      1, 3, 8, 8, 64, 3, 3) == tbn.TBN_CONV_DIRECT
 
 
 def test_linear_and_glue_reject_bad_arguments(L):

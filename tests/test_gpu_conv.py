@@ -153,6 +153,57 @@ def test_smalltap_conv_epilogue(case, layout, ydt):
                   what="smalltap epi %s" % (case,))
 
 
+@pytest.mark.parametrize("case", SMALLTAP)
+def test_smalltap_nchw_in_nhwc_out_matches_oracle(case):
+    """TBN_NCHW_NHWC (NCHW x, NHWC y, codes in (r, s, c) order) on the
+    mma.sync small-tap kernel: bf16 and fp32 output, the residual epilogue."""
+    c = make_case(*case, seed=6700 + sum(case[:7]), wscale=1.2)
+    algo = tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NCHW_NHWC, *case[:7], case[7],
+                                      case[8])
+    assert algo == tbn.TBN_CONV_SMALL_TAPS
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    yb = c.run_gpu(tbn.TBN_NCHW_NHWC, torch.bfloat16, torch.bfloat16)
+    assert_within(yb, y_orc, bound, out_bf16=True, what="smalltap nchw->nhwc bf16 %s" % (case,))
+    y = c.run_gpu(tbn.TBN_NCHW_NHWC, torch.bfloat16, torch.float32)
+    assert_within(y, y_orc, bound, out_bf16=False, what="smalltap nchw->nhwc %s" % (case,))
+    import oracle
+    g = inputs.generator(99)
+    res = torch.randn(*y_orc.shape, generator=g).to(torch.bfloat16)
+    want = oracle.epilogue(y_orc, res.float().numpy(), relu=True)
+    ye = c.run_gpu(tbn.TBN_NCHW_NHWC, torch.bfloat16, torch.bfloat16, relu=True, residual=res)
+    assert_within(ye, want, bound, out_bf16=True, epilogue=True,
+                  what="smalltap nchw->nhwc epi %s" % (case,))
+
+
+@pytest.mark.parametrize("case", DIRECT[:4])
+@pytest.mark.parametrize("xdt", [torch.float32, torch.bfloat16])
+def test_direct_nchw_in_nhwc_out_matches_oracle(case, xdt):
+    c = make_case(*case, seed=7100 + sum(case[:7]), wscale=1.3)
+    y = c.run_gpu(tbn.TBN_NCHW_NHWC, xdt, torch.float32, algo=tbn.TBN_CONV_DIRECT)
+    y_orc, bound = c.oracle_full(xdt)
+    assert_within(y, y_orc, bound, out_bf16=False, what="direct nchw->nhwc %s" % (case,))
+
+
+def test_nchw_in_nhwc_out_auto_falls_back_to_direct():
+    """Long filters with the mixed layout have no tensor-core kernel: AUTO
+    takes the direct kernel, the implicit GEMM refuses."""
+    case = (2, 8, 9, 9, 24, 3, 3, (1, 1), (1, 1))   # C*R*S = 72
+    assert tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NCHW_NHWC, *case[:7], case[7],
+                                      case[8]) == tbn.TBN_CONV_DIRECT
+    c = make_case(*case, seed=71)
+    y_orc, bound = c.oracle_full(torch.bfloat16)
+    y = c.run_gpu(tbn.TBN_NCHW_NHWC, torch.bfloat16, torch.bfloat16, relu=True)
+    assert_within(y, oracle_relu(y_orc), bound, out_bf16=True, epilogue=True, what="auto mixed")
+    with pytest.raises(tbn.TBNError):
+        c.run_gpu(tbn.TBN_NCHW_NHWC, torch.bfloat16, torch.bfloat16,
+                  algo=tbn.TBN_CONV_IMPLICIT_GEMM)
+
+
+def oracle_relu(y):
+    import oracle
+    return oracle.epilogue(y, None, relu=True)
+
+
 def test_smalltap_rejects_long_filters_and_pool():
     c = make_case(1, 8, 6, 6, 16, 3, 3, (1, 1), (1, 1), seed=5)   # n = 72
     with pytest.raises(tbn.TBNError):
