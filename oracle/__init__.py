@@ -14,8 +14,6 @@ follows:
   quantize        Algorithm 1, quantization loop (Eq. 3 + Eq. 5 per filter)
   pack / unpack   two-bit storage; the paper fixes only "two bits per weight",
                   the field layout is documented in tbn_oracle.h
-  pack_e4m3 / unpack_e4m3   the same codes in the second ("e4m3-planar")
-                  word layout, documented there too
   quant_error     Eq. 2 objective, evaluated directly
   conv2d_nchw     Eq. 1, seven nested loops, zero padding, cross-correlation
   conv2d_sites    Eq. 1 at selected output sites
@@ -101,8 +99,6 @@ class Oracle:
             "orc_words_per_filter": ([I], I),
             "orc_pack": ([P, I, I, P], ctypes.c_int),
             "orc_unpack": ([P, I, I, P], ctypes.c_int),
-            "orc_pack_e4m3": ([P, I, I, P], ctypes.c_int),
-            "orc_unpack_e4m3": ([P, I, I, P], ctypes.c_int),
             "orc_quant_error": ([P, P, I, ctypes.c_double], ctypes.c_double),
             "orc_conv2d_nchw": ([P, I, I, I, I, P, P, I, I, I, I, I, I, I, P, P], None),
             "orc_conv2d_nchw_sites": ([P, I, I, I, I, P, P, I, I, I, I, I, I, I, P, I, P, P],
@@ -172,26 +168,6 @@ class Oracle:
             raise ValueError("word count does not match n")
         out = np.empty((K, n), dtype=np.int8)
         if self.lib.orc_unpack(_ptr(w), K, n, _ptr(out)) != 0:
-            raise ValueError("non-zero padding field")
-        return out
-
-    def pack_e4m3(self, wt2d) -> np.ndarray:
-        """Pack int8 codes [K, n] into uint32 words [K, ceil(n/16)], e4m3-planar."""
-        wt = np.ascontiguousarray(np.asarray(wt2d, dtype=np.int8))
-        K, n = wt.shape
-        out = np.empty((K, self.words_per_filter(n)), dtype=np.uint32)
-        if self.lib.orc_pack_e4m3(_ptr(wt), K, n, _ptr(out)) != 0:
-            raise ValueError("codes must be in {-2,-1,1,2}")
-        return out
-
-    def unpack_e4m3(self, words2d, n: int) -> np.ndarray:
-        """Inverse of pack_e4m3; raises if a padding field is non-zero."""
-        w = np.ascontiguousarray(np.asarray(words2d, dtype=np.uint32))
-        K = w.shape[0]
-        if w.shape[1] != self.words_per_filter(n):
-            raise ValueError("word count does not match n")
-        out = np.empty((K, n), dtype=np.int8)
-        if self.lib.orc_unpack_e4m3(_ptr(w), K, n, _ptr(out)) != 0:
             raise ValueError("non-zero padding field")
         return out
 

@@ -145,52 +145,6 @@ int orc_unpack(const uint32_t *words, int64_t K, int64_t n, int8_t *wt)
     return bad_padding ? -1 : 0;
 }
 
-/* ---- second storage layout: "e4m3-planar" --------------------------------
- * Same words as orc_pack (code i of filter k in word k * wpf + i / 16); inside
- * a word, code l = 4 j + b (group j = l / 4, byte b = l mod 4) keeps m at bit
- * 8 b + j and s at bit 8 b + 4 + j. */
-static int magnitude_bit_e4m3(int64_t i)
-{
-    int64_t l = i % 16;
-    return (int)(8 * (l % 4) + l / 4);
-}
-
-int orc_pack_e4m3(const int8_t *wt, int64_t K, int64_t n, uint32_t *words)
-{
-    int64_t wpf = orc_words_per_filter(n);
-    for (int64_t k = 0; k < K; ++k) {
-        for (int64_t j = 0; j < wpf; ++j)
-            words[k * wpf + j] = 0u;
-        for (int64_t i = 0; i < n; ++i) {
-            uint32_t f;
-            if (field_of(wt[k * n + i], &f) != 0)
-                return -1;
-            uint32_t m = f & 1u, s = f >> 1;
-            int mb = magnitude_bit_e4m3(i);
-            words[k * wpf + i / 16] |= (m << mb) | (s << (mb + 4));
-        }
-    }
-    return 0;
-}
-
-int orc_unpack_e4m3(const uint32_t *words, int64_t K, int64_t n, int8_t *wt)
-{
-    int64_t wpf = orc_words_per_filter(n);
-    int bad_padding = 0;
-    for (int64_t k = 0; k < K; ++k) {
-        for (int64_t i = 0; i < wpf * 16; ++i) {
-            uint32_t w = words[k * wpf + i / 16];
-            int mb = magnitude_bit_e4m3(i);
-            uint32_t f = ((w >> mb) & 1u) + 2u * ((w >> (mb + 4)) & 1u);
-            if (i < n)
-                wt[k * n + i] = (int8_t)value_of(f);
-            else if (f != 0u)
-                bad_padding = 1;
-        }
-    }
-    return bad_padding ? -1 : 0;
-}
-
 /* ---- Eq. 2 (Section 2): quantization error ------------------------------ */
 double orc_quant_error(const float *W, const int8_t *wt, int64_t n, double alpha)
 {

@@ -65,16 +65,6 @@ int orc_pack(const int8_t *wt, int64_t K, int64_t n, uint32_t *words);
 /* Inverse of orc_pack.  Returns 0, or -1 if a padding field is non-zero. */
 int orc_unpack(const uint32_t *words, int64_t K, int64_t n, int8_t *wt);
 
-/* The same codes in the "e4m3-planar" word layout used by the batch-1 fp8
- * GEMV: code i of filter k in word k * words_per_filter + i / 16 as above;
- * with l = i mod 16, group j = l / 4 and byte b = l mod 4, its m bit is bit
- * 8 b + j and its s bit is bit 8 b + 4 + j.  Returns 0, or -1 for a wt value
- * outside {-2,-1,1,2}. */
-int orc_pack_e4m3(const int8_t *wt, int64_t K, int64_t n, uint32_t *words);
-
-/* Inverse of orc_pack_e4m3.  Returns 0, or -1 if a padding field is non-zero. */
-int orc_unpack_e4m3(const uint32_t *words, int64_t K, int64_t n, int8_t *wt);
-
 /* Eq. 2 objective evaluated directly: sum_i (W_i - alpha wt_i)^2. */
 double orc_quant_error(const float *W, const int8_t *wt, int64_t n, double alpha);
 

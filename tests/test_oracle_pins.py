@@ -231,43 +231,6 @@ def pin_pack_roundtrip(orc):
                 orc.unpack(bad, n)
 
 
-def _e4m3_value(byte):
-    """An e4m3 byte by the format's definition: sign bit 7, exponent bits
-    6..3 (bias 7), mantissa bits 2..0 (normal numbers only here)."""
-    s, e, m = byte >> 7, (byte >> 3) & 15, byte & 7
-    assert e > 0
-    return (-1.0) ** s * 2.0 ** (e - 7) * (1.0 + m / 8.0)
-
-
-def pin_pack_e4m3_layout(orc):
-    # code l = 4 j + b keeps m at bit 8 b + j and s at bit 8 b + 4 + j:
-    # l = 0 (-1): s -> bit 4; l = 1 (+2): m -> bit 8; l = 5 (-2): bits 9, 13
-    c = np.ones((1, 16), dtype=np.int8)
-    c[0, 0], c[0, 1], c[0, 5] = -1, 2, -2
-    assert int(orc.pack_e4m3(c)[0, 0]) == 0x2310
-    c = np.ones((1, 17), dtype=np.int8)
-    c[0, 16] = -2
-    w = orc.pack_e4m3(c)
-    assert w.shape == (1, 2) and int(w[0, 0]) == 0 and int(w[0, 1]) == 0x11
-    # the layout's purpose: (w & (0x11111111 << j)) * 2^(3-j) + 0x30303030 is
-    # four e4m3 bytes, byte b = W~/2 of code 4 j + b
-    rng = np.random.default_rng(17)
-    codes = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(4, 64))
-    words = orc.pack_e4m3(codes)
-    for k in range(4):
-        for q in range(4):
-            wq = int(words[k, q])
-            for j in range(4):
-                r = (((wq & (0x11111111 << j)) * (1 << (3 - j))) + 0x30303030) & 0xFFFFFFFF
-                for b in range(4):
-                    assert _e4m3_value((r >> (8 * b)) & 0xFF) == codes[k, 16 * q + 4 * j + b] / 2
-    # round trip with partial last words; the same codes as the first layout
-    for n in (1, 27, 64, 100):
-        cc = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(3, n))
-        assert np.array_equal(orc.unpack_e4m3(orc.pack_e4m3(cc), n), cc)
-        assert np.array_equal(orc.unpack(orc.pack(cc), n), orc.unpack_e4m3(orc.pack_e4m3(cc), n))
-
-
 def pin_dequantized_values(orc):
     rng = np.random.default_rng(16)
     W = rng.normal(0, 1.2, size=(8, 50)).astype(F32)
@@ -426,7 +389,7 @@ def pin_all_zero_filter(orc):
 PINS = [pin_quantize_worked_example, pin_discretize_boundaries,
         pin_alpha_is_least_squares_optimum, pin_alpha_minimizes_J, pin_eq4_closed_form,
         pin_bruteforce_tiny, pin_exact_special_case, pin_pack_bit_layout, pin_pack_roundtrip,
-        pin_pack_e4m3_layout, pin_dequantized_values, pin_conv_worked_example, pin_conv_vs_torch,
+        pin_dequantized_values, pin_conv_worked_example, pin_conv_vs_torch,
         pin_conv_vs_im2col, pin_conv_sites, pin_box_filter, pin_linear, pin_glue,
         pin_all_zero_filter]
 
@@ -452,11 +415,6 @@ MUTANTS = [
      "return (int)(16 * (l % 2) + l / 2);", "return (int)(16 * (l / 8) + l % 8);"),
     ("sign bit next to the magnitude bit", "return magnitude_bit(i) + 8;",
      "return magnitude_bit(i) + 1;"),
-    ("e4m3-planar: group and byte swapped", "return (int)(8 * (l % 4) + l / 4);",
-     "return (int)(8 * (l / 4) + l % 4);"),
-    ("e4m3-planar: sign bit 8 above the magnitude bit",
-     "words[k * wpf + i / 16] |= (m << mb) | (s << (mb + 4));",
-     "words[k * wpf + i / 16] |= (m << mb) | (s << (mb + 8));"),
     ("padding ignored in the row index", "int64_t h = p * sh - ph + r;", "int64_t h = p * sh + r;"),
     ("convolution instead of cross-correlation",
      "double wv = (double)wt[((k * C + c) * R + r) * S + s];",
