@@ -392,9 +392,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) conv_smalltap_kernel(Sma
 // ------------------------------------------------------ tensor-core variant
 // NHWC bf16 activations and NHWC bf16 output without a residual (K % 8 == 0,
 // 16-byte aligned y): the configuration the image networks launch.  The
-// mma.sync loop above issues one m16n8k16 per ~30 cycles per SM
-// sub-partition on this GPU.  Here a CTA takes a tile of up to 128 output
-// pixels and 128 filters:
+// mma.sync loop above spends 64 m16n8k16 per warp and tile plus their
+// fragment loads; here the whole tile's products are KP/16 tcgen05.mma
+// issued by one thread.  A CTA takes a tile of up to 128 output pixels and
+// 128 filters:
 //   1. the patch goes to shared memory; its first batch of elements was
 //      loaded into registers while the previous tile computed;
 //   2. the threads build the im2col rows [pixel][64 codes] in the K-major,
