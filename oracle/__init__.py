@@ -17,6 +17,9 @@ follows:
   quant_error     Eq. 2 objective, evaluated directly
   conv2d_nchw     Eq. 1, seven nested loops, zero padding, cross-correlation
   conv2d_sites    Eq. 1 at selected output sites
+  conv2d_bwd_data, conv2d_bwd_filter   Algorithm 1 TwoBitBackward through
+                  Eq. 1: the input gradient (the adjoint of the convolution
+                  with alpha*W~) and the gradient w.r.t. alpha*W~
   linear          Section 3: fully-connected layer treated as a convolution
   epilogue, maxpool2d_nchw   network glue of the benchmark workloads
 """
@@ -104,6 +107,10 @@ class Oracle:
             "orc_conv2d_nchw_sites": ([P, I, I, I, I, P, P, I, I, I, I, I, I, I, P, I, P, P],
                                       None),
             "orc_linear": ([P, I, I, P, P, I, P, P], None),
+            "orc_conv2d_bwd_data_nchw": ([P, I, I, I, I, P, P, I, I, I, I, I, I, I, I, I, P, P],
+                                         None),
+            "orc_conv2d_bwd_filter_nchw": ([P, I, I, I, I, P, I, I, I, I, I, I, I, I, I, P, P],
+                                           None),
             "orc_epilogue": ([P, P, I, ctypes.c_int], None),
             "orc_maxpool2d_nchw": ([P, I, I, I, I, I, I, I, I, P], None),
             "orc_num_threads": ([], ctypes.c_int),
@@ -194,6 +201,41 @@ class Oracle:
         self.lib.orc_conv2d_nchw(_ptr(x), N, C, H, W, _ptr(wt), _ptr(al), K, R, S,
                                  stride[0], stride[1], pad[0], pad[1], _ptr(y), _ptr(bound))
         return y, bound
+
+    def conv2d_bwd_data(self, dy, wt, al, in_hw, stride=(1, 1), pad=(0, 0)):
+        """Algorithm 1 TwoBitBackward: dx through Eq. 1 with alpha*W~ (NCHW).
+
+        dy float32 [N, K, P, Q]; wt int8 [K, C, R, S]; al float64 [K];
+        in_hw = (H, W) of x.  Returns (dx, bound) float64 [N, C, H, W]."""
+        dy = _f32(dy)
+        wt = np.ascontiguousarray(np.asarray(wt, dtype=np.int8))
+        al = np.ascontiguousarray(np.asarray(al, dtype=np.float64))
+        N, K, P, Q = dy.shape
+        K2, C, R, S = wt.shape
+        H, W = in_hw
+        assert K2 == K and al.shape == (K,) and out_hw(H, W, R, S, stride, pad) == (P, Q)
+        dx = np.empty((N, C, H, W), dtype=np.float64)
+        bound = np.empty_like(dx)
+        self.lib.orc_conv2d_bwd_data_nchw(_ptr(dy), N, K, P, Q, _ptr(wt), _ptr(al), C, H, W, R,
+                                          S, stride[0], stride[1], pad[0], pad[1], _ptr(dx),
+                                          _ptr(bound))
+        return dx, bound
+
+    def conv2d_bwd_filter(self, x, dy, RS, stride=(1, 1), pad=(0, 0)):
+        """Algorithm 1 TwoBitBackward: gradient w.r.t. the approximate filters
+        W^ = alpha*W~ of Eq. 1 (NCHW).  x float32 [N, C, H, W]; dy float32
+        [N, K, P, Q]; RS = (R, S).  Returns (dw, bound) float64 [K, C, R, S]."""
+        x, dy = _f32(x), _f32(dy)
+        N, C, H, W = x.shape
+        N2, K, P, Q = dy.shape
+        R, S = RS
+        assert N2 == N and out_hw(H, W, R, S, stride, pad) == (P, Q)
+        dw = np.empty((K, C, R, S), dtype=np.float64)
+        bound = np.empty_like(dw)
+        self.lib.orc_conv2d_bwd_filter_nchw(_ptr(x), N, C, H, W, _ptr(dy), K, P, Q, R, S,
+                                            stride[0], stride[1], pad[0], pad[1], _ptr(dw),
+                                            _ptr(bound))
+        return dw, bound
 
     def conv2d_sites(self, x, wt, al, sites, stride=(1, 1), pad=(0, 0)):
         """Eq. 1 at output sites [(b, k, p, q), ...]; returns (y, bound) [npts]."""

@@ -208,6 +208,80 @@ void orc_conv2d_nchw(const float *x, int64_t N, int64_t C, int64_t H, int64_t W,
     }
 }
 
+/* ---- Algorithm 1, TwoBitBackward: gradients through Eq. 1 -------------- */
+/* dx is the adjoint of the convolution with the approximate filters
+ * alpha[k] wt[k]: every product that Eq. 1 adds into y[b,k,p,q] sends
+ * dy[b,k,p,q] * alpha[k] * wt back to the input element it read. */
+void orc_conv2d_bwd_data_nchw(const float *dy, int64_t N, int64_t K, int64_t P,
+                              int64_t Q, const int8_t *wt, const double *alpha,
+                              int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
+                              int64_t sh, int64_t sw, int64_t ph, int64_t pw,
+                              double *dx, double *bound)
+{
+    for (int64_t i = 0; i < N * C * H * W; ++i) {
+        dx[i] = 0.0;
+        if (bound)
+            bound[i] = 0.0;
+    }
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+    for (int64_t b = 0; b < N; ++b)
+        for (int64_t k = 0; k < K; ++k)
+            for (int64_t p = 0; p < P; ++p)
+                for (int64_t q = 0; q < Q; ++q) {
+                    double g = (double)dy[((b * K + k) * P + p) * Q + q];
+                    for (int64_t c = 0; c < C; ++c)
+                        for (int64_t r = 0; r < R; ++r)
+                            for (int64_t s = 0; s < S; ++s) {
+                                int64_t h = p * sh + r - ph;
+                                int64_t w = q * sw + s - pw;
+                                if (h < 0 || h >= H || w < 0 || w >= W)
+                                    continue;
+                                double wv = alpha[k] * (double)wt[((k * C + c) * R + r) * S + s];
+                                int64_t o = ((b * C + c) * H + h) * W + w;
+                                dx[o] += g * wv;
+                                if (bound)
+                                    bound[o] += fabs(g * wv);
+                            }
+                }
+}
+
+/* dW^[k,c,r,s] = sum over (b, p, q) of dy[b,k,p,q] times the input element
+ * x[b, c, p sh - ph + r, q sw - pw + s] that Eq. 1 multiplies by
+ * W^[k,c,r,s] (zero outside the image). */
+void orc_conv2d_bwd_filter_nchw(const float *x, int64_t N, int64_t C, int64_t H,
+                                int64_t W, const float *dy, int64_t K, int64_t P,
+                                int64_t Q, int64_t R, int64_t S, int64_t sh, int64_t sw,
+                                int64_t ph, int64_t pw, double *dw, double *bound)
+{
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+    for (int64_t k = 0; k < K; ++k)
+        for (int64_t c = 0; c < C; ++c)
+            for (int64_t r = 0; r < R; ++r)
+                for (int64_t s = 0; s < S; ++s) {
+                    double acc = 0.0, mag = 0.0;
+                    for (int64_t b = 0; b < N; ++b)
+                        for (int64_t p = 0; p < P; ++p)
+                            for (int64_t q = 0; q < Q; ++q) {
+                                int64_t h = r + p * sh - ph;
+                                int64_t w = s + q * sw - pw;
+                                if (h < 0 || h >= H || w < 0 || w >= W)
+                                    continue;
+                                double t = (double)dy[((b * K + k) * P + p) * Q + q] *
+                                           (double)x[((b * C + c) * H + h) * W + w];
+                                acc += t;
+                                mag += fabs(t);
+                            }
+                    int64_t o = ((k * C + c) * R + r) * S + s;
+                    dw[o] = acc;
+                    if (bound)
+                        bound[o] = mag;
+                }
+}
+
 void orc_conv2d_nchw_sites(const float *x, int64_t N, int64_t C, int64_t H,
                            int64_t W, const int8_t *wt, const double *alpha,
                            int64_t K, int64_t R, int64_t S, int64_t sh,

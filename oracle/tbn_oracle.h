@@ -92,6 +92,29 @@ void orc_conv2d_nchw_sites(const float *x, int64_t N, int64_t C, int64_t H,
                            const int64_t *sites, int64_t npts, double *y,
                            double *bound);
 
+/* Algorithm 1, TwoBitBackward, through one convolution (Eq. 1) with the
+ * approximate filters W^ = alpha[k] wt[k]:
+ *   dx[b,c,h,w] = sum over (k, p, q, r, s) with p sh - ph + r = h and
+ *                 q sw - pw + s = w of dy[b,k,p,q] * alpha[k] * wt[k,c,r,s]
+ *   bound[...]  = the same sum of absolute values.
+ * dy is [N][K][P][Q] (fp32 values), wt [K][C][R][S], dx and bound
+ * [N][C][H][W]; bound may be NULL. */
+void orc_conv2d_bwd_data_nchw(const float *dy, int64_t N, int64_t K, int64_t P,
+                              int64_t Q, const int8_t *wt, const double *alpha,
+                              int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
+                              int64_t sh, int64_t sw, int64_t ph, int64_t pw,
+                              double *dx, double *bound);
+
+/*   dW^[k,c,r,s] = sum over (b, p, q) of dy[b,k,p,q] *
+ *                  x[b, c, p sh - ph + r, q sw - pw + s]   (zero outside)
+ *   bound[...]   = the same sum of absolute values.
+ * x [N][C][H][W], dy [N][K][P][Q] (fp32 values), dw and bound [K][C][R][S];
+ * bound may be NULL. */
+void orc_conv2d_bwd_filter_nchw(const float *x, int64_t N, int64_t C, int64_t H,
+                                int64_t W, const float *dy, int64_t K, int64_t P,
+                                int64_t Q, int64_t R, int64_t S, int64_t sh, int64_t sw,
+                                int64_t ph, int64_t pw, double *dw, double *bound);
+
 /* Fully-connected layer (Section 3: treated as a convolution):
  *   y[b,k] = alpha[k] * sum_j x[b,j] * wt[k,j],
  *   bound[b,k] = |alpha[k]| * sum_j |x[b,j]|.

@@ -378,6 +378,60 @@ def pin_glue(orc):
     assert np.array_equal(orc.epilogue(y, None, relu=False), y)
 
 
+BWD_CASES = [
+    # N, C, H, W, K, R, S, stride, pad
+    (2, 3, 7, 6, 4, 3, 2, (2, 1), (1, 1)),
+    (1, 2, 9, 9, 3, 3, 3, (1, 1), (1, 1)),
+    (2, 4, 8, 5, 5, 3, 3, (2, 2), (0, 1)),
+    (1, 1, 6, 7, 2, 1, 1, (1, 1), (0, 0)),
+]
+
+
+def _bwd_case(orc, case, seed):
+    N, C, H, W, K, R, S, st, pd = case
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((N, C, H, W)).astype(F32)
+    wt = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(K, C, R, S))
+    al = rng.random(K) + 0.25
+    y, _ = orc.conv2d_nchw(x, wt, al, st, pd)
+    dy = rng.standard_normal(y.shape).astype(F32)
+    return x, wt, al, y, dy
+
+
+def pin_bwd_adjoint(orc):
+    """<conv(x, W^), dy> = <x, dx> = <W^, dW^>: both gradients are the
+    adjoints of the (pinned) forward convolution, which is linear in x and
+    in W^ = alpha W~."""
+    for i, case in enumerate(BWD_CASES):
+        x, wt, al, y, dy = _bwd_case(orc, case, 40 + i)
+        st, pd = case[7], case[8]
+        dx, bx = orc.conv2d_bwd_data(dy, wt, al, x.shape[2:], st, pd)
+        dw, bw = orc.conv2d_bwd_filter(x, dy, wt.shape[2:], st, pd)
+        w_hat = al[:, None, None, None] * wt
+        ref = float((y * dy).sum())
+        scale = float((np.abs(y) * np.abs(dy)).sum())
+        assert abs(float((x.astype(np.float64) * dx).sum()) - ref) <= 1e-12 * scale
+        assert abs(float((w_hat * dw).sum()) - ref) <= 1e-12 * scale
+        assert np.all(bx >= np.abs(dx) - 1e-12) and np.all(bw >= np.abs(dw) - 1e-12)
+
+
+def pin_bwd_vs_torch(orc):
+    """torch's fp64 conv2d_input / conv2d_weight (autograd's routines) give
+    the same gradients."""
+    for i, case in enumerate(BWD_CASES):
+        x, wt, al, y, dy = _bwd_case(orc, case, 50 + i)
+        st, pd = case[7], case[8]
+        dx, _ = orc.conv2d_bwd_data(dy, wt, al, x.shape[2:], st, pd)
+        dw, _ = orc.conv2d_bwd_filter(x, dy, wt.shape[2:], st, pd)
+        w_hat = torch.from_numpy(al[:, None, None, None] * wt.astype(np.float64))
+        g = torch.from_numpy(dy.astype(np.float64))
+        xt = torch.from_numpy(x.astype(np.float64))
+        dx_t = torch.nn.grad.conv2d_input(xt.shape, w_hat, g, stride=st, padding=pd)
+        dw_t = torch.nn.grad.conv2d_weight(xt, w_hat.shape, g, stride=st, padding=pd)
+        assert np.allclose(dx, dx_t.numpy(), rtol=1e-12, atol=1e-12)
+        assert np.allclose(dw, dw_t.numpy(), rtol=1e-12, atol=1e-12)
+
+
 def pin_all_zero_filter(orc):
     # Eq. 5 with every W_i = 0: numerator 0, denominator n -> alpha = 0 (the
     # paper asks alpha > 0; the formula's value is kept), codes all -1.
@@ -391,7 +445,7 @@ PINS = [pin_quantize_worked_example, pin_discretize_boundaries,
         pin_bruteforce_tiny, pin_exact_special_case, pin_pack_bit_layout, pin_pack_roundtrip,
         pin_dequantized_values, pin_conv_worked_example, pin_conv_vs_torch,
         pin_conv_vs_im2col, pin_conv_sites, pin_box_filter, pin_linear, pin_glue,
-        pin_all_zero_filter]
+        pin_all_zero_filter, pin_bwd_adjoint, pin_bwd_vs_torch]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -422,6 +476,14 @@ MUTANTS = [
     ("alpha not applied", "*y_out = alpha[k] * acc;", "*y_out = acc;"),
     ("transposed linear operand", "acc += xv * (double)wt[k * Kin + j];",
      "acc += xv * (double)wt[(j % Kout) * Kin + (k % Kin)];"),
+    ("input gradient without alpha",
+     "double wv = alpha[k] * (double)wt[((k * C + c) * R + r) * S + s];",
+     "double wv = (double)wt[((k * C + c) * R + r) * S + s];"),
+    ("input gradient with the filter taps mirrored", "dx[o] += g * wv;",
+     "dx[o] += g * alpha[k] * (double)wt[((k * C + c) * R + (R - 1 - r)) * S + (S - 1 - s)];"),
+    ("filter gradient ignores the stride in the row index", "int64_t h = r + p * sh - ph;",
+     "int64_t h = r + p - ph;"),
+    ("filter gradient sums magnitudes", "acc += t;", "acc += fabs(t);"),
     ("bound without abs", "acc += xv * wv;\n                abs_sum += fabs(xv);",
      "acc += xv * wv;\n                abs_sum += xv;"),
 ]
