@@ -33,6 +33,9 @@ ranks over the slowest rank's time.
                       {4096, 8192, 16384}: HBM GB/s on the 2-bit stream
 --workload quantize   tbn_quantize_pack on 8192^2 and 16384^2 fp32 matrices:
                       HBM GB/s at 4.25 bytes per weight
+--workload backward   Algorithm 1's TwoBitBackward through the six VGG-small
+                      convolutions at batch 128 (input and filter gradients):
+                      TFLOP/s of both gradients, 2 x 155.5 GFLOP per step
 --impl reference      the CPU oracle (plain C, fp64) on the VGG-small
                       workload: one image of the batch per step through
                       re-quantization + the six convolutions + glue.
@@ -527,6 +530,143 @@ def oracle_forward_one_image(orc, x_img_nchw_f32, Ws, specs):
     return flops
 
 
+def run_backward(args, rank, world, local_rank):
+    """TwoBitBackward for every VGG-small layer: dx (tensor-core forward
+    kernels on the transposed filters) and dW^ (CUDA-core fp32 kernel)."""
+    import paper_1701_00485_gb300 as tbn
+    from paper_1701_00485_gb300 import inputs
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    peaks, peak_kind = load_peaks()
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    N = 128
+    layers = []
+    hw = 32
+    for i, s in enumerate(inputs.VGG_SMALL["convs"]):
+        st, pd = (s.stride, s.stride), (s.pad, s.pad)
+        P, Q = tbn.conv_out_hw(hw, hw, s.R, s.S, st, pd)
+        x = torch.randn((N, hw, hw, s.C), generator=g, device=dev).to(torch.bfloat16)
+        dy = torch.randn((N, P, Q, s.K), generator=g, device=dev).to(torch.bfloat16)
+        W = inputs.he_normal(s.K, s.C, s.R, s.S, inputs.generator(100 + i))
+        codes, alpha = tbn.tbn_quantize_pack(
+            W.permute(0, 2, 3, 1).reshape(s.K, -1).contiguous().to(dev))
+        shape = (N, s.C, hw, hw, s.K, s.R, s.S, st[0], st[1], pd[0], pd[1])
+        wsd = torch.empty(max(256, tbn.lib().tbn_conv2d_bwd_data_workspace_bytes(*shape)),
+                          dtype=torch.uint8, device=dev)
+        wsf = torch.empty(max(256, tbn.lib().tbn_conv2d_bwd_filter_workspace_bytes(*shape)),
+                          dtype=torch.uint8, device=dev)
+        flops = 2 * N * s.K * P * Q * s.C * s.R * s.S
+        layers.append(dict(s=s, hw=hw, st=st, pd=pd, x=x, dy=dy, codes=codes, alpha=alpha,
+                           wsd=wsd, wsf=wsf, flops=flops))
+        if s.pool is not None:
+            hw = (P - s.pool[0]) // s.pool[1] + 1
+        else:
+            hw = P
+
+    def data_fn(L):
+        s = L["s"]
+        return lambda: tbn.tbn_conv2d_bwd_data(L["dy"], L["codes"], L["alpha"], s.C,
+                                               (L["hw"], L["hw"]), s.R, s.S, L["st"], L["pd"],
+                                               workspace=L["wsd"])
+
+    def filt_fn(L):
+        s = L["s"]
+        return lambda: tbn.tbn_conv2d_bwd_filter(L["x"], L["dy"], s.R, s.S, L["st"], L["pd"],
+                                                 workspace=L["wsf"])
+
+    def time_graph(fns, reps):
+        with torch.cuda.stream(stream):
+            for f in fns:
+                f()
+        torch.cuda.synchronize(dev)
+        gr, ev = _rotating_graph(fns, stream, dev)
+        for _ in range(max(3, args.warmup)):
+            gr.replay()
+        ms = []
+        for _ in range(reps):
+            with torch.cuda.stream(stream):
+                flush.fill_(1)
+                gr.replay()
+            stream.synchronize()
+            ms.append(ev[0].elapsed_time(ev[1]))
+        return float(np.median(ms))
+
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    t0 = time.time()
+    reps = max(5, args.steps // 10)
+    ms_all = time_graph([f(L) for L in layers for f in (data_fn, filt_fn)], reps)
+    ms_data = time_graph([data_fn(L) for L in layers], reps)
+    ms_filt = time_graph([filt_fn(L) for L in layers], reps)
+    per_layer = []
+    for i, L in enumerate(layers):
+        per_layer.append({"layer": "c%d" % (i + 1),
+                          "data_us": round(1e3 * time_graph([data_fn(L)], reps), 2),
+                          "filter_us": round(1e3 * time_graph([filt_fn(L)], reps), 2)})
+    clocks = sampler.stop(t0, time.time())
+    gflop = sum(L["flops"] for L in layers) / 1e9
+    value = 2 * gflop / ms_all
+    bf16_peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops"]))
+    sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    mhz = clocks.get("sm_mhz") or 2070.0
+    fp32_peak = sm * 128 * 2 * mhz * 1e6 / 1e12   # FMA lanes x 2 flops x clock
+    filt_tf = gflop / ms_filt
+    return {"metric": "TBN TwoBitBackward TFLOP/s (VGG-small b128, input + filter gradients)",
+            "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": 1, "steps": reps,
+            "warmup": args.warmup, "ms_per_step": round(ms_all, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (N(0,1) activations and output gradients, He-normal weights)",
+            "config": {"workload": "vgg_small_b128_backward", "global_batch": N,
+                       "l2": "512 MiB write between timed steps"},
+            "input_grad_tflops": round(gflop / ms_data, 3),
+            "filter_grad_tflops": round(filt_tf, 3),
+            "per_layer_us": per_layer,
+            "roofline": {"bound": "alu", "achieved": round(filt_tf, 3), "peak": round(fp32_peak, 1),
+                         "unit": "TFLOP/s", "frac": round(filt_tf / fp32_peak, 4), "traffic": None,
+                         "kernel": "bwd_filter_kernel (fp32 FMA on CUDA cores), 6 launches + "
+                                   "slice reductions",
+                         "peak_kind": "derived: %d SMs x 128 FMA lanes x 2 flops x %.0f MHz"
+                                      % (sm, mhz),
+                         "input_grad_vs_bf16_peak": round(gflop / ms_data / bf16_peak, 4)},
+            "clocks": clocks}
+
+
+def run_cpu_oracle_backward(target_s: float = 10.0, max_s: float = 30.0):
+    """The oracle's TwoBitBackward (both gradients) through the six VGG-small
+    layers, one image of the batch at a time."""
+    import oracle
+    from paper_1701_00485_gb300 import inputs
+    orc = oracle.default()
+    rng = np.random.default_rng(5)
+    specs = inputs.VGG_SMALL["convs"]
+    shapes, hw = [], 32
+    for i, s in enumerate(specs):
+        P, Q = oracle.out_hw(hw, hw, s.R, s.S, (s.stride,) * 2, (s.pad,) * 2)
+        wt = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(s.K, s.C, s.R, s.S))
+        shapes.append((s, hw, P, Q, wt, rng.random(s.K) + 0.5))
+        hw = (P - s.pool[0]) // s.pool[1] + 1 if s.pool is not None else P
+    t0 = time.time()
+    flops, images = 0, 0
+    while True:
+        for s, h, P, Q, wt, al in shapes:
+            x = rng.standard_normal((1, s.C, h, h)).astype(np.float32)
+            dy = rng.standard_normal((1, s.K, P, Q)).astype(np.float32)
+            orc.conv2d_bwd_data(dy, wt, al, (h, h), (s.stride,) * 2, (s.pad,) * 2)
+            orc.conv2d_bwd_filter(x, dy, (s.R, s.S), (s.stride,) * 2, (s.pad,) * 2)
+            flops += 2 * 2 * s.K * P * Q * s.C * s.R * s.S
+        images += 1
+        el = time.time() - t0
+        if el >= target_s or el >= max_s:
+            break
+    return {"value": flops / el / 1e12, "unit": "TFLOP/s", "cores": orc.num_threads(),
+            "kind": "oracle",
+            "sample": "%d image(s): input and filter gradients of the six VGG-small layers "
+                      "(fp64 C oracle)" % images}
+
+
 def run_cpu_oracle(target_s: float = 10.0, max_s: float = 30.0, max_images: int | None = None):
     import oracle
     from paper_1701_00485_gb300 import inputs
@@ -559,7 +699,8 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize"], default="vgg_small")
+    ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize", "backward"],
+                    default="vgg_small")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--gemv-sizes", type=int, nargs="+", default=[4096, 8192, 16384],
                     help="K_out = K_in of the GEMV workload")
@@ -612,12 +753,16 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "vgg_small":
         cpu = run_cpu_oracle()
-    runner = {"vgg_small": run_vgg, "gemv": run_gemv, "quantize": run_quantize}[args.workload]
+    elif rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "backward":
+        cpu = run_cpu_oracle_backward()
+    runner = {"vgg_small": run_vgg, "gemv": run_gemv, "quantize": run_quantize,
+              "backward": run_backward}[args.workload]
     res = runner(args, rank, world, local_rank)
     if rank == 0:
         if cpu is not None:
             res["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")}
-            res["cpu_baseline"]["images_per_s"] = round(cpu["images_per_s"], 4)
+            if "images_per_s" in cpu:
+                res["cpu_baseline"]["images_per_s"] = round(cpu["images_per_s"], 4)
         print(json.dumps(res))
     if world > 1:
         torch.distributed.destroy_process_group()

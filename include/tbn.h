@@ -13,6 +13,8 @@
  *   tbn_linear_fwd      fully-connected layer, treated as a convolution
  *                       (Section 3); tbn_linear_fwd_ws with caller-owned
  *                       scratch for the batch-1 fp32 table-lookup GEMV
+ *   tbn_conv2d_bwd_data, tbn_conv2d_bwd_filter   Algorithm 1's
+ *                       TwoBitBackward through a convolution
  *   tbn_maxpool2d_nhwc, tbn_nchw_to_nhwc   network glue between layers
  *
  * Conventions shared by every call
@@ -71,7 +73,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 4
+#define TBN_ABI_VERSION 5
 
 typedef enum {
   TBN_OK = 0,
@@ -224,6 +226,44 @@ tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N
                                      int64_t H, int64_t W, int64_t K, int64_t R, int64_t S,
                                      int64_t stride_h, int64_t stride_w, int64_t pad_h,
                                      int64_t pad_w);
+
+/* TwoBitBackward (Algorithm 1) through one convolution of Eq. 1, whose
+ * filters are the approximate filters W^ = alpha[k] W~[k] (the backward pass
+ * uses them, not the real-valued weights).  Shapes as tbn_conv2d_fwd in NHWC:
+ * x [N][H][W][C], dy = dC/dy [N][P][Q][K], codes [K][tbn_packed_words(R S C)]
+ * in (r, s, c) order; pad_h <= R - 1 and pad_w <= S - 1 (else
+ * TBN_ERR_UNSUPPORTED).  Both calls are asynchronous on `stream`, need a
+ * caller workspace (256-byte aligned, contents on entry irrelevant; calls
+ * that may run concurrently must not share one) and are bitwise
+ * reproducible.
+ *
+ * Input gradient: dx[n,h,w,c] = sum over (k, p, q, r, s) with
+ * p sh - pad_h + r = h and q sw - pad_w + s = w of dy[n,p,q,k] alpha[k]
+ * W~[k,r,s,c], written to dx [N][H][W][C] (bf16 or fp32).  It runs as a
+ * stride-1 convolution (this library's forward kernels) of
+ * bf16(alpha[k] dy) dilated by the stride with the filters transposed and
+ * mirrored; rounding alpha dy to bf16 adds at most 2^-9 relative per term
+ * to the fp32 accumulation. */
+size_t tbn_conv2d_bwd_data_workspace_bytes(int64_t N, int64_t C, int64_t H, int64_t W, int64_t K,
+                                           int64_t R, int64_t S, int64_t stride_h,
+                                           int64_t stride_w, int64_t pad_h, int64_t pad_w);
+tbn_status tbn_conv2d_bwd_data(const void *dy, int64_t N, int64_t C, int64_t H, int64_t W,
+                               const uint32_t *codes, const float *alpha, int64_t K, int64_t R,
+                               int64_t S, int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                               int64_t pad_w, void *dx, tbn_dtype dxdt, void *workspace,
+                               size_t workspace_bytes, tbn_stream stream);
+
+/* Filter gradient: dW^[k,r,s,c] = sum over (n, p, q) of dy[n,p,q,k] *
+ * x[n, p sh - pad_h + r, q sw - pad_w + s, c] (zero outside the image),
+ * fp32 [K][R][S][C] (the codes' order), fp32 accumulation of exact bf16
+ * products; Algorithm 1 applies it to the real-valued weights. */
+size_t tbn_conv2d_bwd_filter_workspace_bytes(int64_t N, int64_t C, int64_t H, int64_t W,
+                                             int64_t K, int64_t R, int64_t S, int64_t stride_h,
+                                             int64_t stride_w, int64_t pad_h, int64_t pad_w);
+tbn_status tbn_conv2d_bwd_filter(const void *x, const void *dy, int64_t N, int64_t C, int64_t H,
+                                 int64_t W, int64_t K, int64_t R, int64_t S, int64_t stride_h,
+                                 int64_t stride_w, int64_t pad_h, int64_t pad_w, float *dw,
+                                 void *workspace, size_t workspace_bytes, tbn_stream stream);
 
 /* Fully-connected layer (Section 3: treated as a convolution):
  *   y[b,k] = alpha[k] * sum_j x[b,j] W~[k,j]

@@ -24,7 +24,7 @@ __all__ = [
     "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack", "tbn_conv2d_fwd",
     "tbn_linear_fwd", "tbn_linear_fwd_ws", "tbn_linear_workspace_bytes",
     "tbn_linear_fwd_noalloc", "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_device_error",
-    "tbn_conv2d_select_algo", "conv_out_hw",
+    "tbn_conv2d_select_algo", "conv_out_hw", "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter",
     "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_NCHW_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
     "TBN_CONV_SMALL_TAPS",
@@ -47,7 +47,8 @@ EXPORTED = [
     "tbn_device_error", "tbn_quantize_pack", "tbn_quantize_pack_group", "tbn_unpack",
     "tbn_conv2d_fwd", "tbn_conv2d_fwd_algo", "tbn_conv2d_select_algo", "tbn_linear_fwd",
     "tbn_linear_workspace_bytes", "tbn_linear_fwd_ws", "tbn_linear_fwd_noalloc",
-    "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc",
+    "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_conv2d_bwd_data_workspace_bytes",
+    "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter_workspace_bytes", "tbn_conv2d_bwd_filter",
 ]
 
 
@@ -71,7 +72,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 4  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 5  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -113,6 +114,11 @@ def lib():
             "tbn_linear_fwd_noalloc": ([P, I32, I64, I64, U32P, P, I64, P, I32,
                                         ctypes.POINTER(Epilogue), P], I32),
             "tbn_maxpool2d_nhwc": ([P, I32, I64, I64, I64, I64, I64, I64, I64, I64, P, P], I32),
+            "tbn_conv2d_bwd_data_workspace_bytes": ([I64] * 11, ctypes.c_size_t),
+            "tbn_conv2d_bwd_data": ([P, I64, I64, I64, I64, U32P, P] + [I64] * 7 +
+                                    [P, I32, P, ctypes.c_size_t, P], I32),
+            "tbn_conv2d_bwd_filter_workspace_bytes": ([I64] * 11, ctypes.c_size_t),
+            "tbn_conv2d_bwd_filter": ([P, P] + [I64] * 11 + [P, P, ctypes.c_size_t, P], I32),
             "tbn_nchw_to_nhwc": ([P, I32, I64, I64, I64, I64, I64, P, P], I32),
         }
         for name, (args, res) in sig.items():
@@ -256,6 +262,52 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
         stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,
         ctypes.byref(e) if e is not None else None, algo, _stream(stream)), "tbn_conv2d_fwd")
     return out
+
+
+def _bwd_shape(N, C, H, W, K, R, S, stride, pad):
+    return (N, C, H, W, K, R, S, stride[0], stride[1], pad[0], pad[1])
+
+
+def tbn_conv2d_bwd_data(dy: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, C: int,
+                        in_hw, R: int, S: int, stride=(1, 1), pad=(0, 0), out_dtype=None,
+                        workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Algorithm 1 TwoBitBackward, input gradient: dy [N,P,Q,K] bf16 (NHWC) ->
+    dx [N,H,W,C] through the convolution with alpha*W~ (codes in (r,s,c) order)."""
+    _cuda(dy, "dy"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
+    N, P, Q, K = dy.shape
+    H, W = in_hw
+    shape = _bwd_shape(N, C, H, W, K, R, S, stride, pad)
+    n = int(lib().tbn_conv2d_bwd_data_workspace_bytes(*shape))
+    if workspace is None:
+        workspace = torch.empty(max(n, 256), dtype=torch.uint8, device=dy.device)
+    ydt = TBN_BF16 if out_dtype in (None, torch.bfloat16) else TBN_F32
+    dx = torch.empty((N, H, W, C), dtype=_torch_dt(ydt), device=dy.device)
+    _check(lib().tbn_conv2d_bwd_data(dy.data_ptr(), N, C, H, W, codes.data_ptr(),
+                                     alpha.data_ptr(), K, R, S, stride[0], stride[1], pad[0],
+                                     pad[1], dx.data_ptr(), ydt, workspace.data_ptr(),
+                                     workspace.numel() * workspace.element_size(),
+                                     _stream(stream)), "tbn_conv2d_bwd_data")
+    return dx
+
+
+def tbn_conv2d_bwd_filter(x: torch.Tensor, dy: torch.Tensor, R: int, S: int, stride=(1, 1),
+                          pad=(0, 0), workspace: torch.Tensor | None = None,
+                          stream=None) -> torch.Tensor:
+    """Algorithm 1 TwoBitBackward, gradient w.r.t. alpha*W~: x [N,H,W,C] and
+    dy [N,P,Q,K] bf16 (NHWC) -> dW^ [K, R*S*C] fp32 in (r,s,c) order."""
+    _cuda(x, "x"), _cuda(dy, "dy")
+    N, H, W, C = x.shape
+    K = dy.shape[3]
+    shape = _bwd_shape(N, C, H, W, K, R, S, stride, pad)
+    n = int(lib().tbn_conv2d_bwd_filter_workspace_bytes(*shape))
+    if workspace is None:
+        workspace = torch.empty(max(n, 256), dtype=torch.uint8, device=x.device)
+    dw = torch.empty((K, R * S * C), dtype=torch.float32, device=x.device)
+    _check(lib().tbn_conv2d_bwd_filter(x.data_ptr(), dy.data_ptr(), *shape, dw.data_ptr(),
+                                       workspace.data_ptr(),
+                                       workspace.numel() * workspace.element_size(),
+                                       _stream(stream)), "tbn_conv2d_bwd_filter")
+    return dw
 
 
 def tbn_conv2d_select_algo(x_dtype, layout, N, C, H, W, K, R, S, stride=(1, 1), pad=(0, 0)):

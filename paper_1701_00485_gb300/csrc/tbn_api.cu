@@ -168,6 +168,12 @@ tbn_status run_conv(const ConvProblem& p, tbn_conv_algo algo, cudaStream_t s) {
 
 }  // namespace
 
+namespace tbn {
+tbn_status run_conv_auto(const ConvProblem& p, cudaStream_t s) {
+  return run_conv(p, TBN_CONV_AUTO, s);
+}
+}  // namespace tbn
+
 extern "C" {
 
 int tbn_abi_version(void) { return TBN_ABI_VERSION; }
@@ -353,6 +359,90 @@ tbn_status tbn_linear_fwd_noalloc(const void* x, tbn_dtype xdt, int64_t B, int64
   if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "linear (no-alloc): %s", why);
   return launch_gemv_lut_static(x, K_in, codes, alpha, K_out, y, ydt, epi ? epi->relu : 0,
                                 epi ? epi->residual : nullptr, as_stream(stream));
+}
+
+}  // extern "C"
+
+namespace {
+
+// Shape checks shared by the backward entry points; fills `sh`.
+tbn_status validate_bwd(int64_t N, int64_t C, int64_t H, int64_t W, int64_t K, int64_t R,
+                        int64_t S, int64_t sh, int64_t sw, int64_t ph, int64_t pw,
+                        BwdConvShape* out) {
+  if (N < 1 || C < 1 || H < 1 || W < 1 || K < 1 || R < 1 || S < 1)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward: sizes must be >= 1");
+  if (sh < 1 || sw < 1 || ph < 0 || pw < 0)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward: bad stride/pad");
+  if (H + 2 * ph < R || W + 2 * pw < S)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward: kernel larger than padded input");
+  BwdConvShape& p = *out;
+  p.N = N; p.C = C; p.H = H; p.W = W; p.K = K; p.R = R; p.S = S;
+  p.sh = sh; p.sw = sw; p.ph = ph; p.pw = pw;
+  p.P = (H + 2 * ph - R) / sh + 1;
+  p.Q = (W + 2 * pw - S) / sw + 1;
+  const char* why = bwd_shape_reason(p);
+  if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
+  return TBN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t tbn_conv2d_bwd_data_workspace_bytes(int64_t N, int64_t C, int64_t H, int64_t W, int64_t K,
+                                           int64_t R, int64_t S, int64_t stride_h,
+                                           int64_t stride_w, int64_t pad_h, int64_t pad_w) {
+  BwdConvShape p{};
+  if (validate_bwd(N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w, &p) != TBN_OK) return 0;
+  return bwd_data_workspace_bytes(p);
+}
+
+tbn_status tbn_conv2d_bwd_data(const void* dy, int64_t N, int64_t C, int64_t H, int64_t W,
+                               const uint32_t* codes, const float* alpha, int64_t K, int64_t R,
+                               int64_t S, int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                               int64_t pad_w, void* dx, tbn_dtype dxdt, void* workspace,
+                               size_t workspace_bytes, tbn_stream stream) {
+  if (!dy || !codes || !alpha || !dx || !workspace)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward data: null pointer");
+  if (dxdt != TBN_F32 && dxdt != TBN_BF16)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward data: bad dx dtype");
+  BwdConvShape p{};
+  const tbn_status st =
+      validate_bwd(N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w, &p);
+  if (st != TBN_OK) return st;
+  if (workspace_bytes < bwd_data_workspace_bytes(p))
+    return fail(TBN_ERR_INVALID_ARG, "conv backward data: workspace smaller than %zu bytes",
+                bwd_data_workspace_bytes(p));
+  if (!is_aligned(dy, 2) || !is_aligned(codes, 4) || !is_aligned(alpha, 4) ||
+      !is_aligned(dx, dtype_size(dxdt)) || !is_aligned(workspace, 256))
+    return fail(TBN_ERR_MISALIGNED, "conv backward data: misaligned pointer");
+  return launch_bwd_data(p, dy, codes, alpha, dx, dxdt, workspace, as_stream(stream));
+}
+
+size_t tbn_conv2d_bwd_filter_workspace_bytes(int64_t N, int64_t C, int64_t H, int64_t W,
+                                             int64_t K, int64_t R, int64_t S, int64_t stride_h,
+                                             int64_t stride_w, int64_t pad_h, int64_t pad_w) {
+  BwdConvShape p{};
+  if (validate_bwd(N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w, &p) != TBN_OK) return 0;
+  return bwd_filter_workspace_bytes(p);
+}
+
+tbn_status tbn_conv2d_bwd_filter(const void* x, const void* dy, int64_t N, int64_t C, int64_t H,
+                                 int64_t W, int64_t K, int64_t R, int64_t S, int64_t stride_h,
+                                 int64_t stride_w, int64_t pad_h, int64_t pad_w, float* dw,
+                                 void* workspace, size_t workspace_bytes, tbn_stream stream) {
+  if (!x || !dy || !dw || !workspace)
+    return fail(TBN_ERR_INVALID_ARG, "conv backward filter: null pointer");
+  BwdConvShape p{};
+  const tbn_status st =
+      validate_bwd(N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w, &p);
+  if (st != TBN_OK) return st;
+  if (workspace_bytes < bwd_filter_workspace_bytes(p))
+    return fail(TBN_ERR_INVALID_ARG, "conv backward filter: workspace smaller than %zu bytes",
+                bwd_filter_workspace_bytes(p));
+  if (!is_aligned(x, 2) || !is_aligned(dy, 2) || !is_aligned(dw, 4) || !is_aligned(workspace, 256))
+    return fail(TBN_ERR_MISALIGNED, "conv backward filter: misaligned pointer");
+  return launch_bwd_filter(p, x, dy, dw, workspace, as_stream(stream));
 }
 
 tbn_status tbn_maxpool2d_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,

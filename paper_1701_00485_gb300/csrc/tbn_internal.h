@@ -59,6 +59,14 @@ struct ConvProblem {
   int pool;  // 0 or 2 (2x2 max pool, stride 2, after ReLU)
 };
 
+// The shape of one convolution for its backward pass (NHWC bf16).
+struct BwdConvShape {
+  int64_t N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
+};
+
+// AUTO algorithm dispatch of tbn_conv2d_fwd for an already validated problem.
+tbn_status run_conv_auto(const ConvProblem& p, cudaStream_t s);
+
 // ---- launchers (each defined next to its kernels) ----
 tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStream_t s);
 tbn_status launch_unpack(const uint32_t* codes, const float* alpha, int64_t K, int64_t n,
@@ -96,6 +104,16 @@ size_t gemv_lut_static_scratch_bytes();
 tbn_status launch_gemv_lut_static(const void* x, int64_t K_in, const uint32_t* codes,
                                   const float* alpha, int64_t K_out, void* y, tbn_dtype ydt,
                                   int relu, const void* residual, cudaStream_t s);
+
+// Algorithm 1 TwoBitBackward through a convolution (tbn_conv_bwd.cu).
+const char* bwd_shape_reason(const BwdConvShape& p);
+size_t bwd_data_workspace_bytes(const BwdConvShape& p);
+tbn_status launch_bwd_data(const BwdConvShape& p, const void* dy, const uint32_t* codes,
+                           const float* alpha, void* dx, tbn_dtype dxdt, void* workspace,
+                           cudaStream_t s);
+size_t bwd_filter_workspace_bytes(const BwdConvShape& p);
+tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* dy, float* dw,
+                             void* workspace, cudaStream_t s);
 
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
