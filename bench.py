@@ -34,8 +34,9 @@ ranks over the slowest rank's time.
 --workload quantize   tbn_quantize_pack on 8192^2 and 16384^2 fp32 matrices:
                       HBM GB/s at 4.25 bytes per weight
 --workload backward   Algorithm 1's TwoBitBackward through the six VGG-small
-                      convolutions at batch 128 (input and filter gradients):
-                      TFLOP/s of both gradients, 2 x 155.5 GFLOP per step
+                      convolutions at batch 128: the filter gradients of all
+                      six layers and the input gradients of c2..c6 (the
+                      image itself needs none), 309.2 GFLOP per step
 --impl reference      the CPU oracle (plain C, fp64) on the VGG-small
                       workload: one image of the batch per step through
                       re-quantization + the six convolutions + glue.
@@ -598,8 +599,10 @@ def run_backward(args, rank, world, local_rank):
     sampler.start()
     t0 = time.time()
     reps = max(5, args.steps // 10)
-    ms_all = time_graph([f(L) for L in layers for f in (data_fn, filt_fn)], reps)
-    ms_data = time_graph([data_fn(L) for L in layers], reps)
+    # the first layer's input gradient (w.r.t. the image) is not part of the pass
+    step_fns = [filt_fn(layers[0])] + [f(L) for L in layers[1:] for f in (data_fn, filt_fn)]
+    ms_all = time_graph(step_fns, reps)
+    ms_data = time_graph([data_fn(L) for L in layers[1:]], reps)
     ms_filt = time_graph([filt_fn(L) for L in layers], reps)
     per_layer = []
     for i, L in enumerate(layers):
@@ -607,12 +610,10 @@ def run_backward(args, rank, world, local_rank):
                           "data_us": round(1e3 * time_graph([data_fn(L)], reps), 2),
                           "filter_us": round(1e3 * time_graph([filt_fn(L)], reps), 2)})
     clocks = sampler.stop(t0, time.time())
-    gflop = sum(L["flops"] for L in layers) / 1e9
-    value = 2 * gflop / ms_all
+    gflop = sum(L["flops"] for L in layers) / 1e9              # one gradient of every layer
+    gflop_data = sum(L["flops"] for L in layers[1:]) / 1e9
+    value = (gflop + gflop_data) / ms_all
     bf16_peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops"]))
-    sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    mhz = clocks.get("sm_mhz") or 2070.0
-    fp32_peak = sm * 128 * 2 * mhz * 1e6 / 1e12   # FMA lanes x 2 flops x clock
     filt_tf = gflop / ms_filt
     return {"metric": "TBN TwoBitBackward TFLOP/s (VGG-small b128, input + filter gradients)",
             "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": 1, "steps": reps,
@@ -621,16 +622,16 @@ def run_backward(args, rank, world, local_rank):
             "data": "synthetic (N(0,1) activations and output gradients, He-normal weights)",
             "config": {"workload": "vgg_small_b128_backward", "global_batch": N,
                        "l2": "512 MiB write between timed steps"},
-            "input_grad_tflops": round(gflop / ms_data, 3),
+            "gflop_per_step": round(gflop + gflop_data, 3),
+            "input_grad_tflops": round(gflop_data / ms_data, 3),
             "filter_grad_tflops": round(filt_tf, 3),
             "per_layer_us": per_layer,
-            "roofline": {"bound": "alu", "achieved": round(filt_tf, 3), "peak": round(fp32_peak, 1),
-                         "unit": "TFLOP/s", "frac": round(filt_tf / fp32_peak, 4), "traffic": None,
-                         "kernel": "bwd_filter_kernel (fp32 FMA on CUDA cores), 6 launches + "
-                                   "slice reductions",
-                         "peak_kind": "derived: %d SMs x 128 FMA lanes x 2 flops x %.0f MHz"
-                                      % (sm, mhz),
-                         "input_grad_vs_bf16_peak": round(gflop / ms_data / bf16_peak, 4)},
+            "roofline": {"bound": "tensor", "achieved": round(filt_tf, 3), "peak": bf16_peak,
+                         "unit": "TFLOP/s", "frac": round(filt_tf / bf16_peak, 4), "traffic": None,
+                         "kernel": "bwd_filter_async_kernel (mma.sync m16n8k16 bf16, cp.async "
+                                   "ring; c1: bwd_filter_kernel), 6 launches + slice reductions",
+                         "peak_kind": "%s bf16 dense, sustained" % peak_kind,
+                         "input_grad_vs_bf16_peak": round(gflop_data / ms_data / bf16_peak, 4)},
             "clocks": clocks}
 
 

@@ -13,8 +13,8 @@
 // * Filter gradient dW^[k, r, s, c] = sum over (n, p, q) of dy[n, p, q, k]
 //   x[n, p sigma - pad + r, q sigma - pad + s, c]: a product of dy^T
 //   (K x pixels) and the im2col view of x (pixels x R S C).  Each CTA
-//   computes a 64 x 64 tile over a slice of the pixels with fp32 FMA on
-//   CUDA cores (bf16 x bf16 products are exact in fp32); a second kernel
+//   computes a 64 x 64 tile over a slice of the pixels on mma.sync
+//   tensor cores (bf16 products exact, fp32 accumulation); a second kernel
 //   adds the slices in slice order, so results are bitwise reproducible.
 #include <cuda_bf16.h>
 
@@ -64,36 +64,55 @@ __global__ void __launch_bounds__(256) transpose_codes_kernel(
 }
 
 // dyd [N][Hd][Wd][K] bf16 = alpha_k dy at (u / sh, v / sw) where both divide,
-// zero elsewhere; also ones[c] = 1 for the transposed filters' scales.
+// zero elsewhere; also ones[c] = 1 for the transposed filters' scales.  One
+// thread per output pixel, eight channels per step (16-byte loads and
+// stores when K % 8 == 0 and dy, dyd are 16-byte aligned).
 __global__ void __launch_bounds__(256) dilate_scale_kernel(
     const __nv_bfloat16* __restrict__ dy, const float* __restrict__ alpha, int N, int P, int Q,
     int K, int Hd, int Wd, int sh, int sw, __nv_bfloat16* __restrict__ dyd,
-    float* __restrict__ ones, int C) {
-  const int64_t total = static_cast<int64_t>(N) * Hd * Wd * K;
+    float* __restrict__ ones, int C, int vec) {
+  const int64_t npix = static_cast<int64_t>(N) * Hd * Wd;
   const int64_t tid = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (tid < C) ones[tid] = 1.0f;
-  for (int64_t e = tid; e < total; e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int k = static_cast<int>(e % K);
-    int64_t t = e / K;
-    const int v = static_cast<int>(t % Wd);
-    t /= Wd;
+  for (int64_t c = tid; c < C; c += static_cast<int64_t>(gridDim.x) * blockDim.x) ones[c] = 1.0f;
+  for (int64_t e = tid; e < npix; e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int v = static_cast<int>(e % Wd);
+    const int64_t t = e / Wd;
     const int u = static_cast<int>(t % Hd);
     const int n = static_cast<int>(t / Hd);
-    float val = 0.0f;
-    if (u % sh == 0 && v % sw == 0) {
-      const int p = u / sh, q = v / sw;
-      if (p < P && q < Q)
-        val = __ldg(alpha + k) *
-              __bfloat162float(dy[((static_cast<int64_t>(n) * P + p) * Q + q) * K + k]);
+    const bool hit = u % sh == 0 && v % sw == 0 && u / sh < P && v / sw < Q;
+    const __nv_bfloat16* src =
+        hit ? dy + ((static_cast<int64_t>(n) * P + u / sh) * Q + v / sw) * K : nullptr;
+    __nv_bfloat16* dst = dyd + e * K;
+    if (vec) {
+      for (int k = 0; k < K; k += 8) {
+        uint4 o = make_uint4(0u, 0u, 0u, 0u);
+        if (hit) {
+          const uint4 i4 = __ldg(reinterpret_cast<const uint4*>(src + k));
+          const uint32_t iw[4] = {i4.x, i4.y, i4.z, i4.w};
+          uint32_t ow[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&iw[q]);
+            const float2 f = __bfloat1622float2(b);
+            const __nv_bfloat162 r =
+                __floats2bfloat162_rn(__ldg(alpha + k + 2 * q) * f.x, __ldg(alpha + k + 2 * q + 1) * f.y);
+            ow[q] = *reinterpret_cast<const uint32_t*>(&r);
+          }
+          o = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+        }
+        *reinterpret_cast<uint4*>(dst + k) = o;
+      }
+    } else {
+      for (int k = 0; k < K; ++k)
+        dst[k] = __float2bfloat16_rn(hit ? __ldg(alpha + k) * __bfloat162float(src[k]) : 0.0f);
     }
-    dyd[e] = __float2bfloat16_rn(val);
   }
 }
 
 // ------------------------------------------------------------ filter grad
 constexpr int kTileM = 64;    // filters k
 constexpr int kTileN = 64;    // (r, s, c) columns
-constexpr int kChunk = 32;    // pixels per shared-memory chunk
+constexpr int kChunk = 64;    // pixels per shared-memory chunk
 constexpr int kBwdThreads = 256;
 
 struct BwdFilterArgs {
@@ -105,17 +124,42 @@ struct BwdFilterArgs {
   int rsc;       // R S C
   int slices;
   int64_t pix_per_slice;
+  int dy_vec, x_vec;   // 16-byte loads possible (K % 8 == 0 / C % 8 == 0, aligned)
 };
 
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                          uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Shared tiles are [pixel][64 bf16]: 128-byte rows of eight 16-byte chunks,
+// chunk c of row r stored at c ^ (r & 7) (conflict-free ldmatrix).
+__device__ __forceinline__ uint32_t tile_off(int row, int chunk) {
+  return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
 // CTA (bx, by, bz): filters 64 bx .., columns 64 by .., pixels of slice bz.
-// Thread (ty, tx) = (tid / 16, tid % 16) accumulates filters 4 ty .. and
-// columns 4 tx .. of the tile.
+// dW^ tile = dy^T (filters x pixels) * im2col(x) (pixels x columns) on
+// mma.m16n8k16 (bf16 products exact, fp32 accumulation): warp w owns
+// filters 16 (w % 4) .. and columns 32 (w / 4) .. (four 8-column n-tiles).
+// Both operands come from the pixel-major tiles by ldmatrix.trans.  Thread
+// i fills chunk i % 8 of pixel row i / 8 (and row i / 8 + 32) of both
+// tiles; the next chunk's loads are issued before the current MMAs.
 __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilterArgs a) {
-  __shared__ __align__(16) float sdy[kChunk][kTileM];
-  __shared__ __align__(16) float sx[kChunk][kTileN];
+  __shared__ __align__(128) uint8_t sdy[kChunk * 128];
+  __shared__ __align__(128) uint8_t sx[kChunk * 128];
   __shared__ int col_r[kTileN], col_s[kTileN], col_c[kTileN];
-  __shared__ int px_n[kChunk], px_h[kChunk], px_w[kChunk];
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int k0 = blockIdx.x * kTileM, j0 = blockIdx.y * kTileN;
   if (tid < kTileN) {
     const int j = j0 + tid;
@@ -124,72 +168,213 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
     col_s[tid] = rs % a.S;
     col_r[tid] = j < a.rsc ? rs / a.S : -1;   // -1: column past R S C
   }
-  const int ty = tid >> 4, tx = tid & 15;
+  __syncthreads();
+  const int my_chunk = tid & 7, my_row = tid >> 3;   // rows my_row and my_row + 32
+  const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
+  const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
+  const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
+
+  // global loads of one chunk into registers: 8 filters of dy and 8 im2col
+  // columns of x for pixels p0 + my_row and p0 + my_row + 32
+  auto load = [&](int64_t p0, uint4 (&vd)[2], uint4 (&vx)[2]) {
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int64_t pix = p0 + my_row + 32 * h2;
+      uint32_t d[4] = {0u, 0u, 0u, 0u}, xv[4] = {0u, 0u, 0u, 0u};
+      if (pix < pend) {
+        const int kb = k0 + 8 * my_chunk;
+        const __nv_bfloat16* dyp = a.dy + pix * a.K + kb;
+        if (a.dy_vec && kb + 8 <= a.K) {
+          const uint4 v = __ldg(reinterpret_cast<const uint4*>(dyp));
+          d[0] = v.x; d[1] = v.y; d[2] = v.z; d[3] = v.w;
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            if (kb + e < a.K)
+              d[e >> 1] |= static_cast<uint32_t>(__bfloat16_as_ushort(dyp[e])) << (16 * (e & 1));
+        }
+        const int n = static_cast<int>(pix / pq);
+        const int rem = static_cast<int>(pix - static_cast<int64_t>(n) * pq);
+        const int h0 = (rem / a.Q) * a.sh - a.ph, w0 = (rem % a.Q) * a.sw - a.pw;
+        const int jc = 8 * my_chunk;
+        const int r = col_r[jc];
+        if (a.x_vec && r >= 0 && jc + 7 < kTileN && col_r[jc + 7] == r && col_s[jc + 7] == col_s[jc]) {
+          // eight consecutive channels of one tap
+          const int hh = h0 + r, ww = w0 + col_s[jc];
+          if (hh >= 0 && hh < a.H && ww >= 0 && ww < a.W) {
+            const uint4 v = __ldg(reinterpret_cast<const uint4*>(
+                a.x + ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + col_c[jc]));
+            xv[0] = v.x; xv[1] = v.y; xv[2] = v.z; xv[3] = v.w;
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int re = col_r[jc + e];
+            if (re < 0) continue;
+            const int hh = h0 + re, ww = w0 + col_s[jc + e];
+            if (hh >= 0 && hh < a.H && ww >= 0 && ww < a.W)
+              xv[e >> 1] |= static_cast<uint32_t>(__bfloat16_as_ushort(
+                                a.x[((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C +
+                                    col_c[jc + e]]))
+                            << (16 * (e & 1));
+          }
+        }
+      }
+      vd[h2] = make_uint4(d[0], d[1], d[2], d[3]);
+      vx[h2] = make_uint4(xv[0], xv[1], xv[2], xv[3]);
+    }
+  };
+
   float acc[4][4];
 #pragma unroll
   for (int i = 0; i < 4; ++i)
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-  const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
-  const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
+  const uint32_t sdy_s = smem_addr(sdy), sx_s = smem_addr(sx);
+  const int wf = 16 * (warp & 3), wj = 32 * (warp >> 2);
+  const int mi = lane >> 3, lr = lane & 7;
+  uint4 vd[2], vx[2];
+  if (pbeg < pend) load(pbeg, vd, vx);
   for (int64_t p0 = pbeg; p0 < pend; p0 += kChunk) {
-    __syncthreads();   // previous chunk consumed; column tables written
-    if (tid < kChunk) {
-      const int64_t pix = p0 + tid;
-      int n = -1, h = 0, w = 0;
-      if (pix < pend) {
-        const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
-        n = static_cast<int>(pix / pq);
-        const int rem = static_cast<int>(pix - static_cast<int64_t>(n) * pq);
-        h = (rem / a.Q) * a.sh - a.ph;
-        w = (rem % a.Q) * a.sw - a.pw;
-      }
-      px_n[tid] = n;
-      px_h[tid] = h;
-      px_w[tid] = w;
-    }
-    // dy chunk: 32 pixels x 64 filters (rows of dy are K-contiguous)
-    for (int e = tid; e < kChunk * kTileM; e += kBwdThreads) {
-      const int pr = e / kTileM, kc = e % kTileM;
-      const int64_t pix = p0 + pr;
-      const int k = k0 + kc;
-      sdy[pr][kc] = (pix < pend && k < a.K) ? __bfloat162float(a.dy[pix * a.K + k]) : 0.0f;
-    }
-    __syncthreads();   // pixel table ready
-    // im2col chunk: 32 pixels x 64 (r, s, c) columns of x
-    for (int e = tid; e < kChunk * kTileN; e += kBwdThreads) {
-      const int pr = e / kTileN, jc = e % kTileN;
-      const int n = px_n[pr], r = col_r[jc];
-      float v = 0.0f;
-      if (n >= 0 && r >= 0) {
-        const int h = px_h[pr] + r, w = px_w[pr] + col_s[jc];
-        if (h >= 0 && h < a.H && w >= 0 && w < a.W)
-          v = __bfloat162float(
-              a.x[((static_cast<int64_t>(n) * a.H + h) * a.W + w) * a.C + col_c[jc]]);
-      }
-      sx[pr][jc] = v;
+    __syncthreads();   // the previous chunk's fragments have been read
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      *reinterpret_cast<uint4*>(sdy + tile_off(my_row + 32 * h2, my_chunk)) = vd[h2];
+      *reinterpret_cast<uint4*>(sx + tile_off(my_row + 32 * h2, my_chunk)) = vx[h2];
     }
     __syncthreads();
-#pragma unroll 8
-    for (int pr = 0; pr < kChunk; ++pr) {
-      const float4 d4 = *reinterpret_cast<const float4*>(&sdy[pr][4 * ty]);
-      const float4 x4 = *reinterpret_cast<const float4*>(&sx[pr][4 * tx]);
-      const float dv[4] = {d4.x, d4.y, d4.z, d4.w}, xv[4] = {x4.x, x4.y, x4.z, x4.w};
+    if (p0 + kChunk < pend) load(p0 + kChunk, vd, vx);
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+    for (int ks = 0; ks < kChunk / 16; ++ks) {
+      // A: filters wf .. wf+15 x pixels 16 ks ..; matrix mi = (pixel half
+      // mi >> 1, filter half mi & 1)
+      uint32_t af[4];
+      ldsm_x4_trans(af, sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr, (wf >> 3) + (mi & 1)));
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(dv[i], xv[j], acc[i][j]);
+      for (int nb = 0; nb < 2; ++nb) {
+        // B: pixels 16 ks .. x columns wj + 16 nb ..; matrix mi = (pixel
+        // half mi & 1, column half mi >> 1)
+        uint32_t bf[4];
+        ldsm_x4_trans(bf, sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr,
+                                          ((wj + 16 * nb) >> 3) + (mi >> 1)));
+        mma_16816(acc[2 * nb], af, bf[0], bf[1]);
+        mma_16816(acc[2 * nb + 1], af, bf[2], bf[3]);
+      }
     }
   }
+  // lane (g, t): filters wf + g (+8), columns wj + 8 nt + 2t (+1)
   float* part = a.part + static_cast<int64_t>(blockIdx.z) * a.K * a.rsc;
+  const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int k = k0 + 4 * ty + i;
-    if (k >= a.K) continue;
+  for (int nt = 0; nt < 4; ++nt) {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int jj = j0 + 4 * tx + j;
-      if (jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[i][j];
+    for (int i = 0; i < 4; ++i) {
+      const int k = k0 + wf + g + 8 * (i >> 1);
+      const int jj = j0 + wj + 8 * nt + 2 * t + (i & 1);
+      if (k < a.K && jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[nt][i];
+    }
+  }
+}
+
+// The same tile computation for aligned operands (K % 8 == 0, C % 8 == 0,
+// 16-byte aligned x and dy): every 16-byte chunk is 8 filters of one pixel or
+// 8 channels of one tap, copied by cp.async into a kStages-deep ring
+// (out-of-image taps and pixels past the slice are zero-filled by a copy of
+// source size 0), so several chunks' loads are in flight per CTA.
+constexpr int kStages = 4;
+constexpr int kStageBytes = 2 * kChunk * 128;   // dy tile + x tile
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const BwdFilterArgs a) {
+  extern __shared__ __align__(128) uint8_t ring[];
+  __shared__ int col_r[kTileN], col_s[kTileN], col_c[kTileN];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int k0 = blockIdx.x * kTileM, j0 = blockIdx.y * kTileN;
+  if (tid < kTileN) {
+    const int j = j0 + tid;
+    const int c = j % a.C, rs = j / a.C;
+    col_c[tid] = c;
+    col_s[tid] = rs % a.S;
+    col_r[tid] = j < a.rsc ? rs / a.S : -1;
+  }
+  __syncthreads();
+  const int my_chunk = tid & 7, my_row = tid >> 3;
+  const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
+  const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
+  const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
+  const int nchunks = pend > pbeg ? static_cast<int>((pend - pbeg + kChunk - 1) / kChunk) : 0;
+  const uint32_t ring_s = smem_addr(ring);
+  const int jc = 8 * my_chunk, tap_r = col_r[jc], tap_s = col_s[jc], tap_c = col_c[jc];
+  const int kb = k0 + 8 * my_chunk;
+
+  auto issue = [&](int ci) {
+    const int64_t p0 = pbeg + static_cast<int64_t>(ci) * kChunk;
+    const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int row = my_row + 32 * h2;
+      const int64_t pix = p0 + row;
+      const bool pv = pix < pend;
+      const int64_t pc = pv ? pix : pbeg;
+      cp_async16(st + tile_off(row, my_chunk), a.dy + pc * a.K + (kb < a.K ? kb : 0),
+                 pv && kb < a.K);
+      const int n = static_cast<int>(pc / pq);
+      const int rem = static_cast<int>(pc - static_cast<int64_t>(n) * pq);
+      const int hh = (rem / a.Q) * a.sh - a.ph + tap_r, ww = (rem % a.Q) * a.sw - a.pw + tap_s;
+      const bool xv = pv && tap_r >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
+      const int64_t xo = xv ? ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + tap_c : 0;
+      cp_async16(st + kChunk * 128 + tile_off(row, my_chunk), a.x + xo, xv);
+    }
+  };
+
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
+  const int wf = 16 * (warp & 3), wj = 32 * (warp >> 2);
+  const int mi = lane >> 3, lr = lane & 7;
+#pragma unroll
+  for (int ci = 0; ci < kStages - 1; ++ci) {
+    if (ci < nchunks) issue(ci);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+  for (int ci = 0; ci < nchunks; ++ci) {
+    asm volatile("cp.async.wait_group %0;" ::"n"(kStages - 2) : "memory");
+    __syncthreads();   // chunk ci visible to all; chunk ci - 1's stage is free
+    if (ci + kStages - 1 < nchunks) issue(ci + kStages - 1);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    const uint32_t sdy_s = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
+    const uint32_t sx_s = sdy_s + kChunk * 128;
+#pragma unroll
+    for (int ks = 0; ks < kChunk / 16; ++ks) {
+      uint32_t af[4];
+      ldsm_x4_trans(af, sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr, (wf >> 3) + (mi & 1)));
+#pragma unroll
+      for (int nb = 0; nb < 2; ++nb) {
+        uint32_t bf[4];
+        ldsm_x4_trans(bf, sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr,
+                                          ((wj + 16 * nb) >> 3) + (mi >> 1)));
+        mma_16816(acc[2 * nb], af, bf[0], bf[1]);
+        mma_16816(acc[2 * nb + 1], af, bf[2], bf[3]);
+      }
+    }
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  float* part = a.part + static_cast<int64_t>(blockIdx.z) * a.K * a.rsc;
+  const int g = lane >> 2, t = lane & 3;
+#pragma unroll
+  for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int k = k0 + wf + g + 8 * (i >> 1);
+      const int jj = j0 + wj + 8 * nt + 2 * t + (i & 1);
+      if (k < a.K && jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[nt][i];
     }
   }
 }
@@ -268,15 +453,16 @@ tbn_status launch_bwd_data(const BwdConvShape& p, const void* dy, const uint32_t
     if (st != TBN_OK) return st;
   }
   {
-    const int64_t total = p.N * b.Hd * b.Wd * p.K;
+    const int64_t total = p.N * b.Hd * b.Wd;
     const int64_t blocks =
         std::max<int64_t>(1, std::min<int64_t>((std::max<int64_t>(total, p.C) + 255) / 256,
                                                static_cast<int64_t>(device_sm_count()) * 16));
+    const int vec = (p.K % 8 == 0 && is_aligned(dy, 16)) ? 1 : 0;   // dyd is 256-aligned
     dilate_scale_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
         static_cast<const __nv_bfloat16*>(dy), alpha, static_cast<int>(p.N),
         static_cast<int>(p.P), static_cast<int>(p.Q), static_cast<int>(p.K),
         static_cast<int>(b.Hd), static_cast<int>(b.Wd), static_cast<int>(p.sh),
-        static_cast<int>(p.sw), dyd, ones, static_cast<int>(p.C));
+        static_cast<int>(p.sw), dyd, ones, static_cast<int>(p.C), vec);
     const tbn_status st = check_launch("dilate_scale_kernel");
     if (st != TBN_OK) return st;
   }
@@ -318,13 +504,29 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   a.npix = p.N * p.P * p.Q;
   a.rsc = static_cast<int>(p.R * p.S * p.C);
   a.slices = bwd_filter_slices(p);
+  a.dy_vec = (p.K % 8 == 0 && is_aligned(dy, 16)) ? 1 : 0;
+  a.x_vec = (p.C % 8 == 0 && is_aligned(x, 16)) ? 1 : 0;
   a.pix_per_slice = (a.npix + a.slices - 1) / a.slices;
   const dim3 grid(static_cast<unsigned>((p.K + kTileM - 1) / kTileM),
                   static_cast<unsigned>((a.rsc + kTileN - 1) / kTileN),
                   static_cast<unsigned>(a.slices));
   if (grid.y > 65535) return fail(TBN_ERR_UNSUPPORTED, "backward filter: R S C too large");
-  bwd_filter_kernel<<<grid, kBwdThreads, 0, s>>>(a);
-  tbn_status st = check_launch("bwd_filter_kernel");
+  tbn_status st;
+  if (a.dy_vec && a.x_vec) {
+    static bool attr_set = false;
+    if (!attr_set) {
+      const cudaError_t e = cudaFuncSetAttribute(bwd_filter_async_kernel,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 kStages * kStageBytes);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(bwd_filter_async_kernel)");
+      attr_set = true;
+    }
+    bwd_filter_async_kernel<<<grid, kBwdThreads, kStages * kStageBytes, s>>>(a);
+    st = check_launch("bwd_filter_async_kernel");
+  } else {
+    bwd_filter_kernel<<<grid, kBwdThreads, 0, s>>>(a);
+    st = check_launch("bwd_filter_kernel");
+  }
   if (st != TBN_OK) return st;
   const int64_t count = p.K * a.rsc;
   const int64_t blocks = std::min<int64_t>((count + 255) / 256, 65536);
