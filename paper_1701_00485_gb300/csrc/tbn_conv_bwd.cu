@@ -276,13 +276,18 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
   }
 }
 
-// The same tile computation for aligned operands (K % 8 == 0, C % 8 == 0,
-// 16-byte aligned x and dy): every 16-byte chunk is 8 filters of one pixel or
-// 8 channels of one tap, copied by cp.async into a kStages-deep ring
-// (out-of-image taps and pixels past the slice are zero-filled by a copy of
-// source size 0), so several chunks' loads are in flight per CTA.
+// The same product for aligned operands (K % 8 == 0, C % 8 == 0, 16-byte
+// aligned x and dy), on tiles of 128 filters x 64 columns: every 16-byte
+// chunk is 8 filters of one pixel or 8 channels of one tap, copied by
+// cp.async into a kStages-deep ring (out-of-image taps and pixels past the
+// slice are zero-filled by a copy of source size 0), so several chunks'
+// loads are in flight per CTA.  Warp w owns filters 32 (w % 4) .. and
+// columns 32 (w / 4) ..: per K step two A and two B fragment loads feed
+// eight mma (twice the mma per ldmatrix of a 16 x 32 warp tile).
+constexpr int kTileMA = 128;
 constexpr int kStages = 4;
-constexpr int kStageBytes = 2 * kChunk * 128;   // dy tile + x tile
+constexpr int kDyTile = kChunk * 128;             // one 64-filter half of dy
+constexpr int kStageBytes = 2 * kDyTile + kChunk * 128;
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
@@ -294,7 +299,7 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
   extern __shared__ __align__(128) uint8_t ring[];
   __shared__ int col_r[kTileN], col_s[kTileN], col_c[kTileN];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int k0 = blockIdx.x * kTileM, j0 = blockIdx.y * kTileN;
+  const int k0 = blockIdx.x * kTileMA, j0 = blockIdx.y * kTileN;
   if (tid < kTileN) {
     const int j = j0 + tid;
     const int c = j % a.C, rs = j / a.C;
@@ -303,14 +308,13 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
     col_r[tid] = j < a.rsc ? rs / a.S : -1;
   }
   __syncthreads();
-  const int my_chunk = tid & 7, my_row = tid >> 3;
+  const int my_chunk = tid & 7, my_row = tid >> 3;   // rows my_row, my_row + 32
   const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
   const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
   const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
   const int nchunks = pend > pbeg ? static_cast<int>((pend - pbeg + kChunk - 1) / kChunk) : 0;
   const uint32_t ring_s = smem_addr(ring);
   const int jc = 8 * my_chunk, tap_r = col_r[jc], tap_s = col_s[jc], tap_c = col_c[jc];
-  const int kb = k0 + 8 * my_chunk;
 
   auto issue = [&](int ci) {
     const int64_t p0 = pbeg + static_cast<int64_t>(ci) * kChunk;
@@ -321,23 +325,29 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
       const int64_t pix = p0 + row;
       const bool pv = pix < pend;
       const int64_t pc = pv ? pix : pbeg;
-      cp_async16(st + tile_off(row, my_chunk), a.dy + pc * a.K + (kb < a.K ? kb : 0),
-                 pv && kb < a.K);
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {   // filter halves 0..63, 64..127
+        const int kb = k0 + 64 * hf + 8 * my_chunk;
+        cp_async16(st + hf * kDyTile + tile_off(row, my_chunk),
+                   a.dy + pc * a.K + (kb < a.K ? kb : 0), pv && kb < a.K);
+      }
       const int n = static_cast<int>(pc / pq);
       const int rem = static_cast<int>(pc - static_cast<int64_t>(n) * pq);
       const int hh = (rem / a.Q) * a.sh - a.ph + tap_r, ww = (rem % a.Q) * a.sw - a.pw + tap_s;
       const bool xv = pv && tap_r >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
       const int64_t xo = xv ? ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + tap_c : 0;
-      cp_async16(st + kChunk * 128 + tile_off(row, my_chunk), a.x + xo, xv);
+      cp_async16(st + 2 * kDyTile + tile_off(row, my_chunk), a.x + xo, xv);
     }
   };
 
-  float acc[4][4];
+  float acc[2][4][4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+  for (int m = 0; m < 2; ++m)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.0f;
-  const int wf = 16 * (warp & 3), wj = 32 * (warp >> 2);
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[m][i][j] = 0.0f;
+  const int wf = 32 * (warp & 3), wj = 32 * (warp >> 2);
   const int mi = lane >> 3, lr = lane & 7;
 #pragma unroll
   for (int ci = 0; ci < kStages - 1; ++ci) {
@@ -349,34 +359,43 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
     __syncthreads();   // chunk ci visible to all; chunk ci - 1's stage is free
     if (ci + kStages - 1 < nchunks) issue(ci + kStages - 1);
     asm volatile("cp.async.commit_group;" ::: "memory");
-    const uint32_t sdy_s = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
-    const uint32_t sx_s = sdy_s + kChunk * 128;
+    const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
+    const uint32_t sdy_s = st + static_cast<uint32_t>((wf >> 6) * kDyTile);   // warp's half
+    const uint32_t sx_s = st + 2 * kDyTile;
+    const int fc = (wf & 63) >> 3;   // the warp's first 16-byte chunk in its half
 #pragma unroll
     for (int ks = 0; ks < kChunk / 16; ++ks) {
-      uint32_t af[4];
-      ldsm_x4_trans(af, sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr, (wf >> 3) + (mi & 1)));
+      uint32_t af[2][4], bf[2][4];
 #pragma unroll
-      for (int nb = 0; nb < 2; ++nb) {
-        uint32_t bf[4];
-        ldsm_x4_trans(bf, sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr,
-                                          ((wj + 16 * nb) >> 3) + (mi >> 1)));
-        mma_16816(acc[2 * nb], af, bf[0], bf[1]);
-        mma_16816(acc[2 * nb + 1], af, bf[2], bf[3]);
-      }
+      for (int mt = 0; mt < 2; ++mt)
+        ldsm_x4_trans(af[mt], sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr,
+                                               fc + 2 * mt + (mi & 1)));
+#pragma unroll
+      for (int nb = 0; nb < 2; ++nb)
+        ldsm_x4_trans(bf[nb], sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr,
+                                              ((wj + 16 * nb) >> 3) + (mi >> 1)));
+#pragma unroll
+      for (int mt = 0; mt < 2; ++mt)
+#pragma unroll
+        for (int nb = 0; nb < 2; ++nb) {
+          mma_16816(acc[mt][2 * nb], af[mt], bf[nb][0], bf[nb][1]);
+          mma_16816(acc[mt][2 * nb + 1], af[mt], bf[nb][2], bf[nb][3]);
+        }
     }
   }
   asm volatile("cp.async.wait_group 0;" ::: "memory");
   float* part = a.part + static_cast<int64_t>(blockIdx.z) * a.K * a.rsc;
   const int g = lane >> 2, t = lane & 3;
 #pragma unroll
-  for (int nt = 0; nt < 4; ++nt) {
+  for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int k = k0 + wf + g + 8 * (i >> 1);
-      const int jj = j0 + wj + 8 * nt + 2 * t + (i & 1);
-      if (k < a.K && jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[nt][i];
-    }
-  }
+    for (int nt = 0; nt < 4; ++nt)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int k = k0 + wf + 16 * mt + g + 8 * (i >> 1);
+        const int jj = j0 + wj + 8 * nt + 2 * t + (i & 1);
+        if (k < a.K && jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[mt][nt][i];
+      }
 }
 
 // dw[e] = sum of the slices' partial values, in slice order.
@@ -507,12 +526,14 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   a.dy_vec = (p.K % 8 == 0 && is_aligned(dy, 16)) ? 1 : 0;
   a.x_vec = (p.C % 8 == 0 && is_aligned(x, 16)) ? 1 : 0;
   a.pix_per_slice = (a.npix + a.slices - 1) / a.slices;
-  const dim3 grid(static_cast<unsigned>((p.K + kTileM - 1) / kTileM),
+  const bool async_path = a.dy_vec && a.x_vec;
+  const int tile_m = async_path ? kTileMA : kTileM;
+  const dim3 grid(static_cast<unsigned>((p.K + tile_m - 1) / tile_m),
                   static_cast<unsigned>((a.rsc + kTileN - 1) / kTileN),
                   static_cast<unsigned>(a.slices));
   if (grid.y > 65535) return fail(TBN_ERR_UNSUPPORTED, "backward filter: R S C too large");
   tbn_status st;
-  if (a.dy_vec && a.x_vec) {
+  if (async_path) {
     static bool attr_set = false;
     if (!attr_set) {
       const cudaError_t e = cudaFuncSetAttribute(bwd_filter_async_kernel,
