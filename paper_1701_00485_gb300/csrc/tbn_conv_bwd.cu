@@ -48,6 +48,22 @@ __global__ void __launch_bounds__(256) transpose_codes_kernel(
     const int c = static_cast<int>(wi / wpf_out);
     const int64_t j = wi - static_cast<int64_t>(c) * wpf_out;
     uint32_t o = 0u;
+    if (K % 16 == 0) {
+      // the word's 16 codes share the tap (r, s); input channels k0 .. k0+15
+      const int64_t i0 = 16 * j;
+      const int k0 = static_cast<int>(i0 % K);
+      const int64_t rs = i0 / K;
+      const int s = static_cast<int>(rs % S), r = static_cast<int>(rs / S);
+      const int64_t src = (static_cast<int64_t>(R - 1 - r) * S + (S - 1 - s)) * C + c;
+#pragma unroll
+      for (int l = 0; l < 16; ++l) {
+        const uint32_t f = field_of_code(codes + static_cast<int64_t>(k0 + l) * wpf_in, src);
+        const int b = 16 * (l & 1) + (l >> 1);
+        o |= ((f & 1u) << b) | ((f >> 1) << (b + 8));
+      }
+      out[wi] = o;
+      continue;
+    }
     for (int l = 0; l < 16; ++l) {
       const int64_t i = 16 * j + l;
       if (i >= n_out) break;
@@ -73,35 +89,40 @@ __global__ void __launch_bounds__(256) dilate_scale_kernel(
     float* __restrict__ ones, int C, int vec) {
   const int64_t npix = static_cast<int64_t>(N) * Hd * Wd;
   const int64_t tid = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  for (int64_t c = tid; c < C; c += static_cast<int64_t>(gridDim.x) * blockDim.x) ones[c] = 1.0f;
-  for (int64_t e = tid; e < npix; e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int v = static_cast<int>(e % Wd);
-    const int64_t t = e / Wd;
+  const int64_t nthreads = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t c = tid; c < C; c += nthreads) ones[c] = 1.0f;
+  // one item = 8 channels of one pixel (vec) or one pixel (scalar path)
+  const int per_pix = vec ? K / 8 : 1;
+  for (int64_t e = tid; e < npix * per_pix; e += nthreads) {
+    const int64_t pix = e / per_pix;
+    const int kv = static_cast<int>(e - pix * per_pix);
+    const int v = static_cast<int>(pix % Wd);
+    const int64_t t = pix / Wd;
     const int u = static_cast<int>(t % Hd);
     const int n = static_cast<int>(t / Hd);
     const bool hit = u % sh == 0 && v % sw == 0 && u / sh < P && v / sw < Q;
     const __nv_bfloat16* src =
         hit ? dy + ((static_cast<int64_t>(n) * P + u / sh) * Q + v / sw) * K : nullptr;
-    __nv_bfloat16* dst = dyd + e * K;
+    __nv_bfloat16* dst = dyd + pix * K;
     if (vec) {
-      for (int k = 0; k < K; k += 8) {
-        uint4 o = make_uint4(0u, 0u, 0u, 0u);
-        if (hit) {
-          const uint4 i4 = __ldg(reinterpret_cast<const uint4*>(src + k));
-          const uint32_t iw[4] = {i4.x, i4.y, i4.z, i4.w};
-          uint32_t ow[4];
+      const int k = 8 * kv;
+      uint4 o = make_uint4(0u, 0u, 0u, 0u);
+      if (hit) {
+        const uint4 i4 = __ldg(reinterpret_cast<const uint4*>(src + k));
+        const float4 a0 = __ldg(reinterpret_cast<const float4*>(alpha + k));
+        const float4 a1 = __ldg(reinterpret_cast<const float4*>(alpha + k + 4));
+        const float al[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        const uint32_t iw[4] = {i4.x, i4.y, i4.z, i4.w};
+        uint32_t ow[4];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&iw[q]);
-            const float2 f = __bfloat1622float2(b);
-            const __nv_bfloat162 r =
-                __floats2bfloat162_rn(__ldg(alpha + k + 2 * q) * f.x, __ldg(alpha + k + 2 * q + 1) * f.y);
-            ow[q] = *reinterpret_cast<const uint32_t*>(&r);
-          }
-          o = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&iw[q]));
+          const __nv_bfloat162 r = __floats2bfloat162_rn(al[2 * q] * f.x, al[2 * q + 1] * f.y);
+          ow[q] = *reinterpret_cast<const uint32_t*>(&r);
         }
-        *reinterpret_cast<uint4*>(dst + k) = o;
+        o = make_uint4(ow[0], ow[1], ow[2], ow[3]);
       }
+      *reinterpret_cast<uint4*>(dst + k) = o;
     } else {
       for (int k = 0; k < K; ++k)
         dst[k] = __float2bfloat16_rn(hit ? __ldg(alpha + k) * __bfloat162float(src[k]) : 0.0f);
@@ -472,11 +493,12 @@ tbn_status launch_bwd_data(const BwdConvShape& p, const void* dy, const uint32_t
     if (st != TBN_OK) return st;
   }
   {
-    const int64_t total = p.N * b.Hd * b.Wd;
+    const int64_t total = p.N * b.Hd * b.Wd * (p.K % 8 == 0 ? p.K / 8 : 1);
     const int64_t blocks =
         std::max<int64_t>(1, std::min<int64_t>((std::max<int64_t>(total, p.C) + 255) / 256,
                                                static_cast<int64_t>(device_sm_count()) * 16));
-    const int vec = (p.K % 8 == 0 && is_aligned(dy, 16)) ? 1 : 0;   // dyd is 256-aligned
+    // dyd is 256-aligned; alpha is read as float4 pairs
+    const int vec = (p.K % 8 == 0 && is_aligned(dy, 16) && is_aligned(alpha, 16)) ? 1 : 0;
     dilate_scale_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(
         static_cast<const __nv_bfloat16*>(dy), alpha, static_cast<int>(p.N),
         static_cast<int>(p.P), static_cast<int>(p.Q), static_cast<int>(p.K),
