@@ -302,13 +302,14 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
 // chunk is 8 filters of one pixel or 8 channels of one tap, copied by
 // cp.async into a kStages-deep ring (out-of-image taps and pixels past the
 // slice are zero-filled by a copy of source size 0), so several chunks'
-// loads are in flight per CTA.  Warp w owns filters 32 (w % 4) .. and
-// columns 32 (w / 4) ..: per K step two A and two B fragment loads feed
-// eight mma (twice the mma per ldmatrix of a 16 x 32 warp tile).
+// loads are in flight per CTA.  Tiles are 128 filters x 128 columns; warp w
+// owns filters 32 (w % 4) .. and columns 64 (w / 4) ..: per K step two A and
+// four B fragment loads feed sixteen mma.
 constexpr int kTileMA = 128;
-constexpr int kStages = 4;
-constexpr int kDyTile = kChunk * 128;             // one 64-filter half of dy
-constexpr int kStageBytes = 2 * kDyTile + kChunk * 128;
+constexpr int kTileNA = 128;
+constexpr int kStages = 3;
+constexpr int kHalfTile = kChunk * 128;           // 64 pixels x 64 bf16
+constexpr int kStageBytes = 4 * kHalfTile;        // dy: 2 halves, x: 2 halves
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
@@ -316,12 +317,12 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
                : "memory");
 }
 
-__global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const BwdFilterArgs a) {
+__global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const BwdFilterArgs a) {
   extern __shared__ __align__(128) uint8_t ring[];
-  __shared__ int col_r[kTileN], col_s[kTileN], col_c[kTileN];
+  __shared__ int col_r[kTileNA], col_s[kTileNA], col_c[kTileNA];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int k0 = blockIdx.x * kTileMA, j0 = blockIdx.y * kTileN;
-  if (tid < kTileN) {
+  const int k0 = blockIdx.x * kTileMA, j0 = blockIdx.y * kTileNA;
+  if (tid < kTileNA) {
     const int j = j0 + tid;
     const int c = j % a.C, rs = j / a.C;
     col_c[tid] = c;
@@ -335,7 +336,14 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
   const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
   const int nchunks = pend > pbeg ? static_cast<int>((pend - pbeg + kChunk - 1) / kChunk) : 0;
   const uint32_t ring_s = smem_addr(ring);
-  const int jc = 8 * my_chunk, tap_r = col_r[jc], tap_s = col_s[jc], tap_c = col_c[jc];
+  int tap_r[2], tap_s[2], tap_c[2];
+#pragma unroll
+  for (int hx = 0; hx < 2; ++hx) {
+    const int jc = 64 * hx + 8 * my_chunk;
+    tap_r[hx] = col_r[jc];
+    tap_s[hx] = col_s[jc];
+    tap_c[hx] = col_c[jc];
+  }
 
   auto issue = [&](int ci) {
     const int64_t p0 = pbeg + static_cast<int64_t>(ci) * kChunk;
@@ -349,26 +357,31 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf) {   // filter halves 0..63, 64..127
         const int kb = k0 + 64 * hf + 8 * my_chunk;
-        cp_async16(st + hf * kDyTile + tile_off(row, my_chunk),
+        cp_async16(st + hf * kHalfTile + tile_off(row, my_chunk),
                    a.dy + pc * a.K + (kb < a.K ? kb : 0), pv && kb < a.K);
       }
       const int n = static_cast<int>(pc / pq);
       const int rem = static_cast<int>(pc - static_cast<int64_t>(n) * pq);
-      const int hh = (rem / a.Q) * a.sh - a.ph + tap_r, ww = (rem % a.Q) * a.sw - a.pw + tap_s;
-      const bool xv = pv && tap_r >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
-      const int64_t xo = xv ? ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + tap_c : 0;
-      cp_async16(st + 2 * kDyTile + tile_off(row, my_chunk), a.x + xo, xv);
+      const int h0 = (rem / a.Q) * a.sh - a.ph, w0 = (rem % a.Q) * a.sw - a.pw;
+#pragma unroll
+      for (int hx = 0; hx < 2; ++hx) {   // column halves 0..63, 64..127
+        const int hh = h0 + tap_r[hx], ww = w0 + tap_s[hx];
+        const bool xv = pv && tap_r[hx] >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
+        const int64_t xo =
+            xv ? ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + tap_c[hx] : 0;
+        cp_async16(st + (2 + hx) * kHalfTile + tile_off(row, my_chunk), a.x + xo, xv);
+      }
     }
   };
 
-  float acc[2][4][4];
+  float acc[2][8][4];
 #pragma unroll
   for (int m = 0; m < 2; ++m)
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) acc[m][i][j] = 0.0f;
-  const int wf = 32 * (warp & 3), wj = 32 * (warp >> 2);
+  const int wf = 32 * (warp & 3), wj = 64 * (warp >> 2);
   const int mi = lane >> 3, lr = lane & 7;
 #pragma unroll
   for (int ci = 0; ci < kStages - 1; ++ci) {
@@ -381,24 +394,23 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
     if (ci + kStages - 1 < nchunks) issue(ci + kStages - 1);
     asm volatile("cp.async.commit_group;" ::: "memory");
     const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
-    const uint32_t sdy_s = st + static_cast<uint32_t>((wf >> 6) * kDyTile);   // warp's half
-    const uint32_t sx_s = st + 2 * kDyTile;
-    const int fc = (wf & 63) >> 3;   // the warp's first 16-byte chunk in its half
+    const uint32_t sdy_s = st + static_cast<uint32_t>((wf >> 6) * kHalfTile);   // warp's half
+    const uint32_t sx_s = st + static_cast<uint32_t>((2 + (wj >> 6)) * kHalfTile);
+    const int fc = (wf & 63) >> 3;   // the warp's first 16-byte chunk in its dy half
 #pragma unroll
     for (int ks = 0; ks < kChunk / 16; ++ks) {
-      uint32_t af[2][4], bf[2][4];
+      uint32_t af[2][4], bf[4][4];
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt)
         ldsm_x4_trans(af[mt], sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr,
                                                fc + 2 * mt + (mi & 1)));
 #pragma unroll
-      for (int nb = 0; nb < 2; ++nb)
-        ldsm_x4_trans(bf[nb], sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr,
-                                              ((wj + 16 * nb) >> 3) + (mi >> 1)));
+      for (int nb = 0; nb < 4; ++nb)
+        ldsm_x4_trans(bf[nb], sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr, 2 * nb + (mi >> 1)));
 #pragma unroll
       for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-        for (int nb = 0; nb < 2; ++nb) {
+        for (int nb = 0; nb < 4; ++nb) {
           mma_16816(acc[mt][2 * nb], af[mt], bf[nb][0], bf[nb][1]);
           mma_16816(acc[mt][2 * nb + 1], af[mt], bf[nb][2], bf[nb][3]);
         }
@@ -410,7 +422,7 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_async_kernel(const Bwd
 #pragma unroll
   for (int mt = 0; mt < 2; ++mt)
 #pragma unroll
-    for (int nt = 0; nt < 4; ++nt)
+    for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const int k = k0 + wf + 16 * mt + g + 8 * (i >> 1);
@@ -451,8 +463,13 @@ BwdDataPlan plan_bwd_data(const BwdConvShape& p) {
   return b;
 }
 
+// Pixel slices of the filter gradient: about 4 x SMs CTAs over the tiles of
+// the kernel the shape selects (a function of the shape only, so the
+// workspace query agrees with the launch).
 int bwd_filter_slices(const BwdConvShape& p) {
-  const int64_t tiles = ((p.K + kTileM - 1) / kTileM) * ((p.R * p.S * p.C + kTileN - 1) / kTileN);
+  const bool big = p.K % 8 == 0 && p.C % 8 == 0;
+  const int tm = big ? kTileMA : kTileM, tn = big ? kTileNA : kTileN;
+  const int64_t tiles = ((p.K + tm - 1) / tm) * ((p.R * p.S * p.C + tn - 1) / tn);
   const int64_t want = 4 * static_cast<int64_t>(device_sm_count());
   const int64_t npix = p.N * p.P * p.Q;
   int64_t s = std::max<int64_t>(1, want / std::max<int64_t>(tiles, 1));
@@ -550,8 +567,9 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   a.pix_per_slice = (a.npix + a.slices - 1) / a.slices;
   const bool async_path = a.dy_vec && a.x_vec;
   const int tile_m = async_path ? kTileMA : kTileM;
+  const int tile_n = async_path ? kTileNA : kTileN;
   const dim3 grid(static_cast<unsigned>((p.K + tile_m - 1) / tile_m),
-                  static_cast<unsigned>((a.rsc + kTileN - 1) / kTileN),
+                  static_cast<unsigned>((a.rsc + tile_n - 1) / tile_n),
                   static_cast<unsigned>(a.slices));
   if (grid.y > 65535) return fail(TBN_ERR_UNSUPPORTED, "backward filter: R S C too large");
   tbn_status st;
