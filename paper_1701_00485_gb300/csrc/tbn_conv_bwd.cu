@@ -463,14 +463,16 @@ BwdDataPlan plan_bwd_data(const BwdConvShape& p) {
   return b;
 }
 
-// Pixel slices of the filter gradient: about 4 x SMs CTAs over the tiles of
-// the kernel the shape selects (a function of the shape only, so the
-// workspace query agrees with the launch).
+// Pixel slices of the filter gradient: one wave of CTAs over the tiles of
+// the kernel the shape selects (2 resident per SM for the 96 KB ring, 4 for
+// the register path), each slice's partial tile costing a write and a read
+// in the reduction.  A function of the shape only, so the workspace query
+// agrees with the launch.
 int bwd_filter_slices(const BwdConvShape& p) {
   const bool big = p.K % 8 == 0 && p.C % 8 == 0;
   const int tm = big ? kTileMA : kTileM, tn = big ? kTileNA : kTileN;
   const int64_t tiles = ((p.K + tm - 1) / tm) * ((p.R * p.S * p.C + tn - 1) / tn);
-  const int64_t want = 4 * static_cast<int64_t>(device_sm_count());
+  const int64_t want = (big ? 2 : 4) * static_cast<int64_t>(device_sm_count());
   const int64_t npix = p.N * p.P * p.Q;
   int64_t s = std::max<int64_t>(1, want / std::max<int64_t>(tiles, 1));
   s = std::min<int64_t>(s, std::max<int64_t>(1, npix / (4 * kChunk)));
