@@ -20,6 +20,7 @@
 
 #include <algorithm>
 #include <cstdint>
+#include <mutex>
 
 #include "tbn_device.cuh"
 #include "tbn_internal.h"
@@ -576,14 +577,15 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   if (grid.y > 65535) return fail(TBN_ERR_UNSUPPORTED, "backward filter: R S C too large");
   tbn_status st;
   if (async_path) {
-    static bool attr_set = false;
-    if (!attr_set) {
-      const cudaError_t e = cudaFuncSetAttribute(bwd_filter_async_kernel,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 kStages * kStageBytes);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(bwd_filter_async_kernel)");
-      attr_set = true;
-    }
+    static std::once_flag attr_once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(attr_once, [] {
+      attr_err = cudaFuncSetAttribute(bwd_filter_async_kernel,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      kStages * kStageBytes);
+    });
+    if (attr_err != cudaSuccess)
+      return cuda_fail(attr_err, "cudaFuncSetAttribute(bwd_filter_async_kernel)");
     bwd_filter_async_kernel<<<grid, kBwdThreads, kStages * kStageBytes, s>>>(a);
     st = check_launch("bwd_filter_async_kernel");
   } else {
