@@ -628,8 +628,9 @@ def run_backward(args, rank, world, local_rank):
             "per_layer_us": per_layer,
             "roofline": {"bound": "tensor", "achieved": round(filt_tf, 3), "peak": bf16_peak,
                          "unit": "TFLOP/s", "frac": round(filt_tf / bf16_peak, 4), "traffic": None,
-                         "kernel": "bwd_filter_async_kernel (mma.sync m16n8k16 bf16, cp.async "
-                                   "ring; c1: bwd_filter_kernel), 6 launches + slice reductions",
+                         "kernel": "bwd_filter_tc_kernel (tcgen05 M128 N128 bf16, accumulator "
+                                   "in tensor memory, cp.async ring; c1: bwd_filter_kernel on "
+                                   "mma.sync), 6 launches + slice reductions",
                          "peak_kind": "%s bf16 dense, sustained" % peak_kind,
                          "input_grad_vs_bf16_peak": round(gflop_data / ms_data / bf16_peak, 4)},
             "clocks": clocks}

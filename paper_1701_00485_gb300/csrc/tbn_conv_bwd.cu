@@ -13,9 +13,11 @@
 // * Filter gradient dW^[k, r, s, c] = sum over (n, p, q) of dy[n, p, q, k]
 //   x[n, p sigma - pad + r, q sigma - pad + s, c]: a product of dy^T
 //   (K x pixels) and the im2col view of x (pixels x R S C).  Each CTA
-//   computes a 64 x 64 tile over a slice of the pixels on mma.sync
-//   tensor cores (bf16 products exact, fp32 accumulation); a second kernel
-//   adds the slices in slice order, so results are bitwise reproducible.
+//   computes a tile over a slice of the pixels: 128 x 128 on tcgen05 with
+//   the accumulator in tensor memory when K and C are multiples of 8, else
+//   64 x 64 on mma.sync (bf16 products exact, fp32 accumulation); a second
+//   kernel adds the slices in a fixed order, so results are bitwise
+//   reproducible.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -147,6 +149,8 @@ struct BwdFilterArgs {
   int slices;
   int64_t pix_per_slice;
   int dy_vec, x_vec;   // 16-byte loads possible (K % 8 == 0 / C % 8 == 0, aligned)
+  uint32_t* err;       // device error word (bounded waits)
+  int part_vec;        // 16-byte partial stores possible (rsc % 4 == 0, aligned)
 };
 
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
@@ -299,13 +303,11 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
 }
 
 // The same product for aligned operands (K % 8 == 0, C % 8 == 0, 16-byte
-// aligned x and dy), on tiles of 128 filters x 64 columns: every 16-byte
+// aligned x and dy), on tiles of 128 filters x 128 columns: every 16-byte
 // chunk is 8 filters of one pixel or 8 channels of one tap, copied by
 // cp.async into a kStages-deep ring (out-of-image taps and pixels past the
 // slice are zero-filled by a copy of source size 0), so several chunks'
-// loads are in flight per CTA.  Tiles are 128 filters x 128 columns; warp w
-// owns filters 32 (w % 4) .. and columns 64 (w / 4) ..: per K step two A and
-// four B fragment loads feed sixteen mma.
+// loads are in flight per CTA.
 constexpr int kTileMA = 128;
 constexpr int kTileNA = 128;
 constexpr int kStages = 3;
@@ -318,9 +320,33 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool v
                : "memory");
 }
 
-__global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const BwdFilterArgs a) {
-  extern __shared__ __align__(128) uint8_t ring[];
+// The product runs on the 5th-generation tensor cores (tcgen05).  The
+// pixel-major tiles are MN-major operands with the 128-byte swizzle: 64
+// filters (or columns) of one pixel are a 128-byte row, 8 pixel rows an
+// atom (SBO = 1 KB apart along the pixels), and the two 64-wide halves
+// LBO = 8 KB apart.  One thread issues four
+// M 128 x N 128 x K 16 MMAs per 64-pixel chunk into a 128-column fp32
+// accumulator in tensor memory and commits them to the stage's mbarrier;
+// a stage is refilled only after the MMAs reading it have completed.
+constexpr uint64_t kBwdWaitLimitNs = 1000000000ull;
+
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(8192u >> 4) << 16;   // LBO: next 64-wide MN half
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;   // SBO: next 8 pixel rows
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;          // 128-byte swizzle
+  return d;
+}
+
+__global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_tc_kernel(const BwdFilterArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* ring = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   __shared__ int col_r[kTileNA], col_s[kTileNA], col_c[kTileNA];
+  __shared__ uint64_t bar[kStages];
+  __shared__ uint32_t tmem_slot;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int k0 = blockIdx.x * kTileMA, j0 = blockIdx.y * kTileNA;
   if (tid < kTileNA) {
@@ -330,8 +356,19 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const 
     col_s[tid] = rs % a.S;
     col_r[tid] = j < a.rsc ? rs / a.S : -1;
   }
+  if (warp == 0) {
+    tmem_alloc(&tmem_slot, 128);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    for (int i = 0; i < kStages; ++i) mbar_init(&bar[i], 1);
+    fence_mbar_init();
+  }
+  tc_fence_before_sync();
   __syncthreads();
-  const int my_chunk = tid & 7, my_row = tid >> 3;   // rows my_row, my_row + 32
+  tc_fence_after_sync();
+  const uint32_t acc = tmem_slot;
+  const int my_chunk = tid & 7, my_row = tid >> 3;
   const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
   const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
   const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
@@ -345,7 +382,6 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const 
     tap_s[hx] = col_s[jc];
     tap_c[hx] = col_c[jc];
   }
-
   auto issue = [&](int ci) {
     const int64_t p0 = pbeg + static_cast<int64_t>(ci) * kChunk;
     const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
@@ -356,7 +392,7 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const 
       const bool pv = pix < pend;
       const int64_t pc = pv ? pix : pbeg;
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {   // filter halves 0..63, 64..127
+      for (int hf = 0; hf < 2; ++hf) {
         const int kb = k0 + 64 * hf + 8 * my_chunk;
         cp_async16(st + hf * kHalfTile + tile_off(row, my_chunk),
                    a.dy + pc * a.K + (kb < a.K ? kb : 0), pv && kb < a.K);
@@ -365,7 +401,7 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const 
       const int rem = static_cast<int>(pc - static_cast<int64_t>(n) * pq);
       const int h0 = (rem / a.Q) * a.sh - a.ph, w0 = (rem % a.Q) * a.sw - a.pw;
 #pragma unroll
-      for (int hx = 0; hx < 2; ++hx) {   // column halves 0..63, 64..127
+      for (int hx = 0; hx < 2; ++hx) {
         const int hh = h0 + tap_r[hx], ww = w0 + tap_s[hx];
         const bool xv = pv && tap_r[hx] >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
         const int64_t xo =
@@ -374,73 +410,101 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_async_kernel(const 
       }
     }
   };
-
-  float acc[2][8][4];
-#pragma unroll
-  for (int m = 0; m < 2; ++m)
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) acc[m][i][j] = 0.0f;
-  const int wf = 32 * (warp & 3), wj = 64 * (warp >> 2);
-  const int mi = lane >> 3, lr = lane & 7;
+  constexpr uint32_t idesc = idesc_bf16_f32(128, 128) | (1u << 15) | (1u << 16);   // MN-major
 #pragma unroll
   for (int ci = 0; ci < kStages - 1; ++ci) {
     if (ci < nchunks) issue(ci);
     asm volatile("cp.async.commit_group;" ::: "memory");
   }
+  bool ok = true;
   for (int ci = 0; ci < nchunks; ++ci) {
     asm volatile("cp.async.wait_group %0;" ::"n"(kStages - 2) : "memory");
-    __syncthreads();   // chunk ci visible to all; chunk ci - 1's stage is free
-    if (ci + kStages - 1 < nchunks) issue(ci + kStages - 1);
-    asm volatile("cp.async.commit_group;" ::: "memory");
-    const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
-    const uint32_t sdy_s = st + static_cast<uint32_t>((wf >> 6) * kHalfTile);   // warp's half
-    const uint32_t sx_s = st + static_cast<uint32_t>((2 + (wj >> 6)) * kHalfTile);
-    const int fc = (wf & 63) >> 3;   // the warp's first 16-byte chunk in its dy half
+    fence_proxy_async_smem();   // this thread's copies -> visible to the tensor core
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after_sync();
+      const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
 #pragma unroll
-    for (int ks = 0; ks < kChunk / 16; ++ks) {
-      uint32_t af[2][4], bf[4][4];
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
-        ldsm_x4_trans(af[mt], sdy_s + tile_off(16 * ks + 8 * (mi >> 1) + lr,
-                                               fc + 2 * mt + (mi & 1)));
-#pragma unroll
-      for (int nb = 0; nb < 4; ++nb)
-        ldsm_x4_trans(bf[nb], sx_s + tile_off(16 * ks + 8 * (mi & 1) + lr, 2 * nb + (mi >> 1)));
-#pragma unroll
-      for (int mt = 0; mt < 2; ++mt)
-#pragma unroll
-        for (int nb = 0; nb < 4; ++nb) {
-          mma_16816(acc[mt][2 * nb], af[mt], bf[nb][0], bf[nb][1]);
-          mma_16816(acc[mt][2 * nb + 1], af[mt], bf[nb][2], bf[nb][3]);
-        }
+      for (int ks = 0; ks < kChunk / 16; ++ks)
+        tc_mma_ss(acc, smem_desc_sw128_mn(st + ks * 2048), smem_desc_sw128_mn(st + 2 * kHalfTile + ks * 2048),
+                  idesc, (ci | ks) != 0 ? 1u : 0u);
+      tc_commit(&bar[ci % kStages]);
     }
+    if (ci + kStages - 1 < nchunks) {
+      // the refilled stage held chunk ci - 1: its MMAs must have finished
+      if (ci >= 1 && tid == 0)
+        ok = mbar_wait(&bar[(ci - 1) % kStages], static_cast<uint32_t>((ci - 1) / kStages) & 1u,
+                       nullptr, a.err, kBwdWaitLimitNs);
+      if (!__syncthreads_and(ok)) break;
+      issue(ci + kStages - 1);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
   }
   asm volatile("cp.async.wait_group 0;" ::: "memory");
+  if (nchunks > 0 && tid == 0)
+    ok = mbar_wait(&bar[(nchunks - 1) % kStages],
+                   static_cast<uint32_t>((nchunks - 1) / kStages) & 1u, nullptr, a.err,
+                   kBwdWaitLimitNs) && ok;
+  ok = __syncthreads_and(ok);
+  tc_fence_after_sync();
+  // epilogue: warp w reads lanes 32 (w % 4) .. (filters) and columns 64 (w / 4) ..
   float* part = a.part + static_cast<int64_t>(blockIdx.z) * a.K * a.rsc;
-  const int g = lane >> 2, t = lane & 3;
+  const int k = k0 + 32 * (warp & 3) + lane;
 #pragma unroll
-  for (int mt = 0; mt < 2; ++mt)
+  for (int q = 0; q < 2; ++q) {
+    const int jb = 64 * (warp >> 2) + 32 * q;
+    uint32_t v[32];
+    tmem_ld_32x32b_x32(acc + (static_cast<uint32_t>(32 * (warp & 3)) << 16) +
+                           static_cast<uint32_t>(jb),
+                       v);
+    tmem_wait_ld();
+    if (nchunks == 0) {
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
+      for (int i = 0; i < 32; ++i) v[i] = 0u;
+    }
+    if (ok && k < a.K) {
+      float* row = part + static_cast<int64_t>(k) * a.rsc + j0 + jb;
+      if (a.part_vec && j0 + jb + 32 <= a.rsc) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int k = k0 + wf + 16 * mt + g + 8 * (i >> 1);
-        const int jj = j0 + wj + 8 * nt + 2 * t + (i & 1);
-        if (k < a.K && jj < a.rsc) part[static_cast<int64_t>(k) * a.rsc + jj] = acc[mt][nt][i];
+        for (int i = 0; i < 32; i += 4)
+          *reinterpret_cast<uint4*>(row + i) = make_uint4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (j0 + jb + i < a.rsc) row[i] = __uint_as_float(v[i]);
       }
+    }
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after_sync();
+    tmem_dealloc(acc, 128);
+  }
 }
 
-// dw[e] = sum of the slices' partial values, in slice order.
-__global__ void __launch_bounds__(256) bwd_filter_reduce_kernel(const float* __restrict__ part,
-                                                                int slices, int64_t count,
-                                                                float* __restrict__ dw) {
-  for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < count;
-       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    float s = part[e];
-    for (int z = 1; z < slices; ++z) s += part[static_cast<int64_t>(z) * count + e];
-    dw[e] = s;
+// dw[e] = sum of the slices' partial values in a fixed order: block b
+// covers elements 32 b .. 32 b + 31; warp w sums slices w, w + 8, w + 16, ...
+// in order, and lane e of warp 0 adds the eight warp sums in warp order.
+constexpr int kReduceGroups = kBwdThreads / 32;
+
+__global__ void __launch_bounds__(kBwdThreads) bwd_filter_reduce_kernel(
+    const float* __restrict__ part, int slices, int64_t count, float* __restrict__ dw) {
+  __shared__ float sums[kReduceGroups][32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t e = static_cast<int64_t>(blockIdx.x) * 32 + lane;
+  float s = 0.0f;
+  if (e < count) {
+#pragma unroll 4
+    for (int z = w; z < slices; z += kReduceGroups) s += part[static_cast<int64_t>(z) * count + e];
+  }
+  sums[w][lane] = s;
+  __syncthreads();
+  if (w == 0 && e < count) {
+    float t = sums[0][lane];
+#pragma unroll
+    for (int g = 1; g < kReduceGroups; ++g) t += sums[g][lane];
+    dw[e] = t;
   }
 }
 
@@ -477,7 +541,10 @@ int bwd_filter_slices(const BwdConvShape& p) {
   const int64_t npix = p.N * p.P * p.Q;
   int64_t s = std::max<int64_t>(1, want / std::max<int64_t>(tiles, 1));
   s = std::min<int64_t>(s, std::max<int64_t>(1, npix / (4 * kChunk)));
-  return static_cast<int>(std::min<int64_t>(s, 64));
+  // at most 64 MB of partial tiles
+  const int64_t per_slice = std::max<int64_t>(1, p.K * p.R * p.S * p.C);
+  s = std::min<int64_t>(s, std::max<int64_t>(1, (int64_t{16} << 20) / per_slice));
+  return static_cast<int>(std::min<int64_t>(s, 1024));
 }
 
 }  // namespace
@@ -557,6 +624,7 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.dy = static_cast<const __nv_bfloat16*>(dy);
   a.part = static_cast<float*>(workspace);
+  a.part_vec = (p.R * p.S * p.C) % 4 == 0 && (reinterpret_cast<uintptr_t>(workspace) & 15) == 0;
   a.N = static_cast<int>(p.N); a.C = static_cast<int>(p.C); a.H = static_cast<int>(p.H);
   a.W = static_cast<int>(p.W); a.K = static_cast<int>(p.K); a.R = static_cast<int>(p.R);
   a.S = static_cast<int>(p.S); a.sh = static_cast<int>(p.sh); a.sw = static_cast<int>(p.sw);
@@ -580,23 +648,25 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
     static std::once_flag attr_once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(attr_once, [] {
-      attr_err = cudaFuncSetAttribute(bwd_filter_async_kernel,
+      attr_err = cudaFuncSetAttribute(bwd_filter_tc_kernel,
                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      kStages * kStageBytes);
+                                      kStages * kStageBytes + 1024);
     });
     if (attr_err != cudaSuccess)
-      return cuda_fail(attr_err, "cudaFuncSetAttribute(bwd_filter_async_kernel)");
-    bwd_filter_async_kernel<<<grid, kBwdThreads, kStages * kStageBytes, s>>>(a);
-    st = check_launch("bwd_filter_async_kernel");
+      return cuda_fail(attr_err, "cudaFuncSetAttribute(bwd_filter_tc_kernel)");
+    a.err = device_error_word();
+    bwd_filter_tc_kernel<<<grid, kBwdThreads, kStages * kStageBytes + 1024, s>>>(a);
+    st = check_launch("bwd_filter_tc_kernel");
   } else {
     bwd_filter_kernel<<<grid, kBwdThreads, 0, s>>>(a);
     st = check_launch("bwd_filter_kernel");
   }
   if (st != TBN_OK) return st;
   const int64_t count = p.K * a.rsc;
-  const int64_t blocks = std::min<int64_t>((count + 255) / 256, 65536);
-  bwd_filter_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(a.part, a.slices, count,
-                                                                          dw);
+  const int64_t blocks = (count + 31) / 32;
+  if (blocks > 0x7fffffff) return fail(TBN_ERR_UNSUPPORTED, "backward filter: too many weights");
+  bwd_filter_reduce_kernel<<<static_cast<unsigned>(blocks), kBwdThreads, 0, s>>>(
+      a.part, a.slices, count, dw);
   return check_launch("bwd_filter_reduce_kernel");
 }
 

@@ -122,3 +122,32 @@ def test_bwd_rejects_large_padding():
     with pytest.raises(tbn.TBNError) as e:
         tbn.tbn_conv2d_bwd_data(dy, codes, alpha, 1, (2, 2), 1, 1, (1, 1), (1, 1))
     assert e.value.status in (tbn.TBN_ERR_UNSUPPORTED, tbn.TBN_ERR_INVALID_ARG)
+
+
+@pytest.mark.parametrize("i", [1, 5])
+def test_bwd_vgg_small_batch128_sampled(i):
+    """Full-size VGG-small layers (batch 128, the backward workload's launch
+    configuration): dx of three whole images and dW of a 3 x 3 block of
+    (filter, channel) pairs, every tap, over the whole batch, against the
+    oracle run on just those images / channels."""
+    s = inputs.VGG_SMALL["convs"][i]
+    hw = 32 >> (i // 2)
+    case = (128, s.C, hw, hw, s.K, s.R, s.S, (s.stride, s.stride), (s.pad, s.pad))
+    N, C, H, W, K, R, S, st, pd = case
+    x, dy, codes, alpha, wt, al = make(case, 7700 + i)
+    dy_nhwc = dy.permute(0, 2, 3, 1).contiguous().cuda()
+    dx = tbn.tbn_conv2d_bwd_data(dy_nhwc, codes, alpha, C, (H, W), R, S, st, pd)
+    dw = tbn.tbn_conv2d_bwd_filter(x.permute(0, 2, 3, 1).contiguous().cuda(), dy_nhwc, R, S, st,
+                                   pd)
+    torch.cuda.synchronize()
+    assert tbn.tbn_device_error() == 0
+    imgs = [0, 77, N - 1]
+    dx_orc, bx = oracle.conv2d_bwd_data(dy[imgs].float().numpy(), wt, al, (H, W), st, pd)
+    got_dx = dx[imgs].float().cpu().permute(0, 3, 1, 2).numpy()
+    assert_within(got_dx, dx_orc, bx, out_bf16=True, extra=BF16_TERM,
+                  what="vgg c%d b128 bwd data" % (i + 1))
+    ks, cs = [0, 37, K - 1], [0, 53, C - 1]
+    dw_orc, bw = oracle.conv2d_bwd_filter(x[:, cs].float().numpy(), dy[:, ks].float().numpy(),
+                                          (R, S), st, pd)
+    got_dw = dw.cpu().reshape(K, R, S, C).permute(0, 3, 1, 2)[ks][:, cs].numpy()
+    assert_within(got_dw, dw_orc, bw, out_bf16=False, what="vgg c%d b128 bwd filter" % (i + 1))
