@@ -168,6 +168,30 @@ __device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4],
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// Pixel index n P Q + p Q + q of one tile row, advanced by kChunk pixels per
+// chunk with the carries of kChunk = dn P Q + dp Q + dq (no divisions in
+// the loop).  Rows past the slice keep advancing but are never loaded.
+struct PixelRow {
+  int64_t pix;
+  int n, p, q;
+  __device__ __forceinline__ void init(int64_t pixel, int P, int Q) {
+    pix = pixel;
+    const int64_t pq = static_cast<int64_t>(P) * Q;
+    n = static_cast<int>(pixel / pq);
+    const int rem = static_cast<int>(pixel - static_cast<int64_t>(n) * pq);
+    p = rem / Q;
+    q = rem - p * Q;
+  }
+  __device__ __forceinline__ void advance(int dn, int dp, int dq, int P, int Q) {
+    pix += kChunk;
+    q += dq;
+    if (q >= Q) { q -= Q; ++p; }
+    p += dp;
+    if (p >= P) { p -= P; ++n; }
+    n += dn;
+  }
+};
+
 // Shared tiles are [pixel][64 bf16]: 128-byte rows of eight 16-byte chunks,
 // chunk c of row r stored at c ^ (r & 7) (conflict-free ldmatrix).
 __device__ __forceinline__ uint32_t tile_off(int row, int chunk) {
@@ -181,7 +205,7 @@ __device__ __forceinline__ uint32_t tile_off(int row, int chunk) {
 // Both operands come from the pixel-major tiles by ldmatrix.trans.  Thread
 // i fills chunk i % 8 of pixel row i / 8 (and row i / 8 + 32) of both
 // tiles; the next chunk's loads are issued before the current MMAs.
-__global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilterArgs a) {
+__global__ void __launch_bounds__(kBwdThreads, 4) bwd_filter_kernel(const BwdFilterArgs a) {
   __shared__ __align__(128) uint8_t sdy[kChunk * 128];
   __shared__ __align__(128) uint8_t sx[kChunk * 128];
   __shared__ int col_r[kTileN], col_s[kTileN], col_c[kTileN];
@@ -199,13 +223,17 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
   const int64_t pbeg = static_cast<int64_t>(blockIdx.z) * a.pix_per_slice;
   const int64_t pend = min(a.npix, pbeg + a.pix_per_slice);
   const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
+  const int dq = kChunk % a.Q, dp = (kChunk / a.Q) % a.P, dn = static_cast<int>(kChunk / pq);
+  PixelRow rows[2];
+  rows[0].init(pbeg + my_row, a.P, a.Q);
+  rows[1].init(pbeg + my_row + 32, a.P, a.Q);
 
-  // global loads of one chunk into registers: 8 filters of dy and 8 im2col
-  // columns of x for pixels p0 + my_row and p0 + my_row + 32
-  auto load = [&](int64_t p0, uint4 (&vd)[2], uint4 (&vx)[2]) {
+  // global loads of the next chunk into registers: 8 filters of dy and 8
+  // im2col columns of x for its pixels my_row and my_row + 32
+  auto load = [&](uint4 (&vd)[2], uint4 (&vx)[2]) {
 #pragma unroll
     for (int h2 = 0; h2 < 2; ++h2) {
-      const int64_t pix = p0 + my_row + 32 * h2;
+      const int64_t pix = rows[h2].pix;
       uint32_t d[4] = {0u, 0u, 0u, 0u}, xv[4] = {0u, 0u, 0u, 0u};
       if (pix < pend) {
         const int kb = k0 + 8 * my_chunk;
@@ -219,9 +247,8 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
             if (kb + e < a.K)
               d[e >> 1] |= static_cast<uint32_t>(__bfloat16_as_ushort(dyp[e])) << (16 * (e & 1));
         }
-        const int n = static_cast<int>(pix / pq);
-        const int rem = static_cast<int>(pix - static_cast<int64_t>(n) * pq);
-        const int h0 = (rem / a.Q) * a.sh - a.ph, w0 = (rem % a.Q) * a.sw - a.pw;
+        const int n = rows[h2].n;
+        const int h0 = rows[h2].p * a.sh - a.ph, w0 = rows[h2].q * a.sw - a.pw;
         const int jc = 8 * my_chunk;
         const int r = col_r[jc];
         if (a.x_vec && r >= 0 && jc + 7 < kTileN && col_r[jc + 7] == r && col_s[jc + 7] == col_s[jc]) {
@@ -248,6 +275,7 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
       }
       vd[h2] = make_uint4(d[0], d[1], d[2], d[3]);
       vx[h2] = make_uint4(xv[0], xv[1], xv[2], xv[3]);
+      rows[h2].advance(dn, dp, dq, a.P, a.Q);
     }
   };
 
@@ -260,7 +288,7 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
   const int wf = 16 * (warp & 3), wj = 32 * (warp >> 2);
   const int mi = lane >> 3, lr = lane & 7;
   uint4 vd[2], vx[2];
-  if (pbeg < pend) load(pbeg, vd, vx);
+  if (pbeg < pend) load(vd, vx);
   for (int64_t p0 = pbeg; p0 < pend; p0 += kChunk) {
     __syncthreads();   // the previous chunk's fragments have been read
 #pragma unroll
@@ -269,7 +297,7 @@ __global__ void __launch_bounds__(kBwdThreads) bwd_filter_kernel(const BwdFilter
       *reinterpret_cast<uint4*>(sx + tile_off(my_row + 32 * h2, my_chunk)) = vx[h2];
     }
     __syncthreads();
-    if (p0 + kChunk < pend) load(p0 + kChunk, vd, vx);
+    if (p0 + kChunk < pend) load(vd, vx);
 #pragma unroll
     for (int ks = 0; ks < kChunk / 16; ++ks) {
       // A: filters wf .. wf+15 x pixels 16 ks ..; matrix mi = (pixel half
@@ -374,40 +402,45 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_tc_kernel(const Bwd
   const int64_t pq = static_cast<int64_t>(a.P) * a.Q;
   const int nchunks = pend > pbeg ? static_cast<int>((pend - pbeg + kChunk - 1) / kChunk) : 0;
   const uint32_t ring_s = smem_addr(ring);
-  int tap_r[2], tap_s[2], tap_c[2];
+  // this thread's two im2col columns: tap (r, s) and channel, and their
+  // offset from the tap-(0, 0) element in x
+  int tap_r[2], tap_s[2];
+  int64_t tap_off[2];
 #pragma unroll
   for (int hx = 0; hx < 2; ++hx) {
     const int jc = 64 * hx + 8 * my_chunk;
     tap_r[hx] = col_r[jc];
     tap_s[hx] = col_s[jc];
-    tap_c[hx] = col_c[jc];
+    tap_off[hx] = (static_cast<int64_t>(tap_r[hx]) * a.W + tap_s[hx]) * a.C + col_c[jc];
   }
+  const int dq = kChunk % a.Q, dp = (kChunk / a.Q) % a.P, dn = static_cast<int>(kChunk / pq);
+  PixelRow rows[2];
+  rows[0].init(pbeg + my_row, a.P, a.Q);
+  rows[1].init(pbeg + my_row + 32, a.P, a.Q);
+  // chunks are issued once each, in order, so the rows advance by kChunk
   auto issue = [&](int ci) {
-    const int64_t p0 = pbeg + static_cast<int64_t>(ci) * kChunk;
     const uint32_t st = ring_s + static_cast<uint32_t>((ci % kStages) * kStageBytes);
 #pragma unroll
     for (int h2 = 0; h2 < 2; ++h2) {
       const int row = my_row + 32 * h2;
-      const int64_t pix = p0 + row;
-      const bool pv = pix < pend;
-      const int64_t pc = pv ? pix : pbeg;
+      const bool pv = rows[h2].pix < pend;
+      const int64_t dy_row = pv ? rows[h2].pix * a.K : 0;
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf) {
         const int kb = k0 + 64 * hf + 8 * my_chunk;
         cp_async16(st + hf * kHalfTile + tile_off(row, my_chunk),
-                   a.dy + pc * a.K + (kb < a.K ? kb : 0), pv && kb < a.K);
+                   a.dy + dy_row + (kb < a.K ? kb : 0), pv && kb < a.K);
       }
-      const int n = static_cast<int>(pc / pq);
-      const int rem = static_cast<int>(pc - static_cast<int64_t>(n) * pq);
-      const int h0 = (rem / a.Q) * a.sh - a.ph, w0 = (rem % a.Q) * a.sw - a.pw;
+      const int h0 = rows[h2].p * a.sh - a.ph, w0 = rows[h2].q * a.sw - a.pw;
+      const int64_t x_row = ((static_cast<int64_t>(rows[h2].n) * a.H + h0) * a.W + w0) * a.C;
 #pragma unroll
       for (int hx = 0; hx < 2; ++hx) {
         const int hh = h0 + tap_r[hx], ww = w0 + tap_s[hx];
         const bool xv = pv && tap_r[hx] >= 0 && hh >= 0 && hh < a.H && ww >= 0 && ww < a.W;
-        const int64_t xo =
-            xv ? ((static_cast<int64_t>(n) * a.H + hh) * a.W + ww) * a.C + tap_c[hx] : 0;
-        cp_async16(st + (2 + hx) * kHalfTile + tile_off(row, my_chunk), a.x + xo, xv);
+        cp_async16(st + (2 + hx) * kHalfTile + tile_off(row, my_chunk),
+                   a.x + (xv ? x_row + tap_off[hx] : 0), xv);
       }
+      rows[h2].advance(dn, dp, dq, a.P, a.Q);
     }
   };
   constexpr uint32_t idesc = idesc_bf16_f32(128, 128) | (1u << 15) | (1u << 16);   // MN-major
@@ -483,27 +516,27 @@ __global__ void __launch_bounds__(kBwdThreads, 2) bwd_filter_tc_kernel(const Bwd
   }
 }
 
-// dw[e] = sum of the slices' partial values in a fixed order: block b
-// covers elements 32 b .. 32 b + 31; warp w sums slices w, w + 8, w + 16, ...
-// in order, and lane e of warp 0 adds the eight warp sums in warp order.
-constexpr int kReduceGroups = kBwdThreads / 32;
-
+// dw[e] = sum of the slices' partial values in a fixed order.  The block's
+// threads form `groups` (1, 2, 4 or 8, a function of the slice count) groups
+// of 256 / groups; group g sums slices g, g + groups, ... in order for one
+// element per thread, and group 0 adds the group sums in group order.
 __global__ void __launch_bounds__(kBwdThreads) bwd_filter_reduce_kernel(
-    const float* __restrict__ part, int slices, int64_t count, float* __restrict__ dw) {
-  __shared__ float sums[kReduceGroups][32];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int64_t e = static_cast<int64_t>(blockIdx.x) * 32 + lane;
+    const float* __restrict__ part, int slices, int groups, int64_t count,
+    float* __restrict__ dw) {
+  __shared__ float sums[kBwdThreads];
+  const int per = kBwdThreads / groups;
+  const int li = threadIdx.x % per, g = threadIdx.x / per;
+  const int64_t e = static_cast<int64_t>(blockIdx.x) * per + li;
   float s = 0.0f;
   if (e < count) {
 #pragma unroll 4
-    for (int z = w; z < slices; z += kReduceGroups) s += part[static_cast<int64_t>(z) * count + e];
+    for (int z = g; z < slices; z += groups) s += part[static_cast<int64_t>(z) * count + e];
   }
-  sums[w][lane] = s;
+  sums[threadIdx.x] = s;
   __syncthreads();
-  if (w == 0 && e < count) {
-    float t = sums[0][lane];
-#pragma unroll
-    for (int g = 1; g < kReduceGroups; ++g) t += sums[g][lane];
+  if (g == 0 && e < count) {
+    float t = sums[li];
+    for (int h = 1; h < groups; ++h) t += sums[h * per + li];
     dw[e] = t;
   }
 }
@@ -663,10 +696,12 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
   }
   if (st != TBN_OK) return st;
   const int64_t count = p.K * a.rsc;
-  const int64_t blocks = (count + 31) / 32;
+  const int groups = a.slices >= 8 ? 8 : a.slices >= 4 ? 4 : a.slices >= 2 ? 2 : 1;
+  const int64_t per = kBwdThreads / groups;
+  const int64_t blocks = (count + per - 1) / per;
   if (blocks > 0x7fffffff) return fail(TBN_ERR_UNSUPPORTED, "backward filter: too many weights");
   bwd_filter_reduce_kernel<<<static_cast<unsigned>(blocks), kBwdThreads, 0, s>>>(
-      a.part, a.slices, count, dw);
+      a.part, a.slices, groups, count, dw);
   return check_launch("bwd_filter_reduce_kernel");
 }
 
