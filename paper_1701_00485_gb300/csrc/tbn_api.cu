@@ -373,6 +373,14 @@ tbn_status validate_bwd(int64_t N, int64_t C, int64_t H, int64_t W, int64_t K, i
     return fail(TBN_ERR_INVALID_ARG, "conv backward: sizes must be >= 1");
   if (sh < 1 || sw < 1 || ph < 0 || pw < 0)
     return fail(TBN_ERR_INVALID_ARG, "conv backward: bad stride/pad");
+  // every size below 2^31 and pad below the kernel size before any sum or
+  // product of them is formed
+  const int64_t lim = int64_t(1) << 31;
+  if (N >= lim || C >= lim || H >= lim || W >= lim || K >= lim || R >= lim || S >= lim ||
+      sh >= lim || sw >= lim)
+    return fail(TBN_ERR_UNSUPPORTED, "conv backward: size too large");
+  if (ph > R - 1 || pw > S - 1)
+    return fail(TBN_ERR_UNSUPPORTED, "conv backward: needs pad <= kernel size - 1");
   if (H + 2 * ph < R || W + 2 * pw < S)
     return fail(TBN_ERR_INVALID_ARG, "conv backward: kernel larger than padded input");
   BwdConvShape& p = *out;

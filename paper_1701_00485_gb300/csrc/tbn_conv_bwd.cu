@@ -584,10 +584,16 @@ int bwd_filter_slices(const BwdConvShape& p) {
 
 const char* bwd_shape_reason(const BwdConvShape& p) {
   if (p.ph > p.R - 1 || p.pw > p.S - 1) return "backward needs pad <= kernel size - 1";
-  if (p.N * p.H * p.W * p.C >= (1ll << 40) || p.N * p.P * p.Q * p.K >= (1ll << 40))
+  // the sizes are below 2^31 here, so each pairwise product fits in int64
+  const int64_t lim = int64_t(1) << 40;
+  const auto prod_below = [lim](int64_t a, int64_t b, int64_t c, int64_t d) {
+    const int64_t ab = a * b, cd = c * d;
+    return ab < lim && cd < lim && (ab == 0 || cd < lim / ab);
+  };
+  if (!prod_below(p.N, p.H, p.W, p.C) || !prod_below(p.N, p.P, p.Q, p.K))
     return "backward: tensor too large";
-  if (p.C >= (1 << 30) || p.K >= (1 << 30) || p.R * p.S * p.C >= (1ll << 30) ||
-      p.R * p.S * p.K >= (1ll << 30))
+  if (p.C >= (1 << 30) || p.K >= (1 << 30) || !prod_below(p.R, p.S, p.C, 1024) ||
+      !prod_below(p.R, p.S, p.K, 1024))
     return "backward: filter too large";
   return "";
 }

@@ -145,3 +145,68 @@ def test_python_binding_requires_cuda_tensors():
     import torch
     with pytest.raises(ValueError):
         tbn.tbn_quantize_pack(torch.zeros(2, 16))
+
+
+def _bwd_data(L, **kw):
+    d = ctypes.c_void_p(256)
+    a = dict(dy=d, N=2, C=64, H=8, W=8, codes=d, alpha=d, K=64, R=3, S=3, sh=1, sw=1, ph=1,
+             pw=1, dx=d, dxdt=1, ws=d, wsb=1 << 30)
+    a.update(kw)
+    return L.tbn_conv2d_bwd_data(a["dy"], a["N"], a["C"], a["H"], a["W"], a["codes"],
+                                 a["alpha"], a["K"], a["R"], a["S"], a["sh"], a["sw"], a["ph"],
+                                 a["pw"], a["dx"], a["dxdt"], a["ws"], a["wsb"], None)
+
+
+def _bwd_filter(L, **kw):
+    d = ctypes.c_void_p(256)
+    a = dict(x=d, dy=d, N=2, C=64, H=8, W=8, K=64, R=3, S=3, sh=1, sw=1, ph=1, pw=1, dw=d,
+             ws=d, wsb=1 << 30)
+    a.update(kw)
+    return L.tbn_conv2d_bwd_filter(a["x"], a["dy"], a["N"], a["C"], a["H"], a["W"], a["K"],
+                                   a["R"], a["S"], a["sh"], a["sw"], a["ph"], a["pw"], a["dw"],
+                                   a["ws"], a["wsb"], None)
+
+
+@pytest.mark.parametrize("call", [_bwd_data, _bwd_filter])
+def test_bwd_rejects_bad_arguments(L, call):
+    """Every check of the TwoBitBackward entry points returns before a launch."""
+    first = "dy" if call is _bwd_data else "x"
+    assert call(L, **{first: None}) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, ws=None) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, N=0) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, K=-1) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, sh=0) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, pw=-1) == tbn.TBN_ERR_INVALID_ARG
+    assert call(L, H=1, W=1, ph=0, pw=0) == tbn.TBN_ERR_INVALID_ARG   # kernel > input
+    assert call(L, ph=3) == tbn.TBN_ERR_UNSUPPORTED                    # pad > R - 1
+    assert call(L, ph=1 << 62) == tbn.TBN_ERR_UNSUPPORTED              # no overflow first
+    assert call(L, N=1 << 31) == tbn.TBN_ERR_UNSUPPORTED
+    assert call(L, N=1 << 20, H=1 << 10, W=1 << 10) == tbn.TBN_ERR_UNSUPPORTED
+    assert call(L, C=1 << 28) == tbn.TBN_ERR_UNSUPPORTED               # R S C >= 2^30
+    assert call(L, wsb=0) == tbn.TBN_ERR_INVALID_ARG                   # workspace too small
+    assert call(L, ws=ctypes.c_void_p(128)) == tbn.TBN_ERR_MISALIGNED  # workspace 256-aligned
+    assert call(L, dy=ctypes.c_void_p(257)) == tbn.TBN_ERR_MISALIGNED
+    if call is _bwd_data:
+        assert call(L, dxdt=7) == tbn.TBN_ERR_INVALID_ARG
+        assert call(L, codes=None) == tbn.TBN_ERR_INVALID_ARG
+    else:
+        assert call(L, dw=ctypes.c_void_p(258)) == tbn.TBN_ERR_MISALIGNED
+
+
+def test_bwd_workspace_queries(L):
+    """Zero for shapes the entry points refuse; for valid shapes the input
+    gradient's scratch covers the transposed codes, the unit scales and the
+    dilated alpha-scaled dy, and the filter gradient's holds at least one
+    fp32 partial of dW."""
+    qd, qf = L.tbn_conv2d_bwd_data_workspace_bytes, L.tbn_conv2d_bwd_filter_workspace_bytes
+    assert qd(0, 64, 8, 8, 64, 3, 3, 1, 1, 1, 1) == 0
+    assert qf(2, 64, 8, 8, 64, 3, 3, 1, 1, 3, 1) == 0
+    assert qf(2, 64, 8, 8, 64, 3, 3, 1, 1, 1 << 62, 1) == 0
+    N, C, H, W, K, R, S = 2, 64, 8, 8, 96, 3, 3
+    wd = qd(N, C, H, W, K, R, S, 2, 2, 1, 1)
+    words_t = C * ((R * S * K + 15) // 16) * 4
+    Hd, Wd = H + 2 - R + 1, W + 2 - S + 1                      # dilated dy extent
+    assert wd >= words_t + C * 4 + N * Hd * Wd * K * 2 and wd % 256 == 0
+    wf = qf(N, C, H, W, K, R, S, 1, 1, 1, 1)
+    assert wf >= K * R * S * C * 4 and wf % 256 == 0
+    assert wf <= (64 << 20) + 256                              # partial tiles capped at 64 MB
