@@ -108,15 +108,21 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
   if (N < 1 || C < 1 || H < 1 || W < 1 || K < 1 || R < 1 || S < 1)
     return fail(TBN_ERR_INVALID_ARG, "conv: sizes must be >= 1");
   if (sh < 1 || sw < 1 || ph < 0 || pw < 0) return fail(TBN_ERR_INVALID_ARG, "conv: bad stride/pad");
-  if (H + 2 * ph < R || W + 2 * pw < S)
-    return fail(TBN_ERR_INVALID_ARG, "conv: kernel larger than padded input");
+  // bounds first, so that no sum or product below can overflow
+  const int64_t lim31 = int64_t(1) << 31;
+  if (N >= lim31 || C >= lim31 || H >= lim31 || W >= lim31 || K >= lim31)
+    return fail(TBN_ERR_UNSUPPORTED, "conv: a size is 2^31 or more");
   if (R > 0xFFFF || S > 0xFFFF || sh > 0xFFFF || sw > 0xFFFF || ph > 0xFFFF || pw > 0xFFFF)
     return fail(TBN_ERR_UNSUPPORTED, "conv: kernel/stride/pad above 65535");
+  if (H + 2 * ph < R || W + 2 * pw < S)
+    return fail(TBN_ERR_INVALID_ARG, "conv: kernel larger than padded input");
   const int64_t lim = int64_t(1) << 31;
   if (!mul_ok(C * R, S, lim) || !mul_ok(C, H * W, lim) || H * W >= lim)
     return fail(TBN_ERR_UNSUPPORTED, "conv: C*R*S or C*H*W exceeds 2^31");
   const int64_t P = (H + 2 * ph - R) / sh + 1, Q = (W + 2 * pw - S) / sw + 1;
-  if (!mul_ok(N, H * W * C, int64_t(1) << 46) || !mul_ok(N * P * Q, K, int64_t(1) << 46))
+  const int64_t lim46 = int64_t(1) << 46;
+  if (!mul_ok(N, H * W * C, lim46) || !mul_ok(N, P, lim46) || !mul_ok(N * P, Q, lim46) ||
+      !mul_ok(N * P * Q, K, lim46))
     return fail(TBN_ERR_UNSUPPORTED, "conv: tensor too large");
   const size_t xs = dtype_size(xdt), ys = dtype_size(ydt);
   if (!is_aligned(x, xs) || !is_aligned(y, ys) || !is_aligned(codes, 4) || !is_aligned(alpha, 4))
@@ -296,8 +302,8 @@ tbn_status validate_linear(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in
   if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad x dtype");
   if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "linear: bad y dtype");
   if (B < 1 || K_in < 1 || K_out < 1) return fail(TBN_ERR_INVALID_ARG, "linear: sizes must be >= 1");
-  if (K_in >= (int64_t(1) << 31) || K_out >= (int64_t(1) << 31))
-    return fail(TBN_ERR_UNSUPPORTED, "linear: K_in / K_out >= 2^31");
+  if (B >= (int64_t(1) << 31) || K_in >= (int64_t(1) << 31) || K_out >= (int64_t(1) << 31))
+    return fail(TBN_ERR_UNSUPPORTED, "linear: B / K_in / K_out >= 2^31");
   const size_t ys = dtype_size(ydt);
   if (!is_aligned(x, dtype_size(xdt)) || !is_aligned(y, ys) || !is_aligned(codes, 4) ||
       !is_aligned(alpha, 4) || (epi && epi->residual && !is_aligned(epi->residual, ys)))

@@ -88,6 +88,12 @@ def test_conv_rejects_bad_arguments(L):
     assert _conv(L, x=ctypes.c_void_p(257)) == tbn.TBN_ERR_MISALIGNED
     assert _conv(L, C=1 << 20, H=1 << 12, W=1) == tbn.TBN_ERR_UNSUPPORTED
     assert _conv(L, algo=11) == tbn.TBN_ERR_INVALID_ARG
+    # huge sizes are refused before any sum or product of them is formed
+    assert _conv(L, ph=1 << 62) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, N=1 << 62) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, C=1 << 40, R=1 << 30) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, N=1 << 20, H=8, W=8, C=1, ph=0xFFFF, pw=0xFFFF) == \
+        tbn.TBN_ERR_UNSUPPORTED                                      # N P Q above 2^46
 
 
 def test_select_algo_host_rules(L):
@@ -118,6 +124,8 @@ def test_linear_and_glue_reject_bad_arguments(L):
     d = ctypes.c_void_p(256)
     assert L.tbn_linear_fwd(None, 1, 1, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_linear_fwd(d, 1, 0, 64, d, d, 8, d, 1, None, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_linear_fwd(d, 1, 1 << 40, 64, d, d, 8, d, 1, None, None) == \
+        tbn.TBN_ERR_UNSUPPORTED
     assert L.tbn_linear_fwd_ws(None, 1, 1, 64, d, d, 8, d, 1, None, d, 4096, None) == \
         tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_linear_fwd_ws(d, 1, 1, 64, d, d, 8, ctypes.c_void_p(257), 1, None, d, 4096,
