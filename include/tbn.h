@@ -25,8 +25,8 @@
  *   per-process kernel attributes.
  * - One process drives one GPU (run one process per GPU for replicas): the
  *   kernels' shared-memory attributes are set on the device that is current
- *   at a kernel's first launch in the process, and a launch on another
- *   device would fail with TBN_ERR_CUDA.
+ *   at a kernel's first launch in the process, so a later launch of a
+ *   large-shared-memory kernel on another device can fail with TBN_ERR_CUDA.
  * - Every compute call is asynchronous on `stream` (a cudaStream_t; NULL is
  *   the legacy default stream).  Arguments are validated on the host before
  *   anything is launched; an invalid call returns a status and launches
