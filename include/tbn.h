@@ -154,6 +154,15 @@ const char *tbn_last_error(void);
  * error was recorded. */
 tbn_status tbn_device_error(uint32_t *flags);
 
+/* Self-check of the failure detection that every kernel's waits rely on:
+ * launches one thread that waits, through the same bounded wait, on a
+ * shared-memory mbarrier that nothing arrives at.  After limit_us
+ * microseconds (1 .. 1000000) the wait gives up, sets bit 1 (timeout) of
+ * the current device's error word and the kernel returns; the device stays
+ * usable.  Asynchronous on `stream`; read the result with tbn_device_error.
+ * TBN_ERR_INVALID_ARG for a limit out of range. */
+tbn_status tbn_selftest_wait_timeout(uint32_t limit_us, tbn_stream stream);
+
 /* Quantize and pack one layer -- Algorithm 1, quantization loop; Eq. 3
  * (discretization) and Eq. 5 (optimal scaling factor), Section 2.
  *

@@ -27,7 +27,8 @@ __all__ = [
     "tbn_conv2d_select_algo", "conv_out_hw", "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter",
     "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_NCHW_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
-    "TBN_CONV_SMALL_TAPS",
+    "TBN_CONV_SMALL_TAPS", "TBN_DEVERR_TIMEOUT", "TBN_DEVERR_BAD_LAUNCH",
+    "tbn_selftest_wait_timeout",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -40,6 +41,7 @@ TBN_NCHW, TBN_NHWC, TBN_NCHW_NHWC = 0, 1, 2
 TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
 TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM, TBN_CONV_SMALL_TAPS = 0, 1, 2, 3
 TBN_MAX_QUANT_JOBS = 16
+TBN_DEVERR_TIMEOUT, TBN_DEVERR_BAD_LAUNCH = 1, 2   # bits of the device error word
 
 # every symbol include/tbn.h declares
 EXPORTED = [
@@ -49,6 +51,7 @@ EXPORTED = [
     "tbn_linear_workspace_bytes", "tbn_linear_fwd_ws", "tbn_linear_fwd_noalloc",
     "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_conv2d_bwd_data_workspace_bytes",
     "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter_workspace_bytes", "tbn_conv2d_bwd_filter",
+    "tbn_selftest_wait_timeout",
 ]
 
 
@@ -96,6 +99,7 @@ def lib():
             "tbn_status_string": ([I32], ctypes.c_char_p),
             "tbn_last_error": ([], ctypes.c_char_p),
             "tbn_device_error": ([ctypes.POINTER(ctypes.c_uint32)], I32),
+            "tbn_selftest_wait_timeout": ([ctypes.c_uint32, P], I32),
             "tbn_quantize_pack": ([P, I64, I64, U32P, P, P], I32),
             "tbn_quantize_pack_group": ([ctypes.POINTER(QuantJob), I32, P], I32),
             "tbn_unpack": ([U32P, P, I64, I64, P, I32, P], I32),
@@ -412,3 +416,10 @@ def tbn_device_error() -> int:
     v = ctypes.c_uint32(0)
     _check(lib().tbn_device_error(ctypes.byref(v)), "tbn_device_error")
     return int(v.value)
+
+
+def tbn_selftest_wait_timeout(limit_us: int, stream=None) -> None:
+    """Launch the bounded-wait self-check: a wait that nothing ends runs out
+    after limit_us and sets TBN_DEVERR_TIMEOUT in the device error word."""
+    _check(lib().tbn_selftest_wait_timeout(limit_us, _stream(stream)),
+           "tbn_selftest_wait_timeout")

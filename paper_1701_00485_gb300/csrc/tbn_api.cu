@@ -8,6 +8,7 @@
 #include <mutex>
 
 #include "tbn.h"
+#include "tbn_device.cuh"
 #include "tbn_internal.h"
 
 namespace tbn {
@@ -18,6 +19,18 @@ __device__ uint32_t g_tbn_device_error;
 namespace {
 
 thread_local char t_last_error[512] = "";
+
+// One thread waits on a fresh mbarrier (phase 0 never completes: nothing
+// arrives) through the library's bounded wait, which records the timeout in
+// the error word after limit_ns and returns.
+__global__ void selftest_wait_timeout_kernel(uint32_t* err, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    mbar_wait(&bar, 0u, nullptr, err, limit_ns);
+  }
+}
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -215,6 +228,16 @@ tbn_status tbn_device_error(uint32_t* flags) {
   if (e != cudaSuccess) return cuda_fail(e, "device_error: clear");
   *flags = v;
   return TBN_OK;
+}
+
+tbn_status tbn_selftest_wait_timeout(uint32_t limit_us, tbn_stream stream) {
+  if (limit_us < 1 || limit_us > 1000000)
+    return fail(TBN_ERR_INVALID_ARG, "selftest_wait_timeout: limit must be 1 .. 1000000 us");
+  uint32_t* err = device_error_word();
+  if (!err) return fail(TBN_ERR_CUDA, "selftest_wait_timeout: cannot resolve the error word");
+  selftest_wait_timeout_kernel<<<1, 32, 0, as_stream(stream)>>>(err,
+                                                                uint64_t(limit_us) * 1000u);
+  return check_launch("selftest_wait_timeout_kernel");
 }
 
 tbn_status tbn_quantize_pack_group(const tbn_quant_job* jobs, int njobs, tbn_stream stream) {

@@ -218,3 +218,8 @@ def test_bwd_workspace_queries(L):
     wf = qf(N, C, H, W, K, R, S, 1, 1, 1, 1)
     assert wf >= K * R * S * C * 4 and wf % 256 == 0
     assert wf <= (64 << 20) + 256                              # partial tiles capped at 64 MB
+
+
+def test_selftest_wait_timeout_rejects_bad_limits(L):
+    assert L.tbn_selftest_wait_timeout(0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_selftest_wait_timeout(1000001, None) == tbn.TBN_ERR_INVALID_ARG
