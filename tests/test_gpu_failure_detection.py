@@ -14,7 +14,7 @@ pytestmark = pytest.mark.gpu
 
 
 def test_bounded_wait_runs_out_and_is_reported():
-    assert tbn.tbn_device_error() == 0
+    tbn.tbn_device_error()                         # start from a clear word
     t0 = time.perf_counter()
     tbn.tbn_selftest_wait_timeout(2000)            # 2 ms
     flags = tbn.tbn_device_error()                 # synchronizes
