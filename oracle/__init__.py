@@ -14,6 +14,9 @@ follows:
   quantize        Algorithm 1, quantization loop (Eq. 3 + Eq. 5 per filter)
   pack / unpack   two-bit storage; the paper fixes only "two bits per weight",
                   the field layout is documented in tbn_oracle.h
+  pack_canonical / unpack_canonical   the canonical (sequential) two-bit
+                  layout, the interchange format (same fields, code i at bits
+                  2i, 2i+1 of its word)
   quant_error     Eq. 2 objective, evaluated directly
   conv2d_nchw     Eq. 1, seven nested loops, zero padding, cross-correlation
   conv2d_sites    Eq. 1 at selected output sites
@@ -22,6 +25,10 @@ follows:
                   with alpha*W~) and the gradient w.r.t. alpha*W~
   linear          Section 3: fully-connected layer treated as a convolution
   epilogue, maxpool2d_nchw   network glue of the benchmark workloads
+  dense_conv2d_nchw, avgpool_global_nchw, dense_linear   the full-precision
+                  first convolution, global average pool and last
+                  fully-connected layer of the ResNet-18 workload (not part
+                  of the paper's method)
 """
 from __future__ import annotations
 
@@ -112,7 +119,12 @@ class Oracle:
             "orc_conv2d_bwd_filter_nchw": ([P, I, I, I, I, P, I, I, I, I, I, I, I, I, I, P, P],
                                            None),
             "orc_epilogue": ([P, P, I, ctypes.c_int], None),
-            "orc_maxpool2d_nchw": ([P, I, I, I, I, I, I, I, I, P], None),
+            "orc_maxpool2d_nchw": ([P, I, I, I, I, I, I, I, I, I, I, P], None),
+            "orc_pack_canonical": ([P, I, I, P], ctypes.c_int),
+            "orc_unpack_canonical": ([P, I, I, P], ctypes.c_int),
+            "orc_dense_conv2d_nchw": ([P, I, I, I, I, P, I, I, I, I, I, I, I, P, P], None),
+            "orc_avgpool_global_nchw": ([P, I, I, I, I, P], None),
+            "orc_dense_linear": ([P, I, I, P, I, P, P], None),
             "orc_num_threads": ([], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
@@ -278,15 +290,69 @@ class Oracle:
                               out.size, int(bool(relu)))
         return out
 
-    def maxpool2d_nchw(self, x, k=(2, 2), stride=(2, 2)):
-        """Max pooling without padding, NCHW."""
+    def maxpool2d_nchw(self, x, k=(2, 2), stride=(2, 2), pad=(0, 0)):
+        """Max pooling, NCHW; taps in the padding are skipped (-inf padding)."""
         x = np.ascontiguousarray(np.asarray(x, dtype=np.float64))
         N, C, H, W = x.shape
-        Ho, Wo = (H - k[0]) // stride[0] + 1, (W - k[1]) // stride[1] + 1
+        Ho, Wo = out_hw(H, W, k[0], k[1], stride, pad)
         y = np.empty((N, C, Ho, Wo), dtype=np.float64)
         self.lib.orc_maxpool2d_nchw(_ptr(x), N, C, H, W, k[0], k[1], stride[0], stride[1],
-                                    _ptr(y))
+                                    pad[0], pad[1], _ptr(y))
         return y
+
+    def pack_canonical(self, wt2d) -> np.ndarray:
+        """Pack int8 codes [K, n] in the canonical layout (code i at bits 2i, 2i+1)."""
+        wt = np.ascontiguousarray(np.asarray(wt2d, dtype=np.int8))
+        K, n = wt.shape
+        out = np.empty((K, self.words_per_filter(n)), dtype=np.uint32)
+        if self.lib.orc_pack_canonical(_ptr(wt), K, n, _ptr(out)) != 0:
+            raise ValueError("codes must be in {-2,-1,1,2}")
+        return out
+
+    def unpack_canonical(self, words2d, n: int) -> np.ndarray:
+        """Inverse of pack_canonical; raises if a padding field is non-zero."""
+        w = np.ascontiguousarray(np.asarray(words2d, dtype=np.uint32))
+        K = w.shape[0]
+        if w.shape[1] != self.words_per_filter(n):
+            raise ValueError("word count does not match n")
+        out = np.empty((K, n), dtype=np.int8)
+        if self.lib.orc_unpack_canonical(_ptr(w), K, n, _ptr(out)) != 0:
+            raise ValueError("non-zero padding field")
+        return out
+
+    def dense_conv2d_nchw(self, x, w, stride=(1, 1), pad=(0, 0)):
+        """Full-precision convolution (fp32 weights), NCHW; returns (y, bound)
+        float64 [N, K, P, Q], bound = sum of |x * w| over the taps."""
+        x, w = _f32(x), _f32(w)
+        N, C, H, W = x.shape
+        K, C2, R, S = w.shape
+        assert C2 == C
+        P, Q = out_hw(H, W, R, S, stride, pad)
+        y = np.empty((N, K, P, Q), dtype=np.float64)
+        bound = np.empty_like(y)
+        self.lib.orc_dense_conv2d_nchw(_ptr(x), N, C, H, W, _ptr(w), K, R, S, stride[0],
+                                       stride[1], pad[0], pad[1], _ptr(y), _ptr(bound))
+        return y, bound
+
+    def avgpool_global_nchw(self, x):
+        """Mean over H and W of x [N, C, H, W]; returns float64 [N, C]."""
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+        N, C, H, W = x.shape
+        y = np.empty((N, C), dtype=np.float64)
+        self.lib.orc_avgpool_global_nchw(_ptr(x), N, C, H, W, _ptr(y))
+        return y
+
+    def dense_linear(self, x, w):
+        """Full-precision fully-connected layer: x [B, Kin], w [Kout, Kin] fp32;
+        returns (y, bound) float64 [B, Kout]."""
+        x, w = _f32(x), _f32(w)
+        B, Kin = x.shape
+        Kout = w.shape[0]
+        assert w.shape[1] == Kin
+        y = np.empty((B, Kout), dtype=np.float64)
+        bound = np.empty_like(y)
+        self.lib.orc_dense_linear(_ptr(x), B, Kin, _ptr(w), Kout, _ptr(y), _ptr(bound))
+        return y, bound
 
 
 def default() -> Oracle:

@@ -145,6 +145,46 @@ int orc_unpack(const uint32_t *words, int64_t K, int64_t n, int8_t *wt)
     return bad_padding ? -1 : 0;
 }
 
+/* Canonical ("sequential") two-bit layout, the interchange format: the same
+ * field f = m + 2 s per code, code i of a filter in word i / 16 at bits
+ * 2 (i mod 16) (the bit m) and 2 (i mod 16) + 1 (the bit s), little-endian,
+ * unused fields 0. */
+static uint32_t canonical_field_at(const uint32_t *words, int64_t wpf, int64_t k, int64_t i)
+{
+    uint32_t w = words[k * wpf + i / 16];
+    return (w >> (2 * (i % 16))) & 3u;
+}
+
+int orc_pack_canonical(const int8_t *wt, int64_t K, int64_t n, uint32_t *words)
+{
+    int64_t wpf = orc_words_per_filter(n);
+    for (int64_t k = 0; k < K; ++k) {
+        for (int64_t j = 0; j < wpf; ++j)
+            words[k * wpf + j] = 0u;
+        for (int64_t i = 0; i < n; ++i) {
+            uint32_t f;
+            if (field_of(wt[k * n + i], &f) != 0)
+                return -1;
+            words[k * wpf + i / 16] |= f << (2 * (i % 16));
+        }
+    }
+    return 0;
+}
+
+int orc_unpack_canonical(const uint32_t *words, int64_t K, int64_t n, int8_t *wt)
+{
+    int64_t wpf = orc_words_per_filter(n);
+    int bad_padding = 0;
+    for (int64_t k = 0; k < K; ++k) {
+        for (int64_t i = 0; i < n; ++i)
+            wt[k * n + i] = (int8_t)value_of(canonical_field_at(words, wpf, k, i));
+        for (int64_t i = n; i < wpf * 16; ++i)
+            if (canonical_field_at(words, wpf, k, i) != 0u)
+                bad_padding = 1;
+    }
+    return bad_padding ? -1 : 0;
+}
+
 /* ---- Eq. 2 (Section 2): quantization error ------------------------------ */
 double orc_quant_error(const float *W, const int8_t *wt, int64_t n, double alpha)
 {
@@ -337,9 +377,9 @@ void orc_epilogue(double *y, const double *residual, int64_t count, int relu)
 
 void orc_maxpool2d_nchw(const double *x, int64_t N, int64_t C, int64_t H,
                         int64_t W, int64_t kh, int64_t kw, int64_t sh,
-                        int64_t sw, double *y)
+                        int64_t sw, int64_t ph, int64_t pw, double *y)
 {
-    int64_t Ho = (H - kh) / sh + 1, Wo = (W - kw) / sw + 1;
+    int64_t Ho = (H + 2 * ph - kh) / sh + 1, Wo = (W + 2 * pw - kw) / sw + 1;
     for (int64_t b = 0; b < N; ++b)
         for (int64_t c = 0; c < C; ++c)
             for (int64_t i = 0; i < Ho; ++i)
@@ -347,12 +387,85 @@ void orc_maxpool2d_nchw(const double *x, int64_t N, int64_t C, int64_t H,
                     double m = -INFINITY;
                     for (int64_t u = 0; u < kh; ++u)
                         for (int64_t v = 0; v < kw; ++v) {
-                            double t = x[((b * C + c) * H + i * sh + u) * W + j * sw + v];
+                            int64_t h = i * sh - ph + u, w = j * sw - pw + v;
+                            if (h < 0 || h >= H || w < 0 || w >= W)
+                                continue; /* padding never wins the max */
+                            double t = x[((b * C + c) * H + h) * W + w];
                             if (t > m)
                                 m = t;
                         }
                     y[((b * C + c) * Ho + i) * Wo + j] = m;
                 }
+}
+
+/* ---- the full-precision layers around the two-bit ones ------------------ */
+/* Networks keep their first convolution and last fully-connected layer in
+ * full precision (the ResNet-18 workload); these are their definitions. */
+void orc_dense_conv2d_nchw(const float *x, int64_t N, int64_t C, int64_t H, int64_t W,
+                           const float *w, int64_t K, int64_t R, int64_t S, int64_t sh,
+                           int64_t sw, int64_t ph, int64_t pw, double *y, double *bound)
+{
+    int64_t P = out_extent(H, R, sh, ph);
+    int64_t Q = out_extent(W, S, sw, pw);
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+    for (int64_t bk = 0; bk < N * K; ++bk) {
+        int64_t b = bk / K, k = bk % K;
+        for (int64_t p = 0; p < P; ++p)
+            for (int64_t q = 0; q < Q; ++q) {
+                double acc = 0.0, mag = 0.0;
+                for (int64_t c = 0; c < C; ++c)
+                    for (int64_t r = 0; r < R; ++r)
+                        for (int64_t s = 0; s < S; ++s) {
+                            int64_t h_in = p * sh - ph + r;
+                            int64_t w_in = q * sw - pw + s;
+                            if (h_in < 0 || h_in >= H || w_in < 0 || w_in >= W)
+                                continue; /* zero padding */
+                            double xw = (double)x[((b * C + c) * H + h_in) * W + w_in] *
+                                       (double)w[((k * C + c) * R + r) * S + s];
+                            acc += xw;
+                            mag += fabs(xw);
+                        }
+                int64_t o = ((b * K + k) * P + p) * Q + q;
+                y[o] = acc;
+                if (bound)
+                    bound[o] = mag;
+            }
+    }
+}
+
+void orc_avgpool_global_nchw(const double *x, int64_t N, int64_t C, int64_t H, int64_t W,
+                             double *y)
+{
+    for (int64_t b = 0; b < N; ++b)
+        for (int64_t c = 0; c < C; ++c) {
+            double acc = 0.0;
+            for (int64_t h = 0; h < H; ++h)
+                for (int64_t w = 0; w < W; ++w)
+                    acc += x[((b * C + c) * H + h) * W + w];
+            y[b * C + c] = acc / (double)(H * W);
+        }
+}
+
+void orc_dense_linear(const float *x, int64_t B, int64_t Kin, const float *w, int64_t Kout,
+                      double *y, double *bound)
+{
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static)
+#endif
+    for (int64_t bk = 0; bk < B * Kout; ++bk) {
+        int64_t b = bk / Kout, k = bk % Kout;
+        double acc = 0.0, mag = 0.0;
+        for (int64_t j = 0; j < Kin; ++j) {
+            double prod = (double)x[b * Kin + j] * (double)w[k * Kin + j];
+            acc += prod;
+            mag += fabs(prod);
+        }
+        y[bk] = acc;
+        if (bound)
+            bound[bk] = mag;
+    }
 }
 
 int orc_num_threads(void)

@@ -65,6 +65,13 @@ int orc_pack(const int8_t *wt, int64_t K, int64_t n, uint32_t *words);
 /* Inverse of orc_pack.  Returns 0, or -1 if a padding field is non-zero. */
 int orc_unpack(const uint32_t *words, int64_t K, int64_t n, int8_t *wt);
 
+/* Canonical two-bit layout (the interchange format): the same field
+ * f = m + 2 s, code i of filter k at bits 2 (i mod 16) .. 2 (i mod 16) + 1 of
+ * word k * words_per_filter + i / 16 (bit m low, bit s high), unused fields
+ * 0.  Same return values as orc_pack / orc_unpack. */
+int orc_pack_canonical(const int8_t *wt, int64_t K, int64_t n, uint32_t *words);
+int orc_unpack_canonical(const uint32_t *words, int64_t K, int64_t n, int8_t *wt);
+
 /* Eq. 2 objective evaluated directly: sum_i (W_i - alpha wt_i)^2. */
 double orc_quant_error(const float *W, const int8_t *wt, int64_t n, double alpha);
 
@@ -128,10 +135,28 @@ void orc_linear(const float *x, int64_t B, int64_t Kin, const int8_t *wt,
 void orc_epilogue(double *y, const double *residual, int64_t count, int relu);
 
 /* Max pooling in NCHW (network glue between TBN layers): window kh x kw,
- * stride sh x sw, no padding.  y is [N][C][Ho][Wo]. */
+ * stride sh x sw, padding ph x pw (taps outside the image are skipped, i.e.
+ * padded with -infinity).  y is [N][C][Ho][Wo], Ho = (H + 2 ph - kh)/sh + 1. */
 void orc_maxpool2d_nchw(const double *x, int64_t N, int64_t C, int64_t H,
                         int64_t W, int64_t kh, int64_t kw, int64_t sh,
-                        int64_t sw, double *y);
+                        int64_t sw, int64_t ph, int64_t pw, double *y);
+
+/* Full-precision layers of the networks (first convolution and last
+ * fully-connected layer of ResNet-18; not part of the paper's method):
+ *   dense conv:   y[b,k,p,q] = sum_{c,r,s} x[b,c,p sh-ph+r,q sw-pw+s] w[k,c,r,s]
+ *                 (zero padding), bound = the same sum of |products|;
+ *                 x [N][C][H][W], w [K][C][R][S] fp32, y/bound [N][K][P][Q];
+ *   global average pool: y[b,c] = mean of x[b,c,:,:]; x [N][C][H][W];
+ *   dense linear: y[b,k] = sum_j x[b,j] w[k,j], bound = sum_j |x[b,j] w[k,j]|;
+ *                 x [B][Kin], w [Kout][Kin] fp32.
+ * bound may be NULL. */
+void orc_dense_conv2d_nchw(const float *x, int64_t N, int64_t C, int64_t H, int64_t W,
+                           const float *w, int64_t K, int64_t R, int64_t S, int64_t sh,
+                           int64_t sw, int64_t ph, int64_t pw, double *y, double *bound);
+void orc_avgpool_global_nchw(const double *x, int64_t N, int64_t C, int64_t H, int64_t W,
+                             double *y);
+void orc_dense_linear(const float *x, int64_t B, int64_t Kin, const float *w, int64_t Kout,
+                      double *y, double *bound);
 
 /* Threads the parallel loops use (1 without OpenMP). */
 int orc_num_threads(void);

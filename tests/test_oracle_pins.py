@@ -378,6 +378,89 @@ def pin_glue(orc):
     assert np.array_equal(orc.epilogue(y, None, relu=False), y)
 
 
+
+def pin_canonical_layout(orc):
+    """The canonical interchange layout: the hand-derived words of both worked
+    examples (0x50AB, 0x6C: field f = m + 2 s of code i at bits 2i, 2i+1),
+    round trips, the padding check, and the same field values as the
+    byte-planar layout code by code."""
+    gq = read_golden("quantize_worked_example.txt")
+    wq = np.array([[int(v) for v in gq["codes"]]], dtype=np.int8)
+    assert int(orc.pack_canonical(wq)[0, 0]) == int(gq["packed_canonical"][0], 16)
+    gc = read_golden("conv_worked_example.txt")
+    wc = np.array([[int(v) for v in gc["codes"]]], dtype=np.int8)
+    assert int(orc.pack_canonical(wc)[0, 0]) == int(gc["packed_canonical"][0], 16)
+    rng = np.random.default_rng(31)
+    field = {1: 0, 2: 1, -1: 2, -2: 3}
+    for n in (1, 7, 16, 17, 40, 363):
+        codes = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(3, n))
+        words = orc.pack_canonical(codes)
+        assert words.shape == (3, (n + 15) // 16)
+        assert np.array_equal(orc.unpack_canonical(words, n), codes)
+        # bit positions written out from the definition
+        for k in range(3):
+            for i in range(n):
+                f = (int(words[k, i // 16]) >> (2 * (i % 16))) & 3
+                assert f == field[int(codes[k, i])]
+        if n % 16:
+            bad = words.copy()
+            bad[0, -1] |= np.uint32(1 << 30)
+            with pytest.raises(ValueError):
+                orc.unpack_canonical(bad, n)
+    # both layouts hold the same codes
+    codes = rng.choice(np.array([-2, -1, 1, 2], dtype=np.int8), size=(4, 50))
+    assert np.array_equal(orc.unpack(orc.pack(codes), 50),
+                          orc.unpack_canonical(orc.pack_canonical(codes), 50))
+
+
+def pin_maxpool_padding(orc):
+    """Max pooling with padding (ResNet-18's 3x3/2, pad 1) against torch,
+    including all-negative inputs, where a zero pad would wrongly win."""
+    rng = np.random.default_rng(32)
+    for shape, k, st, pd in (((2, 3, 9, 8), (3, 3), (2, 2), (1, 1)),
+                             ((1, 2, 7, 7), (3, 3), (2, 2), (1, 1)),
+                             ((1, 1, 6, 5), (2, 3), (1, 2), (1, 0))):
+        x = rng.normal(0, 1, size=shape) - 3.0
+        ref = torch.nn.functional.max_pool2d(torch.from_numpy(x), k, st, pd).numpy()
+        assert np.array_equal(orc.maxpool2d_nchw(x, k, st, pd), ref)
+
+
+def pin_dense_layers(orc):
+    """The full-precision first convolution, global average pool and last
+    fully-connected layer: the hand-worked example, torch's fp64 conv2d, numpy
+    means and matmuls."""
+    g = read_golden("conv_worked_example.txt")
+    x = np.array([float(v) for v in g["x"]], dtype=F32).reshape(1, 1, 3, 3)
+    W = np.array([float(v) for v in g["W"]], dtype=F32).reshape(1, 1, 2, 2)
+    y, bound = orc.dense_conv2d_nchw(x, W)
+    assert y.ravel().tolist() == [float(v) for v in g["dense_y"]]
+    assert bound.ravel().tolist() == [float(v) for v in g["dense_abs"]]
+    rng = np.random.default_rng(33)
+    for N, C, H, Wd, K, R, S, st, pd in ((2, 3, 15, 13, 4, 7, 7, (2, 2), (3, 3)),
+                                        (1, 2, 8, 9, 3, 3, 1, (1, 2), (1, 0))):
+        x = rng.normal(0, 1, size=(N, C, H, Wd)).astype(F32)
+        w = rng.normal(0, 0.3, size=(K, C, R, S)).astype(F32)
+        y, bound = orc.dense_conv2d_nchw(x, w, st, pd)
+        xt, wt_ = torch.from_numpy(x.astype(np.float64)), torch.from_numpy(w.astype(np.float64))
+        ref = torch.nn.functional.conv2d(xt, wt_, stride=st, padding=pd).numpy()
+        mag = torch.nn.functional.conv2d(xt.abs(), wt_.abs(), stride=st, padding=pd).numpy()
+        assert np.allclose(y, ref, rtol=1e-12, atol=1e-12)
+        assert np.allclose(bound, mag, rtol=1e-12, atol=1e-12)
+    x = rng.normal(0, 1, size=(3, 5, 7, 6))
+    assert np.allclose(orc.avgpool_global_nchw(x), x.mean(axis=(2, 3)), rtol=1e-14, atol=1e-15)
+    assert np.array_equal(orc.avgpool_global_nchw(np.full((1, 2, 4, 4), 2.5)),
+                          np.full((1, 2), 2.5))
+    xb = rng.normal(0, 1, size=(4, 37)).astype(F32)
+    wb = rng.normal(0, 0.2, size=(9, 37)).astype(F32)
+    y, bound = orc.dense_linear(xb, wb)
+    xd, wd = xb.astype(np.float64), wb.astype(np.float64)
+    assert np.allclose(y, xd @ wd.T, rtol=1e-12, atol=1e-12)
+    assert np.allclose(bound, np.abs(xd) @ np.abs(wd).T, rtol=1e-12, atol=1e-12)
+    # a fully-connected layer is a 1x1 convolution on a 1x1 image
+    yc, bc = orc.dense_conv2d_nchw(xb.reshape(4, 37, 1, 1), wb.reshape(9, 37, 1, 1))
+    assert np.array_equal(yc.reshape(4, 9), y) and np.array_equal(bc.reshape(4, 9), bound)
+
+
 BWD_CASES = [
     # N, C, H, W, K, R, S, stride, pad
     (2, 3, 7, 6, 4, 3, 2, (2, 1), (1, 1)),
@@ -445,7 +528,8 @@ PINS = [pin_quantize_worked_example, pin_discretize_boundaries,
         pin_bruteforce_tiny, pin_exact_special_case, pin_pack_bit_layout, pin_pack_roundtrip,
         pin_dequantized_values, pin_conv_worked_example, pin_conv_vs_torch,
         pin_conv_vs_im2col, pin_conv_sites, pin_box_filter, pin_linear, pin_glue,
-        pin_all_zero_filter, pin_bwd_adjoint, pin_bwd_vs_torch]
+        pin_all_zero_filter, pin_bwd_adjoint, pin_bwd_vs_torch, pin_canonical_layout,
+        pin_maxpool_padding, pin_dense_layers]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -486,6 +570,21 @@ MUTANTS = [
     ("filter gradient sums magnitudes", "acc += t;", "acc += fabs(t);"),
     ("bound without abs", "acc += xv * wv;\n                abs_sum += fabs(xv);",
      "acc += xv * wv;\n                abs_sum += xv;"),
+    ("canonical layout with the sign bit low", "words[k * wpf + i / 16] |= f << (2 * (i % 16));",
+     "words[k * wpf + i / 16] |= ((f >> 1) | ((f & 1u) << 1)) << (2 * (i % 16));"),
+    ("canonical layout codes in reverse order within a word",
+     "return (w >> (2 * (i % 16))) & 3u;", "return (w >> (2 * (15 - i % 16))) & 3u;"),
+    ("max pool padding not subtracted", "int64_t h = i * sh - ph + u, w = j * sw - pw + v;",
+     "int64_t h = i * sh + u, w = j * sw + v;"),
+    ("max pool padding counted as zero", "continue; /* padding never wins the max */",
+     "{ if (0.0 > m) m = 0.0; continue; }"),
+    ("dense convolution ignores the column stride", "int64_t w_in = q * sw - pw + s;",
+     "int64_t w_in = q - pw + s;"),
+    ("dense convolution bound without abs", "mag += fabs(xw);", "mag += xw;"),
+    ("average over H only", "y[b * C + c] = acc / (double)(H * W);",
+     "y[b * C + c] = acc / (double)H;"),
+    ("dense linear transposed weight", "(double)w[k * Kin + j];",
+     "(double)w[(j % Kout) * Kin + (k % Kin)];"),
 ]
 
 
