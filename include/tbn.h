@@ -15,7 +15,12 @@
  *                       scratch for the batch-1 fp32 table-lookup GEMV
  *   tbn_conv2d_bwd_data, tbn_conv2d_bwd_filter   Algorithm 1's
  *                       TwoBitBackward through a convolution
+ *   tbn_repack          byte-planar codes <-> the canonical interchange layout
  *   tbn_maxpool2d_nhwc, tbn_nchw_to_nhwc   network glue between layers
+ *   tbn_dense_conv2d_fwd, tbn_avgpool2d_global_nhwc, tbn_dense_linear_fwd
+ *                       the full-precision layers a network keeps around its
+ *                       two-bit layers (first convolution, global average
+ *                       pool, last fully-connected layer)
  *
  * Conventions shared by every call
  * --------------------------------
@@ -77,7 +82,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 5
+#define TBN_ABI_VERSION 6
 
 typedef enum {
   TBN_OK = 0,
@@ -200,6 +205,25 @@ tbn_status tbn_quantize_pack_group(const tbn_quant_job *jobs, int njobs, tbn_str
  * Padding fields are ignored. */
 tbn_status tbn_unpack(const uint32_t *codes, const float *alpha, int64_t K, int64_t n,
                       void *out, tbn_unpack_format fmt, tbn_stream stream);
+
+/* Canonical ("sequential") two-bit layout, the interchange format for codes
+ * exchanged with other software: the same field f = m + 2 s per code (Section
+ * 1: two bits per weight), code i of filter k in word
+ * k * tbn_packed_words(n) + i / 16 at bits 2 (i mod 16) (m) and
+ * 2 (i mod 16) + 1 (s), little-endian, unused fields 0.  The worked example
+ * W~ = (-2, -1, -1, -1, 1, 1, 2, 2) is 0x000050AB in this layout and
+ * 0x03080309 in the library's byte-planar one. */
+typedef enum {
+  TBN_REPACK_CANONICAL_TO_PLANAR = 0,
+  TBN_REPACK_PLANAR_TO_CANONICAL = 1
+} tbn_repack_direction;
+
+/* Repack codes [K][tbn_packed_words(n)] between the two layouts (a fixed
+ * permutation of the bits of each word; unused fields stay 0).  in and out
+ * are 4-byte aligned device arrays of the same size; they may be the same
+ * array (in place) but must not otherwise overlap.  Asynchronous on `stream`. */
+tbn_status tbn_repack(const uint32_t *in, int64_t K, int64_t n, uint32_t *out,
+                      tbn_repack_direction dir, tbn_stream stream);
 
 /* Two-bit convolution, Eq. 1 (Section 2): cross-correlation with zero
  * padding, no bias, groups = 1, dilation = 1 (the paper states none of
@@ -333,17 +357,48 @@ tbn_status tbn_linear_fwd_noalloc(const void *x, tbn_dtype xdt, int64_t B, int64
                                   void *y, tbn_dtype ydt, const tbn_epilogue *epi,
                                   tbn_stream stream);
 
-/* Max pooling over NHWC (network glue): window kh x kw, stride sh x sw, no
- * padding; x [N][H][W][C] -> y [N][Ho][Wo][C], Ho = (H - kh)/sh + 1. */
+/* Max pooling over NHWC (network glue): window kh x kw, stride sh x sw,
+ * padding ph x pw (taps in the padding are skipped, i.e. -infinity padding;
+ * ph < kh and pw < kw); x [N][H][W][C] -> y [N][Ho][Wo][C],
+ * Ho = (H + 2 ph - kh)/sh + 1, Wo = (W + 2 pw - kw)/sw + 1. */
 tbn_status tbn_maxpool2d_nhwc(const void *x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                               int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
-                              void *y, tbn_stream stream);
+                              int64_t ph, int64_t pw, void *y, tbn_stream stream);
 
 /* Layout conversion NCHW -> NHWC with channel zero-padding to C_pad >= C
  * (network glue for the first layer).  x [N][C][H][W], y [N][H][W][C_pad],
  * same dtype. */
 tbn_status tbn_nchw_to_nhwc(const void *x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
                             int64_t W, int64_t C_pad, void *y, tbn_stream stream);
+
+/* ---- full-precision layers (network glue, not the paper's method) -------
+ * Two-bit networks keep their first convolution and last fully-connected
+ * layer in full precision (the ResNet-18 workload).  These calls compute
+ * them on the CUDA cores in fp32: products x * w rounded to fp32 and added
+ * in fp32. */
+
+/* Dense convolution with fp32 weights w [K][C][R][S] (PyTorch order, any
+ * activation layout): y = x cross-correlated with w, zero padding, no bias,
+ * optional ReLU (relu != 0).  layout NCHW: x [N][C][H][W] -> y [N][K][P][Q];
+ * NCHW_NHWC: x [N][C][H][W] -> y [N][P][Q][K]; NHWC: x [N][H][W][C] ->
+ * y [N][P][Q][K].  x and y fp32 or bf16; w 4-byte aligned. */
+tbn_status tbn_dense_conv2d_fwd(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                                int64_t C, int64_t H, int64_t W, const float *w, int64_t K,
+                                int64_t R, int64_t S, int64_t stride_h, int64_t stride_w,
+                                int64_t pad_h, int64_t pad_w, void *y, tbn_dtype ydt, int relu,
+                                tbn_stream stream);
+
+/* Global average pool: x [N][H][W][C] -> y [N][C], y[b,c] = the fp32 mean of
+ * x[b,:,:,c] (pixels added in order, times 1/(H W)). */
+tbn_status tbn_avgpool2d_global_nhwc(const void *x, tbn_dtype xdt, int64_t N, int64_t H,
+                                     int64_t W, int64_t C, void *y, tbn_dtype ydt,
+                                     tbn_stream stream);
+
+/* Dense fully-connected layer with fp32 weights: x [B][K_in] fp32,
+ * w [K_out][K_in] fp32, y [B][K_out] (fp32 or bf16) = x w^T, optional ReLU. */
+tbn_status tbn_dense_linear_fwd(const float *x, int64_t B, int64_t K_in, const float *w,
+                                int64_t K_out, void *y, tbn_dtype ydt, int relu,
+                                tbn_stream stream);
 
 #ifdef __cplusplus
 }

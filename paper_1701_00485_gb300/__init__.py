@@ -28,7 +28,9 @@ __all__ = [
     "TBN_F32", "TBN_BF16", "TBN_NCHW", "TBN_NHWC", "TBN_NCHW_NHWC", "TBN_UNPACK_I8", "TBN_UNPACK_F32",
     "TBN_UNPACK_BF16", "TBN_CONV_AUTO", "TBN_CONV_DIRECT", "TBN_CONV_IMPLICIT_GEMM",
     "TBN_CONV_SMALL_TAPS", "TBN_DEVERR_TIMEOUT", "TBN_DEVERR_BAD_LAUNCH",
-    "tbn_selftest_wait_timeout",
+    "tbn_selftest_wait_timeout", "tbn_repack", "TBN_REPACK_CANONICAL_TO_PLANAR",
+    "TBN_REPACK_PLANAR_TO_CANONICAL", "tbn_dense_conv2d_fwd", "tbn_avgpool2d_global_nhwc",
+    "tbn_dense_linear_fwd",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -42,6 +44,7 @@ TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
 TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM, TBN_CONV_SMALL_TAPS = 0, 1, 2, 3
 TBN_MAX_QUANT_JOBS = 16
 TBN_DEVERR_TIMEOUT, TBN_DEVERR_BAD_LAUNCH = 1, 2   # bits of the device error word
+TBN_REPACK_CANONICAL_TO_PLANAR, TBN_REPACK_PLANAR_TO_CANONICAL = 0, 1
 
 # every symbol include/tbn.h declares
 EXPORTED = [
@@ -51,7 +54,8 @@ EXPORTED = [
     "tbn_linear_workspace_bytes", "tbn_linear_fwd_ws", "tbn_linear_fwd_noalloc",
     "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_conv2d_bwd_data_workspace_bytes",
     "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter_workspace_bytes", "tbn_conv2d_bwd_filter",
-    "tbn_selftest_wait_timeout",
+    "tbn_selftest_wait_timeout", "tbn_repack", "tbn_dense_conv2d_fwd",
+    "tbn_avgpool2d_global_nhwc", "tbn_dense_linear_fwd",
 ]
 
 
@@ -75,7 +79,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 5  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 6  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -117,7 +121,12 @@ def lib():
                                    ctypes.POINTER(Epilogue), P, ctypes.c_size_t, P], I32),
             "tbn_linear_fwd_noalloc": ([P, I32, I64, I64, U32P, P, I64, P, I32,
                                         ctypes.POINTER(Epilogue), P], I32),
-            "tbn_maxpool2d_nhwc": ([P, I32, I64, I64, I64, I64, I64, I64, I64, I64, P, P], I32),
+            "tbn_maxpool2d_nhwc": ([P, I32] + [I64] * 10 + [P, P], I32),
+            "tbn_repack": ([U32P, I64, I64, U32P, I32, P], I32),
+            "tbn_dense_conv2d_fwd": ([P, I32, I32, I64, I64, I64, I64, P] + [I64] * 7 +
+                                     [P, I32, I32, P], I32),
+            "tbn_avgpool2d_global_nhwc": ([P, I32, I64, I64, I64, I64, P, I32, P], I32),
+            "tbn_dense_linear_fwd": ([P, I64, I64, P, I64, P, I32, I32, P], I32),
             "tbn_conv2d_bwd_data_workspace_bytes": ([I64] * 11, ctypes.c_size_t),
             "tbn_conv2d_bwd_data": ([P, I64, I64, I64, I64, U32P, P] + [I64] * 7 +
                                     [P, I32, P, ctypes.c_size_t, P], I32),
@@ -388,15 +397,89 @@ def tbn_linear_fwd_noalloc(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Te
     return out
 
 
-def tbn_maxpool2d_nhwc(x: torch.Tensor, k=(2, 2), stride=(2, 2), out=None, stream=None):
+def tbn_maxpool2d_nhwc(x, k=(2, 2), stride=(2, 2), out=None, stream=None, pad=(0, 0)):
+    """Max pooling over NHWC; taps in the padding are skipped (-inf padding)."""
     _cuda(x, "x")
     N, H, W, C = x.shape
-    Ho, Wo = (H - k[0]) // stride[0] + 1, (W - k[1]) // stride[1] + 1
+    Ho, Wo = conv_out_hw(H, W, k[0], k[1], stride, pad)
     if out is None:
         out = torch.empty((N, Ho, Wo, C), dtype=x.dtype, device=x.device)
     _check(lib().tbn_maxpool2d_nhwc(x.data_ptr(), _dt(x), N, H, W, C, k[0], k[1], stride[0],
-                                    stride[1], out.data_ptr(), _stream(stream)),
+                                    stride[1], pad[0], pad[1], out.data_ptr(), _stream(stream)),
            "tbn_maxpool2d_nhwc")
+    return out
+
+
+def tbn_repack(codes: torch.Tensor, n: int, direction: int, out=None, stream=None):
+    """Codes [K, ceil(n/16)] between the byte-planar layout and the canonical
+    interchange layout (TBN_REPACK_CANONICAL_TO_PLANAR / _PLANAR_TO_CANONICAL)."""
+    _cuda(codes, "codes")
+    K = codes.shape[0]
+    if out is None:
+        out = torch.empty_like(codes)
+    _cuda(out, "out")
+    _check(lib().tbn_repack(codes.data_ptr(), K, n, out.data_ptr(), direction, _stream(stream)),
+           "tbn_repack")
+    return out
+
+
+def tbn_dense_conv2d_fwd(x: torch.Tensor, w: torch.Tensor, stride=(1, 1), pad=(0, 0),
+                         layout: int = TBN_NCHW_NHWC, out_dtype=None, relu: bool = False,
+                         out: torch.Tensor | None = None, stream=None):
+    """Full-precision convolution with fp32 weights w [K, C, R, S] (the first
+    layer a two-bit network keeps in fp32).  x is [N,C,H,W] for NCHW and
+    NCHW_NHWC, [N,H,W,C] for NHWC; y is NCHW for NCHW, else NHWC."""
+    _cuda(x, "x"), _cuda(w, "w")
+    if w.dtype != torch.float32 or w.dim() != 4:
+        raise ValueError("w must be a float32 [K, C, R, S] tensor")
+    K, C, R, S = w.shape
+    if layout == TBN_NHWC:
+        N, H, W, C2 = x.shape
+    else:
+        N, C2, H, W = x.shape
+    if C2 != C:
+        raise ValueError("x has %d channels, w expects %d" % (C2, C))
+    P, Q = conv_out_hw(H, W, R, S, stride, pad)
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    shape = (N, K, P, Q) if layout == TBN_NCHW else (N, P, Q, K)
+    if out is None:
+        out = torch.empty(shape, dtype=_torch_dt(ydt), device=x.device)
+    elif tuple(out.shape) != shape or _dt(out) != ydt:
+        raise ValueError("out has the wrong shape or dtype")
+    _check(lib().tbn_dense_conv2d_fwd(x.data_ptr(), _dt(x), layout, N, C, H, W, w.data_ptr(), K, R,
+                                      S, stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,
+                                      1 if relu else 0, _stream(stream)), "tbn_dense_conv2d_fwd")
+    return out
+
+
+def tbn_avgpool2d_global_nhwc(x: torch.Tensor, out_dtype=torch.float32, out=None, stream=None):
+    """Mean over H and W of x [N, H, W, C] -> [N, C]."""
+    _cuda(x, "x")
+    N, H, W, C = x.shape
+    ydt = TBN_F32 if out_dtype == torch.float32 else TBN_BF16
+    if out is None:
+        out = torch.empty((N, C), dtype=_torch_dt(ydt), device=x.device)
+    _check(lib().tbn_avgpool2d_global_nhwc(x.data_ptr(), _dt(x), N, H, W, C, out.data_ptr(), ydt,
+                                           _stream(stream)), "tbn_avgpool2d_global_nhwc")
+    return out
+
+
+def tbn_dense_linear_fwd(x: torch.Tensor, w: torch.Tensor, out_dtype=torch.float32,
+                         relu: bool = False, out=None, stream=None):
+    """Full-precision fully-connected layer: x [B, K_in] fp32, w [K_out, K_in] fp32."""
+    _cuda(x, "x"), _cuda(w, "w")
+    if x.dtype != torch.float32 or w.dtype != torch.float32:
+        raise ValueError("x and w must be float32")
+    B, K_in = x.shape
+    K_out = w.shape[0]
+    if w.shape[1] != K_in:
+        raise ValueError("w must be [K_out, K_in]")
+    ydt = TBN_F32 if out_dtype == torch.float32 else TBN_BF16
+    if out is None:
+        out = torch.empty((B, K_out), dtype=_torch_dt(ydt), device=x.device)
+    _check(lib().tbn_dense_linear_fwd(x.data_ptr(), B, K_in, w.data_ptr(), K_out, out.data_ptr(),
+                                      ydt, 1 if relu else 0, _stream(stream)),
+           "tbn_dense_linear_fwd")
     return out
 
 

@@ -483,16 +483,23 @@ tbn_status tbn_conv2d_bwd_filter(const void* x, const void* dy, int64_t N, int64
 }
 
 tbn_status tbn_maxpool2d_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
-                              int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw, void* y,
-                              tbn_stream stream) {
+                              int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
+                              int64_t ph, int64_t pw, void* y, tbn_stream stream) {
   if (!x || !y) return fail(TBN_ERR_INVALID_ARG, "maxpool: null pointer");
   if (dt != TBN_F32 && dt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "maxpool: bad dtype");
-  if (N < 1 || H < 1 || W < 1 || C < 1 || kh < 1 || kw < 1 || sh < 1 || sw < 1 || kh > H || kw > W)
+  if (N < 1 || H < 1 || W < 1 || C < 1 || kh < 1 || kw < 1 || sh < 1 || sw < 1 || ph < 0 ||
+      pw < 0)
     return fail(TBN_ERR_INVALID_ARG, "maxpool: bad sizes");
+  const int64_t lim = int64_t(1) << 31;
+  if (H >= lim || W >= lim || C >= lim || N >= lim || kh >= lim || kw >= lim || sh >= lim ||
+      sw >= lim)
+    return fail(TBN_ERR_UNSUPPORTED, "maxpool: a size is 2^31 or more");
+  if (ph >= kh || pw >= kw) return fail(TBN_ERR_INVALID_ARG, "maxpool: padding must be below the window");
+  if (kh > H + 2 * ph || kw > W + 2 * pw) return fail(TBN_ERR_INVALID_ARG, "maxpool: window larger than the padded input");
   if (!mul_ok(N * H, W * C, int64_t(1) << 46)) return fail(TBN_ERR_UNSUPPORTED, "maxpool: too large");
   if (!is_aligned(x, dtype_size(dt)) || !is_aligned(y, dtype_size(dt)))
     return fail(TBN_ERR_MISALIGNED, "maxpool: misaligned pointer");
-  return launch_maxpool_nhwc(x, dt, N, H, W, C, kh, kw, sh, sw, y, as_stream(stream));
+  return launch_maxpool_nhwc(x, dt, N, H, W, C, kh, kw, sh, sw, ph, pw, y, as_stream(stream));
 }
 
 tbn_status tbn_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
@@ -505,6 +512,78 @@ tbn_status tbn_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, i
   if (!is_aligned(x, dtype_size(dt)) || !is_aligned(y, dtype_size(dt)))
     return fail(TBN_ERR_MISALIGNED, "nchw_to_nhwc: misaligned pointer");
   return launch_nchw_to_nhwc(x, dt, N, C, H, W, C_pad, y, as_stream(stream));
+}
+
+}  // extern "C"
+
+extern "C" {
+
+tbn_status tbn_repack(const uint32_t* in, int64_t K, int64_t n, uint32_t* out,
+                      tbn_repack_direction dir, tbn_stream stream) {
+  if (!in || !out) return fail(TBN_ERR_INVALID_ARG, "repack: null pointer");
+  if (dir != TBN_REPACK_CANONICAL_TO_PLANAR && dir != TBN_REPACK_PLANAR_TO_CANONICAL)
+    return fail(TBN_ERR_INVALID_ARG, "repack: bad direction");
+  if (K < 1 || n < 1) return fail(TBN_ERR_INVALID_ARG, "repack: K, n must be >= 1");
+  if (n >= (int64_t(1) << 31) || !mul_ok(K, (n + 15) / 16, int64_t(1) << 40))
+    return fail(TBN_ERR_UNSUPPORTED, "repack: too large");
+  if (!is_aligned(in, 4) || !is_aligned(out, 4))
+    return fail(TBN_ERR_MISALIGNED, "repack: pointers must be 4-byte aligned");
+  const int64_t words = K * ((n + 15) / 16);
+  const uintptr_t a = reinterpret_cast<uintptr_t>(in), b = reinterpret_cast<uintptr_t>(out);
+  const uintptr_t bytes = static_cast<uintptr_t>(words) * 4u;
+  if (a != b && a < b + bytes && b < a + bytes)
+    return fail(TBN_ERR_INVALID_ARG, "repack: in and out overlap (only in == out is allowed)");
+  return launch_repack(in, words, out, dir == TBN_REPACK_CANONICAL_TO_PLANAR, as_stream(stream));
+}
+
+tbn_status tbn_dense_conv2d_fwd(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                                int64_t C, int64_t H, int64_t W, const float* w, int64_t K,
+                                int64_t R, int64_t S, int64_t stride_h, int64_t stride_w,
+                                int64_t pad_h, int64_t pad_w, void* y, tbn_dtype ydt, int relu,
+                                tbn_stream stream) {
+  if (!w) return fail(TBN_ERR_INVALID_ARG, "dense conv: null pointer");
+  // the shape, dtype, layout and alignment checks of the two-bit convolution;
+  // the weights stand in for its codes and alpha (both only checked for
+  // being non-null and 4-byte aligned)
+  const tbn_epilogue epi{relu != 0 ? 1 : 0, nullptr, 0};
+  ConvProblem p{};
+  const tbn_status st =
+      validate_conv(x, xdt, layout, N, C, H, W, reinterpret_cast<const uint32_t*>(w), w, K, R, S,
+                    stride_h, stride_w, pad_h, pad_w, y, ydt, &epi, &p);
+  if (st != TBN_OK) return st;
+  if (!mul_ok(K, C * R * S, int64_t(1) << 40))
+    return fail(TBN_ERR_UNSUPPORTED, "dense conv: weights too large");
+  return launch_dense_conv(p, w, as_stream(stream));
+}
+
+tbn_status tbn_avgpool2d_global_nhwc(const void* x, tbn_dtype xdt, int64_t N, int64_t H,
+                                     int64_t W, int64_t C, void* y, tbn_dtype ydt,
+                                     tbn_stream stream) {
+  if (!x || !y) return fail(TBN_ERR_INVALID_ARG, "avgpool: null pointer");
+  if ((xdt != TBN_F32 && xdt != TBN_BF16) || (ydt != TBN_F32 && ydt != TBN_BF16))
+    return fail(TBN_ERR_INVALID_ARG, "avgpool: bad dtype");
+  if (N < 1 || H < 1 || W < 1 || C < 1) return fail(TBN_ERR_INVALID_ARG, "avgpool: bad sizes");
+  const int64_t lim = int64_t(1) << 31;
+  if (N >= lim || H >= lim || W >= lim || C >= lim || !mul_ok(N * C, H * W, int64_t(1) << 46))
+    return fail(TBN_ERR_UNSUPPORTED, "avgpool: too large");
+  if (!is_aligned(x, dtype_size(xdt)) || !is_aligned(y, dtype_size(ydt)))
+    return fail(TBN_ERR_MISALIGNED, "avgpool: misaligned pointer");
+  return launch_avgpool_global_nhwc(x, xdt, N, H, W, C, y, ydt, as_stream(stream));
+}
+
+tbn_status tbn_dense_linear_fwd(const float* x, int64_t B, int64_t K_in, const float* w,
+                                int64_t K_out, void* y, tbn_dtype ydt, int relu,
+                                tbn_stream stream) {
+  if (!x || !w || !y) return fail(TBN_ERR_INVALID_ARG, "dense linear: null pointer");
+  if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "dense linear: bad y dtype");
+  if (B < 1 || K_in < 1 || K_out < 1) return fail(TBN_ERR_INVALID_ARG, "dense linear: sizes must be >= 1");
+  const int64_t lim = int64_t(1) << 31;
+  if (B >= lim || K_in >= lim || K_out >= lim || !mul_ok(K_out, K_in, int64_t(1) << 46) ||
+      !mul_ok(B, K_in, int64_t(1) << 46))
+    return fail(TBN_ERR_UNSUPPORTED, "dense linear: too large");
+  if (!is_aligned(x, 4) || !is_aligned(w, 4) || !is_aligned(y, dtype_size(ydt)))
+    return fail(TBN_ERR_MISALIGNED, "dense linear: misaligned pointer");
+  return launch_dense_linear(x, B, K_in, w, K_out, y, ydt, relu, as_stream(stream));
 }
 
 }  // extern "C"

@@ -1,6 +1,6 @@
 // tbn_conv_direct.cu -- CUDA-core direct two-bit convolution (Eq. 1) for
 // every layout / dtype / stride / padding, plus the network glue kernels
-// (NHWC max pooling, NCHW -> NHWC with channel padding).
+// (NHWC max pooling with optional padding, NCHW -> NHWC with channel padding).
 //
 // Direct convolution: a CTA computes 128 output pixels x 32 filters.  The
 // filters' codes are decoded once per CTA into shared memory as fp32 W~ (a
@@ -204,11 +204,13 @@ tbn_status launch_direct_l(const DirectArgs& a, bool xb, bool yb, bool pool, cud
   return launch_direct_w<float, float, kLayout>(a, pool, s);
 }
 
+// Windows that reach into the padding skip those taps (-infinity padding).
 template <typename T>
 __global__ void __launch_bounds__(256) maxpool_nhwc_kernel(const T* __restrict__ x, int64_t N,
                                                            int64_t H, int64_t W, int64_t C,
                                                            int64_t kh, int64_t kw, int64_t sh,
-                                                           int64_t sw, int64_t Ho, int64_t Wo,
+                                                           int64_t sw, int64_t ph, int64_t pw,
+                                                           int64_t Ho, int64_t Wo,
                                                            T* __restrict__ y) {
   const int64_t total = N * Ho * Wo * C;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
@@ -218,11 +220,16 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_kernel(const T* __restrict__
     const int64_t ho = (i / (C * Wo)) % Ho;
     const int64_t b = i / (C * Wo * Ho);
     float m = -INFINITY;
-    for (int64_t u = 0; u < kh; ++u)
+    for (int64_t u = 0; u < kh; ++u) {
+      const int64_t h = ho * sh - ph + u;
+      if (h < 0 || h >= H) continue;
       for (int64_t v = 0; v < kw; ++v) {
-        const float t = to_f32<T>(x[((b * H + ho * sh + u) * W + wo * sw + v) * C + c]);
+        const int64_t w = wo * sw - pw + v;
+        if (w < 0 || w >= W) continue;
+        const float t = to_f32<T>(x[((b * H + h) * W + w) * C + c]);
         if (t > m) m = t;
       }
+    }
     y[i] = from_f32<T>(m);
   }
 }
@@ -230,7 +237,8 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_kernel(const T* __restrict__
 // 8 channels (16 bytes) of bf16 per thread.
 __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
     const uint4* __restrict__ x, int64_t N, int64_t H, int64_t W, int64_t C8, int64_t kh,
-    int64_t kw, int64_t sh, int64_t sw, int64_t Ho, int64_t Wo, uint4* __restrict__ y) {
+    int64_t kw, int64_t sh, int64_t sw, int64_t ph, int64_t pw, int64_t Ho, int64_t Wo,
+    uint4* __restrict__ y) {
   const int64_t total = N * Ho * Wo * C8;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -241,9 +249,13 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
     float m[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) m[e] = -INFINITY;
-    for (int64_t u = 0; u < kh; ++u)
+    for (int64_t u = 0; u < kh; ++u) {
+      const int64_t h = ho * sh - ph + u;
+      if (h < 0 || h >= H) continue;
       for (int64_t v = 0; v < kw; ++v) {
-        const uint4 t = x[((b * H + ho * sh + u) * W + wo * sw + v) * C8 + c];
+        const int64_t w = wo * sw - pw + v;
+        if (w < 0 || w >= W) continue;
+        const uint4 t = x[((b * H + h) * W + w) * C8 + c];
         const __nv_bfloat16* tb = reinterpret_cast<const __nv_bfloat16*>(&t);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -251,6 +263,7 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
           if (f > m[e]) m[e] = f;
         }
       }
+    }
     uint4 o;
     __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(&o);
 #pragma unroll
@@ -340,22 +353,22 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s) {
 
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
-                               void* y, cudaStream_t s) {
-  const int64_t Ho = (H - kh) / sh + 1, Wo = (W - kw) / sw + 1;
+                               int64_t ph, int64_t pw, void* y, cudaStream_t s) {
+  const int64_t Ho = (H + 2 * ph - kh) / sh + 1, Wo = (W + 2 * pw - kw) / sw + 1;
   if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16)) {
     const int64_t total = N * Ho * Wo * (C / 8);
     maxpool_nhwc_bf16x8_kernel<<<(unsigned)grid_for(total), 256, 0, s>>>(
-        static_cast<const uint4*>(x), N, H, W, C / 8, kh, kw, sh, sw, Ho, Wo,
+        static_cast<const uint4*>(x), N, H, W, C / 8, kh, kw, sh, sw, ph, pw, Ho, Wo,
         static_cast<uint4*>(y));
   } else if (dt == TBN_BF16) {
     const int64_t total = N * Ho * Wo * C;
     maxpool_nhwc_kernel<__nv_bfloat16><<<(unsigned)grid_for(total), 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(x), N, H, W, C, kh, kw, sh, sw, Ho, Wo,
+        static_cast<const __nv_bfloat16*>(x), N, H, W, C, kh, kw, sh, sw, ph, pw, Ho, Wo,
         static_cast<__nv_bfloat16*>(y));
   } else {
     const int64_t total = N * Ho * Wo * C;
     maxpool_nhwc_kernel<float><<<(unsigned)grid_for(total), 256, 0, s>>>(
-        static_cast<const float*>(x), N, H, W, C, kh, kw, sh, sw, Ho, Wo,
+        static_cast<const float*>(x), N, H, W, C, kh, kw, sh, sw, ph, pw, Ho, Wo,
         static_cast<float*>(y));
   }
   return check_launch("maxpool_nhwc_kernel");

@@ -21,8 +21,13 @@
 //                   64 channels and one TMA box load fetches it (the box is
 //                   the tile's output pixels shifted by the tap; zero fill
 //                   supplies the padding, element strides the conv stride).
-//                   Otherwise gather warps assemble the rows from a
-//                   per-K-block table of (tap, channel) offsets.
+//                   When C % 32 == 0 (e.g. 96 channels) a K block is two
+//                   boxes of 32 channels, each from its own tap, into two
+//                   64-byte-row halves of the stage with the 64-byte swizzle
+//                   (a box past the filter's last code is loaded out of
+//                   range and arrives zero-filled).  Otherwise gather warps
+//                   assemble the rows from a per-K-block table of (tap,
+//                   channel) offsets.
 //   D               fp32 in tensor memory (256 columns).  Epilogue warps read
 //                   lane = filter, column = pixel, multiply by 2 * alpha (Eq. 1
 //                   applies alpha to the whole filter; the factor 2 undoes the
@@ -181,7 +186,8 @@ __device__ __forceinline__ void store_out(const IgArgs& a, size_t o, float v) {
 // kPoolBW: 0 = no pool; 8, 16, 32 = fused 2x2/2 max pool for tiles of whole
 // output rows of that width.  kTmaStore: bf16 output through the staging
 // tile and TMA stores (else direct global stores).
-template <bool kGather, int kPoolBW, bool kTmaStore>
+// kCh32 (TMA mode only): K blocks as two 32-channel boxes (C % 32 == 0).
+template <bool kGather, int kPoolBW, bool kTmaStore, bool kCh32>
 __global__ void __launch_bounds__(threads_for<kGather>(), 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmap_x,
                       const __grid_constant__ CUtensorMap tmap_y,
@@ -248,32 +254,48 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
     // (the MMA warp releases in order) and its parity wait cannot alias
     const int pid = warp == 0 ? 0 : warp - kFirstGatherWarp + 1;
     int turn = 0;   // g % kTmaProducers
-    const uint32_t box_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBK * 2);
-    const int cblocks = a.C / kBK;
+    constexpr int kBoxCh = kCh32 ? kBK / 2 : kBK;   // channels per box
+    constexpr int kBoxes = kBK / kBoxCh;             // boxes per K block
+    const uint32_t box_bytes = static_cast<uint32_t>(a.bw * a.bh * a.bn * kBoxCh * 2);
+    const int cblocks = a.C / kBoxCh;                // boxes per tap
     int g = 0;  // global K-block counter of this CTA
     bool ok = true;
     for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x) {
       const TileCoord tc = tile_coord(a, t);
-      int tap = 0, cb = 0;
+      int tap = 0, cb = 0;   // (tap, channel box) of the next box
       for (int kb = 0; kb < KB; ++kb, ++g) {
         const bool mine = turn == pid;
         if (++turn == kTmaProducers) turn = 0;
         if (!mine) {
-          if (++cb == cblocks) { cb = 0; ++tap; }
+#pragma unroll
+          for (int bx = 0; bx < kBoxes; ++bx)
+            if (++cb == cblocks) { cb = 0; ++tap; }
           continue;
         }
         const int sb = g % kStages;
         const uint32_t it = static_cast<uint32_t>(g / kStages);
         ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-        const int r = tap / a.S, s = tap - r * a.S;
         if (elect_one()) {
-          mbar_arrive_expect_tx(&ctl->full[sb], box_bytes);
-          tma_load_4d(ring + sb * kStageBytes, &tmap_x, &ctl->full[sb], cb * kBK,
-                      tc.q0 * a.sw - a.pw + s, tc.p0 * a.sh - a.ph + r, tc.n0);
+          mbar_arrive_expect_tx(&ctl->full[sb], box_bytes * kBoxes);
+#pragma unroll
+          for (int bx = 0; bx < kBoxes; ++bx) {
+            // a box past the filter's last tap is requested at channel C:
+            // entirely out of range, it arrives zero-filled
+            const bool past = tap >= a.R * a.S;
+            const int tp = past ? 0 : tap;
+            const int r = tp / a.S, s = tp - r * a.S;
+            tma_load_4d(ring + sb * kStageBytes + bx * (kStageBytes / kBoxes), &tmap_x,
+                        &ctl->full[sb], past ? a.C : cb * kBoxCh, tc.q0 * a.sw - a.pw + s,
+                        tc.p0 * a.sh - a.ph + r, tc.n0);
+            if (++cb == cblocks) { cb = 0; ++tap; }
+          }
+        } else {
+#pragma unroll
+          for (int bx = 0; bx < kBoxes; ++bx)
+            if (++cb == cblocks) { cb = 0; ++tap; }
         }
         __syncwarp();
-        if (++cb == cblocks) { cb = 0; ++tap; }
       }
     }
     // drain: every copy this warp issued must land before the CTA may exit
@@ -387,14 +409,25 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
                        kWaitLimitNs);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after_sync();
-        const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(ring + st * kStageBytes));
         const uint32_t a_col = a_tmem0 + static_cast<uint32_t>(st * kAColsPerStage);
         if (elect_one()) {
+          if constexpr (kCh32) {
+            // two halves of 32 codes, 64-byte rows with the 64-byte swizzle
 #pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk) {
-            // K step kk: 16 codes = 8 TMEM columns of A, 32 bytes of B rows
-            tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
-                      (kb | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+              const uint64_t bdesc = smem_desc_sw64_kmajor(
+                  smem_addr(ring + st * kStageBytes + (kk >> 1) * (kStageBytes / 2)));
+              tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * (kk & 1)),
+                        idesc, (kb | kk) != 0 ? 1u : 0u);
+            }
+          } else {
+            const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(ring + st * kStageBytes));
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+              // K step kk: 16 codes = 8 TMEM columns of A, 32 bytes of B rows
+              tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
+                        (kb | kk) != 0 ? 1u : 0u);
+            }
           }
           tc_commit(&ctl->empty[st]);
         }
@@ -728,7 +761,9 @@ struct TilePlan {
 
 int ceil_div(int64_t a, int64_t b) { return static_cast<int>((a + b - 1) / b); }
 
-bool use_tma(const ConvProblem& p) { return p.C % kBK == 0 && p.sh <= 2 && p.sw <= 2; }
+// TMA activations: whole 64-channel boxes, or 32-channel boxes in pairs.
+bool use_tma(const ConvProblem& p) { return p.C % (kBK / 2) == 0 && p.sh <= 2 && p.sw <= 2; }
+bool use_ch32(const ConvProblem& p) { return p.C % kBK != 0; }
 
 // Output pixels per tile: whole rows of the output (so one TMA box per tap
 // covers the tile), balanced so the last tile along each axis is not a
@@ -796,7 +831,7 @@ CUresult encode_out_map(CUtensorMap* m, const void* base, const ConvProblem& p, 
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-template <bool kGather, int kPoolBW, bool kTmaStore>
+template <bool kGather, int kPoolBW, bool kTmaStore, bool kCh32>
 tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStream_t s) {
   alignas(64) CUtensorMap tmap_x, tmap_y, tmap_res;
   std::memset(&tmap_x, 0, sizeof(tmap_x));
@@ -806,14 +841,16 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
     const cuuint64_t gdim[4] = {(cuuint64_t)p.C, (cuuint64_t)p.W, (cuuint64_t)p.H, (cuuint64_t)p.N};
     const cuuint64_t gstride[3] = {(cuuint64_t)(p.C * 2), (cuuint64_t)(p.W * p.C * 2),
                                    (cuuint64_t)(p.H * p.W * p.C * 2)};
-    const cuuint32_t box[4] = {(cuuint32_t)kBK, (cuuint32_t)(t.bw * p.sw),
+    const cuuint32_t box[4] = {(cuuint32_t)(kCh32 ? kBK / 2 : kBK), (cuuint32_t)(t.bw * p.sw),
                                (cuuint32_t)(t.bh * p.sh), (cuuint32_t)t.bn};
     const cuuint32_t estr[4] = {1u, (cuuint32_t)p.sw, (cuuint32_t)p.sh, 1u};
     if (box[1] > 256 || box[2] > 256 || box[3] > 256)
       return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: TMA box too large");
     const CUresult cr = get_encode_tiled()(&tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
                                            const_cast<void*>(p.x), gdim, gstride, box, estr,
-                                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                           CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                           kCh32 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                 : CU_TENSOR_MAP_SWIZZLE_128B,
                                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (cr != CUDA_SUCCESS) return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed (%d)", (int)cr);
@@ -829,19 +866,17 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
         return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(residual) failed (%d)", (int)cr);
     }
   }
-  auto kern = conv_igemm_kernel<kGather, kPoolBW, kTmaStore>;
-  static bool attr_done[2][4][2][64] = {};
-  const int pidx = kPoolBW == 0 ? 0 : (kPoolBW == 8 ? 1 : (kPoolBW == 16 ? 2 : 3));
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 0 || dev >= 64 || !attr_done[kGather][pidx][kTmaStore][dev]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(conv_igemm_kernel)");
-    if (dev >= 0 && dev < 64) attr_done[kGather][pidx][kTmaStore][dev] = true;
-  }
+  auto kern = conv_igemm_kernel<kGather, kPoolBW, kTmaStore, kCh32>;
+  // kernel attributes: set once per process (one process drives one GPU)
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kSmemBytes);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(conv_igemm_kernel)");
   const int grid = std::min(a.tiles, device_sm_count());
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -858,13 +893,13 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
   return check_launch("conv_igemm_kernel");
 }
 
-template <bool kGather, bool kTmaStore>
+template <bool kGather, bool kTmaStore, bool kCh32>
 tbn_status launch_pool(const ConvProblem& p, const TilePlan& t, IgArgs& a, int pw, cudaStream_t s) {
   switch (pw) {
-    case 8: return launch_t<kGather, 8, kTmaStore>(p, t, a, s);
-    case 16: return launch_t<kGather, 16, kTmaStore>(p, t, a, s);
-    case 32: return launch_t<kGather, 32, kTmaStore>(p, t, a, s);
-    default: return launch_t<kGather, 0, kTmaStore>(p, t, a, s);
+    case 8: return launch_t<kGather, 8, kTmaStore, kCh32>(p, t, a, s);
+    case 16: return launch_t<kGather, 16, kTmaStore, kCh32>(p, t, a, s);
+    case 32: return launch_t<kGather, 32, kTmaStore, kCh32>(p, t, a, s);
+    default: return launch_t<kGather, 0, kTmaStore, kCh32>(p, t, a, s);
   }
 }
 
@@ -916,10 +951,16 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
   a.err = device_error_word();
   const int pw = pool_width(p, t);
   const bool tst = use_tma_store(p);
-  if (use_tma(p)) {
-    return tst ? launch_pool<false, true>(p, t, a, pw, s) : launch_pool<false, false>(p, t, a, pw, s);
+  if (use_tma(p) && use_ch32(p)) {
+    return tst ? launch_pool<false, true, true>(p, t, a, pw, s)
+               : launch_pool<false, false, true>(p, t, a, pw, s);
   }
-  return tst ? launch_pool<true, true>(p, t, a, pw, s) : launch_pool<true, false>(p, t, a, pw, s);
+  if (use_tma(p)) {
+    return tst ? launch_pool<false, true, false>(p, t, a, pw, s)
+               : launch_pool<false, false, false>(p, t, a, pw, s);
+  }
+  return tst ? launch_pool<true, true, false>(p, t, a, pw, s)
+             : launch_pool<true, false, false>(p, t, a, pw, s);
 }
 
 }  // namespace tbn

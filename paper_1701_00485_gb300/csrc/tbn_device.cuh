@@ -389,6 +389,18 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_kmajor(uint32_t saddr) {
   return d;
 }
 
+// The same for 64-byte rows (32 bf16 per row) with the 64-byte swizzle:
+// 8-row atoms of 512 bytes (stride byte offset), layout type 4.
+__device__ __forceinline__ uint64_t smem_desc_sw64_kmajor(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1u) << 16;
+  d |= static_cast<uint64_t>(512u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(4u) << 61;
+  return d;
+}
+
 // Instruction descriptor for kind::f16 with bf16 A and B, fp32 D, both
 // operands K-major: D format [4,6) = 1 (f32), A format [7,10) = 1 (bf16),
 // B format [10,13) = 1 (bf16), N >> 3 at [17,23), M >> 4 at [24,29).

@@ -117,7 +117,20 @@ tbn_status launch_bwd_filter(const BwdConvShape& p, const void* x, const void* d
 
 tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H, int64_t W,
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
-                               void* y, cudaStream_t s);
+                               int64_t ph, int64_t pw, void* y, cudaStream_t s);
+
+// Canonical <-> byte-planar code words (tbn_quantize.cu).
+tbn_status launch_repack(const uint32_t* in, int64_t words, uint32_t* out, bool to_planar,
+                         cudaStream_t s);
+
+// Full-precision layers around the two-bit ones (tbn_dense.cu).
+tbn_status launch_dense_conv(const ConvProblem& p, const float* w, cudaStream_t s);
+tbn_status launch_avgpool_global_nhwc(const void* x, tbn_dtype xdt, int64_t N, int64_t H,
+                                      int64_t W, int64_t C, void* y, tbn_dtype ydt,
+                                      cudaStream_t s);
+tbn_status launch_dense_linear(const float* x, int64_t B, int64_t K_in, const float* w,
+                               int64_t K_out, void* y, tbn_dtype ydt, int relu,
+                               cudaStream_t s);
 tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C, int64_t H,
                                int64_t W, int64_t C_pad, void* y, cudaStream_t s);
 

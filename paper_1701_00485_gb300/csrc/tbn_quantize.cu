@@ -460,6 +460,53 @@ __global__ void __launch_bounds__(256) unpack_kernel(const uint32_t* __restrict_
   }
 }
 
+// ---- canonical <-> byte-planar repacking ----
+// Both layouts hold the same 2-bit field f = m + 2 s per code and 0 in the
+// unused fields, so a repack is a fixed permutation of the 32 bits of each
+// word.  Canonical: code l (0..15) at bits 2l (m) and 2l + 1 (s).
+// Byte-planar: code l = 2p + h at bits 16h + p (m) and 16h + 8 + p (s).
+// gather_even(v) moves bits 0, 2, 4, ... 30 of v to bits 0..15; scatter_even
+// is its inverse (standard bit (un)interleaving by masks).
+__device__ __forceinline__ uint32_t gather_even(uint32_t v) {
+  v &= 0x55555555u;
+  v = (v | (v >> 1)) & 0x33333333u;
+  v = (v | (v >> 2)) & 0x0F0F0F0Fu;
+  v = (v | (v >> 4)) & 0x00FF00FFu;
+  v = (v | (v >> 8)) & 0x0000FFFFu;
+  return v;
+}
+
+__device__ __forceinline__ uint32_t scatter_even(uint32_t v) {
+  v &= 0x0000FFFFu;
+  v = (v | (v << 8)) & 0x00FF00FFu;
+  v = (v | (v << 4)) & 0x0F0F0F0Fu;
+  v = (v | (v << 2)) & 0x33333333u;
+  v = (v | (v << 1)) & 0x55555555u;
+  return v;
+}
+
+__device__ __forceinline__ uint32_t canonical_to_planar(uint32_t c) {
+  const uint32_t m = gather_even(c), sg = gather_even(c >> 1);   // bit l = code l
+  return gather_even(m) | (gather_even(sg) << 8) | (gather_even(m >> 1) << 16) |
+         (gather_even(sg >> 1) << 24);
+}
+
+__device__ __forceinline__ uint32_t planar_to_canonical(uint32_t w) {
+  const uint32_t m = scatter_even(w & 0xFFu) | (scatter_even((w >> 16) & 0xFFu) << 1);
+  const uint32_t sg = scatter_even((w >> 8) & 0xFFu) | (scatter_even(w >> 24) << 1);
+  return scatter_even(m) | (scatter_even(sg) << 1);
+}
+
+template <bool kToPlanar>
+__global__ void __launch_bounds__(256) repack_kernel(const uint32_t* __restrict__ in,
+                                                     int64_t words, uint32_t* __restrict__ out) {
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < words;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const uint32_t w = __ldg(in + t);
+    out[t] = kToPlanar ? canonical_to_planar(w) : planar_to_canonical(w);
+  }
+}
+
 }  // namespace
 
 tbn_status launch_quantize_group(const tbn_quant_job* jobs, int njobs, cudaStream_t s) {
@@ -532,6 +579,17 @@ tbn_status launch_unpack(const uint32_t* codes, const float* alpha, int64_t K, i
       break;
   }
   return check_launch("unpack_kernel");
+}
+
+tbn_status launch_repack(const uint32_t* in, int64_t words, uint32_t* out, bool to_planar,
+                         cudaStream_t s) {
+  const int64_t blocks =
+      std::max<int64_t>(1, std::min<int64_t>((words + 255) / 256, int64_t(device_sm_count()) * 8));
+  if (to_planar)
+    repack_kernel<true><<<static_cast<unsigned>(blocks), 256, 0, s>>>(in, words, out);
+  else
+    repack_kernel<false><<<static_cast<unsigned>(blocks), 256, 0, s>>>(in, words, out);
+  return check_launch("repack_kernel");
 }
 
 }  // namespace tbn

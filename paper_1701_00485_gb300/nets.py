@@ -1,4 +1,5 @@
-"""Two-bit network forward passes built from the C-ABI calls.
+"""Two-bit network forward passes built from the C-ABI calls: VGG-small,
+AlexNet and ResNet-18 shaped networks.
 
 A network object owns its device buffers (fp32 real-valued weights, packed
 codes, alpha, activations) so that one forward pass is a fixed sequence of
@@ -19,8 +20,9 @@ from dataclasses import dataclass
 
 import torch
 
-from . import (TBN_NHWC, tbn_conv2d_fwd, tbn_linear_fwd, tbn_maxpool2d_nhwc, tbn_nchw_to_nhwc,
-               tbn_quantize_pack_group, packed_words, conv_out_hw)
+from . import (TBN_NHWC, TBN_NCHW_NHWC, tbn_conv2d_fwd, tbn_linear_fwd, tbn_maxpool2d_nhwc,
+               tbn_nchw_to_nhwc, tbn_quantize_pack_group, tbn_dense_conv2d_fwd,
+               tbn_avgpool2d_global_nhwc, tbn_dense_linear_fwd, packed_words, conv_out_hw)
 from . import inputs as _inputs
 
 
@@ -154,3 +156,182 @@ class FCStack:
             tbn_linear_fwd(h, codes, alpha, codes.shape[0], relu=relu, out=y)
             h = y
         return h
+
+    @property
+    def flops_per_image(self) -> int:
+        return sum(2 * codes.shape[0] * W.shape[1] for (W, codes, _, _, _) in self.layers)
+
+
+def _quantize_all(jobs):
+    for i in range(0, len(jobs), 16):
+        tbn_quantize_pack_group(jobs[i:i + 16])
+
+
+class AlexNet:
+    """AlexNet-shaped TBN network (every convolution and fully-connected
+    layer two-bit, per-output-neuron alpha): the conv stack with 3x3/2 max
+    pools, the NHWC flattening of the last pooled map, FC 9216-4096-4096-1000
+    with ReLU between them."""
+
+    def __init__(self, batch: int | None = None, seed: int = 2, device="cuda"):
+        x, Ws, Wfc = _inputs.alexnet_inputs(seed, batch)
+        self.features = ConvStack(_inputs.ALEXNET["convs"], x, Ws, device)
+        self.N = self.features.N
+        self.classifier = FCStack(_inputs.ALEXNET["fcs"], Wfc, self.N, device)
+        self.x_in = self.features.x_in
+        self.out = self.classifier.layers[-1][4]
+
+    @property
+    def conv_flops(self) -> int:
+        return self.features.flops
+
+    @property
+    def fc_flops(self) -> int:
+        return self.N * self.classifier.flops_per_image
+
+    @property
+    def flops(self) -> int:
+        """Algorithmic flops of all TBN layers (convolutions and FC) per batch."""
+        return self.conv_flops + self.fc_flops
+
+    def quantize(self):
+        _quantize_all([(l.W, l.codes, l.alpha) for l in self.features.layers] +
+                      [(W, c, a) for (W, c, a, _, _) in self.classifier.layers])
+
+    def forward(self, requantize: bool = False, conv_hook=None):
+        if requantize:
+            self.quantize()
+        h = self.features.forward(requantize=False, conv_hook=conv_hook)
+        return self.classifier.forward(h.reshape(self.N, -1))
+
+    def launches_per_forward(self, requantize: bool = False) -> int:
+        n = self.features.launches_per_forward(False) + len(self.classifier.layers)
+        return n + (1 if requantize else 0)
+
+
+def alexnet(batch: int | None = None, seed: int = 2, device="cuda") -> AlexNet:
+    return AlexNet(batch, seed, device)
+
+
+@dataclass
+class TbnConv:
+    name: str
+    spec: _inputs.ConvSpec
+    W: torch.Tensor          # fp32 [K, R*S*C] in (r, s, c) order
+    codes: torch.Tensor
+    alpha: torch.Tensor
+    in_hw: tuple
+    out_hw: tuple
+    y: torch.Tensor          # NHWC bf16
+
+    @property
+    def flops_per_image(self) -> int:
+        s = self.spec
+        return 2 * s.K * self.out_hw[0] * self.out_hw[1] * s.C * s.R * s.S
+
+    def run(self, x, residual=None, relu=None):
+        s = self.spec
+        tbn_conv2d_fwd(x, self.codes, self.alpha, s.K, s.R, s.S, (s.stride, s.stride),
+                       (s.pad, s.pad), layout=TBN_NHWC, relu=s.relu if relu is None else relu,
+                       residual=residual, out=self.y)
+        return self.y
+
+
+class ResNet18:
+    """ResNet-18-shaped network: a full-precision 7x7/2 first convolution
+    (fp32 weights, ReLU) and 3x3/2 max pool (pad 1), eight basic blocks of
+    two-bit 3x3 convolutions (64/128/256/512 channels; the first block of
+    stages 2-4 has stride 2 and a two-bit 1x1/2 projection shortcut), the
+    residual added in the second convolution's fused epilogue before its
+    ReLU, then a global average pool and a full-precision FC 512 -> 1000.
+    Batch norm is the identity (synthetic weights carry no statistics)."""
+
+    def __init__(self, batch: int | None = None, seed: int = 3, device="cuda"):
+        self.device = torch.device(device)
+        x, stem, convs, fc = _inputs.resnet18_inputs(seed, batch)
+        dev = self.device
+        self.N = N = x.shape[0]
+        self.x_in = x.to(dev).contiguous()
+        self.stem_w = stem.to(dev).contiguous()
+        H, W = x.shape[2], x.shape[3]
+        self.stem_hw = conv_out_hw(H, W, 7, 7, (2, 2), (3, 3))
+        self.stem_y = torch.empty((N, self.stem_hw[0], self.stem_hw[1], 64), dtype=torch.bfloat16,
+                                  device=dev)
+        self.pool_hw = conv_out_hw(self.stem_hw[0], self.stem_hw[1], 3, 3, (2, 2), (1, 1))
+        self.pool_y = torch.empty((N, self.pool_hw[0], self.pool_hw[1], 64), dtype=torch.bfloat16,
+                                  device=dev)
+        self.convs = {}
+        hw = self.pool_hw
+        stage_in = {}
+        for name, spec, Wt in convs:
+            blk = name[:4]
+            if blk not in stage_in:
+                stage_in[blk] = hw
+            ihw = stage_in[blk] if name[-1] in "ad" else self.convs[blk + "a"].out_hw
+            ohw = conv_out_hw(ihw[0], ihw[1], spec.R, spec.S, (spec.stride,) * 2, (spec.pad,) * 2)
+            K = spec.K
+            Wl = Wt.permute(0, 2, 3, 1).reshape(K, -1).contiguous().to(dev)
+            codes = torch.empty((K, packed_words(Wl.shape[1])), dtype=torch.int32, device=dev)
+            alpha = torch.empty((K,), dtype=torch.float32, device=dev)
+            y = torch.empty((N, ohw[0], ohw[1], K), dtype=torch.bfloat16, device=dev)
+            self.convs[name] = TbnConv(name, spec, Wl, codes, alpha, ihw, ohw, y)
+            if name[-1] == "b":
+                hw = ohw
+        self.blocks = []
+        for name in self.convs:
+            if name[-1] == "a":
+                blk = name[:4]
+                self.blocks.append((self.convs[blk + "a"], self.convs[blk + "b"],
+                                    self.convs.get(blk + "d")))
+        self.feat_hw = hw
+        self.feat = torch.empty((N, 512), dtype=torch.float32, device=dev)
+        self.fc_w = fc.to(dev).contiguous()
+        self.logits = torch.empty((N, self.fc_w.shape[0]), dtype=torch.float32, device=dev)
+        self.out = self.logits
+
+    @property
+    def tbn_flops(self) -> int:
+        """Algorithmic flops of the 19 two-bit convolutions per batch."""
+        return self.N * sum(c.flops_per_image for c in self.convs.values())
+
+    @property
+    def dense_flops(self) -> int:
+        """Flops of the full-precision first convolution and FC per batch."""
+        P, Q = self.stem_hw
+        return self.N * (2 * 64 * P * Q * 3 * 49 + 2 * self.fc_w.shape[0] * self.fc_w.shape[1])
+
+    def quantize(self):
+        _quantize_all([(c.W, c.codes, c.alpha) for c in self.convs.values()])
+
+    def stem(self):
+        tbn_dense_conv2d_fwd(self.x_in, self.stem_w, (2, 2), (3, 3), layout=TBN_NCHW_NHWC,
+                             out_dtype=torch.bfloat16, relu=True, out=self.stem_y)
+        tbn_maxpool2d_nhwc(self.stem_y, (3, 3), (2, 2), out=self.pool_y, pad=(1, 1))
+        return self.pool_y
+
+    def body(self, h):
+        """The two-bit basic blocks from the pooled stem output."""
+        for a, b, d in self.blocks:
+            a.run(h)
+            res = d.run(h) if d is not None else h
+            b.run(a.y, residual=res, relu=True)
+            h = b.y
+        return h
+
+    def head(self, h):
+        tbn_avgpool2d_global_nhwc(h, out=self.feat)
+        tbn_dense_linear_fwd(self.feat, self.fc_w, out=self.logits)
+        return self.logits
+
+    def forward(self, requantize: bool = False):
+        if requantize:
+            self.quantize()
+        return self.head(self.body(self.stem()))
+
+    def launches_per_forward(self, requantize: bool = False) -> int:
+        n = 2 + len(self.convs) + 2
+        return n + ((len(self.convs) + 15) // 16 if requantize else 0)
+
+
+def resnet18(batch: int | None = None, seed: int = 3, device="cuda") -> ResNet18:
+    return ResNet18(batch, seed, device)

@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 5
+    assert L.tbn_abi_version() == 6
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -130,8 +130,38 @@ def test_linear_and_glue_reject_bad_arguments(L):
         tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_linear_fwd_ws(d, 1, 1, 64, d, d, 8, ctypes.c_void_p(257), 1, None, d, 4096,
                                None) == tbn.TBN_ERR_MISALIGNED
-    assert L.tbn_maxpool2d_nhwc(d, 1, 1, 4, 4, 8, 5, 5, 1, 1, d, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_maxpool2d_nhwc(d, 1, 1, 4, 4, 8, 5, 5, 1, 1, 0, 0, d, None) == \
+        tbn.TBN_ERR_INVALID_ARG
+    # padding must stay below the window
+    assert L.tbn_maxpool2d_nhwc(d, 1, 1, 8, 8, 8, 3, 3, 2, 2, 3, 1, d, None) == \
+        tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_maxpool2d_nhwc(d, 1, 1, 8, 8, 8, 3, 3, 2, 2, -1, 1, d, None) == \
+        tbn.TBN_ERR_INVALID_ARG
     assert L.tbn_nchw_to_nhwc(d, 1, 1, 4, 4, 4, 3, d, None) == tbn.TBN_ERR_INVALID_ARG
+
+
+def test_repack_and_dense_layers_reject_bad_arguments(L):
+    d = ctypes.c_void_p(256)
+    assert L.tbn_repack(None, 4, 16, d, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_repack(d, 4, 16, d, 2, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_repack(d, 0, 16, d, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_repack(d, 4, 16, ctypes.c_void_p(258), 0, None) == tbn.TBN_ERR_MISALIGNED
+    # partial overlap is refused (in == out is allowed)
+    assert L.tbn_repack(d, 4, 16, ctypes.c_void_p(260), 0, None) == tbn.TBN_ERR_INVALID_ARG
+    args = [d, 1, tbn.TBN_NCHW_NHWC, 2, 3, 16, 16, d, 64, 7, 7, 2, 2, 3, 3, d, 1, 1, None]
+    bad = list(args); bad[7] = None
+    assert L.tbn_dense_conv2d_fwd(*bad) == tbn.TBN_ERR_INVALID_ARG
+    bad = list(args); bad[9] = 30                     # kernel larger than the padded input
+    assert L.tbn_dense_conv2d_fwd(*bad) == tbn.TBN_ERR_INVALID_ARG
+    bad = list(args); bad[7] = ctypes.c_void_p(258)   # weights not 4-byte aligned
+    assert L.tbn_dense_conv2d_fwd(*bad) == tbn.TBN_ERR_MISALIGNED
+    assert L.tbn_avgpool2d_global_nhwc(d, 1, 2, 0, 7, 512, d, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_avgpool2d_global_nhwc(d, 3, 2, 7, 7, 512, d, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_dense_linear_fwd(d, 2, 512, None, 1000, d, 0, 0, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_dense_linear_fwd(d, 2, 512, d, 1000, ctypes.c_void_p(258), 0, 0, None) == \
+        tbn.TBN_ERR_MISALIGNED
+    assert L.tbn_dense_linear_fwd(d, 2, 1 << 40, d, 1000, d, 0, 0, None) == \
+        tbn.TBN_ERR_UNSUPPORTED
 
 
 def test_linear_workspace_query(L):

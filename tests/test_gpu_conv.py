@@ -2,6 +2,8 @@
 against the oracle's seven-loop convolution, per output:
 |y_gpu - y_orc| <= 2e-3 * |alpha| * sum|x| (fp32 output), plus the bf16
 output rounding for bf16 output."""
+import zlib
+
 import numpy as np
 import pytest
 import torch
@@ -59,7 +61,7 @@ def test_lenet_layer_full():
 
 # ---------------------------------------------------------------- implicit GEMM
 IGEMM = [
-    # N, C, H, W, K, R, S, stride, pad    (all NHWC bf16, C % 64 == 0)
+    # N, C, H, W, K, R, S, stride, pad    (all NHWC bf16, C % 32 == 0, stride <= 2)
     (1, 64, 8, 8, 128, 3, 3, (1, 1), (1, 1)),       # one tile, exact
     (2, 64, 8, 8, 128, 1, 1, (1, 1), (0, 0)),       # 1x1
     (3, 128, 16, 16, 256, 3, 3, (1, 1), (1, 1)),    # two filter tiles
@@ -73,6 +75,12 @@ IGEMM = [
     (1, 192, 6, 5, 136, 2, 3, (1, 1), (1, 0)),      # R != S, asymmetric pad
     (1, 64, 300, 4, 128, 3, 3, (1, 1), (1, 1)),     # Q < P, tall image
     (1, 64, 3, 300, 128, 3, 3, (1, 1), (1, 1)),     # Q > 256: several q tiles
+    # C % 32 == 0, not % 64: two 32-channel boxes per K block (64-byte swizzle)
+    (2, 96, 13, 13, 128, 5, 5, (1, 1), (2, 2)),     # AlexNet conv2 taps, n % 64 == 32
+    (2, 32, 9, 9, 64, 3, 3, (1, 1), (1, 1)),        # one box per tap, ragged last block
+    (2, 160, 8, 8, 128, 1, 1, (1, 1), (0, 0)),      # 1x1, n = 160
+    (2, 96, 14, 14, 128, 3, 3, (2, 2), (1, 1)),     # stride 2
+    (1, 96, 27, 27, 256, 5, 5, (1, 1), (2, 2)),     # AlexNet conv2 image, two filter tiles
 ]
 
 
@@ -87,11 +95,11 @@ def test_igemm_conv_matches_oracle_fp32_out(case):
 
 
 GATHER = [
-    # C % 64 != 0 (activations gathered by threads) or stride > 2
+    # C % 32 != 0 (activations gathered by threads) or stride > 2
     (2, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)),      # VGG first layer shape (C=3)
     (1, 1, 28, 28, 20, 5, 5, (1, 1), (0, 0)),       # C=1
     (1, 3, 35, 35, 96, 11, 11, (4, 4), (0, 0)),     # AlexNet conv1 geometry
-    (2, 96, 13, 13, 128, 5, 5, (1, 1), (2, 2)),     # C % 8 == 0, not % 64 (vector gather)
+    (2, 40, 13, 13, 128, 5, 5, (1, 1), (2, 2)),     # C % 8 == 0, not % 32 (vector gather)
     (2, 5, 9, 7, 70, 3, 3, (1, 1), (1, 1)),         # odd C, ragged K
     (1, 16, 12, 12, 64, 3, 3, (2, 2), (1, 1)),      # stride 2 gathered
     (1, 64, 20, 20, 128, 3, 3, (3, 3), (1, 1)),     # C % 64 == 0 but stride 3
@@ -219,6 +227,7 @@ POOL = [
     (3, 128, 16, 16, 200, 3, 3, (1, 1), (1, 1)),    # 16-wide rows, ragged K
     (2, 3, 32, 32, 128, 3, 3, (1, 1), (1, 1)),      # gathered activations
     (5, 64, 9, 8, 64, 3, 3, (1, 1), (1, 1)),        # odd P (floor), images per tile
+    (2, 96, 16, 16, 128, 3, 3, (1, 1), (1, 1)),     # 32-channel boxes
 ]
 POOL_OTHER = [
     (1, 64, 13, 11, 72, 3, 3, (1, 1), (1, 1)),      # odd P, Q: direct kernel
@@ -344,7 +353,7 @@ def test_workload_layer_sampled(name, N, spec, hw):
     """Each conv layer of the VGG-small / AlexNet / ResNet-18 workloads at its
     full batch and size, in the launch configuration the networks use
     (NHWC bf16 in, bf16 out, AUTO algorithm), checked at sampled outputs."""
-    g = inputs.generator(hash(name) % 100000)
+    g = inputs.generator(zlib.crc32(name.encode()) % 100000)
     x = torch.randn(N, spec.C, hw, hw, generator=g).to(torch.bfloat16)
     W = inputs.he_normal(spec.K, spec.C, spec.R, spec.S, g)
     c = ConvCase(x, W, (spec.stride, spec.stride), (spec.pad, spec.pad))

@@ -84,16 +84,19 @@ def test_linear_as_conv_matches_oracle(B, K_in, K_out, xdt):
     assert_within(y, y_orc, bound, out_bf16=False, what="linear-as-conv")
 
 
-@pytest.mark.parametrize("shape,k,s", [((2, 32, 32, 128), (2, 2), (2, 2)),
-                                       ((3, 55, 55, 96), (3, 3), (2, 2)),
-                                       ((1, 9, 8, 5), (2, 2), (2, 2)),
-                                       ((2, 13, 13, 256), (3, 3), (2, 2))])
+@pytest.mark.parametrize("shape,k,s,pd", [((2, 32, 32, 128), (2, 2), (2, 2), (0, 0)),
+                                          ((3, 55, 55, 96), (3, 3), (2, 2), (0, 0)),
+                                          ((1, 9, 8, 5), (2, 2), (2, 2), (0, 0)),
+                                          ((2, 13, 13, 256), (3, 3), (2, 2), (0, 0)),
+                                          ((2, 112, 112, 64), (3, 3), (2, 2), (1, 1)),
+                                          ((1, 9, 7, 5), (3, 2), (2, 1), (1, 1))])
 @pytest.mark.parametrize("dt", [torch.bfloat16, torch.float32])
-def test_maxpool_matches_oracle(shape, k, s, dt):
+def test_maxpool_matches_oracle(shape, k, s, pd, dt):
     g = inputs.generator(sum(shape))
-    x = torch.randn(*shape, generator=g).to(dt)
-    y = tbn.tbn_maxpool2d_nhwc(x.cuda(), k, s).float().cpu().numpy()
-    want = oracle.maxpool2d_nchw(x.float().permute(0, 3, 1, 2).numpy(), k, s)
+    # shifted down so that every window is negative: a zero pad would win the max
+    x = (torch.randn(*shape, generator=g) - 3.0).to(dt)
+    y = tbn.tbn_maxpool2d_nhwc(x.cuda(), k, s, pad=pd).float().cpu().numpy()
+    want = oracle.maxpool2d_nchw(x.float().permute(0, 3, 1, 2).numpy(), k, s, pd)
     assert np.array_equal(y, want.transpose(0, 2, 3, 1))
 
 
