@@ -92,6 +92,7 @@ constexpr int kTmemCols = 512;      // accumulator [0,256) + weight ring [256,41
 constexpr int kExpWarps = 8;
 constexpr int kEpiWarps = 8;
 constexpr int kGatherWarps = 4;
+constexpr int kPatchWarps = 8;      // patch mode: one operand row per thread
 constexpr int kTmaProducers = 2;    // TMA mode: warp 0 and warps 18 .. 18 + kTmaProducers - 2
 static_assert(kTmaProducers <= kStages, "a producer's parity wait needs kStages >= producers");
 constexpr int kFirstExpWarp = 2;
@@ -103,9 +104,26 @@ constexpr uint64_t kWaitLimitNs = 1000000000ull;    // 1 s
 
 static_assert(kAccCols + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
-template <bool kGather>
+// How the activation operand reaches the stage ring.
+constexpr int kModeTma64 = 0;   // one 64-channel TMA box per K block (C % 64 == 0)
+constexpr int kModeTma32 = 1;   // two 32-channel TMA boxes per K block (C % 32 == 0)
+constexpr int kModeGather = 2;  // threads gather each code's activation from global memory
+constexpr int kModePatch = 3;   // the tile's input rows are staged in shared memory (bulk
+                                // copy, double-buffered) and threads build the rows from there
+
+__host__ __device__ constexpr bool mode_gathers(int mode) { return mode >= kModeGather; }
+// the patch buffers take the room of two ring stages
+__host__ __device__ constexpr int stages_for(int mode) { return mode == kModePatch ? kStages - 2 : kStages; }
+
+// Producer warps of a mode (warps kFirstGatherWarp.. in the gathering modes).
+__host__ __device__ constexpr int producer_warps(int mode) {
+  return mode == kModePatch ? kPatchWarps : (mode == kModeGather ? kGatherWarps : 0);
+}
+
+template <int kMode>
 constexpr int threads_for() {
-  return 32 * (kFirstGatherWarp + (kGather ? kGatherWarps : kTmaProducers - 1));
+  return 32 * (kFirstGatherWarp +
+               (mode_gathers(kMode) ? producer_warps(kMode) : kTmaProducers - 1));
 }
 
 struct IgArgs {
@@ -123,6 +141,11 @@ struct IgArgs {
   const void* residual;
   int relu, y_bf16;
   uint32_t* err;
+  // patch mode: the patch is rows [p0 sh - ph, + PR) x columns [-pw, W + pw)
+  int PR, PW;              // patch rows, patch columns (W + 2 pw)
+  int patch_cap;           // bytes per patch buffer (multiple of 16)
+  int patch_bulk;          // pw == 0: in-image rows are one contiguous range of x
+  long long x_bytes;       // size of x (bulk copies never read past it)
 };
 
 struct SmemCtl {
@@ -139,17 +162,31 @@ struct SmemCtl {
   int abort;
   int gtab_off[2][kBK];    // gather: element offset of each code of the K block
   int gtab_rs[2][kBK];     // gather: (r << 16 | s), or -1 beyond the filter
+  uint64_t patch_full[2];  // patch mode: a buffer's bulk copy has landed
 };
 
-constexpr size_t kSmemBytes =
-    1024 /*align slack*/ + kStages * kStageBytes + kOutStageBytes + sizeof(SmemCtl);
-static_assert(kSmemBytes <= 232448, "shared memory budget");
+constexpr int kSmemLimit = 232448;
+constexpr int kPatchMaxKBlocks = 16;   // patch mode keeps a table of every K block's codes
+
+// Dynamic shared memory of a mode: ring, output staging, control block; in
+// patch mode also two patch buffers and the code-offset table.
+constexpr size_t smem_bytes_for(int mode, size_t patch_cap, int kblocks) {
+  return 1024 /*align slack*/ + stages_for(mode) * kStageBytes + kOutStageBytes +
+         ((sizeof(SmemCtl) + 15) / 16) * 16 +
+         (mode == kModePatch ? 2 * patch_cap + static_cast<size_t>(kblocks) * kBK * 4 : 0);
+}
+static_assert(smem_bytes_for(kModeTma64, 0, 0) <= kSmemLimit, "shared memory budget");
 
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint4 v) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
                "r"(v.z), "r"(v.w)
                : "memory");
+}
+
+// 16-bit shared-memory store by 32-bit shared address.
+__device__ __forceinline__ void st_shared_u16(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared.u16 [%0], %1;" ::"r"(addr), "h"(static_cast<uint16_t>(v)) : "memory");
 }
 
 struct TileCoord {
@@ -186,19 +223,27 @@ __device__ __forceinline__ void store_out(const IgArgs& a, size_t o, float v) {
 // kPoolBW: 0 = no pool; 8, 16, 32 = fused 2x2/2 max pool for tiles of whole
 // output rows of that width.  kTmaStore: bf16 output through the staging
 // tile and TMA stores (else direct global stores).
-// kCh32 (TMA mode only): K blocks as two 32-channel boxes (C % 32 == 0).
-template <bool kGather, int kPoolBW, bool kTmaStore, bool kCh32>
-__global__ void __launch_bounds__(threads_for<kGather>(), 1)
+// kMode: how activations reach the ring (kModeTma64 / kModeTma32 /
+// kModeGather / kModePatch).
+template <int kMode, int kPoolBW, bool kTmaStore>
+__global__ void __launch_bounds__(threads_for<kMode>(), 1)
     conv_igemm_kernel(const __grid_constant__ CUtensorMap tmap_x,
                       const __grid_constant__ CUtensorMap tmap_y,
                       const __grid_constant__ CUtensorMap tmap_res,
                       const __grid_constant__ IgArgs a) {
+  constexpr bool kGather = mode_gathers(kMode);
+  constexpr bool kCh32 = kMode == kModeTma32;
+  constexpr bool kPatch = kMode == kModePatch;
+  constexpr int kSt = stages_for(kMode);   // ring stages
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
-  uint8_t* ring = smem;                                   // kStages x 32 KiB
-  uint8_t* out_stage = smem + kStages * kStageBytes;      // 64 KiB
+  // 1024-byte aligned by pointer arithmetic on the shared array, so that the
+  // compiler keeps every access derived from it in the shared state space
+  uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+  uint8_t* ring = smem;                                   // kSt x 32 KiB
+  uint8_t* out_stage = smem + kSt * kStageBytes;          // 64 KiB
   SmemCtl* ctl = reinterpret_cast<SmemCtl*>(out_stage + kOutStageBytes);
+  // patch mode: two patch buffers, then the code-offset table
+  uint8_t* patch_buf = reinterpret_cast<uint8_t*>(ctl) + ((sizeof(SmemCtl) + 15) / 16) * 16;
   volatile int* abort_flag = &ctl->abort;
 
   const int warp = threadIdx.x >> 5;
@@ -206,10 +251,12 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
   const int KB = a.kblocks;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) {
-      mbar_init(&ctl->full[i], 32 * kExpWarps + (kGather ? 32 * kGatherWarps : 1));
+    for (int i = 0; i < kSt; ++i) {
+      mbar_init(&ctl->full[i], 32 * kExpWarps + (kGather ? 32 * producer_warps(kMode) : 1));
       mbar_init(&ctl->empty[i], 1);
     }
+    mbar_init(&ctl->patch_full[0], 1);
+    mbar_init(&ctl->patch_full[1], 1);
     mbar_init(&ctl->acc_full, 1);
     mbar_init(&ctl->acc_empty, 32 * kEpiWarps);
     mbar_init(&ctl->res_full, 1);
@@ -272,8 +319,8 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
             if (++cb == cblocks) { cb = 0; ++tap; }
           continue;
         }
-        const int sb = g % kStages;
-        const uint32_t it = static_cast<uint32_t>(g / kStages);
+        const int sb = g % kSt;
+        const uint32_t it = static_cast<uint32_t>(g / kSt);
         ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         if (elect_one()) {
@@ -299,11 +346,11 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       }
     }
     // drain: every copy this warp issued must land before the CTA may exit
-    for (int i = g > kStages ? g - kStages : 0; i < g; ++i)
+    for (int i = g > kSt ? g - kSt : 0; i < g; ++i)
       if (i % kTmaProducers == pid)
-        mbar_wait(&ctl->full[i % kStages], static_cast<uint32_t>(i / kStages) & 1u, nullptr,
+        mbar_wait(&ctl->full[i % kSt], static_cast<uint32_t>(i / kSt) & 1u, nullptr,
                   a.err, kWaitLimitNs);
-  } else if (kGather && warp >= kFirstGatherWarp) {
+  } else if (kMode == kModeGather && warp >= kFirstGatherWarp) {
     // ================= gather producers =================
     // The gather warps meet at a named barrier every K block, so none of them
     // may leave the loops early: after a failed wait a warp keeps walking the
@@ -347,8 +394,8 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
           }
         }
         named_barrier_sync(2, 32 * kGatherWarps);
-        const int sb = g % kStages;
-        const uint32_t it = static_cast<uint32_t>(g / kStages);
+        const int sb = g % kSt;
+        const uint32_t it = static_cast<uint32_t>(g / kSt);
         if (ok) ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) continue;
@@ -392,6 +439,221 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
         mbar_arrive(&ctl->full[sb]);
       }
     }
+  } else if (kPatch && warp >= kFirstGatherWarp) {
+    // ================= patch producers =================
+    // Tiles are whole output rows of one image (bn = 1, tiles_q = 1).  The
+    // input rows a tile reads, [p0 sh - ph, + PR) x [-pw, W + pw) x C, are
+    // staged in a shared-memory patch (zero outside the image); each K block
+    // row is then built from the patch with one 32-bit load per pair of codes
+    // when the pair is contiguous there, two 16-bit loads otherwise.  With no
+    // column padding the in-image rows are one contiguous range of x and one
+    // bulk copy (issued a tile ahead, into the other buffer) fetches them.
+    const int gt = threadIdx.x - 32 * kFirstGatherWarp;   // 0..255
+    const int pitch = a.PW * a.C;                          // patch row, elements
+    const int patch_elems = a.PR * pitch;
+    const int* ptab = reinterpret_cast<const int*>(patch_buf + 2 * a.patch_cap);
+    int* ptab_w = reinterpret_cast<int*>(patch_buf + 2 * a.patch_cap);
+    const uint8_t* xb = reinterpret_cast<const uint8_t*>(a.x);
+    // offset table of every K block: patch element of code k relative to the
+    // pixel's (tap 0, channel 0) element, -1 past the filter
+    for (int i = gt; i < KB * kBK; i += 32 * kPatchWarps) {
+      const int k = i;
+      int off = -1;
+      if (k < a.ncodes) {
+        const int c = k % a.C, tap = k / a.C;
+        const int r = tap / a.S, s = tap - r * a.S;
+        off = (r * a.PW + s) * a.C + c;
+      }
+      asm volatile("st.shared.s32 [%0], %1;" ::"r"(smem_addr(ptab_w + i)), "r"(off) : "memory");
+    }
+    grid_dependency_wait();   // activations may come from the previous kernel
+    grid_dependents_launch();
+    named_barrier_sync(2, 32 * kPatchWarps);
+
+    // geometry of tile t's patch: in-image patch rows [lo, hi), the byte
+    // offset `src` in x of its first in-image element, and the byte offset of
+    // patch element 0 in its buffer (chosen so that the bulk copy's
+    // destination is 16-byte aligned)
+    auto geom = [&](int t, int& lo, int& hi, long long& src, uint32_t& off0) {
+      const TileCoord tc = tile_coord(a, t);
+      const int h0 = tc.p0 * a.sh - a.ph;
+      lo = max(0, -h0);
+      hi = min(a.PR, a.H - h0);
+      if (hi < lo) hi = lo;
+      const long long e0 = static_cast<long long>(lo) * pitch;
+      src = ((static_cast<long long>(tc.n0) * a.H + h0 + lo) * a.W) * a.C * 2;
+      off0 = static_cast<uint32_t>(((src & 15) - 2 * e0) & 15);
+    };
+    // one thread: the bulk copy of tile t's in-image rows into buffer b
+    auto issue = [&](int t, int b) {
+      int lo, hi;
+      long long src;
+      uint32_t off0;
+      geom(t, lo, hi, src, off0);
+      const long long len = static_cast<long long>(hi - lo) * pitch * 2;
+      const long long a0 = src & ~15LL;
+      long long a1 = (src + len + 15) & ~15LL;
+      if (a1 > a.x_bytes) a1 = a.x_bytes & ~15LL;   // the rest is copied by threads
+      const uint32_t bytes = a1 > a0 ? static_cast<uint32_t>(a1 - a0) : 0u;
+      uint8_t* dst = patch_buf + b * a.patch_cap + off0 + 2 * static_cast<long long>(lo) * pitch -
+                     (src & 15);
+      fence_proxy_async_smem();   // earlier generic accesses of the buffer come first
+      mbar_arrive_expect_tx(&ctl->patch_full[b], bytes);
+      if (bytes) bulk_load_1d(dst, xb + a0, bytes, &ctl->patch_full[b]);
+    };
+
+    int g = 0;
+    bool ok = true;
+    uint32_t issued[2] = {0u, 0u};   // bulk copies issued into each buffer (thread 0)
+    uint32_t landed[2] = {0u, 0u};   // copies this thread has seen complete
+    uint32_t tiles_done = 0;
+    if (a.patch_bulk && gt == 0 && static_cast<int>(blockIdx.x) < a.tiles) {
+      issue(blockIdx.x, 0);
+      ++issued[0];
+    }
+    __syncwarp();   // reconverge before the aligned named barriers below
+    const int T = a.bw * a.bh;
+    for (int t = blockIdx.x; t < a.tiles; t += gridDim.x, ++tiles_done) {
+      const int b = tiles_done & 1;
+      uint8_t* buf = patch_buf + b * a.patch_cap;
+      int lo, hi;
+      long long src;
+      uint32_t off0;
+      geom(t, lo, hi, src, off0);
+      const uint32_t buf_s = smem_addr(buf);
+      const uint32_t pe_s = buf_s + off0;   // patch element e at pe_s + 2 e
+      // everyone has finished building the previous tile (the buffer filled
+      // next was last read two tiles ago)
+      named_barrier_sync(2, 32 * kPatchWarps);
+      if (a.patch_bulk) {
+        if (gt == 0 && ok && t + static_cast<int>(gridDim.x) < a.tiles) {
+          issue(t + gridDim.x, b ^ 1);
+          ++issued[b ^ 1];
+        }
+        if (ok) {
+          ok = mbar_wait(&ctl->patch_full[b], landed[b] & 1u, abort_flag, a.err, kWaitLimitNs);
+          if (ok) ++landed[b];
+        }
+        ok = __all_sync(0xffffffffu, ok);
+        // rows outside the image are zero; the copy's rounding may have
+        // written neighbouring bytes there
+        for (int e = gt; e < lo * pitch; e += 32 * kPatchWarps) st_shared_u16(pe_s + 2 * e, 0u);
+        for (int e = hi * pitch + gt; e < patch_elems; e += 32 * kPatchWarps)
+          st_shared_u16(pe_s + 2 * e, 0u);
+        // the last bytes of x that no 16-byte chunk of the copy covered
+        const long long len = static_cast<long long>(hi - lo) * pitch * 2;
+        const long long cov = a.x_bytes & ~15LL;
+        if (src + len > cov) {
+          const long long first = max(src, cov);
+          for (long long bpos = first + 2 * gt; bpos < src + len; bpos += 2 * 32 * kPatchWarps)
+            st_shared_u16(pe_s + 2 * static_cast<uint32_t>(lo * pitch + (bpos - src) / 2),
+                          *reinterpret_cast<const uint16_t*>(xb + bpos));
+        }
+      } else {
+        // column padding: element by element, zero outside the image
+        const TileCoord tc = tile_coord(a, t);
+        const int h0 = tc.p0 * a.sh - a.ph;
+        const uint16_t* xs = reinterpret_cast<const uint16_t*>(a.x);
+        for (int e = gt; e < patch_elems; e += 32 * kPatchWarps) {
+          const int rho = e / pitch, rem = e - rho * pitch;
+          const int u = rem / a.C, c = rem - u * a.C;
+          const int h = h0 + rho, w = u - a.pw;
+          uint16_t v = 0;
+          if (h >= 0 && h < a.H && w >= 0 && w < a.W)
+            v = __ldg(xs + ((static_cast<long long>(tc.n0) * a.H + h) * a.W + w) * a.C + c);
+          st_shared_u16(pe_s + 2 * e, v);
+        }
+      }
+      named_barrier_sync(2, 32 * kPatchWarps);   // patch complete
+      // this thread's rows: pixel (i, q) of the tile reads from patch element
+      // i sh pitch + q sw C on; base in 16-bit units from the buffer start
+      constexpr int kRows = kMaxTileN / (32 * kPatchWarps);   // operand rows per thread
+      int base[kRows];
+      bool valid[kRows];
+#pragma unroll
+      for (int j = 0; j < kRows; ++j) {
+        const int px = gt + 32 * kPatchWarps * j;
+        const int i = px / a.bw, q = px - i * a.bw;
+        valid[j] = px < T;
+        base[j] = static_cast<int>(off0 / 2) + i * a.sh * pitch + q * a.sw * a.C;
+      }
+      for (int kb = 0; kb < KB; ++kb, ++g) {
+        const int sb = g % kSt;
+        const uint32_t it = static_cast<uint32_t>(g / kSt);
+        if (ok) ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) continue;
+        const int* __restrict__ tab = ptab + kb * kBK;
+        uint8_t* __restrict__ stage = ring + sb * kStageBytes;
+        const uint16_t* __restrict__ p16 = reinterpret_cast<const uint16_t*>(buf);
+        const uint32_t* __restrict__ p32 = reinterpret_cast<const uint32_t*>(buf);
+#pragma unroll
+        for (int j = 0; j < kRows; ++j) {
+          const int row = gt + 32 * kPatchWarps * j;
+          if (row >= a.tile_n) continue;
+          // four chunks at a time: every load of the group is issued before
+          // the first shift or store
+#pragma unroll
+          for (int cg = 0; cg < 2; ++cg) {
+            int4 o[8];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+              o[2 * c] = *reinterpret_cast<const int4*>(tab + 8 * (4 * cg + c));
+              o[2 * c + 1] = *reinterpret_cast<const int4*>(tab + 8 * (4 * cg + c) + 4);
+            }
+            uint32_t wv[4][5];
+            bool run[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+              // the chunk's 8 codes are 8 consecutive patch elements (one run
+              // of a filter row): 5 aligned words, 4 funnel shifts
+              run[c] = valid[j] && o[2 * c].x >= 0 && o[2 * c + 1].w == o[2 * c].x + 7;
+              const int e = base[j] + (o[2 * c].x >= 0 ? o[2 * c].x : 0);
+              const uint32_t* w = p32 + (e >> 1);
+#pragma unroll
+              for (int u = 0; u < 5; ++u) wv[c][u] = run[c] ? w[u] : 0u;
+            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+              const int ch = 4 * cg + c;
+              uint4 v = make_uint4(0u, 0u, 0u, 0u);
+              if (run[c]) {
+                const int e = base[j] + o[2 * c].x;
+                const uint32_t sh = static_cast<uint32_t>(e & 1) * 16u;
+                v.x = __funnelshift_r(wv[c][0], wv[c][1], sh);
+                v.y = __funnelshift_r(wv[c][1], wv[c][2], sh);
+                v.z = __funnelshift_r(wv[c][2], wv[c][3], sh);
+                v.w = __funnelshift_r(wv[c][3], wv[c][4], sh);
+              } else if (valid[j]) {
+                // a chunk across two filter rows, or past the filter's end
+                const int off[8] = {o[2 * c].x, o[2 * c].y, o[2 * c].z, o[2 * c].w,
+                                    o[2 * c + 1].x, o[2 * c + 1].y, o[2 * c + 1].z,
+                                    o[2 * c + 1].w};
+                uint32_t h[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                  h[u] = off[u] >= 0 ? static_cast<uint32_t>(p16[base[j] + off[u]]) : 0u;
+                v = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                               h[6] | (h[7] << 16));
+              }
+              // 128-byte swizzle: chunk XOR (row mod 8)
+              *reinterpret_cast<uint4*>(stage + row * 128 + (((ch ^ (row & 7)) & 7) << 4)) = v;
+            }
+          }
+        }
+        fence_proxy_async_smem();   // generic-proxy writes -> visible to tcgen05.mma
+        mbar_arrive(&ctl->full[sb]);
+      }
+    }
+    // drain (after an abort): every bulk copy issued must land before the
+    // CTA may exit
+    if (a.patch_bulk && gt == 0) {
+      for (int b = 0; b < 2; ++b)
+        while (landed[b] < issued[b] &&
+               mbar_wait(&ctl->patch_full[b], landed[b] & 1u, nullptr, a.err, kWaitLimitNs))
+          ++landed[b];
+    }
+    __syncwarp();
   } else if (warp == 1) {
     // ================= MMA issuer =================
     const uint32_t idesc = idesc_bf16_f32(kBM, static_cast<uint32_t>(a.tile_n));
@@ -404,8 +666,8 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after_sync();
       for (int kb = 0; kb < KB; ++kb, ++g) {
-        const int st = g % kStages;
-        ok = mbar_wait(&ctl->full[st], static_cast<uint32_t>(g / kStages) & 1u, abort_flag, a.err,
+        const int st = g % kSt;
+        ok = mbar_wait(&ctl->full[st], static_cast<uint32_t>(g / kSt) & 1u, abort_flag, a.err,
                        kWaitLimitNs);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after_sync();
@@ -495,12 +757,19 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
       q1 = q3;
       q2 = next_codes();
       q3 = next_codes();
-      const int s0 = g % kStages, s1 = (g + 1) % kStages;
-      bool ok = mbar_wait(&ctl->empty[s0], (static_cast<uint32_t>(g / kStages) & 1u) ^ 1u,
-                          abort_flag, a.err, kWaitLimitNs);
+      const int s0 = g % kSt, s1 = (g + 1) % kSt;
+      // in patch mode the operand builders are the bottleneck: waiting
+      // expanders park instead of spinning, leaving the issue slots to them
+      bool ok = kPatch ? mbar_wait_sleep(&ctl->empty[s0], (static_cast<uint32_t>(g / kSt) & 1u) ^ 1u,
+                                         abort_flag, a.err, kWaitLimitNs)
+                       : mbar_wait(&ctl->empty[s0], (static_cast<uint32_t>(g / kSt) & 1u) ^ 1u,
+                                   abort_flag, a.err, kWaitLimitNs);
       if (ok && two)
-        ok = mbar_wait(&ctl->empty[s1], (static_cast<uint32_t>((g + 1) / kStages) & 1u) ^ 1u,
-                       abort_flag, a.err, kWaitLimitNs);
+        ok = kPatch ? mbar_wait_sleep(&ctl->empty[s1],
+                                      (static_cast<uint32_t>((g + 1) / kSt) & 1u) ^ 1u, abort_flag,
+                                      a.err, kWaitLimitNs)
+                    : mbar_wait(&ctl->empty[s1], (static_cast<uint32_t>((g + 1) / kSt) & 1u) ^ 1u,
+                                abort_flag, a.err, kWaitLimitNs);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after_sync();
       tmem_st_32x32b_x16(col + static_cast<uint32_t>(s0 * kAColsPerStage), v0);
@@ -549,7 +818,9 @@ __global__ void __launch_bounds__(threads_for<kGather>(), 1)
               : "memory");
         }
       }
-      if (ok) ok = mbar_wait(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs);
+      if (ok)
+        ok = kPatch ? mbar_wait_sleep(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs)
+                    : mbar_wait(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs);
       if (kTmaStore && a.residual && ok)
         ok = mbar_wait(&ctl->res_full, par, abort_flag, a.err, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok);
@@ -831,8 +1102,10 @@ CUresult encode_out_map(CUtensorMap* m, const void* base, const ConvProblem& p, 
                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-template <bool kGather, int kPoolBW, bool kTmaStore, bool kCh32>
+template <int kMode, int kPoolBW, bool kTmaStore>
 tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStream_t s) {
+  constexpr bool kGather = mode_gathers(kMode);
+  constexpr bool kCh32 = kMode == kModeTma32;
   alignas(64) CUtensorMap tmap_x, tmap_y, tmap_res;
   std::memset(&tmap_x, 0, sizeof(tmap_x));
   std::memset(&tmap_y, 0, sizeof(tmap_y));
@@ -866,13 +1139,15 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
         return fail(TBN_ERR_CUDA, "cuTensorMapEncodeTiled(residual) failed (%d)", (int)cr);
     }
   }
-  auto kern = conv_igemm_kernel<kGather, kPoolBW, kTmaStore, kCh32>;
-  // kernel attributes: set once per process (one process drives one GPU)
+  auto kern = conv_igemm_kernel<kMode, kPoolBW, kTmaStore>;
+  const size_t smem = smem_bytes_for(kMode, static_cast<size_t>(a.patch_cap), a.kblocks);
+  // kernel attributes: set once per process (one process drives one GPU);
+  // the shared-memory limit is the largest any launch of the mode can need
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)kSmemBytes);
+                                    kSmemLimit);
     if (attr_err == cudaSuccess)
       attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
   });
@@ -880,8 +1155,8 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
   const int grid = std::min(a.tiles, device_sm_count());
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(grid));
-  cfg.blockDim = dim3(threads_for<kGather>());
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.blockDim = dim3(threads_for<kMode>());
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -893,14 +1168,31 @@ tbn_status launch_t(const ConvProblem& p, const TilePlan& t, IgArgs& a, cudaStre
   return check_launch("conv_igemm_kernel");
 }
 
-template <bool kGather, bool kTmaStore, bool kCh32>
+template <int kMode, bool kTmaStore>
 tbn_status launch_pool(const ConvProblem& p, const TilePlan& t, IgArgs& a, int pw, cudaStream_t s) {
   switch (pw) {
-    case 8: return launch_t<kGather, 8, kTmaStore, kCh32>(p, t, a, s);
-    case 16: return launch_t<kGather, 16, kTmaStore, kCh32>(p, t, a, s);
-    case 32: return launch_t<kGather, 32, kTmaStore, kCh32>(p, t, a, s);
-    default: return launch_t<kGather, 0, kTmaStore, kCh32>(p, t, a, s);
+    case 8: return launch_t<kMode, 8, kTmaStore>(p, t, a, s);
+    case 16: return launch_t<kMode, 16, kTmaStore>(p, t, a, s);
+    case 32: return launch_t<kMode, 32, kTmaStore>(p, t, a, s);
+    default: return launch_t<kMode, 0, kTmaStore>(p, t, a, s);
   }
+}
+
+// Patch mode (gathered activations staged per tile in shared memory) when a
+// tile is whole output rows of one image, the filter spans at most
+// kPatchMaxKBlocks K blocks and two patches fit beside the ring.
+int patch_cap_bytes(const ConvProblem& p, const TilePlan& t) {
+  if (use_tma(p) || t.tiles_q != 1 || t.bn != 1) return 0;
+  const int64_t kblocks = (p.C * p.R * p.S + kBK - 1) / kBK;
+  if (kblocks > kPatchMaxKBlocks) return 0;
+  const int64_t rows = static_cast<int64_t>(t.bh - 1) * p.sh + p.R;
+  const int64_t elems = rows * (p.W + 2 * p.pw) * p.C;
+  const int64_t cap = ((2 * elems + 32) + 15) / 16 * 16;
+  if (cap > (int64_t(1) << 20)) return 0;
+  if (smem_bytes_for(kModePatch, static_cast<size_t>(cap), static_cast<int>(kblocks)) >
+      static_cast<size_t>(kSmemLimit))
+    return 0;
+  return static_cast<int>(cap);
 }
 
 }  // namespace
@@ -952,15 +1244,25 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
   const int pw = pool_width(p, t);
   const bool tst = use_tma_store(p);
   if (use_tma(p) && use_ch32(p)) {
-    return tst ? launch_pool<false, true, true>(p, t, a, pw, s)
-               : launch_pool<false, false, true>(p, t, a, pw, s);
+    return tst ? launch_pool<kModeTma32, true>(p, t, a, pw, s)
+               : launch_pool<kModeTma32, false>(p, t, a, pw, s);
   }
   if (use_tma(p)) {
-    return tst ? launch_pool<false, true, false>(p, t, a, pw, s)
-               : launch_pool<false, false, false>(p, t, a, pw, s);
+    return tst ? launch_pool<kModeTma64, true>(p, t, a, pw, s)
+               : launch_pool<kModeTma64, false>(p, t, a, pw, s);
   }
-  return tst ? launch_pool<true, true, false>(p, t, a, pw, s)
-             : launch_pool<true, false, false>(p, t, a, pw, s);
+  const int cap = patch_cap_bytes(p, t);
+  if (cap > 0) {
+    a.PR = (t.bh - 1) * a.sh + a.R;
+    a.PW = a.W + 2 * a.pw;
+    a.patch_cap = cap;
+    a.patch_bulk = a.pw == 0 ? 1 : 0;
+    a.x_bytes = static_cast<long long>(p.N) * p.H * p.W * p.C * 2;
+    return tst ? launch_pool<kModePatch, true>(p, t, a, pw, s)
+               : launch_pool<kModePatch, false>(p, t, a, pw, s);
+  }
+  return tst ? launch_pool<kModeGather, true>(p, t, a, pw, s)
+             : launch_pool<kModeGather, false>(p, t, a, pw, s);
 }
 
 }  // namespace tbn
