@@ -272,6 +272,61 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
   }
 }
 
+// One output row (image b, row ho) per block, bf16 NHWC with C % 8 == 0: a
+// thread takes (column, 8-channel vector) items, so consecutive threads read
+// consecutive 16-byte vectors of each tap; the max is taken on bf16 pairs
+// (exact: max of two bf16 values is one of them).  Taps in the padding are
+// skipped.
+__global__ void __launch_bounds__(256) maxpool_row_bf16x8_kernel(
+    const uint4* __restrict__ x, int H, int W, int C8, int kh, int kw, int sh, int sw, int ph,
+    int pw, int Ho, int Wo, uint4* __restrict__ y) {
+  const int b = blockIdx.x / Ho, ho = blockIdx.x - b * Ho;
+  const int items = Wo * C8;
+  const uint4* xb = x + static_cast<int64_t>(b) * H * W * C8;
+  uint4* yrow = y + (static_cast<int64_t>(b) * Ho + ho) * Wo * C8;
+  const int h_lo = max(0, ho * sh - ph), h_hi = min(H, ho * sh - ph + kh);
+  for (int i = threadIdx.x; i < items; i += 256) {
+    const int wo = i / C8, c = i - wo * C8;
+    const int w_lo = max(0, wo * sw - pw), w_hi = min(W, wo * sw - pw + kw);
+    __nv_bfloat162 m[4];
+    const __nv_bfloat162 ninf = __floats2bfloat162_rn(-INFINITY, -INFINITY);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) m[e] = ninf;
+    for (int h = h_lo; h < h_hi; ++h) {
+      const uint4* xr = xb + (static_cast<int64_t>(h) * W) * C8 + c;
+      for (int w = w_lo; w < w_hi; ++w) {
+        const uint4 t = __ldg(xr + static_cast<int64_t>(w) * C8);
+        const __nv_bfloat162* tb = reinterpret_cast<const __nv_bfloat162*>(&t);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) m[e] = __hmax2(m[e], tb[e]);
+      }
+    }
+    yrow[i] = *reinterpret_cast<const uint4*>(m);
+  }
+}
+
+// NCHW -> NHWC for any H*W (the vector kernel below needs H*W % 8 == 0):
+// a block moves 1024 pixels of one image through shared memory, reading
+// each channel plane with consecutive 2-byte loads and writing the pixels'
+// Cp channels as one contiguous run of 2-byte stores.
+constexpr int kT2Pix = 1024;
+
+__global__ void __launch_bounds__(256) nchw_to_nhwc_tiled_kernel(
+    const uint16_t* __restrict__ x, int C, int HW, int Cp, uint16_t* __restrict__ y) {
+  extern __shared__ uint16_t t2[];   // [kT2Pix][Cp]
+  grid_dependents_launch();
+  const int b = blockIdx.y;
+  const int p0 = blockIdx.x * kT2Pix;
+  const int np = min(kT2Pix, HW - p0);
+  const uint16_t* xb = x + static_cast<int64_t>(b) * C * HW + p0;
+  for (int c = 0; c < Cp; ++c)
+    for (int i = threadIdx.x; i < np; i += 256)
+      t2[i * Cp + c] = c < C ? __ldg(xb + static_cast<int64_t>(c) * HW + i) : uint16_t(0);
+  __syncthreads();
+  uint16_t* yb = y + (static_cast<int64_t>(b) * HW + p0) * Cp;
+  for (int i = threadIdx.x; i < np * Cp; i += 256) yb[i] = t2[i];
+}
+
 // One thread per pixel of one image (blockIdx.y): reads the pixel's C
 // values from the C planes (coalesced across the warp's consecutive pixels)
 // and writes its Cp channels contiguously; no index divisions.
@@ -355,7 +410,12 @@ tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H
                                int64_t C, int64_t kh, int64_t kw, int64_t sh, int64_t sw,
                                int64_t ph, int64_t pw, void* y, cudaStream_t s) {
   const int64_t Ho = (H + 2 * ph - kh) / sh + 1, Wo = (W + 2 * pw - kw) / sw + 1;
-  if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16)) {
+  if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16) &&
+      N * Ho < (int64_t(1) << 31) && H * W * C < (int64_t(1) << 31)) {
+    maxpool_row_bf16x8_kernel<<<static_cast<unsigned>(N * Ho), 256, 0, s>>>(
+        static_cast<const uint4*>(x), (int)H, (int)W, (int)(C / 8), (int)kh, (int)kw, (int)sh,
+        (int)sw, (int)ph, (int)pw, (int)Ho, (int)Wo, static_cast<uint4*>(y));
+  } else if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16)) {
     const int64_t total = N * Ho * Wo * (C / 8);
     maxpool_nhwc_bf16x8_kernel<<<(unsigned)grid_for(total), 256, 0, s>>>(
         static_cast<const uint4*>(x), N, H, W, C / 8, kh, kw, sh, sw, ph, pw, Ho, Wo,
@@ -383,7 +443,7 @@ tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, [] {
-    const void* fns[10] = {(const void*)nchw_to_nhwc_bf16x8_kernel<1>,
+    const void* fns[11] = {(const void*)nchw_to_nhwc_bf16x8_kernel<1>,
                            (const void*)nchw_to_nhwc_bf16x8_kernel<2>,
                            (const void*)nchw_to_nhwc_bf16x8_kernel<3>,
                            (const void*)nchw_to_nhwc_bf16x8_kernel<4>,
@@ -392,7 +452,8 @@ tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C
                            (const void*)nchw_to_nhwc_bf16x8_kernel<7>,
                            (const void*)nchw_to_nhwc_bf16x8_kernel<8>,
                            (const void*)nchw_to_nhwc_kernel<__nv_bfloat16>,
-                           (const void*)nchw_to_nhwc_kernel<float>};
+                           (const void*)nchw_to_nhwc_kernel<float>,
+                           (const void*)nchw_to_nhwc_tiled_kernel};
     for (const void* f : fns) {
       const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
       if (e != cudaSuccess && attr_err == cudaSuccess) attr_err = e;
@@ -417,6 +478,13 @@ tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C
       default: nchw_to_nhwc_bf16x8_kernel<8><<<blocks, 256, 0, s>>>(xv, c, HW8, total, yv); break;
     }
     return check_launch("nchw_to_nhwc_bf16x8_kernel");
+  }
+  if (dt == TBN_BF16 && C_pad <= 16) {
+    const dim3 grid(static_cast<unsigned>((H * W + kT2Pix - 1) / kT2Pix), static_cast<unsigned>(N));
+    nchw_to_nhwc_tiled_kernel<<<grid, 256, kT2Pix * C_pad * 2, s>>>(
+        static_cast<const uint16_t*>(x), (int)C, (int)(H * W), (int)C_pad,
+        static_cast<uint16_t*>(y));
+    return check_launch("nchw_to_nhwc_tiled_kernel");
   }
   const dim3 grid(static_cast<unsigned>((H * W + 255) / 256), static_cast<unsigned>(N));
   if (dt == TBN_BF16)

@@ -126,3 +126,17 @@ def test_nchw_to_nhwc_vector_path(N, C, H, W, C_pad):
 
 def test_device_error_word_is_clear():
     assert tbn.tbn_device_error() == 0
+
+
+@pytest.mark.parametrize("N,C,H,W,C_pad", [(2, 3, 227, 227, 3), (1, 3, 33, 35, 4), (3, 1, 7, 5, 1),
+                                           (2, 5, 31, 33, 12), (1, 3, 3, 3, 16)])
+def test_nchw_to_nhwc_tiled_path(N, C, H, W, C_pad):
+    """bf16 with H*W % 8 != 0 (AlexNet's 227 x 227 input) or C_pad > 8 takes
+    the shared-memory tiled kernel: every element and the zero padding,
+    exactly, including images that end inside a tile."""
+    g = inputs.generator(N * 1000 + C * 10 + H)
+    x = torch.randn(N, C, H, W, generator=g).to(torch.bfloat16)
+    y = tbn.tbn_nchw_to_nhwc(x.cuda(), C_pad=C_pad).cpu()
+    want = torch.zeros(N, H, W, C_pad, dtype=torch.bfloat16)
+    want[..., :C] = x.permute(0, 2, 3, 1)
+    assert torch.equal(y, want)
