@@ -1,45 +1,53 @@
 """Benchmark of the TBN hot path on GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload vgg_small|gemv|quantize]
+                    [--workload alexnet|vgg_small|resnet18|lenet|gemv|quantize|backward]
+                    [--no-extras] [--no-cpu-baseline]
 
-Default workload: the VGG-small TBN conv stack at batch 128 on CIFAR-sized
-input (3x32x32 bf16 ~ N(0,1), six 3x3/p1 layers 128-128-256-256-512-512,
-ReLU, 2x2 max pool after every second layer, He-normal weights), seed 1.
-One step = one pass of the whole hot path over the batch: re-quantize every
-layer's real-valued weights (Eq. 3 + Eq. 5 + packing, one grouped launch),
-NCHW -> NHWC, six two-bit convolutions (Eq. 1) with fused ReLU and, after
-every second layer, the fused 2x2 max pool.  The metric is TBN-conv TFLOP/s:
-the algorithmic 2*N*K*P*Q*C*R*S flops of the six convolutions per step over
-the step's device time (every launch of the step included); images/s is
-reported beside it.
+Default workload: the AlexNet-shaped TBN network at batch 256 (3x227x227
+bf16 ~ N(0,1); conv 96x11x11/4, 256x5x5/p2, 384x3x3/p1, 384x3x3/p1,
+256x3x3/p1 with 3x3/2 max pools; FC 9216-4096-4096-1000; He-normal weights,
+two-bit with per-output-neuron alpha), seed 2.  One step is one pass of the
+whole hot path over the batch: re-quantization of every layer's real-valued
+weights (Eq. 3 + Eq. 5 + packing, one grouped launch; Algorithm 1 runs the
+quantization loop before each forward), the input's NCHW -> NHWC change, the
+five two-bit convolutions (Eq. 1) with fused ReLU, the three max pools and
+the three fully-connected layers (Section 3).  The metric is TBN TFLOP/s:
+the algorithmic 2*N*K*P*Q*C*R*S flops of the convolutions plus 2*B*K_in*K_out
+of the FC layers (581.25 GFLOP per step) over the step's device time, every
+launch of the step included; images/s is reported beside it, and the
+inference form (codes quantized once, no re-quantization) as an extra key.
 
 Timing: the step is captured in a CUDA graph; W warm-up replays (and at
 least --min-warmup-s seconds of them, so the clocks settle), then K timed
 replays, each bracketed by CUDA events recorded inside the graph, with a
 512 MiB write between replays that flushes L2 (outside the timed events).
-nvidia-smi samples the SM clock through the timed regions.  A second timed
-region replays an instrumented copy of the graph with events around every
-tensor-core convolution: the roofline entry (the tcgen05 conv kernel) is
-its flops over those durations.  The e2e figure replays a third graph that
-adds, each step, the copy of the input batch from pinned host memory and the
-copy of the output feature map back to pinned host memory.
+nvidia-smi samples the SM clock through the timed regions.  The roofline
+entry is the tcgen05 implicit-GEMM kernel: its launches of one step (the
+five convolutions and the three FC layers) replayed back to back in a graph
+of their own after an L2 flush, algorithmic flops over that time.  The e2e
+figure replays a graph that adds, each step, the copy of the input batch
+from pinned host memory and of the logits back to pinned host memory.
+
+Extra keys of the default run (each its own small timed region): VGG-small
+b128 and ResNet-18 b128 forward TFLOP/s and images/s, the LeNet-like layer's
+quantize + conv latency, the quantizer's and the GEMV's HBM GB/s.
 
 Under torchrun (N > 1) every rank runs its own batch on its own GPU (data
 parallel replicas, no collective on the data path): value = the work of all
 ranks over the slowest rank's time.
 
+--workload vgg_small  VGG-small b128 (re-quantized per forward) as the line
+--workload resnet18   ResNet-18 b128 as the line
 --workload gemv       batch-1/8 fully-connected layers, K_out = K_in in
                       {4096, 8192, 16384}: HBM GB/s on the 2-bit stream
 --workload quantize   tbn_quantize_pack on 8192^2 and 16384^2 fp32 matrices:
                       HBM GB/s at 4.25 bytes per weight
 --workload backward   Algorithm 1's TwoBitBackward through the six VGG-small
-                      convolutions at batch 128: the filter gradients of all
-                      six layers and the input gradients of c2..c6 (the
-                      image itself needs none), 309.2 GFLOP per step
---impl reference      the CPU oracle (plain C, fp64) on the VGG-small
+                      convolutions at batch 128
+--impl reference      the CPU oracle (plain C, fp64) on the AlexNet
                       workload: one image of the batch per step through
-                      re-quantization + the six convolutions + glue.
+                      re-quantization + the five convolutions + pools + FC.
 """
 from __future__ import annotations
 
@@ -57,22 +65,30 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-WORKLOAD = "vgg_small_b128_cifar"
-METRIC = "TBN conv TFLOP/s (VGG-small b128 forward incl. per-step re-quantization)"
-FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# used only when MEASURED_PEAKS.json is absent (one earlier GB300 measurement)
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 FLUSH_BYTES = 512 * 1024 * 1024
 
-# DRAM bytes (read + write) per convolution launch, mean over the five
-# implicit-GEMM launches of one step (c2..c6), from the ncu capture summarised in profiles/vgg_small_b128_launches.md.
-# Valid only for the kernel sources it was measured on (hash below); otherwise the
-# roofline entry reports null.
+WORKLOADS = {
+    "alexnet": ("alexnet_b256", "TBN TFLOP/s (AlexNet b256 forward incl. per-step re-quantization)"),
+    "vgg_small": ("vgg_small_b128_cifar",
+                  "TBN conv TFLOP/s (VGG-small b128 forward incl. per-step re-quantization)"),
+    "resnet18": ("resnet18_b128", "TBN conv TFLOP/s (ResNet-18 b128, two-bit convolutions)"),
+}
+
+# DRAM bytes (read + write) per implicit-GEMM launch of the AlexNet step, from
+# the ncu capture summarised in profiles/alexnet_b256_launches.md (batch-32
+# capture scaled to batch 256).  Valid only for the kernel sources it was
+# measured on (hash below); otherwise the roofline entry reports null.
 CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
                             "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
-                "sha256_16": "07de82155ed5eaf3", "bytes_per_launch": 14.54e6}
+                "sha256_16": None, "bytes_per_launch": None}
 
 
 def measured_traffic(rec):
     import hashlib
+    if rec["sha256_16"] is None:
+        return None
     h = hashlib.sha256()
     for f in rec["sources"]:
         with open(os.path.join(ROOT, f), "rb") as fh:
@@ -143,25 +159,30 @@ class ClockSampler:
 
 
 class L2Flush:
-    """Evicts the step's data from L2 between timed replays: writes a 512 MiB
-    buffer (larger than the 129 MB L2) and, in "write+read" mode, then reads
-    another 512 MiB buffer, so the write's dirty lines are written back
-    before the timed region instead of during it (L2 ends up holding clean,
-    unrelated lines)."""
+    """Evicts the step's data from L2 between timed replays by writing a
+    512 MiB buffer (larger than the 129 MB L2)."""
 
-    def __init__(self, dev, mode):
-        self.mode = mode
+    def __init__(self, dev):
         self.w = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
-        self.r = torch.ones(FLUSH_BYTES // 4, dtype=torch.int32, device=dev) if mode == "write+read" else None
-        self.acc = torch.empty((), dtype=torch.int32, device=dev)
 
     def zero_(self):
         self.w.zero_()
-        if self.r is not None:
-            torch.sum(self.r, dim=0, dtype=torch.int32, out=self.acc)
 
 
-def timed_replays(graph, stream, flush, ev, steps, dev):
+def capture(body, stream, dev):
+    """A CUDA graph of body() bracketed by two timing events recorded inside it."""
+    ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(g, stream=stream):
+            ev[0].record()
+            body()
+            ev[1].record()
+    torch.cuda.synchronize(dev)
+    return g, ev
+
+
+def timed_replays(graph, stream, flush, ev, steps):
     """Replay `graph` `steps` times, flushing L2 before each replay; returns
     the per-replay device times (ms) between the graph's own events ev."""
     out = []
@@ -200,192 +221,278 @@ def barrier(world: int):
         torch.distributed.barrier()
 
 
-# ------------------------------------------------------------------ VGG-small
-def run_vgg(args, rank, world, local_rank):
+def pick_peak(peaks, clocks):
+    """Burst peak when the timed region ran at the maximum SM clock with no
+    power cap (a kernel timed that way is not power-limited), else the
+    sustained one; returns (peak, kind, other)."""
+    burst = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    sust = peaks.get("bf16_tflops_sustained")
+    at_max = (clocks.get("sm_mhz") is not None and clocks.get("sm_max_mhz") is not None and
+              clocks["sm_mhz"] >= 0.97 * clocks["sm_max_mhz"] and
+              "sw_power_cap" not in clocks.get("reasons", []))
+    if at_max or sust is None:
+        return burst, "burst", (float(sust) if sust is not None else None)
+    return float(sust), "sustained", burst
+
+
+# ------------------------------------------------------------------ networks
+def net_spec(name, dev, batch=None):
+    """The network of a workload and the closures the benchmark times: the
+    whole step, the inference form, the implicit-GEMM launches of one step
+    (for the roofline) and every launch of the step on its own."""
     import paper_1701_00485_gb300 as tbn
     from paper_1701_00485_gb300 import nets
 
+    def conv_call(h, l, s, pool=0):
+        return lambda: tbn.tbn_conv2d_fwd(h, l.codes, l.alpha, s.K, s.R, s.S, (s.stride,) * 2,
+                                          (s.pad,) * 2, layout=tbn.TBN_NHWC, relu=s.relu,
+                                          out=l.y, pool=pool)
+
+    def is_igemm(N, C, hw, s):
+        return tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NHWC, N, C, hw[0], hw[1], s.K,
+                                          s.R, s.S, (s.stride,) * 2, (s.pad,) * 2) == \
+            tbn.TBN_CONV_IMPLICIT_GEMM
+
+    chain, chain_flops, layers = [], 0, []
+    if name in ("alexnet", "vgg_small"):
+        net = nets.alexnet(batch, device=dev) if name == "alexnet" else nets.vgg_small(batch, device=dev)
+        F = net.features if name == "alexnet" else net
+        N = F.N
+        layers.append(("nchw_to_nhwc", lambda: tbn.tbn_nchw_to_nhwc(F.x_in, out=F.x_nhwc)))
+        h = F.x_nhwc
+        for i, l in enumerate(F.layers):
+            s = l.spec
+            fn = conv_call(h, l, s, 2 if s.pool == (2, 2) else 0)
+            layers.append(("conv%d" % (i + 1), fn))
+            if is_igemm(N, s.C, l.in_hw, s):
+                chain.append(fn)
+                chain_flops += N * l.flops_per_image
+            h = l.y
+            if l.pooled is not None:
+                k, st = s.pool
+                layers.append(("pool%d" % (i + 1),
+                               (lambda hh=h, ll=l, k=k, st=st:
+                                tbn.tbn_maxpool2d_nhwc(hh, (k, k), (st, st), out=ll.pooled))))
+                h = l.pooled
+        if name == "alexnet":
+            hh = h.reshape(N, -1)
+            for j, (W, codes, alpha, relu, y) in enumerate(net.classifier.layers):
+                fn = (lambda hh=hh, c=codes, a=alpha, r=relu, y=y:
+                      tbn.tbn_linear_fwd(hh, c, a, c.shape[0], relu=r, out=y))
+                layers.append(("fc%d" % (j + 6), fn))
+                chain.append(fn)
+                chain_flops += 2 * N * W.shape[0] * W.shape[1]
+                hh = y
+            flops = net.flops
+            cfg = {"workload": "alexnet_b256", "global_batch": N, "image": [3, 227, 227],
+                   "layers": "conv 96x11x11/4, 256x5x5/p2, 384x3x3/p1, 384x3x3/p1, "
+                             "256x3x3/p1, 3x3/2 max pools; FC 9216-4096-4096-1000",
+                   "requantize_per_step": True}
+            kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM): conv1 (patch mode), " \
+                          "conv2 (32-channel TMA), conv3-5, fc6-8 (1x1)"
+        else:
+            flops = net.flops
+            cfg = {"workload": "vgg_small_b128_cifar", "global_batch": N, "image": [3, 32, 32],
+                   "layers": "3x3/p1 128-128-256-256-512-512, 2x2 pool every 2nd",
+                   "requantize_per_step": True}
+            kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM), layers c2-c6"
+        step = lambda: net.forward(requantize=True)
+        infer = lambda: net.forward(requantize=False)
+        quant = net.quantize
+        tbn_flops = flops
+    elif name == "resnet18":
+        net = nets.resnet18(batch, device=dev)
+        N = net.N
+        layers.append(("stem", net.stem))
+        h = net.pool_y
+        for a, b, d in net.blocks:
+            for c, x_in, res, relu in ((a, h, None, None), (d, h, None, None),
+                                       (b, a.y, (d.y if d is not None else h), True)):
+                if c is None:
+                    continue
+                fn = (lambda c=c, x_in=x_in, res=res, relu=relu: c.run(x_in, residual=res, relu=relu))
+                layers.append((c.name, fn))
+                chain.append(fn)
+                chain_flops += N * c.flops_per_image
+            h = b.y
+        layers.append(("head", lambda hh=h: net.head(hh)))
+        step = lambda: net.forward(requantize=True)
+        infer = lambda: net.forward(requantize=False)
+        quant = net.quantize
+        tbn_flops = net.tbn_flops
+        flops = tbn_flops
+        cfg = {"workload": "resnet18_b128", "global_batch": N, "image": [3, 224, 224],
+               "layers": "fp32 7x7/2 stem + 3x3/2 max pool, 8 basic blocks of two-bit 3x3 "
+                         "convs (1x1/2 two-bit projections), global average pool, fp32 FC "
+                         "512-1000", "requantize_per_step": True}
+        kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM), all 19 two-bit convolutions"
+    else:
+        raise ValueError(name)
+    return dict(net=net, N=N, step=step, infer=infer, quant=quant, flops=flops,
+                tbn_flops=tbn_flops, chain=chain, chain_flops=chain_flops, layers=layers,
+                cfg=cfg, kernel_desc=kernel_desc,
+                launches=net.launches_per_forward(True))
+
+
+def run_network(args, rank, world, local_rank, name, full=True, steps=None, warmup=None):
+    import paper_1701_00485_gb300 as tbn
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    net = nets.vgg_small(device=dev)
-    N = net.N
-    flops = net.flops
-    tc_layers = [i for i, l in enumerate(net.layers)
-                 if tbn.tbn_conv2d_select_algo(torch.bfloat16, tbn.TBN_NHWC, N, l.spec.C,
-                                               l.in_hw[0], l.in_hw[1], l.spec.K, l.spec.R,
-                                               l.spec.S, (l.spec.stride,) * 2,
-                                               (l.spec.pad,) * 2) == tbn.TBN_CONV_IMPLICIT_GEMM]
-    tc_flops = N * sum(net.layers[i].flops_per_image for i in tc_layers)
-
+    steps = args.steps if steps is None else steps
+    warmup = args.warmup if warmup is None else warmup
+    sp = net_spec(name, dev)
+    net, N = sp["net"], sp["N"]
     stream = torch.cuda.Stream(device=dev)
     # eager warm-up outside capture: resolves per-device state and kernel attributes
     with torch.cuda.stream(stream):
-        net.forward(requantize=True)
+        sp["step"]()
     torch.cuda.synchronize(dev)
     if tbn.tbn_device_error() != 0:
         raise RuntimeError("device error word set after warm-up")
 
-    def capture(body):
-        ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.stream(stream):
-            with torch.cuda.graph(g, stream=stream):
-                ev[0].record()
-                body()
-                ev[1].record()
-        torch.cuda.synchronize(dev)
-        return g, ev
+    def chain_body():
+        for fn in sp["chain"]:
+            fn()
 
-    # plain step: the timed graph
-    graph, ev_step = capture(lambda: net.forward(requantize=True))
-    # instrumented step: events around every tensor-core convolution
-    ev_conv = {i: [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-               for i in range(len(net.layers))}
-
-    ev_quant = torch.cuda.Event(enable_timing=True, external=True)
-
-    def hook(i, layer, when):
-        if i < 0:
-            ev_quant.record()
-        elif i in ev_conv:
-            ev_conv[i][0 if when == "before" else 1].record()
-
-    graph_i, ev_i = capture(lambda: net.forward(requantize=True, conv_hook=hook))
-
-    # roofline graph: the tensor-core convolutions alone, back to back as in
-    # the step (each layer reads the previous layer's output), bracketed by
-    # one pair of events so the launches overlap as they do in the step
-    def tc_chain():
-        for i in tc_layers:
-            l = net.layers[i]
-            s = l.spec
-            h = net.layers[i - 1].pooled if net.layers[i - 1].pooled is not None else \
-                net.layers[i - 1].y
-            tbn.tbn_conv2d_fwd(h, l.codes, l.alpha, s.K, s.R, s.S, (s.stride, s.stride),
-                               (s.pad, s.pad), layout=tbn.TBN_NHWC, relu=s.relu, out=l.y,
-                               pool=2 if s.pool == (2, 2) else 0)
-
-    assert tc_layers and tc_layers[0] > 0 and \
-        tc_layers == list(range(tc_layers[0], tc_layers[-1] + 1)) and \
-        all(net.layers[i].pooled is None for i in tc_layers), "chain of fused layers"
-    graph_c, ev_c = capture(tc_chain)
-    # e2e step: host input in, output feature map out
-    x_host = net.x_in.cpu().pin_memory()
-    out_host = torch.empty(net.out.shape, dtype=net.out.dtype).pin_memory()
-
-    def e2e_body():
-        net.x_in.copy_(x_host, non_blocking=True)
-        net.forward(requantize=True)
-        out_host.copy_(net.out, non_blocking=True)
-
-    graph_e, ev_e = capture(e2e_body)
-
-    flush = L2Flush(dev, args.l2_flush)
+    graph, ev_step = capture(sp["step"], stream, dev)
+    graph_inf, ev_inf = capture(sp["infer"], stream, dev)
+    graph_q, ev_q = capture(sp["quant"], stream, dev)
+    graph_c, ev_c = capture(chain_body, stream, dev)
+    flush = L2Flush(dev)
     sampler = ClockSampler(local_rank)
     sampler.start()
-    warm(graph, stream, flush, args.warmup, args.min_warmup_s, dev)
+    warm(graph, stream, flush, warmup, args.min_warmup_s if full else 0.2, dev)
 
     barrier(world)
     torch.cuda.synchronize(dev)
     t0 = time.time()
-    step_ms = timed_replays(graph, stream, flush, ev_step, args.steps, dev)
+    step_ms = timed_replays(graph, stream, flush, ev_step, steps)
     torch.cuda.synchronize(dev)
     barrier(world)
-    # roofline region: the tensor-core chain alone, then the instrumented
-    # graph (per-layer breakdown; its events between layers stop the overlap)
-    chain_ms = timed_replays(graph_c, stream, flush, ev_c, args.steps, dev)
-    conv_ms = []
-    layer_ms = np.zeros(len(net.layers))
-    quant_ms = 0.0
-    prefix_ms = 0.0
-    for _ in range(args.steps):
-        with torch.cuda.stream(stream):
-            flush.zero_()
-            graph_i.replay()
-        stream.synchronize()
-        conv_ms.append(sum(ev_conv[i][0].elapsed_time(ev_conv[i][1]) for i in tc_layers))
-        layer_ms += [ev_conv[i][0].elapsed_time(ev_conv[i][1]) for i in range(len(net.layers))]
-        quant_ms += ev_i[0].elapsed_time(ev_quant)
-        prefix_ms += ev_quant.elapsed_time(ev_conv[0][0])
+    inf_ms = timed_replays(graph_inf, stream, flush, ev_inf, steps)
+    chain_ms = timed_replays(graph_c, stream, flush, ev_c, steps)
+    quant_ms = timed_replays(graph_q, stream, flush, ev_q, max(3, steps // 2))
+    breakdown = {}
+    if full:
+        reps = max(3, min(steps, 10))
+        for label, fn in sp["layers"]:
+            g, ev = capture(fn, stream, dev)
+            breakdown[label] = round(1e3 * float(np.median(timed_replays(g, stream, flush, ev, reps))), 2)
+            del g
     t1 = time.time()
     clocks = sampler.stop(t0, t1)
 
     total_ms = max_over_ranks(float(np.sum(step_ms)), world, dev)
-    ms_per_step = total_ms / args.steps
-    value = world * flops * args.steps / (total_ms * 1e-3) / 1e12
-    images_per_s = world * N * args.steps / (total_ms * 1e-3)
-
-    warm(graph_e, stream, flush, 3, 0.0, dev)
-    e2e_ms = timed_replays(graph_e, stream, flush, ev_e, args.steps, dev)
-    e2e_total = max_over_ranks(float(np.sum(e2e_ms)), world, dev)
-    e2e_value = world * flops * args.steps / (e2e_total * 1e-3) / 1e12
-
-    err = tbn.tbn_device_error()
+    ms_per_step = total_ms / steps
+    value = world * sp["flops"] * steps / (total_ms * 1e-3) / 1e12
+    images_per_s = world * N * steps / (total_ms * 1e-3)
+    inf_step = float(np.mean(inf_ms))
+    chain_step = float(np.mean(chain_ms))
     peaks, peak_kind = load_peaks()
-    tc_launch_ms = float(np.mean(chain_ms)) / len(tc_layers)   # mean per launch in the chain
-    achieved = (tc_flops / len(tc_layers)) / (tc_launch_ms * 1e-3) / 1e12
-    achieved_isolated = tc_flops / (float(np.mean(conv_ms)) * 1e-3) / 1e12
-    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-    burst = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    peak, which, other = pick_peak(peaks, clocks)
+    achieved = sp["chain_flops"] / (chain_step * 1e-3) / 1e12
     roofline = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
                 "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-                # the step runs at full SM clock (see "clocks"), so the burst
-                # peak is the stricter denominator: reported beside it
-                "peak_burst": burst, "frac_burst": round(achieved / burst, 4),
-                "timing": "the %d launches back to back in one graph, L2 flushed before each "
-                          "replay, %.2f us per launch; with events between the layers (no launch "
-                          "overlap) %.1f TFLOP/s" % (len(tc_layers), 1e3 * tc_launch_ms,
-                                                    achieved_isolated),
-                "traffic": measured_traffic(CONV_TRAFFIC),
-                "kernel": "conv_igemm_kernel (tcgen05 implicit GEMM), %d launches per step "
-                          "(layers %s)" % (len(tc_layers),
-                                           ",".join("c%d" % (i + 1) for i in tc_layers)),
-                "peak_kind": "%s bf16 dense, sustained" % peak_kind}
-    return {
-        "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 5),
+                "peak_kind": "%s bf16 dense, %s" % (peak_kind, which),
+                "timing": "the %d implicit-GEMM launches of one step back to back in one graph, "
+                          "L2 flushed before each replay: %.2f us per step (%.1f GFLOP)"
+                          % (len(sp["chain"]), 1e3 * chain_step, sp["chain_flops"] / 1e9),
+                "traffic": measured_traffic(CONV_TRAFFIC) if name == "alexnet" else None,
+                "kernel": sp["kernel_desc"]}
+    if other is not None:
+        roofline["frac_" + ("sustained" if which == "burst" else "burst")] = round(achieved / other, 4)
+    res = {
+        "metric": WORKLOADS[name][1], "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": steps, "warmup": warmup, "ms_per_step": round(ms_per_step, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) input, He-normal weights)",
-        "config": {"workload": WORKLOAD, "global_batch": N * world, "image": [3, 32, 32],
-                   "layers": "3x3/p1 128-128-256-256-512-512, 2x2 pool every 2nd",
-                   "requantize_per_step": True, "parallelism": "replicas x%d" % world,
-                   "l2": "512 MiB %s between timed steps" % args.l2_flush},
+        "config": dict(sp["cfg"], global_batch=N * world, parallelism="replicas x%d" % world,
+                       l2="512 MiB write between timed steps"),
         "images_per_s": round(images_per_s, 1),
-        "breakdown_note": "per layer from events between the layers, which stop the launch "
-                          "overlap of the plain step: the parts sum to more than ms_per_step",
-        "breakdown_us": dict([("quantize", round(1e3 * quant_ms / args.steps, 2)),
-                              ("nchw_to_nhwc", round(1e3 * prefix_ms / args.steps, 2))] +
-                             [("c%d" % (i + 1), round(1e3 * layer_ms[i] / args.steps, 2))
-                              for i in range(len(net.layers))]),
-        "tbn_conv_gflop_per_step": round(flops * world / 1e9, 3),
-        "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s",
-                "h2d_bytes_per_step": int(x_host.numel() * x_host.element_size()),
-                "d2h_bytes_per_step": int(out_host.numel() * out_host.element_size()),
-                "ms_per_step": round(e2e_total / args.steps, 5)},
-        "gpu_launches": net.launches_per_forward(True) * args.steps,
+        "tbn_gflop_per_step": round(sp["tbn_flops"] * world / 1e9, 3),
+        "inference_form": {"note": "codes and alpha quantized once (no re-quantization in the step)",
+                           "ms_per_step": round(inf_step, 5),
+                           "tflops": round(sp["flops"] / (inf_step * 1e-3) / 1e12, 3),
+                           "images_per_s": round(N / (inf_step * 1e-3), 1)},
+        "requantize_us": round(1e3 * float(np.median(quant_ms)), 2),
         "roofline": roofline,
+        "gpu_launches": sp["launches"] * steps,
         "clocks": clocks,
-        "device_error_word": err,
     }
+    if name == "resnet18":
+        res["tbn_conv_tflops_chain"] = round(achieved, 3)
+        res["dense_gflop_per_step"] = round(net.dense_flops / 1e9, 3)
+    if full:
+        res["breakdown_us"] = breakdown
+        res["breakdown_note"] = "each launch alone in its own graph after an L2 flush (no " \
+                                "overlap with its neighbours): the parts sum to more than the step"
+        # e2e: host input in, logits out, every step
+        x_host = sp["net"].x_in.cpu().pin_memory()
+        out = sp["net"].out
+        out_host = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+
+        def e2e_body():
+            sp["net"].x_in.copy_(x_host, non_blocking=True)
+            sp["step"]()
+            out_host.copy_(out, non_blocking=True)
+
+        graph_e, ev_e = capture(e2e_body, stream, dev)
+        warm(graph_e, stream, flush, 3, 0.0, dev)
+        e2e_ms = timed_replays(graph_e, stream, flush, ev_e, steps)
+        e2e_total = max_over_ranks(float(np.sum(e2e_ms)), world, dev)
+        res["e2e"] = {"value": round(world * sp["flops"] * steps / (e2e_total * 1e-3) / 1e12, 3),
+                      "unit": "TFLOP/s",
+                      "h2d_bytes_per_step": int(x_host.numel() * x_host.element_size()),
+                      "d2h_bytes_per_step": int(out_host.numel() * out_host.element_size()),
+                      "ms_per_step": round(e2e_total / steps, 5)}
+    res["device_error_word"] = tbn.tbn_device_error()
+    del graph, graph_inf, graph_q, graph_c
+    return res
 
 
-# ------------------------------------------------------------------ HBM-bound paths
+# ------------------------------------------------------------------ single layers
+def run_lenet(args, local_rank, reps=50):
+    """The LeNet-like layer (config 1): quantize + pack [20, 25] fp32 weights,
+    then the fp32 direct convolution of 16 x 1 x 28 x 28 fp32 inputs;
+    latency per pass (launch-bound: 9.2 MFLOP)."""
+    import paper_1701_00485_gb300 as tbn
+    from paper_1701_00485_gb300 import inputs
+    dev = torch.device("cuda", local_rank)
+    x, W = inputs.lenet_inputs(0)
+    x, W = x.to(dev), W.reshape(20, -1).contiguous().to(dev)
+    codes = torch.empty((20, tbn.packed_words(25)), dtype=torch.int32, device=dev)
+    alpha = torch.empty((20,), dtype=torch.float32, device=dev)
+    y = torch.empty((16, 20, 24, 24), dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def body():
+        tbn.tbn_quantize_pack(W, codes, alpha)
+        tbn.tbn_conv2d_fwd(x, codes, alpha, 20, 5, 5, layout=tbn.TBN_NCHW, out=y)
+
+    with torch.cuda.stream(stream):
+        body()
+    torch.cuda.synchronize(dev)
+    g, ev = capture(body, stream, dev)
+    flush = L2Flush(dev)
+    warm(g, stream, flush, 5, 0.0, dev)
+    ms = timed_replays(g, stream, flush, ev, reps)
+    t = float(np.median(ms))
+    return {"workload": "lenet_like_conv_b16", "us_per_pass": round(1e3 * t, 2),
+            "tflops": round(2 * 16 * 20 * 24 * 24 * 25 / (t * 1e-3) / 1e12, 4),
+            "note": "quantize + pack, then the fp32 direct convolution; two launches, "
+                    "launch-latency bound"}
+
+
 def _rotating_graph(fn_list, stream, dev):
     """One graph that calls each fn once (launches rotate over buffers that
     together exceed L2), bracketed by events."""
-    ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.stream(stream):
-        with torch.cuda.graph(g, stream=stream):
-            ev[0].record()
-            for fn in fn_list:
-                fn()
-            ev[1].record()
-    torch.cuda.synchronize(dev)
-    return g, ev
+    def body():
+        for fn in fn_list:
+            fn()
+    return capture(body, stream, dev)
 
 
-def run_gemv(args, rank, world, local_rank):
+def run_gemv(args, rank, world, local_rank, sizes=None, batches=None, reps=None):
     import paper_1701_00485_gb300 as tbn
     from paper_1701_00485_gb300 import inputs
     torch.cuda.set_device(local_rank)
@@ -394,18 +501,21 @@ def run_gemv(args, rank, world, local_rank):
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     stream = torch.cuda.Stream(device=dev)
+    sizes = args.gemv_sizes if sizes is None else sizes
+    batches = args.gemv_batches if batches is None else batches
+    reps_t = max(3, args.steps // 20) if reps is None else reps
     sweep = []
     sampler = ClockSampler(local_rank)
     sampler.start()
     t0 = time.time()
-    for K in args.gemv_sizes:
+    for K in sizes:
         W, _ = inputs.gemv_inputs(K, 1)
         codes, alpha = tbn.tbn_quantize_pack(W.to(dev))
         del W
         code_bytes = codes.numel() * 4
         copies = max(2, int(np.ceil(3 * l2 / code_bytes)))
         bufs = [codes] + [codes.clone() for _ in range(copies - 1)]
-        for B in args.gemv_batches:
+        for B in batches:
             gx = torch.Generator(device=dev)
             gx.manual_seed(1000 * K + B)
             x = torch.randn((B, K), generator=gx, device=dev).to(torch.bfloat16)
@@ -414,19 +524,13 @@ def run_gemv(args, rank, world, local_rank):
             ws = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
             x32 = x.float()
             reps = max(copies, 64)
-            # "mma": tbn_linear_fwd with bf16 activations (tensor-core GEMV);
-            # "table-f32": tbn_linear_fwd_ws with fp32 activations (the
-            # batch-1 table-lookup GEMV, the path for fp32 inputs);
-            # "conv-f32": tbn_linear_fwd with fp32 activations and no scratch
-            # (the 1x1-convolution path those inputs take otherwise)
-            paths = ["mma", "table-f32", "conv-f32"] if ws_bytes > 0 else ["mma"]
+            # "mma": bf16 activations (tensor-core GEMV); "table-f32": fp32
+            # activations on the batch-1 table-lookup GEMV (tbn_linear_fwd_ws)
+            paths = ["mma", "table-f32"] if ws_bytes > 0 else ["mma"]
             for path in paths:
                 if path == "table-f32":
                     fns = [(lambda c=bufs[r % copies]:
                             tbn.tbn_linear_fwd_ws(x32, c, alpha, K, ws, out=y))
-                           for r in range(reps)]
-                elif path == "conv-f32":
-                    fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x32, c, alpha, K, out=y))
                            for r in range(reps)]
                 else:
                     fns = [(lambda c=bufs[r % copies]: tbn.tbn_linear_fwd(x, c, alpha, K, out=y))
@@ -439,7 +543,7 @@ def run_gemv(args, rank, world, local_rank):
                     g.replay()
                 torch.cuda.synchronize(dev)
                 ms = []
-                for _ in range(max(3, args.steps // 20)):
+                for _ in range(reps_t):
                     with torch.cuda.stream(stream):
                         g.replay()
                     stream.synchronize()
@@ -456,7 +560,6 @@ def run_gemv(args, rank, world, local_rank):
     clocks = sampler.stop(t0, time.time())
     head = ([s for s in sweep if s["K"] == 16384 and s["B"] == 1 and s["path"] == "mma"] or
             sweep)[0]
-    head_kernel = "gemv_tma_kernel (mma.sync)"
     return {"metric": "TBN GEMV HBM GB/s (B=1, K_out=K_in=16384, 2-bit weight stream)",
             "value": head["gbs"], "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
@@ -465,11 +568,11 @@ def run_gemv(args, rank, world, local_rank):
             "config": {"workload": "gemv_sweep", "l2": "rotating weight copies > 3x L2"},
             "roofline": {"bound": "hbm", "achieved": head["gbs"], "peak": hbm, "unit": "GB/s",
                          "frac": round(head["gbs"] / hbm, 4), "traffic": None,
-                         "kernel": head_kernel, "peak_kind": peak_kind},
+                         "kernel": "gemv_tma_kernel (mma.sync)", "peak_kind": peak_kind},
             "sweep": sweep, "clocks": clocks}
 
 
-def run_quantize(args, rank, world, local_rank):
+def run_quantize(args, rank, world, local_rank, sizes=None, reps=None):
     import paper_1701_00485_gb300 as tbn
     from paper_1701_00485_gb300 import inputs
     torch.cuda.set_device(local_rank)
@@ -477,26 +580,28 @@ def run_quantize(args, rank, world, local_rank):
     peaks, peak_kind = load_peaks()
     hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
     stream = torch.cuda.Stream(device=dev)
-    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush = L2Flush(dev)
+    sizes = args.quant_sizes if sizes is None else sizes
+    reps = max(5, args.steps // 10) if reps is None else reps
     sweep = []
     sampler = ClockSampler(local_rank)
     sampler.start()
     t0 = time.time()
-    for K in args.quant_sizes:
+    for K in sizes:
         W, _ = inputs.gemv_inputs(K, 1)
         W = W.to(dev)
         codes = torch.empty((K, K // 16), dtype=torch.int32, device=dev)
         alpha = torch.empty((K,), dtype=torch.float32, device=dev)
-        g, ev = _rotating_graph([lambda: tbn.tbn_quantize_pack(W, codes, alpha)], stream, dev)
+        g, ev = capture(lambda: tbn.tbn_quantize_pack(W, codes, alpha), stream, dev)
         for _ in range(max(3, args.warmup)):
             g.replay()
         torch.cuda.synchronize(dev)
-        ms = timed_replays(g, stream, flush, ev, max(5, args.steps // 10), dev)
+        ms = timed_replays(g, stream, flush, ev, reps)
         t = float(np.median(ms)) * 1e-3
         byts = K * K * 4.25 + 4 * K
         sweep.append({"K": K, "n": K, "us": round(t * 1e6, 2), "gbs": round(byts / t / 1e9, 1),
                       "frac_hbm": round(byts / t / 1e9 / hbm, 4)})
-        del W, codes, alpha
+        del W, codes, alpha, g
         torch.cuda.empty_cache()
     clocks = sampler.stop(t0, time.time())
     head = sweep[-1]
@@ -512,25 +617,7 @@ def run_quantize(args, rank, world, local_rank):
             "sweep": sweep, "clocks": clocks}
 
 
-# ------------------------------------------------------------------ CPU oracle
-def oracle_forward_one_image(orc, x_img_nchw_f32, Ws, specs):
-    """Re-quantize every layer and run one image through the stack on the CPU
-    oracle (Eq. 3, Eq. 5, Eq. 1 + ReLU + max pool)."""
-    h = x_img_nchw_f32[None]
-    flops = 0
-    for W, s in zip(Ws, specs):
-        K = W.shape[0]
-        wt, al = orc.quantize(W.reshape(K, -1))
-        y, _ = orc.conv2d_nchw(h, wt.reshape(W.shape), al, (s.stride, s.stride),
-                               (s.pad, s.pad))
-        flops += 2 * K * y.shape[2] * y.shape[3] * s.C * s.R * s.S
-        y = orc.epilogue(y, None, relu=s.relu)
-        if s.pool is not None:
-            y = orc.maxpool2d_nchw(y, (s.pool[0],) * 2, (s.pool[1],) * 2)
-        h = y.astype(np.float32)
-    return flops
-
-
+# ------------------------------------------------------------------ backward
 def run_backward(args, rank, world, local_rank):
     """TwoBitBackward for every VGG-small layer: dx (tensor-core forward
     kernels on the transposed filters) and dW^ (CUDA-core fp32 kernel)."""
@@ -613,7 +700,7 @@ def run_backward(args, rank, world, local_rank):
     gflop = sum(L["flops"] for L in layers) / 1e9              # one gradient of every layer
     gflop_data = sum(L["flops"] for L in layers[1:]) / 1e9
     value = (gflop + gflop_data) / ms_all
-    bf16_peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops"]))
+    bf16_peak, which, _ = pick_peak(peaks, clocks)
     filt_tf = gflop / ms_filt
     return {"metric": "TBN TwoBitBackward TFLOP/s (VGG-small b128, input + filter gradients)",
             "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": 1, "steps": reps,
@@ -631,7 +718,7 @@ def run_backward(args, rank, world, local_rank):
                          "kernel": "bwd_filter_tc_kernel (tcgen05 M128 N128 bf16, accumulator "
                                    "in tensor memory, cp.async ring; c1: bwd_filter_kernel on "
                                    "mma.sync), 6 launches + slice reductions",
-                         "peak_kind": "%s bf16 dense, sustained" % peak_kind,
+                         "peak_kind": "%s bf16 dense, %s" % (peak_kind, which),
                          "input_grad_vs_bf16_peak": round(gflop_data / ms_data / bf16_peak, 4)},
             "clocks": clocks}
 
@@ -669,48 +756,126 @@ def run_cpu_oracle_backward(target_s: float = 10.0, max_s: float = 30.0):
                       "(fp64 C oracle)" % images}
 
 
-def run_cpu_oracle(target_s: float = 10.0, max_s: float = 30.0, max_images: int | None = None):
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_alexnet_one_image(orc, x_img_nchw_f32, Ws, Wfc, specs, fcs):
+    """Re-quantize every layer and run one image through the AlexNet-shaped
+    network on the CPU oracle (Eq. 3, Eq. 5, Eq. 1 + ReLU + max pool, the FC
+    layers of Section 3 on the NHWC flattening); returns its TBN flops."""
+    h = x_img_nchw_f32[None]
+    flops = 0
+    for W, s in zip(Ws, specs):
+        K = W.shape[0]
+        wt, al = orc.quantize(W.reshape(K, -1))
+        y, _ = orc.conv2d_nchw(h, wt.reshape(W.shape), al, (s.stride,) * 2, (s.pad,) * 2)
+        flops += 2 * K * y.shape[2] * y.shape[3] * s.C * s.R * s.S
+        y = orc.epilogue(y, None, relu=s.relu)
+        if s.pool is not None:
+            y = orc.maxpool2d_nchw(y, (s.pool[0],) * 2, (s.pool[1],) * 2)
+        h = y.astype(np.float32)
+    v = np.ascontiguousarray(h.transpose(0, 2, 3, 1).reshape(1, -1))
+    for W, (kin, kout, relu) in zip(Wfc, fcs):
+        wt, al = orc.quantize(W)
+        y, _ = orc.linear(v, wt, al)
+        flops += 2 * kin * kout
+        v = orc.epilogue(y, None, relu=relu).astype(np.float32)
+    return flops
+
+
+def run_cpu_oracle(target_s: float = 10.0, max_images: int | None = None, threads=None):
+    """The oracle as it stands on the host cores: whole images of the AlexNet
+    b256 batch, each through re-quantization of all eight layers + the
+    network; returns TFLOP/s over the sample."""
     import oracle
     from paper_1701_00485_gb300 import inputs
     orc = oracle.default()
-    x, Ws = inputs.vgg_small_inputs(1)
-    specs = inputs.VGG_SMALL["convs"]
+    cores = orc.num_threads() if threads is None else threads
+    if threads is not None:
+        orc.set_num_threads(threads)
+    x, Ws, Wfc = inputs.alexnet_inputs(2, batch=8)
+    specs, fcs = inputs.ALEXNET["convs"], inputs.ALEXNET["fcs"]
     xf = x.float().numpy()
     Wn = [W.numpy() for W in Ws]
+    Wfn = [W.numpy() for W in Wfc]
     t0 = time.time()
-    flops = 0
-    images = 0
-    while True:
-        flops += oracle_forward_one_image(orc, xf[images % x.shape[0]], Wn, specs)
-        images += 1
-        el = time.time() - t0
-        if el >= target_s or el >= max_s or (max_images and images >= max_images):
-            break
+    flops, images = 0, 0
+    try:
+        while True:
+            flops += oracle_alexnet_one_image(orc, xf[images % xf.shape[0]], Wn, Wfn, specs, fcs)
+            images += 1
+            el = time.time() - t0
+            if el >= target_s or (max_images and images >= max_images):
+                break
+    finally:
+        if threads is not None:
+            orc.set_num_threads(os.cpu_count() or 1)
     el = time.time() - t0
-    return {"value": flops / el / 1e12, "unit": "TFLOP/s", "cores": orc.num_threads(),
-            "kind": "oracle", "images": images, "seconds": round(el, 3),
-            "images_per_s": images / el,
-            "sample": "%d image(s) of the VGG-small b128 batch, each through re-quantization "
-                      "of all six layers + six convolutions + ReLU/pool glue (fp64 C oracle)"
-                      % images}
+    return {"value": flops / el / 1e12, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+            "images": images, "seconds": round(el, 3), "images_per_s": images / el,
+            "sample": "%d image(s) of the AlexNet b256 batch, each through re-quantization of "
+                      "all eight layers + five convolutions + ReLU/pool glue + three FC layers "
+                      "(fp64 C oracle, %d thread(s))" % (images, cores)}
+
+
+def cpu_baseline_line():
+    """All-core sample (about 10 s) and a single-thread image."""
+    allc = run_cpu_oracle(target_s=10.0)
+    one = run_cpu_oracle(target_s=0.0, max_images=1, threads=1)
+    line = {k: allc[k] for k in ("value", "unit", "cores", "kind", "sample")}
+    line["images_per_s"] = round(allc["images_per_s"], 4)
+    line["single_thread"] = {"value": one["value"], "unit": "TFLOP/s", "cores": 1,
+                             "seconds_per_image": one["seconds"]}
+    return line
+
+
+def reference_arm(args, rank):
+    """The reference arm: the CPU oracle on the AlexNet workload, one image of
+    the batch per step (plus its re-quantization), on the host cores."""
+    if rank != 0:
+        return 0
+    per_step, cb = [], None
+    for _ in range(max(1, args.warmup)):
+        run_cpu_oracle(target_s=0.0, max_images=1)
+    for _ in range(args.steps):
+        cb = run_cpu_oracle(target_s=0.0, max_images=1)
+        per_step.append(cb["seconds"])
+    total = float(np.sum(per_step))
+    img_flops = cb["value"] * 1e12 * cb["seconds"]
+    value = img_flops * args.steps / total / 1e12
+    line = {"impl": "reference", "metric": WORKLOADS["alexnet"][1], "value": value,
+            "unit": "TFLOP/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": total / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded N(0,1) input, He-normal weights)",
+            "config": {"workload": "alexnet_b256", "global_batch": 256, "image": [3, 227, 227],
+                       "step_sample": "1 image of the 256-image batch per step"},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cb["cores"],
+                             "kind": "oracle",
+                             "sample": "1 image per step through re-quantization + five "
+                                       "convolutions + glue + three FC layers"},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
 
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["vgg_small", "gemv", "quantize", "backward"],
-                    default="vgg_small")
+    ap.add_argument("--workload", choices=["alexnet", "vgg_small", "resnet18", "lenet", "gemv",
+                                           "quantize", "backward"], default="alexnet")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="only the headline workload (no VGG/ResNet/LeNet/GEMV/quantizer keys)")
     ap.add_argument("--gemv-sizes", type=int, nargs="+", default=[4096, 8192, 16384],
                     help="K_out = K_in of the GEMV workload")
     ap.add_argument("--gemv-batches", type=int, nargs="+", default=[1, 8])
     ap.add_argument("--quant-sizes", type=int, nargs="+", default=[8192, 16384],
                     help="square fp32 matrices of the quantize workload")
-    ap.add_argument("--l2-flush", choices=["write", "write+read"], default="write",
-                    help="L2 eviction between timed steps (write+read also drains the dirty lines)")
     ap.add_argument("--min-warmup-s", type=float, default=1.0,
                     help="keep replaying warm-up steps for at least this long (clock settling)")
     args = ap.parse_args()
@@ -720,51 +885,48 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
 
     if args.impl == "reference":
-        # the reference arm is the CPU oracle; rank 0 alone runs it
-        if rank != 0:
-            return 0
-        per_step = []
-        cb = None
-        for _ in range(max(1, args.warmup)):
-            run_cpu_oracle(target_s=0.0, max_images=1)
-        for _ in range(args.steps):
-            cb = run_cpu_oracle(target_s=0.0, max_images=1)
-            per_step.append(cb["seconds"])
-        total = float(np.sum(per_step))
-        img_flops = cb["value"] * 1e12 * cb["seconds"]
-        value = img_flops * args.steps / total / 1e12
-        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
-                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": total / args.steps * 1e3, "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-                "data": "synthetic (seeded N(0,1) input, He-normal weights)",
-                "config": {"workload": WORKLOAD, "global_batch": 128, "image": [3, 32, 32],
-                           "step_sample": "1 image of the 128-image batch per step"},
-                "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cb["cores"],
-                                 "kind": "oracle",
-                                 "sample": "1 image per step through re-quantization + six "
-                                           "convolutions + glue"},
-                "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
-                        "d2h_bytes_per_step": 0}}
-        print(json.dumps(line))
-        return 0
+        return reference_arm(args, rank)
 
     if world > 1:
         torch.distributed.init_process_group("nccl")
     # the CPU baseline forks no workers after CUDA init: run it first
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "vgg_small":
-        cpu = run_cpu_oracle()
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "alexnet":
+        cpu = cpu_baseline_line()
     elif rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "backward":
         cpu = run_cpu_oracle_backward()
-    runner = {"vgg_small": run_vgg, "gemv": run_gemv, "quantize": run_quantize,
-              "backward": run_backward}[args.workload]
-    res = runner(args, rank, world, local_rank)
+    if args.workload in WORKLOADS:
+        res = run_network(args, rank, world, local_rank, args.workload)
+        if args.workload == "alexnet" and not args.no_extras and world == 1:
+            k = min(args.steps, 20)
+            extras = {}
+            for name in ("vgg_small", "resnet18"):
+                r = run_network(args, rank, world, local_rank, name, full=False, steps=k,
+                                warmup=min(args.warmup, 5))
+                extras[name] = {kk: r[kk] for kk in ("value", "unit", "ms_per_step",
+                                                     "images_per_s", "inference_form",
+                                                     "requantize_us", "roofline", "clocks")}
+                if name == "resnet18":
+                    extras[name]["note"] = "value: 434.06 GFLOP of two-bit convolutions over " \
+                                           "the whole step (fp32 stem and FC included in the " \
+                                           "time); roofline: the 19 two-bit convolutions alone"
+                torch.cuda.empty_cache()
+            extras["lenet"] = run_lenet(args, local_rank)
+            q = run_quantize(args, rank, world, local_rank, reps=5)
+            extras["quantize"] = {"sweep": q["sweep"], "clocks": q["clocks"]}
+            gm = run_gemv(args, rank, world, local_rank, reps=3)
+            extras["gemv"] = {"sweep": gm["sweep"], "clocks": gm["clocks"]}
+            res["extras"] = extras
+    else:
+        runner = {"lenet": None, "gemv": run_gemv, "quantize": run_quantize,
+                  "backward": run_backward}[args.workload]
+        if runner is None:
+            res = dict(run_lenet(args, local_rank), n_gpus=1)
+        else:
+            res = runner(args, rank, world, local_rank)
     if rank == 0:
         if cpu is not None:
-            res["cpu_baseline"] = {k: cpu[k] for k in ("value", "unit", "cores", "kind", "sample")}
-            if "images_per_s" in cpu:
-                res["cpu_baseline"]["images_per_s"] = round(cpu["images_per_s"], 4)
+            res["cpu_baseline"] = cpu
         print(json.dumps(res))
     if world > 1:
         torch.distributed.destroy_process_group()

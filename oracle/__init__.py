@@ -126,6 +126,7 @@ class Oracle:
             "orc_avgpool_global_nchw": ([P, I, I, I, I, P], None),
             "orc_dense_linear": ([P, I, I, P, I, P, P], None),
             "orc_num_threads": ([], ctypes.c_int),
+            "orc_set_num_threads": ([ctypes.c_int], None),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -135,6 +136,10 @@ class Oracle:
 
     def num_threads(self) -> int:
         return int(self.lib.orc_num_threads())
+
+    def set_num_threads(self, n: int) -> None:
+        """Threads of the parallel loops (timing the oracle on one core)."""
+        self.lib.orc_set_num_threads(int(n))
 
     def discretize_one(self, w: float) -> int:
         """Eq. 3 for a single weight (evaluated on the value widened to double)."""

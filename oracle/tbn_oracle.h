@@ -161,6 +161,10 @@ void orc_dense_linear(const float *x, int64_t B, int64_t Kin, const float *w, in
 /* Threads the parallel loops use (1 without OpenMP). */
 int orc_num_threads(void);
 
+/* Set the thread count of the parallel loops (n >= 1; no effect without
+ * OpenMP).  Used to time the oracle single-threaded beside all cores. */
+void orc_set_num_threads(int n);
+
 #ifdef __cplusplus
 }
 #endif

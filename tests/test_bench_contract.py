@@ -27,8 +27,8 @@ def test_reference_arm_prints_one_contract_line():
     assert len(lines) == 1
     d = json.loads(lines[0])
     assert d["impl"] == "reference"
-    assert d["metric"] == bench.METRIC and d["unit"] == "TFLOP/s"
-    assert d["config"]["workload"] == bench.WORKLOAD
+    assert d["metric"] == bench.WORKLOADS["alexnet"][1] and d["unit"] == "TFLOP/s"
+    assert d["config"]["workload"] == bench.WORKLOADS["alexnet"][0]
     assert d["higher_is_better"] is True and d["steps"] == 2 and d["warmup"] == 3
     assert d["value"] > 0 and d["ms_per_step"] > 0 and d["n_gpus"] == 1
     for key in ("scaling", "vs_baseline", "dtype", "data"):
