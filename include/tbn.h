@@ -309,8 +309,10 @@ tbn_status tbn_conv2d_bwd_filter(const void *x, const void *dy, int64_t N, int64
  * residual [B][K_out] of y's dtype; pool is invalid here).
  * Equivalent to tbn_linear_fwd_ws with no workspace: bf16 x with B <= 8,
  * K_in % 64 == 0 and 16-byte aligned x and codes runs the tensor-core GEMV;
- * fp32 x with B == 1, K_in <= 512 (K_in % 64 == 0) the table-lookup GEMV;
- * every other shape a 1x1 convolution. */
+ * fp32 x with B == 1 and K_in % 64 == 0 runs only on the table-lookup GEMV,
+ * which needs no workspace for K_in <= 512 -- larger layers return
+ * TBN_ERR_UNSUPPORTED here (use tbn_linear_fwd_ws or tbn_linear_fwd_noalloc);
+ * every other shape runs as a 1x1 convolution (tensor cores for bf16 x). */
 tbn_status tbn_linear_fwd(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
                           const uint32_t *codes, const float *alpha, int64_t K_out, void *y,
                           tbn_dtype ydt, const tbn_epilogue *epi, tbn_stream stream);
@@ -332,7 +334,9 @@ size_t tbn_linear_workspace_bytes(tbn_dtype xdt, int64_t B, int64_t K_in, int64_
  * aligned, contents on entry irrelevant), and a second kernel on `stream`
  * adds them in chunk order, so results are bitwise reproducible.  Calls
  * that may run concurrently must not share a workspace.  Otherwise the call
- * behaves as tbn_linear_fwd and does not touch `workspace` (NULL allowed). */
+ * behaves as tbn_linear_fwd and does not touch `workspace` (NULL allowed);
+ * a batch-1 fp32 layer of the table kernel's shape with a smaller workspace
+ * returns TBN_ERR_UNSUPPORTED (16-byte misaligned codes: TBN_ERR_MISALIGNED). */
 tbn_status tbn_linear_fwd_ws(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
                              const uint32_t *codes, const float *alpha, int64_t K_out, void *y,
                              tbn_dtype ydt, const tbn_epilogue *epi, void *workspace,

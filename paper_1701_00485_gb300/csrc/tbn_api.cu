@@ -364,8 +364,19 @@ tbn_status tbn_linear_fwd_ws(const void* x, tbn_dtype xdt, int64_t B, int64_t K_
   if (st != TBN_OK) return st;
   const int relu = epi ? epi->relu : 0;
   const void* residual = epi ? epi->residual : nullptr;
-  if (linear_uses_table(xdt, B, K_in, K_out, codes) &&
-      workspace_bytes >= gemv_lut_workspace_bytes(K_in, K_out)) {
+  if (gemv_lut_shape_reason(xdt, B, K_in, K_out)[0] == '\0') {
+    // a batch-1 fp32 layer runs on the table-lookup GEMV only: the CUDA-core
+    // 1x1 convolution it would fall back to reads the codes about a hundred
+    // times slower than the table kernel, so that path is refused
+    const size_t need = gemv_lut_workspace_bytes(K_in, K_out);
+    if (workspace_bytes < need || (need > 0 && workspace == nullptr))
+      return fail(TBN_ERR_UNSUPPORTED,
+                  "linear: fp32 activations at batch 1 run on the table-lookup GEMV, which needs "
+                  "%zu bytes of workspace for this shape: call tbn_linear_fwd_ws with "
+                  "tbn_linear_workspace_bytes(...) bytes, or tbn_linear_fwd_noalloc",
+                  need);
+    if (!linear_uses_table(xdt, B, K_in, K_out, codes))
+      return fail(TBN_ERR_MISALIGNED, "linear: the table-lookup GEMV needs 16-byte aligned codes");
     return launch_gemv_lut(x, K_in, codes, alpha, K_out, y, ydt, relu, residual, workspace,
                            workspace_bytes, as_stream(stream));
   }

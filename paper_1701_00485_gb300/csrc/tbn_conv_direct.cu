@@ -277,6 +277,9 @@ __global__ void __launch_bounds__(256) maxpool_nhwc_bf16x8_kernel(
 // consecutive 16-byte vectors of each tap; the max is taken on bf16 pairs
 // (exact: max of two bf16 values is one of them).  Taps in the padding are
 // skipped.
+// kK > 0: a kK x kK window, all of its loads issued before the first max
+// (taps in the padding load nothing and count as -infinity).
+template <int kK>
 __global__ void __launch_bounds__(256) maxpool_row_bf16x8_kernel(
     const uint4* __restrict__ x, int H, int W, int C8, int kh, int kw, int sh, int sw, int ph,
     int pw, int Ho, int Wo, uint4* __restrict__ y) {
@@ -285,6 +288,33 @@ __global__ void __launch_bounds__(256) maxpool_row_bf16x8_kernel(
   const uint4* xb = x + static_cast<int64_t>(b) * H * W * C8;
   uint4* yrow = y + (static_cast<int64_t>(b) * Ho + ho) * Wo * C8;
   const int h_lo = max(0, ho * sh - ph), h_hi = min(H, ho * sh - ph + kh);
+  if constexpr (kK > 0) {
+    const uint4 ninf4 = make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+    for (int i = threadIdx.x; i < items; i += 256) {
+      const int wo = i / C8, c = i - wo * C8;
+      const int h0 = ho * sh - ph, w0 = wo * sw - pw;
+      uint4 t[kK * kK];
+#pragma unroll
+      for (int u = 0; u < kK; ++u)
+#pragma unroll
+        for (int v = 0; v < kK; ++v) {
+          const int h = h0 + u, w = w0 + v;
+          t[u * kK + v] = (h >= 0 && h < H && w >= 0 && w < W)
+                              ? __ldg(xb + (static_cast<int64_t>(h) * W + w) * C8 + c)
+                              : ninf4;
+        }
+      __nv_bfloat162 m[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) m[e] = reinterpret_cast<const __nv_bfloat162*>(&t[0])[e];
+#pragma unroll
+      for (int j = 1; j < kK * kK; ++j)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          m[e] = __hmax2(m[e], reinterpret_cast<const __nv_bfloat162*>(&t[j])[e]);
+      yrow[i] = *reinterpret_cast<const uint4*>(m);
+    }
+    return;
+  }
   for (int i = threadIdx.x; i < items; i += 256) {
     const int wo = i / C8, c = i - wo * C8;
     const int w_lo = max(0, wo * sw - pw), w_hi = min(W, wo * sw - pw + kw);
@@ -412,9 +442,18 @@ tbn_status launch_maxpool_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t H
   const int64_t Ho = (H + 2 * ph - kh) / sh + 1, Wo = (W + 2 * pw - kw) / sw + 1;
   if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16) &&
       N * Ho < (int64_t(1) << 31) && H * W * C < (int64_t(1) << 31)) {
-    maxpool_row_bf16x8_kernel<<<static_cast<unsigned>(N * Ho), 256, 0, s>>>(
-        static_cast<const uint4*>(x), (int)H, (int)W, (int)(C / 8), (int)kh, (int)kw, (int)sh,
-        (int)sw, (int)ph, (int)pw, (int)Ho, (int)Wo, static_cast<uint4*>(y));
+    if (kh == 3 && kw == 3)
+      maxpool_row_bf16x8_kernel<3><<<static_cast<unsigned>(N * Ho), 256, 0, s>>>(
+          static_cast<const uint4*>(x), (int)H, (int)W, (int)(C / 8), (int)kh, (int)kw, (int)sh,
+          (int)sw, (int)ph, (int)pw, (int)Ho, (int)Wo, static_cast<uint4*>(y));
+    else if (kh == 2 && kw == 2)
+      maxpool_row_bf16x8_kernel<2><<<static_cast<unsigned>(N * Ho), 256, 0, s>>>(
+          static_cast<const uint4*>(x), (int)H, (int)W, (int)(C / 8), (int)kh, (int)kw, (int)sh,
+          (int)sw, (int)ph, (int)pw, (int)Ho, (int)Wo, static_cast<uint4*>(y));
+    else
+      maxpool_row_bf16x8_kernel<0><<<static_cast<unsigned>(N * Ho), 256, 0, s>>>(
+          static_cast<const uint4*>(x), (int)H, (int)W, (int)(C / 8), (int)kh, (int)kw, (int)sh,
+          (int)sw, (int)ph, (int)pw, (int)Ho, (int)Wo, static_cast<uint4*>(y));
   } else if (dt == TBN_BF16 && C % 8 == 0 && is_aligned(x, 16) && is_aligned(y, 16)) {
     const int64_t total = N * Ho * Wo * (C / 8);
     maxpool_nhwc_bf16x8_kernel<<<(unsigned)grid_for(total), 256, 0, s>>>(

@@ -1036,6 +1036,55 @@ int ceil_div(int64_t a, int64_t b) { return static_cast<int>((a + b - 1) / b); }
 bool use_tma(const ConvProblem& p) { return p.C % (kBK / 2) == 0 && p.sh <= 2 && p.sw <= 2; }
 bool use_ch32(const ConvProblem& p) { return p.C % kBK != 0; }
 
+// Cost of a tile plan in SM cycles (a model, used only to compare plans):
+// the persistent CTAs take the tiles in waves; a tile costs per K block the
+// larger of the weight decode (about 320 cycles for 128 filters x 64 codes,
+// independent of the pixel count) and the MMAs (about 684 cycles at 256
+// pixels), plus a fixed cost for the pipeline fill and the epilogue.
+int64_t plan_cost(const ConvProblem& p, const TilePlan& t, int sms) {
+  const int64_t kblocks = (p.C * p.R * p.S + kBK - 1) / kBK;
+  const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n *
+                        ((p.K + kBM - 1) / kBM);
+  const int64_t waves = (tiles + sms - 1) / sms;
+  const int64_t mma = 684 * t.tile_n / kMaxTileN;
+  return waves * (kblocks * std::max<int64_t>(320, mma) + 2000);
+}
+
+// A fully-connected layer whose default plan leaves SMs idle (at batch 256:
+// 256 images per tile, K_out / 128 tiles) gets tiles of fewer images when
+// the cost model says the extra CTAs outweigh the longer decode per pixel.
+TilePlan shrink_for_occupancy(const ConvProblem& p, TilePlan t) {
+  const int sms = device_sm_count();
+  const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n *
+                        ((p.K + kBM - 1) / kBM);
+  // only fully-connected shapes (a 1x1 image): for convolutions the model
+  // misjudged the smaller tiles (ResNet-18's 7x7 layers ran slower)
+  if (tiles >= sms || t.tiles_q != 1 || p.P != 1 || p.Q != 1) return t;
+  TilePlan best = t;
+  int64_t best_cost = plan_cost(p, t, sms);
+  TilePlan c = t;
+  while (true) {
+    if (c.bn > 1) {
+      c.bn = (c.bn + 1) / 2;
+    } else if (c.bh > (p.pool ? 2 : 1)) {
+      c.bh = p.pool ? std::max(2, (c.bh / 2) & ~1) : (c.bh + 1) / 2;
+    } else {
+      break;
+    }
+    c.tiles_p = ceil_div(p.P, c.bh);
+    c.tiles_n = ceil_div(p.N, c.bn);
+    c.T = c.bw * c.bh * c.bn;
+    c.tile_n = ((c.T + 15) / 16) * 16;
+    if (c.tile_n < 32) break;
+    const int64_t cost = plan_cost(p, c, sms);
+    if (cost < best_cost) {
+      best = c;
+      best_cost = cost;
+    }
+  }
+  return best;
+}
+
 // Output pixels per tile: whole rows of the output (so one TMA box per tap
 // covers the tile), balanced so the last tile along each axis is not a
 // sliver, at most 256 pixels.  With a fused 2x2 pool a tile holds whole
@@ -1069,7 +1118,7 @@ TilePlan plan_tiles(const ConvProblem& p) {
   t.tiles_n = ceil_div(p.N, t.bn);
   t.T = t.bw * t.bh * t.bn;
   t.tile_n = ((t.T + 15) / 16) * 16;
-  return t;
+  return shrink_for_occupancy(p, t);
 }
 
 int pool_width(const ConvProblem& p, const TilePlan& t) {

@@ -6,8 +6,8 @@
 // x * w products are rounded to fp32 and accumulated in fp32, which is what
 // "kept in fp32" means for these layers.
 //
-// Dense convolution: a CTA computes a tile of 4 output rows x 32 output
-// columns of one image for 64 filters.  Per chunk of input channels it
+// Dense convolution: a persistent CTA takes tiles of 4 output rows x 32
+// output columns of one image for 64 filters.  Per chunk of input channels it
 // stages the fp32 weights [tap][64 filters] and the input patch the tile
 // reads (zero outside the image) in shared memory; each warp owns 8
 // filters (its weight reads are broadcasts), each lane one output column of
@@ -52,8 +52,12 @@ struct DenseConvArgs {
 };
 
 // kXNhwc: x is [N][H][W][C] (else [N][C][H][W]); kYNhwc: y is [N][P][Q][K]
-// (else [N][K][P][Q]).
-template <typename TX, typename TY, bool kXNhwc, bool kYNhwc>
+// (else [N][K][P][Q]).  kR, kS, kSH, kSW > 0 fix the kernel extent and
+// stride at compile time (the 7x7/2 first layer of ResNet-18): the tap loop
+// unrolls and every shared-memory address is an immediate offset; 0 = taken
+// from the arguments.
+template <typename TX, typename TY, bool kXNhwc, bool kYNhwc, int kR = 0, int kS = 0,
+          int kSH = 0, int kSW = 0>
 __global__ void __launch_bounds__(kDcThreads) dense_conv_kernel(const DenseConvArgs a) {
   extern __shared__ __align__(16) float dsm[];
   const int RS = a.R * a.S;
@@ -61,99 +65,123 @@ __global__ void __launch_bounds__(kDcThreads) dense_conv_kernel(const DenseConvA
   float* s_x = dsm + static_cast<size_t>(a.cc) * RS * kDcFilt;   // [cc][prows][pcols]
   const TX* __restrict__ x = static_cast<const TX*>(a.x);
 
-  int t = blockIdx.x;
-  const int tq = t % a.tiles_q;
-  t /= a.tiles_q;
-  const int tp = t % a.tiles_p;
-  const int b = t / a.tiles_p;
   const int k0 = blockIdx.y * kDcFilt;
-  const int q0 = tq * kDcCols, p0 = tp * kDcRows;
-  const int h_base = p0 * a.sh - a.ph, w_base = q0 * a.sw - a.pw;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int f0 = warp * 8;
-
-  float acc[kDcRows][8];
-#pragma unroll
-  for (int i = 0; i < kDcRows; ++i)
-#pragma unroll
-    for (int f = 0; f < 8; ++f) acc[i][f] = 0.0f;
-
+  const int R = kR > 0 ? kR : a.R, S = kS > 0 ? kS : a.S;
+  const int sh = kSH > 0 ? kSH : a.sh, sw = kSW > 0 ? kSW : a.sw;
   const int patch = a.prows * a.pcols;
-  for (int c0 = 0; c0 < a.C; c0 += a.cc) {
-    const int cn = min(a.cc, a.C - c0);
-    __syncthreads();
-    // weights of this channel chunk, tap-major: s_w[(c * R + r) * S + s][f]
+  const int ntiles = a.N * a.tiles_p * a.tiles_q;
+  // column stride 2 (compile time): each patch row keeps its even columns,
+  // then its odd ones, so that for a tap the 32 lanes (output columns) read
+  // 32 consecutive words instead of every other one (no bank conflicts)
+  constexpr bool kSplit = kSW == 2;
+  const int half = (a.pcols + 1) / 2;
+  // all input channels in one chunk: the CTA's weights are staged once and
+  // serve every tile it takes (persistent grid)
+  const bool w_once = a.cc >= a.C;
+  auto load_weights = [&](int c0, int cn) {
     for (int i = threadIdx.x; i < cn * RS * kDcFilt; i += kDcThreads) {
       const int f = i % kDcFilt, tap = i / kDcFilt;
       const int k = k0 + f;
       s_w[i] = k < a.K ? __ldg(a.w + (static_cast<int64_t>(k) * a.C + c0) * RS + tap) : 0.0f;
     }
-    // input patch of this channel chunk, zero outside the image
-    for (int i = threadIdx.x; i < cn * patch; i += kDcThreads) {
-      const int c = i / patch, rem = i - c * patch;
-      const int pr = rem / a.pcols, pc = rem - pr * a.pcols;
-      const int h = h_base + pr, w = w_base + pc;
-      float v = 0.0f;
-      if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
-        const int64_t o = kXNhwc
-                              ? ((static_cast<int64_t>(b) * a.H + h) * a.W + w) * a.C + c0 + c
-                              : ((static_cast<int64_t>(b) * a.C + c0 + c) * a.H + h) * a.W + w;
-        v = ld_f32<TX>(x, o);
-      }
-      s_x[i] = v;
-    }
-    __syncthreads();
-    for (int c = 0; c < cn; ++c) {
-      const float* xc = s_x + c * patch + lane * a.sw;
-      for (int r = 0; r < a.R; ++r) {
-        const float* xr = xc + r * a.pcols;
-        const float* wr = s_w + ((c * a.R + r) * a.S) * kDcFilt + f0;
-        for (int s = 0; s < a.S; ++s) {
-          const float4 w0 = *reinterpret_cast<const float4*>(wr + s * kDcFilt);
-          const float4 w1 = *reinterpret_cast<const float4*>(wr + s * kDcFilt + 4);
+  };
+  if (w_once) load_weights(0, a.C);
+  TY* __restrict__ y = static_cast<TY*>(a.y);
+
+  for (int t0 = blockIdx.x; t0 < ntiles; t0 += gridDim.x) {
+    int t = t0;
+    const int tq = t % a.tiles_q;
+    t /= a.tiles_q;
+    const int tp = t % a.tiles_p;
+    const int b = t / a.tiles_p;
+    const int q0 = tq * kDcCols, p0 = tp * kDcRows;
+    const int h_base = p0 * sh - a.ph, w_base = q0 * sw - a.pw;
+
+    float acc[kDcRows][8];
 #pragma unroll
-          for (int i = 0; i < kDcRows; ++i) {
-            const float xv = xr[i * a.sh * a.pcols + s];
-            acc[i][0] = fmaf(xv, w0.x, acc[i][0]);
-            acc[i][1] = fmaf(xv, w0.y, acc[i][1]);
-            acc[i][2] = fmaf(xv, w0.z, acc[i][2]);
-            acc[i][3] = fmaf(xv, w0.w, acc[i][3]);
-            acc[i][4] = fmaf(xv, w1.x, acc[i][4]);
-            acc[i][5] = fmaf(xv, w1.y, acc[i][5]);
-            acc[i][6] = fmaf(xv, w1.z, acc[i][6]);
-            acc[i][7] = fmaf(xv, w1.w, acc[i][7]);
+    for (int i = 0; i < kDcRows; ++i)
+#pragma unroll
+      for (int f = 0; f < 8; ++f) acc[i][f] = 0.0f;
+
+    for (int c0 = 0; c0 < a.C; c0 += a.cc) {
+      const int cn = min(a.cc, a.C - c0);
+      __syncthreads();   // the previous chunk / tile is done with the buffers
+      if (!w_once) load_weights(c0, cn);
+      // input patch of this channel chunk, zero outside the image
+      for (int i = threadIdx.x; i < cn * patch; i += kDcThreads) {
+        const int c = i / patch, rem = i - c * patch;
+        const int pr = rem / a.pcols, pc = rem - pr * a.pcols;
+        const int h = h_base + pr, w = w_base + pc;
+        float v = 0.0f;
+        if (h >= 0 && h < a.H && w >= 0 && w < a.W) {
+          const int64_t o = kXNhwc
+                                ? ((static_cast<int64_t>(b) * a.H + h) * a.W + w) * a.C + c0 + c
+                                : ((static_cast<int64_t>(b) * a.C + c0 + c) * a.H + h) * a.W + w;
+          v = ld_f32<TX>(x, o);
+        }
+        if constexpr (kSplit)
+          s_x[c * patch + pr * a.pcols + ((pc & 1) ? half + (pc >> 1) : (pc >> 1))] = v;
+        else
+          s_x[i] = v;
+      }
+      __syncthreads();
+      for (int c = 0; c < cn; ++c) {
+        const float* xc = s_x + c * patch + (kSplit ? lane : lane * sw);
+#pragma unroll 1
+        for (int r = 0; r < R; ++r) {
+          const float* xr = xc + r * a.pcols;
+          const float* wr = s_w + ((c * R + r) * S) * kDcFilt + f0;
+#pragma unroll
+          for (int s = 0; s < S; ++s) {
+            const float4 w0 = *reinterpret_cast<const float4*>(wr + s * kDcFilt);
+            const float4 w1 = *reinterpret_cast<const float4*>(wr + s * kDcFilt + 4);
+#pragma unroll
+            for (int i = 0; i < kDcRows; ++i) {
+              const float xv =
+                  kSplit ? xr[i * sh * a.pcols + (s & 1) * half + (s >> 1)] : xr[i * sh * a.pcols + s];
+              acc[i][0] = fmaf(xv, w0.x, acc[i][0]);
+              acc[i][1] = fmaf(xv, w0.y, acc[i][1]);
+              acc[i][2] = fmaf(xv, w0.z, acc[i][2]);
+              acc[i][3] = fmaf(xv, w0.w, acc[i][3]);
+              acc[i][4] = fmaf(xv, w1.x, acc[i][4]);
+              acc[i][5] = fmaf(xv, w1.y, acc[i][5]);
+              acc[i][6] = fmaf(xv, w1.z, acc[i][6]);
+              acc[i][7] = fmaf(xv, w1.w, acc[i][7]);
+            }
           }
         }
       }
     }
-  }
 
-  TY* __restrict__ y = static_cast<TY*>(a.y);
-  const int q = q0 + lane;
-  if (q >= a.Q) return;
+    const int q = q0 + lane;
+    if (q >= a.Q) continue;
 #pragma unroll
-  for (int i = 0; i < kDcRows; ++i) {
-    const int p = p0 + i;
-    if (p >= a.P) continue;
+    for (int i = 0; i < kDcRows; ++i) {
+      const int p = p0 + i;
+      if (p >= a.P) continue;
 #pragma unroll
-    for (int f = 0; f < 8; ++f) {
-      const int k = k0 + f0 + f;
-      if (k >= a.K) continue;
-      float v = acc[i][f];
-      if (a.relu) v = fmaxf(v, 0.0f);
-      const int64_t o = kYNhwc ? ((static_cast<int64_t>(b) * a.P + p) * a.Q + q) * a.K + k
-                               : ((static_cast<int64_t>(b) * a.K + k) * a.P + p) * a.Q + q;
-      if constexpr (sizeof(TY) == 2)
-        y[o] = __float2bfloat16_rn(v);
-      else
-        y[o] = v;
+      for (int f = 0; f < 8; ++f) {
+        const int k = k0 + f0 + f;
+        if (k >= a.K) continue;
+        float v = acc[i][f];
+        if (a.relu) v = fmaxf(v, 0.0f);
+        const int64_t o = kYNhwc ? ((static_cast<int64_t>(b) * a.P + p) * a.Q + q) * a.K + k
+                                 : ((static_cast<int64_t>(b) * a.K + k) * a.P + p) * a.Q + q;
+        if constexpr (sizeof(TY) == 2)
+          y[o] = __float2bfloat16_rn(v);
+        else
+          y[o] = v;
+      }
     }
   }
 }
 
-template <typename TX, typename TY, bool kXNhwc, bool kYNhwc>
+template <typename TX, typename TY, bool kXNhwc, bool kYNhwc, int kR = 0, int kS = 0,
+          int kSH = 0, int kSW = 0>
 tbn_status launch_dense_conv_t(const DenseConvArgs& a, size_t smem, cudaStream_t s) {
-  auto kern = dense_conv_kernel<TX, TY, kXNhwc, kYNhwc>;
+  auto kern = dense_conv_kernel<TX, TY, kXNhwc, kYNhwc, kR, kS, kSH, kSW>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -164,13 +192,23 @@ tbn_status launch_dense_conv_t(const DenseConvArgs& a, size_t smem, cudaStream_t
   const int64_t gy = (a.K + kDcFilt - 1) / kDcFilt;
   if (tiles > 0x7fffffffLL || gy > 65535)
     return fail(TBN_ERR_UNSUPPORTED, "dense conv: grid too large");
-  kern<<<dim3(static_cast<unsigned>(tiles), static_cast<unsigned>(gy)), kDcThreads, smem, s>>>(a);
+  // persistent: as many CTAs as fit at once (the weights are staged once per CTA)
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kDcThreads, smem) !=
+          cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  const int64_t slots = static_cast<int64_t>(device_sm_count()) * per_sm;
+  const int64_t gx = std::max<int64_t>(1, std::min<int64_t>(tiles, (slots + gy - 1) / gy));
+  kern<<<dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy)), kDcThreads, smem, s>>>(a);
   return check_launch("dense_conv_kernel");
 }
 
 template <typename TX, typename TY>
 tbn_status launch_dense_conv_l(const DenseConvArgs& a, size_t smem, bool xn, bool yn,
                                cudaStream_t s) {
+  if (!xn && yn && a.R == 7 && a.S == 7 && a.sh == 2 && a.sw == 2)
+    return launch_dense_conv_t<TX, TY, false, true, 7, 7, 2, 2>(a, smem, s);
   if (xn && yn) return launch_dense_conv_t<TX, TY, true, true>(a, smem, s);
   if (!xn && yn) return launch_dense_conv_t<TX, TY, false, true>(a, smem, s);
   if (!xn && !yn) return launch_dense_conv_t<TX, TY, false, false>(a, smem, s);

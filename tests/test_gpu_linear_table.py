@@ -101,15 +101,30 @@ def test_table_gemv_is_reproducible_and_ignores_stale_workspace():
     assert torch.equal(y1, y2) and torch.equal(y1, y3)
 
 
-def test_small_workspace_falls_back_to_the_convolution():
-    """A workspace smaller than the query asks for is not used: the layer runs
-    as a 1x1 convolution (same results within the bound)."""
+def test_batch1_fp32_without_enough_workspace_is_refused():
+    """A batch-1 fp32 layer of the table kernel's shape runs only there: with
+    a workspace smaller than the query asks for (or none) the call returns
+    TBN_ERR_UNSUPPORTED instead of taking the CUDA-core 1x1 convolution,
+    and launches nothing."""
     g = inputs.generator(8)
     W = inputs.normal((300, 2048), 1.2, g)
-    x = torch.randn(1, 2048, generator=g)
+    codes, alpha = tbn.tbn_quantize_pack(W.cuda())
+    x = torch.randn(1, 2048, generator=g).cuda()
     small = torch.empty(64, dtype=torch.uint8, device="cuda")
-    y, y_orc, bound = run_table(W, x, torch.float32, ws=small)
-    assert_within(y, y_orc, bound, out_bf16=False, what="fallback linear")
+    y = torch.full((1, 300), 7.0, device="cuda")
+    for ws in (small, None):
+        with pytest.raises(tbn.TBNError) as e:
+            tbn.tbn_linear_fwd_ws(x, codes, alpha, 300, ws, out=y)
+        assert e.value.status == tbn.TBN_ERR_UNSUPPORTED
+    with pytest.raises(tbn.TBNError) as e:
+        tbn.tbn_linear_fwd(x, codes, alpha, 300, out=y)
+    assert e.value.status == tbn.TBN_ERR_UNSUPPORTED
+    torch.cuda.synchronize()
+    assert torch.all(y == 7.0)
+    # one chunk (K_in <= 512) needs no workspace
+    x2 = torch.randn(1, 512, generator=g).cuda()
+    c2, a2 = tbn.tbn_quantize_pack(inputs.normal((40, 512), 1.2, g).cuda())
+    tbn.tbn_linear_fwd(x2, c2, a2, 40)
 
 
 @pytest.mark.parametrize("K", inputs.GEMV_SIZES)
