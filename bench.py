@@ -2,7 +2,7 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload alexnet|vgg_small|resnet18|lenet|gemv|quantize|backward]
-                    [--no-extras] [--no-cpu-baseline]
+                    [--no-extras] [--no-cpu-baseline] [--eager-steps K]
 
 Default workload: the AlexNet-shaped TBN network at batch 256 (3x227x227
 bf16 ~ N(0,1); conv 96x11x11/4, 256x5x5/p2, 384x3x3/p1, 384x3x3/p1,
@@ -76,13 +76,13 @@ WORKLOADS = {
     "resnet18": ("resnet18_b128", "TBN conv TFLOP/s (ResNet-18 b128, two-bit convolutions)"),
 }
 
-# DRAM bytes (read + write) per implicit-GEMM launch of the AlexNet step, from
-# the ncu capture summarised in profiles/alexnet_b256_launches.md (batch-32
-# capture scaled to batch 256).  Valid only for the kernel sources it was
+# DRAM bytes (read + write) per implicit-GEMM launch of the AlexNet b256 step,
+# mean over its eight launches, from the full-size ncu capture summarised in
+# profiles/alexnet_b256_launches.md.  Valid only for the kernel sources it was
 # measured on (hash below); otherwise the roofline entry reports null.
 CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
                             "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
-                "sha256_16": None, "bytes_per_launch": None}
+                "sha256_16": "6f5b73eeeb7677d7", "bytes_per_launch": 43.90e6}
 
 
 def measured_traffic(rec):
@@ -878,6 +878,9 @@ def main():
                     help="square fp32 matrices of the quantize workload")
     ap.add_argument("--min-warmup-s", type=float, default=1.0,
                     help="keep replaying warm-up steps for at least this long (clock settling)")
+    ap.add_argument("--eager-steps", type=int, default=0,
+                    help="for profilers: run the network workload's step eagerly this many "
+                         "times (no graphs, no timing, no JSON line) and exit")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -886,6 +889,15 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, rank)
+    if args.eager_steps > 0:
+        import paper_1701_00485_gb300 as tbn
+        torch.cuda.set_device(local_rank)
+        sp = net_spec(args.workload, torch.device("cuda", local_rank))
+        for _ in range(args.eager_steps):
+            sp["step"]()
+        torch.cuda.synchronize()
+        print("eager steps %d, device error word %d" % (args.eager_steps, tbn.tbn_device_error()))
+        return 0
 
     if world > 1:
         torch.distributed.init_process_group("nccl")

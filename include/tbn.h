@@ -26,8 +26,10 @@
  * --------------------------------
  * - Pointers to tensors are DEVICE pointers, allocated and owned by the
  *   caller.  The library allocates no device memory and keeps no state
- *   between calls except the per-device error word (tbn_device_error) and
- *   per-process kernel attributes.
+ *   between calls except the per-device error word (tbn_device_error),
+ *   per-process kernel attributes and the 4 MiB scratch array of
+ *   tbn_linear_fwd_noalloc (one per device and process; calls of that entry
+ *   point that could overlap must be serialized, see its declaration).
  * - One process drives one GPU (run one process per GPU for replicas): the
  *   kernels' shared-memory attributes are set on the device that is current
  *   at a kernel's first launch in the process, so a later launch of a
@@ -154,7 +156,8 @@ const char *tbn_status_string(tbn_status s);
 const char *tbn_last_error(void);
 
 /* Reads and clears the error word of the current device (synchronous:
- * waits for the device's pending work).  Bit 1: a kernel wait timed out;
+ * waits for the device's pending work; the read and the clear are one atomic
+ * step on the device).  Bit 1: a kernel wait timed out;
  * bit 2: a kernel saw a launch shape it could not run.  *flags = 0 when no
  * error was recorded. */
 tbn_status tbn_device_error(uint32_t *flags);
@@ -176,8 +179,10 @@ tbn_status tbn_selftest_wait_timeout(uint32_t limit_us, tbn_stream stream);
  *   codes  [K][tbn_packed_words(n)] uint32 (device, output), 4-byte aligned.
  *   alpha  [K] fp32 (device, output):
  *          alpha_k = (sum_{|W|<=1} |W| + 2 sum_{|W|>1} |W|) / (n + 3 |{|W|>1}|)
- *          accumulated in fp32 per 16 weights and fp64 across them, rounded
- *          once to fp32.  An all-zero filter gets alpha = 0.
+ *          the sum of 16 weights of a word in fp32, the word sums added
+ *          exactly as fp32 pairs (two-float TwoSum; fp64 only when a word sum
+ *          overflows fp32), rounded once to fp32.  An all-zero filter gets
+ *          alpha = 0.
  *   Eq. 3 per weight: W < -1 -> -2; -1 <= W <= 0 -> -1 (including -0.0);
  *          0 < W <= 1 -> 1; W > 1 -> 2.  NaN weights are undefined input.
  * K >= 1, 1 <= n < 2^31, K * tbn_packed_words(n) < 2^40. */

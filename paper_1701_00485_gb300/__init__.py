@@ -357,8 +357,8 @@ def tbn_linear_fwd_ws(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor,
                       residual: torch.Tensor | None = None, out: torch.Tensor | None = None,
                       stream=None):
     """tbn_linear_fwd with caller-owned device scratch: a CUDA tensor of at least
-    tbn_linear_workspace_bytes(...) bytes, zero-filled before its first use
-    (e.g. torch.zeros), or None."""
+    tbn_linear_workspace_bytes(...) bytes (its contents on entry do not
+    matter), or None."""
     _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
     B, K_in = x.shape
     ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)

@@ -15,6 +15,8 @@ namespace tbn {
 
 // Per-device error word written by kernels (timeouts, bad launch shapes).
 __device__ uint32_t g_tbn_device_error;
+// Where tbn_device_error's one-thread kernel leaves the word it took.
+__device__ uint32_t g_tbn_error_snapshot;
 
 namespace {
 
@@ -31,6 +33,14 @@ __global__ void selftest_wait_timeout_kernel(uint32_t* err, uint64_t limit_ns) {
     mbar_wait(&bar, 0u, nullptr, err, limit_ns);
   }
 }
+
+// Reads and clears the error word in one atomic step, so that a bit a
+// kernel of another stream sets meanwhile stays for the next read.
+__global__ void take_error_kernel(uint32_t* err) {
+  g_tbn_error_snapshot = atomicExch(err, 0u);
+}
+
+std::mutex g_error_read_mutex;   // one reader of the snapshot slot at a time
 
 constexpr int kMaxDevices = 64;
 uint32_t* g_err_ptr[kMaxDevices] = {};
@@ -218,14 +228,15 @@ tbn_status tbn_device_error(uint32_t* flags) {
   *flags = 0;
   uint32_t* p = device_error_word();
   if (!p) return fail(TBN_ERR_CUDA, "device_error: cannot resolve the error word");
+  std::lock_guard<std::mutex> g(g_error_read_mutex);
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "device_error: synchronize");
+  take_error_kernel<<<1, 1>>>(p);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "device_error: launch");
   uint32_t v = 0;
-  e = cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost);
+  e = cudaMemcpyFromSymbol(&v, g_tbn_error_snapshot, sizeof(v));   // synchronous, after the kernel
   if (e != cudaSuccess) return cuda_fail(e, "device_error: read");
-  const uint32_t zero = 0;
-  e = cudaMemcpy(p, &zero, sizeof(zero), cudaMemcpyHostToDevice);
-  if (e != cudaSuccess) return cuda_fail(e, "device_error: clear");
   *flags = v;
   return TBN_OK;
 }
