@@ -278,7 +278,8 @@ def net_spec(name, dev, batch=None):
             hh = h.reshape(N, -1)
             for j, (W, codes, alpha, relu, y) in enumerate(net.classifier.layers):
                 fn = (lambda hh=hh, c=codes, a=alpha, r=relu, y=y:
-                      tbn.tbn_linear_fwd(hh, c, a, c.shape[0], relu=r, out=y))
+                      tbn.tbn_linear_fwd_ws(hh, c, a, c.shape[0], net.classifier.workspace,
+                                            relu=r, out=y))
                 layers.append(("fc%d" % (j + 6), fn))
                 chain.append(fn)
                 chain_flops += 2 * N * W.shape[0] * W.shape[1]
@@ -289,7 +290,8 @@ def net_spec(name, dev, batch=None):
                              "256x3x3/p1, 3x3/2 max pools; FC 9216-4096-4096-1000",
                    "requantize_per_step": True}
             kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM): conv1 (patch mode), " \
-                          "conv2 (32-channel TMA), conv3-5, fc6-8 (1x1)"
+                          "conv2 (32-channel TMA), conv3-5, fc6-8 (1x1, split K; their " \
+                          "ordered split sums included in the chain time)"
         else:
             flops = net.flops
             cfg = {"workload": "vgg_small_b128_cifar", "global_batch": N, "image": [3, 32, 32],

@@ -346,6 +346,15 @@ tbn_status validate_linear(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in
   return TBN_OK;
 }
 
+// The 1x1-convolution form of a fully-connected layer (Section 3), with
+// 256-byte aligned stand-in pointers for shape-only queries.
+bool linear_as_conv(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in, const uint32_t* codes,
+                    const float* alpha, int64_t K_out, void* y, tbn_dtype ydt,
+                    const tbn_epilogue* epi, ConvProblem* p) {
+  return validate_conv(x, xdt, TBN_NHWC, B, K_in, 1, 1, codes, alpha, K_out, 1, 1, 1, 1, 0, 0, y,
+                       ydt, epi, p) == TBN_OK;
+}
+
 bool linear_uses_table(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out,
                        const uint32_t* codes) {
   return gemv_lut_unsupported_reason(xdt, B, K_in, K_out, codes)[0] == '\0';
@@ -363,8 +372,17 @@ tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
 
 size_t tbn_linear_workspace_bytes(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out) {
   if ((xdt != TBN_F32 && xdt != TBN_BF16) || B < 1 || K_in < 1 || K_out < 1) return 0;
-  if (gemv_lut_shape_reason(xdt, B, K_in, K_out)[0] != '\0') return 0;
-  return gemv_lut_workspace_bytes(K_in, K_out);
+  if (gemv_lut_shape_reason(xdt, B, K_in, K_out)[0] == '\0')
+    return gemv_lut_workspace_bytes(K_in, K_out);
+  if (xdt != TBN_BF16 || (B <= 8 && K_in % 64 == 0)) return 0;   // tensor-core GEMV, or no split
+  static const uint32_t dummy[64] __attribute__((aligned(256))) = {};
+  ConvProblem p{};
+  if (!linear_as_conv(dummy, xdt, B, K_in, dummy, reinterpret_cast<const float*>(dummy), K_out,
+                      const_cast<uint32_t*>(dummy), TBN_BF16, nullptr, &p))
+    return 0;
+  if (conv_igemm_unsupported_reason(p)[0] != '\0') return 0;
+  size_t bytes = 0;
+  return conv_igemm_splitk(p, &bytes) > 1 ? bytes : 0;
 }
 
 tbn_status tbn_linear_fwd_ws(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
@@ -395,9 +413,23 @@ tbn_status tbn_linear_fwd_ws(const void* x, tbn_dtype xdt, int64_t B, int64_t K_
     return launch_gemv(x, B, K_in, codes, alpha, K_out, y, ydt, relu, residual,
                        as_stream(stream));
   }
-  // a fully-connected layer is a 1x1 convolution over a 1x1 image (Section 3)
-  return tbn_conv2d_fwd(x, xdt, TBN_NHWC, B, K_in, 1, 1, codes, alpha, K_out, 1, 1, 1, 1, 0, 0, y,
-                        ydt, epi, stream);
+  // a fully-connected layer is a 1x1 convolution over a 1x1 image (Section 3);
+  // with the workspace the query asks for, its K blocks are split over the
+  // SMs its output tiles leave idle
+  ConvProblem p{};
+  const tbn_status vs = validate_conv(x, xdt, TBN_NHWC, B, K_in, 1, 1, codes, alpha, K_out, 1, 1,
+                                      1, 1, 0, 0, y, ydt, epi, &p);
+  if (vs != TBN_OK) return vs;
+  if (workspace != nullptr && is_aligned(workspace, 16) &&
+      conv_igemm_unsupported_reason(p)[0] == '\0') {
+    size_t need = 0;
+    const int splits = conv_igemm_splitk(p, &need);
+    if (splits > 1 && workspace_bytes >= need) {
+      p.partial = static_cast<float*>(workspace);
+      p.ksplit = splits;
+    }
+  }
+  return run_conv_auto(p, as_stream(stream));
 }
 
 tbn_status tbn_linear_fwd_noalloc(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,

@@ -146,6 +146,11 @@ struct IgArgs {
   int patch_cap;           // bytes per patch buffer (multiple of 16)
   int patch_bulk;          // pw == 0: in-image rows are one contiguous range of x
   long long x_bytes;       // size of x (bulk copies never read past it)
+  // split K: tile t is K-block range `split` (t / base_tiles) of the output
+  // tile t % base_tiles; the fp32 partial sums go to `partial`
+  // [ksplit][N][P][Q][K] and a second kernel adds them in split order
+  int ksplit, kb_per, base_tiles;
+  float* partial;
 };
 
 struct SmemCtl {
@@ -191,10 +196,15 @@ __device__ __forceinline__ void st_shared_u16(uint32_t addr, uint32_t v) {
 
 struct TileCoord {
   int ktile, q0, p0, n0;
+  int split, kb0, kb1;   // K blocks [kb0, kb1) of the filter (split K)
 };
 
 __device__ __forceinline__ TileCoord tile_coord(const IgArgs& a, int t) {
   TileCoord c;
+  c.split = t / a.base_tiles;
+  t -= c.split * a.base_tiles;
+  c.kb0 = c.split * a.kb_per;
+  c.kb1 = min(a.kblocks, c.kb0 + a.kb_per);
   c.ktile = t % a.tiles_k;
   const int pt_lin = t / a.tiles_k;
   const int qt = pt_lin % a.tiles_q;
@@ -309,8 +319,9 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     bool ok = true;
     for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x) {
       const TileCoord tc = tile_coord(a, t);
-      int tap = 0, cb = 0;   // (tap, channel box) of the next box
-      for (int kb = 0; kb < KB; ++kb, ++g) {
+      // (tap, channel box) of the next box
+      int tap = (tc.kb0 * kBoxes) / cblocks, cb = (tc.kb0 * kBoxes) % cblocks;
+      for (int kb = tc.kb0; kb < tc.kb1; ++kb, ++g) {
         const bool mine = turn == pid;
         if (++turn == kTmaProducers) turn = 0;
         if (!mine) {
@@ -378,7 +389,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         pbase[i] = ((static_cast<int64_t>(rv[i] ? tc.n0 + ni : 0) * a.H + rh[i]) * a.W + rw[i]) *
                    static_cast<int64_t>(a.C);
       }
-      for (int kb = 0; kb < KB; ++kb, ++g) {
+      for (int kb = tc.kb0; kb < tc.kb1; ++kb, ++g) {
         // table of this K block's 64 codes: offset from the tap-(0,0) pixel
         const int tb = g & 1;
         if (gt < kBK) {
@@ -514,6 +525,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     __syncwarp();   // reconverge before the aligned named barriers below
     const int T = a.bw * a.bh;
     for (int t = blockIdx.x; t < a.tiles; t += gridDim.x, ++tiles_done) {
+      const TileCoord tc = tile_coord(a, t);
       const int b = tiles_done & 1;
       uint8_t* buf = patch_buf + b * a.patch_cap;
       int lo, hi;
@@ -577,7 +589,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         valid[j] = px < T;
         base[j] = static_cast<int>(off0 / 2) + i * a.sh * pitch + q * a.sw * a.C;
       }
-      for (int kb = 0; kb < KB; ++kb, ++g) {
+      for (int kb = tc.kb0; kb < tc.kb1; ++kb, ++g) {
         const int sb = g % kSt;
         const uint32_t it = static_cast<uint32_t>(g / kSt);
         if (ok) ok = mbar_wait(&ctl->empty[sb], (it & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
@@ -661,11 +673,12 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     uint32_t tiles_done = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x, ++tiles_done) {
+      const TileCoord tc = tile_coord(a, t);
       // the epilogue must have drained the previous tile's accumulator
       ok = mbar_wait(&ctl->acc_empty, (tiles_done & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after_sync();
-      for (int kb = 0; kb < KB; ++kb, ++g) {
+      for (int kb = tc.kb0; kb < tc.kb1; ++kb, ++g) {
         const int st = g % kSt;
         ok = mbar_wait(&ctl->full[st], static_cast<uint32_t>(g / kSt) & 1u, abort_flag, a.err,
                        kWaitLimitNs);
@@ -680,7 +693,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
               const uint64_t bdesc = smem_desc_sw64_kmajor(
                   smem_addr(ring + st * kStageBytes + (kk >> 1) * (kStageBytes / 2)));
               tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * (kk & 1)),
-                        idesc, (kb | kk) != 0 ? 1u : 0u);
+                        idesc, ((kb - tc.kb0) | kk) != 0 ? 1u : 0u);
             }
           } else {
             const uint64_t bdesc = smem_desc_sw128_kmajor(smem_addr(ring + st * kStageBytes));
@@ -688,7 +701,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
             for (int kk = 0; kk < kBK / 16; ++kk) {
               // K step kk: 16 codes = 8 TMEM columns of A, 32 bytes of B rows
               tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
-                        (kb | kk) != 0 ? 1u : 0u);
+                        ((kb - tc.kb0) | kk) != 0 ? 1u : 0u);
             }
           }
           tc_commit(&ctl->empty[st]);
@@ -715,15 +728,20 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     const uint32_t lane_off = static_cast<uint32_t>(sub * 32) << 16;
     const bool pair_ok = ((a.wpf & 1) == 0) && ((reinterpret_cast<uintptr_t>(a.codes) & 7) == 0);
     // this CTA's K blocks, all tiles in sequence (g = tile_index * KB + kb)
-    const int my_tiles = (a.tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                         static_cast<int>(gridDim.x);
-    const int total = my_tiles * KB;
+    int total = 0;   // K blocks of all this CTA's tiles
+    for (int t = blockIdx.x; t < a.tiles; t += gridDim.x) {
+      const TileCoord tc = tile_coord(a, t);
+      total += tc.kb1 - tc.kb0;
+    }
     // prefetch cursor over (tile, kb): the codes of K block kb of a filter
     // are words [4 kb, 4 kb + 4) of its row; this warp takes two of them
-    int t_ld = blockIdx.x, kb_ld = 0;
+    int t_ld = blockIdx.x, kb_ld = 0, kb_end = 0;
     const uint32_t* crow_ld = nullptr;
     auto set_row = [&]() {
-      const int k = (t_ld % a.tiles_k) * kBM + m;
+      const TileCoord tc = tile_coord(a, t_ld < a.tiles ? t_ld : 0);
+      kb_ld = tc.kb0;
+      kb_end = tc.kb1;
+      const int k = tc.ktile * kBM + m;
       crow_ld = (t_ld < a.tiles && k < a.K) ? a.codes + static_cast<size_t>(k) * a.wpf : nullptr;
     };
     set_row();
@@ -734,8 +752,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         if (pair_ok) r = __ldg(reinterpret_cast<const uint2*>(crow_ld + w0));
         else r = make_uint2(__ldg(crow_ld + w0), w0 + 1 < a.wpf ? __ldg(crow_ld + w0 + 1) : 0u);
       }
-      if (++kb_ld == KB) {
-        kb_ld = 0;
+      if (++kb_ld == kb_end) {
         t_ld += gridDim.x;
         set_row();
       }
@@ -911,7 +928,15 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
             tc_fence_before_sync();
             mbar_arrive(&ctl->acc_empty);
           }
-          if (kTmaStore) {
+          if (!kTmaStore && a.partial != nullptr) {
+            // split K (1x1 image): pixel px is image n0 + px; the raw sum of
+            // this K range goes to partial[split][n][k]
+            float* dst = a.partial + (static_cast<size_t>(tc.split) * a.N + tc.n0 + 32 * j) * a.K + k;
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (kvalid && 32 * j + i < T && tc.n0 + 32 * j + i < a.N)
+                dst[static_cast<size_t>(i) * a.K] = __uint_as_float(v[i]);
+          } else if (kTmaStore) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               const int px = 32 * j + i;
@@ -1025,6 +1050,49 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
   }
 }
 
+// Split K: y = 2 alpha[k] * (sum of the K ranges' partial sums, in range
+// order) (+ residual), ReLU, rounded to y's dtype.  Deterministic.  Four
+// consecutive outputs per thread (K % 4 == 0: 16-byte partial loads).
+template <bool kVec>
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const float* __restrict__ partial,
+                                                           int S, int64_t mk, int K,
+                                                           const float* __restrict__ alpha,
+                                                           const void* residual, int relu,
+                                                           void* y, int y_bf16) {
+  constexpr int kV = kVec ? 4 : 1;
+  const int64_t n = mk / kV;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float acc[kV];
+    if constexpr (kVec) {
+      float4 t = __ldg(reinterpret_cast<const float4*>(partial) + i);
+      for (int s = 1; s < S; ++s) {
+        const float4 u = __ldg(reinterpret_cast<const float4*>(partial + s * mk) + i);
+        t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
+      }
+      acc[0] = t.x; acc[1] = t.y; acc[2] = t.z; acc[3] = t.w;
+    } else {
+      acc[0] = 0.0f;
+      for (int s = 0; s < S; ++s) acc[0] += __ldg(partial + s * mk + i);
+    }
+    const int64_t o = i * kV;
+    const int k0 = static_cast<int>(o % K);
+#pragma unroll
+    for (int e = 0; e < kV; ++e) {
+      float v = 2.0f * __ldg(alpha + k0 + e) * acc[e];
+      if (y_bf16) {
+        if (residual) v += __bfloat162float(static_cast<const __nv_bfloat16*>(residual)[o + e]);
+        if (relu) v = fmaxf(v, 0.0f);
+        static_cast<__nv_bfloat16*>(y)[o + e] = __float2bfloat16_rn(v);
+      } else {
+        if (residual) v += static_cast<const float*>(residual)[o + e];
+        if (relu) v = fmaxf(v, 0.0f);
+        static_cast<float*>(y)[o + e] = v;
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------- host side
 struct TilePlan {
   int bw, bh, bn, T, tile_n, tiles_q, tiles_p, tiles_n;
@@ -1035,55 +1103,6 @@ int ceil_div(int64_t a, int64_t b) { return static_cast<int>((a + b - 1) / b); }
 // TMA activations: whole 64-channel boxes, or 32-channel boxes in pairs.
 bool use_tma(const ConvProblem& p) { return p.C % (kBK / 2) == 0 && p.sh <= 2 && p.sw <= 2; }
 bool use_ch32(const ConvProblem& p) { return p.C % kBK != 0; }
-
-// Cost of a tile plan in SM cycles (a model, used only to compare plans):
-// the persistent CTAs take the tiles in waves; a tile costs per K block the
-// larger of the weight decode (about 320 cycles for 128 filters x 64 codes,
-// independent of the pixel count) and the MMAs (about 684 cycles at 256
-// pixels), plus a fixed cost for the pipeline fill and the epilogue.
-int64_t plan_cost(const ConvProblem& p, const TilePlan& t, int sms) {
-  const int64_t kblocks = (p.C * p.R * p.S + kBK - 1) / kBK;
-  const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n *
-                        ((p.K + kBM - 1) / kBM);
-  const int64_t waves = (tiles + sms - 1) / sms;
-  const int64_t mma = 684 * t.tile_n / kMaxTileN;
-  return waves * (kblocks * std::max<int64_t>(320, mma) + 2000);
-}
-
-// A fully-connected layer whose default plan leaves SMs idle (at batch 256:
-// 256 images per tile, K_out / 128 tiles) gets tiles of fewer images when
-// the cost model says the extra CTAs outweigh the longer decode per pixel.
-TilePlan shrink_for_occupancy(const ConvProblem& p, TilePlan t) {
-  const int sms = device_sm_count();
-  const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n *
-                        ((p.K + kBM - 1) / kBM);
-  // only fully-connected shapes (a 1x1 image): for convolutions the model
-  // misjudged the smaller tiles (ResNet-18's 7x7 layers ran slower)
-  if (tiles >= sms || t.tiles_q != 1 || p.P != 1 || p.Q != 1) return t;
-  TilePlan best = t;
-  int64_t best_cost = plan_cost(p, t, sms);
-  TilePlan c = t;
-  while (true) {
-    if (c.bn > 1) {
-      c.bn = (c.bn + 1) / 2;
-    } else if (c.bh > (p.pool ? 2 : 1)) {
-      c.bh = p.pool ? std::max(2, (c.bh / 2) & ~1) : (c.bh + 1) / 2;
-    } else {
-      break;
-    }
-    c.tiles_p = ceil_div(p.P, c.bh);
-    c.tiles_n = ceil_div(p.N, c.bn);
-    c.T = c.bw * c.bh * c.bn;
-    c.tile_n = ((c.T + 15) / 16) * 16;
-    if (c.tile_n < 32) break;
-    const int64_t cost = plan_cost(p, c, sms);
-    if (cost < best_cost) {
-      best = c;
-      best_cost = cost;
-    }
-  }
-  return best;
-}
 
 // Output pixels per tile: whole rows of the output (so one TMA box per tap
 // covers the tile), balanced so the last tile along each axis is not a
@@ -1118,7 +1137,7 @@ TilePlan plan_tiles(const ConvProblem& p) {
   t.tiles_n = ceil_div(p.N, t.bn);
   t.T = t.bw * t.bh * t.bn;
   t.tile_n = ((t.T + 15) / 16) * 16;
-  return shrink_for_occupancy(p, t);
+  return t;
 }
 
 int pool_width(const ConvProblem& p, const TilePlan& t) {
@@ -1248,6 +1267,31 @@ int patch_cap_bytes(const ConvProblem& p, const TilePlan& t) {
 
 bool conv_igemm_uses_tma(const ConvProblem& p) { return use_tma(p); }
 
+// Split K when the output tiles fill fewer than half the SMs and the filter
+// has at least 8 K blocks: every MMA instruction costs about as much at 64
+// pixels as at 256 (measured: the per-K-block time of one CTA barely moves
+// between 32 and 256 pixels), so idle SMs are filled with K ranges of
+// full-width tiles rather than with narrower tiles.
+int conv_igemm_splitk(const ConvProblem& p, size_t* workspace_bytes) {
+  *workspace_bytes = 0;
+  // fully-connected shapes only (a 1x1 convolution over a 1x1 image): a
+  // tile's pixel i is then image n0 + i, and the partial sums are stored
+  // without the pixel walk of a general tile
+  if (!use_tma(p) || p.pool || p.P != 1 || p.Q != 1 || p.R != 1 || p.S != 1) return 1;
+  const TilePlan t = plan_tiles(p);
+  const int64_t base = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n *
+                       ((p.K + kBM - 1) / kBM);
+  const int64_t kblocks = (p.C * p.R * p.S + kBK - 1) / kBK;
+  const int sms = device_sm_count();
+  if (2 * base > sms || kblocks < 8) return 1;
+  int64_t S = std::min<int64_t>(sms / base, kblocks / 4);
+  if (S < 2) return 1;
+  const int64_t per = (kblocks + S - 1) / S;
+  S = (kblocks + per - 1) / per;
+  *workspace_bytes = static_cast<size_t>(S) * p.N * p.P * p.Q * p.K * 4;
+  return static_cast<int>(S);
+}
+
 const char* conv_igemm_unsupported_reason(const ConvProblem& p) {
   if (p.layout != TBN_NHWC) return "implicit GEMM needs NHWC";
   if (p.xdt != TBN_BF16) return "implicit GEMM needs bf16 activations";
@@ -1281,17 +1325,44 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
   a.tiles_q = t.tiles_q; a.tiles_p = t.tiles_p;
   a.tiles_k = ceil_div(p.K, kBM);
   const int64_t tiles = static_cast<int64_t>(t.tiles_q) * t.tiles_p * t.tiles_n * a.tiles_k;
-  if (tiles > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: too many tiles");
-  a.tiles = static_cast<int>(tiles);
   a.ncodes = (int)(p.C * p.R * p.S);
   a.kblocks = ceil_div(a.ncodes, kBK);
+  const bool split = p.ksplit > 1 && p.partial != nullptr;
+  a.ksplit = split ? p.ksplit : 1;
+  a.kb_per = ceil_div(a.kblocks, a.ksplit);
+  if (split && (!use_tma(p) || p.pool || p.P != 1 || p.Q != 1 || p.R != 1 || p.S != 1 ||
+                (a.ksplit - 1) * a.kb_per >= a.kblocks))
+    return fail(TBN_ERR_INVALID_ARG, "implicit GEMM: bad split-K request");
+  if (tiles * a.ksplit > 0x7fffffffLL) return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: too many tiles");
+  a.base_tiles = static_cast<int>(tiles);
+  a.tiles = static_cast<int>(tiles * a.ksplit);
+  a.partial = split ? p.partial : nullptr;
   a.wpf = (a.ncodes + 15) / 16;
   a.x = static_cast<const __nv_bfloat16*>(p.x);
   a.codes = p.codes; a.alpha = p.alpha; a.y = p.y; a.residual = p.residual;
   a.relu = p.relu; a.y_bf16 = p.ydt == TBN_BF16 ? 1 : 0;
   a.err = device_error_word();
   const int pw = pool_width(p, t);
-  const bool tst = use_tma_store(p);
+  const bool tst = use_tma_store(p) && !split;   // partial sums: direct fp32 stores
+  if (split) {
+    // the K ranges' partial sums, then their ordered sum with the epilogue
+    const tbn_status st = use_ch32(p) ? launch_pool<kModeTma32, false>(p, t, a, pw, s)
+                                      : launch_pool<kModeTma64, false>(p, t, a, pw, s);
+    if (st != TBN_OK) return st;
+    const int64_t mk = p.N * p.P * p.Q * p.K;
+    const bool vec = p.K % 4 == 0 && is_aligned(p.partial, 16);
+    const int64_t items = vec ? mk / 4 : mk;
+    const int64_t blocks = std::min<int64_t>((items + 255) / 256, int64_t(device_sm_count()) * 16);
+    if (vec)
+      splitk_reduce_kernel<true><<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+          p.partial, a.ksplit, mk, (int)p.K, p.alpha, p.residual, p.relu, p.y,
+          p.ydt == TBN_BF16 ? 1 : 0);
+    else
+      splitk_reduce_kernel<false><<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+          p.partial, a.ksplit, mk, (int)p.K, p.alpha, p.residual, p.relu, p.y,
+          p.ydt == TBN_BF16 ? 1 : 0);
+    return check_launch("splitk_reduce_kernel");
+  }
   if (use_tma(p) && use_ch32(p)) {
     return tst ? launch_pool<kModeTma32, true>(p, t, a, pw, s)
                : launch_pool<kModeTma32, false>(p, t, a, pw, s);

@@ -57,6 +57,11 @@ struct ConvProblem {
   int relu;
   const void* residual;
   int pool;  // 0 or 2 (2x2 max pool, stride 2, after ReLU)
+  // split K (implicit GEMM only; set by tbn_linear_fwd_ws): ksplit > 1 K
+  // ranges accumulate into fp32 `partial` [ksplit][N][P][Q][K], then a
+  // second kernel adds them in order and applies the epilogue
+  float* partial;
+  int ksplit;
 };
 
 // The shape of one convolution for its backward pass (NHWC bf16).
@@ -77,6 +82,10 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s);
 // Empty string when the implicit-GEMM kernel can run `p`, else the reason.
 const char* conv_igemm_unsupported_reason(const ConvProblem& p);
 tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s);
+// Split-K plan of the implicit GEMM for `p` (a layer whose output tiles
+// leave most SMs idle, e.g. a fully-connected layer at batch 256): the number
+// of K ranges (1 = no split) and the fp32 workspace bytes it needs.
+int conv_igemm_splitk(const ConvProblem& p, size_t* workspace_bytes);
 // True when the implicit-GEMM kernel would feed activations by TMA (its fast mode).
 bool conv_igemm_uses_tma(const ConvProblem& p);
 

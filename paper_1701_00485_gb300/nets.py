@@ -20,7 +20,8 @@ from dataclasses import dataclass
 
 import torch
 
-from . import (TBN_NHWC, TBN_NCHW_NHWC, tbn_conv2d_fwd, tbn_linear_fwd, tbn_maxpool2d_nhwc,
+from . import (TBN_NHWC, TBN_NCHW_NHWC, tbn_conv2d_fwd, tbn_linear_fwd_ws,
+               tbn_linear_workspace_bytes, tbn_maxpool2d_nhwc,
                tbn_nchw_to_nhwc, tbn_quantize_pack_group, tbn_dense_conv2d_fwd,
                tbn_avgpool2d_global_nhwc, tbn_dense_linear_fwd, packed_words, conv_out_hw)
 from . import inputs as _inputs
@@ -133,17 +134,27 @@ def vgg_small(batch: int | None = None, seed: int = 1, device="cuda") -> ConvSta
 
 
 class FCStack:
-    """Fully-connected TBN layers (Section 3), ReLU between them."""
+    """Fully-connected TBN layers (Section 3), ReLU between them.  One device
+    workspace, sized by tbn_linear_workspace_bytes for the largest layer and
+    shared by all (they run one after another on the stream), lets a layer
+    whose output tiles leave SMs idle split its K dimension over them."""
 
     def __init__(self, fcs, weights, batch, device="cuda"):
         self.device = torch.device(device)
         self.layers = []
+        self.launches = 0
+        ws = 0
         for (kin, kout, relu), W in zip(fcs, weights):
             W = W.contiguous().to(self.device)
             codes = torch.empty((kout, packed_words(kin)), dtype=torch.int32, device=self.device)
             alpha = torch.empty((kout,), dtype=torch.float32, device=self.device)
             y = torch.empty((batch, kout), dtype=torch.bfloat16, device=self.device)
             self.layers.append((W, codes, alpha, relu, y))
+            need = tbn_linear_workspace_bytes(batch, kin, kout)
+            self.launches += 2 if need > 0 else 1     # split K adds the ordered sum
+            ws = max(ws, need)
+        self.workspace = (torch.empty(ws, dtype=torch.uint8, device=self.device)
+                          if ws > 0 else None)
 
     def quantize(self):
         tbn_quantize_pack_group([(W, c, a) for (W, c, a, _, _) in self.layers])
@@ -153,7 +164,7 @@ class FCStack:
             self.quantize()
         h = x
         for (W, codes, alpha, relu, y) in self.layers:
-            tbn_linear_fwd(h, codes, alpha, codes.shape[0], relu=relu, out=y)
+            tbn_linear_fwd_ws(h, codes, alpha, codes.shape[0], self.workspace, relu=relu, out=y)
             h = y
         return h
 
@@ -205,7 +216,7 @@ class AlexNet:
         return self.classifier.forward(h.reshape(self.N, -1))
 
     def launches_per_forward(self, requantize: bool = False) -> int:
-        n = self.features.launches_per_forward(False) + len(self.classifier.layers)
+        n = self.features.launches_per_forward(False) + self.classifier.launches
         return n + (1 if requantize else 0)
 
 

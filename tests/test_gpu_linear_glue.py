@@ -140,3 +140,33 @@ def test_nchw_to_nhwc_tiled_path(N, C, H, W, C_pad):
     want = torch.zeros(N, H, W, C_pad, dtype=torch.bfloat16)
     want[..., :C] = x.permute(0, 2, 3, 1)
     assert torch.equal(y, want)
+
+
+@pytest.mark.parametrize("B,K_in,K_out,relu,res", [(256, 9216, 4096, True, False),
+                                                   (256, 4096, 1000, False, False),
+                                                   (64, 2048, 300, True, True)])
+def test_linear_split_k_matches_oracle(B, K_in, K_out, relu, res):
+    """A fully-connected layer whose output tiles leave SMs idle (AlexNet's FC
+    layers at batch 256) runs with split K when given the workspace the query
+    asks for: every output within the bound, and the same results as the
+    unsplit call within the bound (the sum order differs)."""
+    ws_bytes = tbn.tbn_linear_workspace_bytes(B, K_in, K_out)
+    assert ws_bytes >= 4 * B * K_out * 2      # at least two K ranges of fp32 partial sums
+    g = inputs.generator(B + K_in + K_out)
+    W = inputs.normal((K_out, K_in), 1.1, g)
+    x = torch.randn(B, K_in, generator=g).to(torch.bfloat16)
+    r = torch.randn(B, K_out, generator=g).to(torch.bfloat16) if res else None
+    codes, alpha = tbn.tbn_quantize_pack(W.cuda())
+    ws = torch.full((ws_bytes,), 0xFF, dtype=torch.uint8, device="cuda")   # stale contents
+    y = tbn.tbn_linear_fwd_ws(x.cuda(), codes, alpha, K_out, ws, relu=relu,
+                              residual=r.cuda() if res else None)
+    y1 = tbn.tbn_linear_fwd(x.cuda(), codes, alpha, K_out, relu=relu,
+                            residual=r.cuda() if res else None)
+    torch.cuda.synchronize()
+    assert tbn.tbn_device_error() == 0
+    wt, al = oracle.quantize(W.numpy())
+    y_orc, bound = oracle.linear(x.float().numpy(), wt, al)
+    want = oracle.epilogue(y_orc, r.float().numpy() if res else None, relu=relu)
+    for got, what in ((y, "split K"), (y1, "unsplit")):
+        assert_within(got.float().cpu().numpy(), want, bound, out_bf16=True, epilogue=True,
+                      what="linear %s %s" % (what, (B, K_in, K_out)))
