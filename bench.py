@@ -258,13 +258,25 @@ def net_spec(name, dev, batch=None):
         net = nets.alexnet(batch, device=dev) if name == "alexnet" else nets.vgg_small(batch, device=dev)
         F = net.features if name == "alexnet" else net
         N = F.N
-        layers.append(("nchw_to_nhwc", lambda: tbn.tbn_nchw_to_nhwc(F.x_in, out=F.x_nhwc)))
-        h = F.x_nhwc
+        if F.s2d:
+            s0 = F.layers[0].spec
+            layers.append(("space_to_depth", lambda: tbn.tbn_space_to_depth(
+                F.x_in, s0.R, s0.S, (s0.stride,) * 2, (s0.pad,) * 2, layout=tbn.TBN_NCHW,
+                out=F.x_s2d)))
+            h = F.x_s2d
+        else:
+            layers.append(("nchw_to_nhwc", lambda: tbn.tbn_nchw_to_nhwc(F.x_in, out=F.x_nhwc)))
+            h = F.x_nhwc
         for i, l in enumerate(F.layers):
             s = l.spec
-            fn = conv_call(h, l, s, 2 if s.pool == (2, 2) else 0)
+            if i == 0 and F.s2d:
+                fn = (lambda h=h, l=l, s=s: tbn.tbn_conv2d_fwd(
+                    h, l.codes, l.alpha, s.K, s.R, s.S, (s.stride,) * 2, (s.pad,) * 2,
+                    layout=tbn.TBN_S2D_NHWC, in_chw=F.in_chw, relu=s.relu, out=l.y))
+            else:
+                fn = conv_call(h, l, s, 2 if s.pool == (2, 2) else 0)
             layers.append(("conv%d" % (i + 1), fn))
-            if is_igemm(N, s.C, l.in_hw, s):
+            if (i == 0 and F.s2d) or is_igemm(N, s.C, l.in_hw, s):
                 chain.append(fn)
                 chain_flops += N * l.flops_per_image
             h = l.y
@@ -289,7 +301,8 @@ def net_spec(name, dev, batch=None):
                    "layers": "conv 96x11x11/4, 256x5x5/p2, 384x3x3/p1, 384x3x3/p1, "
                              "256x3x3/p1, 3x3/2 max pools; FC 9216-4096-4096-1000",
                    "requantize_per_step": True}
-            kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM): conv1 (patch mode), " \
+            kernel_desc = "conv_igemm_kernel (tcgen05 implicit GEMM): conv1 (space-to-depth " \
+                          "input, filter resident in tensor memory), " \
                           "conv2 (32-channel TMA), conv3-5, fc6-8 (1x1, split K; their " \
                           "ordered split sums included in the chain time)"
         else:

@@ -84,7 +84,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 6
+#define TBN_ABI_VERSION 7
 
 typedef enum {
   TBN_OK = 0,
@@ -100,8 +100,12 @@ typedef enum { TBN_F32 = 0, TBN_BF16 = 1 } tbn_dtype;
 /* Activation layouts.  TBN_NCHW_NHWC (convolutions only) reads an NCHW x
  * and writes an NHWC y (and residual), with codes in the NHWC order
  * (r, s, c): the first layer of an NHWC network can read its NCHW input
- * batch without a converted copy (small-tap and direct kernels). */
-typedef enum { TBN_NCHW = 0, TBN_NHWC = 1, TBN_NCHW_NHWC = 2 } tbn_layout;
+ * batch without a converted copy (small-tap and direct kernels).
+ * TBN_S2D_NHWC (convolutions only) reads x in the space-to-depth form that
+ * tbn_space_to_depth writes for the same convolution and writes an NHWC y;
+ * sizes, stride, padding and codes ((r, s, c) order) are those of the
+ * convolution on the original input. */
+typedef enum { TBN_NCHW = 0, TBN_NHWC = 1, TBN_NCHW_NHWC = 2, TBN_S2D_NHWC = 3 } tbn_layout;
 
 typedef enum {
   TBN_UNPACK_I8 = 0,   /* int8 W~ in {-2,-1,1,2}                 */
@@ -253,6 +257,32 @@ tbn_status tbn_conv2d_fwd(const void *x, tbn_dtype xdt, tbn_layout layout, int64
                           const float *alpha, int64_t K, int64_t R, int64_t S,
                           int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
                           void *y, tbn_dtype ydt, const tbn_epilogue *epi, tbn_stream stream);
+
+/* Space-to-depth input of a strided convolution with few channels (not in
+ * the paper; a layout change that lets a first layer such as AlexNet's
+ * 11x11 stride-4 convolution over 3 channels run on the tensor-core
+ * implicit GEMM).  With s = stride_h = stride_w >= 2, s*s*C <= 64,
+ * P, Q the output size, R' = ceil(R / s), S' = ceil(S / s), it writes
+ *   out [N][Hs][Ws][64] bf16,  Hs = P + R' - 1,  Ws = Q + S' - 1,
+ *   out[n][Y][X][(dy s + dx) C + c] = x[n, c, s Y + dy - pad_h, s X + dx - pad_w]
+ * (dy, dx in [0, s); zero outside the image and for channels >= s*s*C).
+ * x is bf16, NCHW or NHWC, 2-byte aligned; out is 16-byte aligned and must
+ * not overlap x.  The convolution of Eq. 1 over x then equals
+ * tbn_conv2d_fwd with layout TBN_S2D_NHWC over out (a stride-1 R' x S'
+ * convolution of the 64 channels, whose weights the kernel gathers from the
+ * original codes; weights past the filter are zero).  That call needs
+ * K <= 128, bf16 output or fp32, no pool and no residual, and R' S' K blocks
+ * that fit in tensor memory beside the output tile (AlexNet's first layer:
+ * R' = S' = 3).  Asynchronous on `stream`.
+ * tbn_space_to_depth_elems returns the element count of out, or -1 when the
+ * geometry is invalid or unsupported. */
+int64_t tbn_space_to_depth_elems(int64_t N, int64_t C, int64_t H, int64_t W, int64_t R,
+                                 int64_t S, int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                                 int64_t pad_w);
+tbn_status tbn_space_to_depth(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                              int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
+                              int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
+                              void *out, tbn_stream stream);
 
 /* tbn_conv2d_fwd with an explicit algorithm.  Returns TBN_ERR_UNSUPPORTED if
  * the requested algorithm cannot run this shape. */

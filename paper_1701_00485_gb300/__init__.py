@@ -30,7 +30,7 @@ __all__ = [
     "TBN_CONV_SMALL_TAPS", "TBN_DEVERR_TIMEOUT", "TBN_DEVERR_BAD_LAUNCH",
     "tbn_selftest_wait_timeout", "tbn_repack", "TBN_REPACK_CANONICAL_TO_PLANAR",
     "TBN_REPACK_PLANAR_TO_CANONICAL", "tbn_dense_conv2d_fwd", "tbn_avgpool2d_global_nhwc",
-    "tbn_dense_linear_fwd",
+    "tbn_dense_linear_fwd", "tbn_space_to_depth", "space_to_depth_shape", "TBN_S2D_NHWC",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -39,7 +39,7 @@ _LIB_PATH = os.path.join(_HERE, "libtbn.so")
 TBN_OK, TBN_ERR_INVALID_ARG, TBN_ERR_UNSUPPORTED, TBN_ERR_MISALIGNED, TBN_ERR_CUDA, \
     TBN_ERR_TIMEOUT = range(6)
 TBN_F32, TBN_BF16 = 0, 1
-TBN_NCHW, TBN_NHWC, TBN_NCHW_NHWC = 0, 1, 2
+TBN_NCHW, TBN_NHWC, TBN_NCHW_NHWC, TBN_S2D_NHWC = 0, 1, 2, 3
 TBN_UNPACK_I8, TBN_UNPACK_F32, TBN_UNPACK_BF16 = 0, 1, 2
 TBN_CONV_AUTO, TBN_CONV_DIRECT, TBN_CONV_IMPLICIT_GEMM, TBN_CONV_SMALL_TAPS = 0, 1, 2, 3
 TBN_MAX_QUANT_JOBS = 16
@@ -55,7 +55,8 @@ EXPORTED = [
     "tbn_maxpool2d_nhwc", "tbn_nchw_to_nhwc", "tbn_conv2d_bwd_data_workspace_bytes",
     "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter_workspace_bytes", "tbn_conv2d_bwd_filter",
     "tbn_selftest_wait_timeout", "tbn_repack", "tbn_dense_conv2d_fwd",
-    "tbn_avgpool2d_global_nhwc", "tbn_dense_linear_fwd",
+    "tbn_avgpool2d_global_nhwc", "tbn_dense_linear_fwd", "tbn_space_to_depth_elems",
+    "tbn_space_to_depth",
 ]
 
 
@@ -79,7 +80,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 6  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 7  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -133,6 +134,8 @@ def lib():
             "tbn_conv2d_bwd_filter_workspace_bytes": ([I64] * 11, ctypes.c_size_t),
             "tbn_conv2d_bwd_filter": ([P, P] + [I64] * 11 + [P, P, ctypes.c_size_t, P], I32),
             "tbn_nchw_to_nhwc": ([P, I32, I64, I64, I64, I64, I64, P, P], I32),
+            "tbn_space_to_depth_elems": ([I64] * 10, I64),
+            "tbn_space_to_depth": ([P, I32, I32] + [I64] * 10 + [P, P], I32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(L, name)
@@ -247,12 +250,21 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
                    S: int, stride=(1, 1), pad=(0, 0), layout: int = TBN_NHWC,
                    out_dtype=None, relu: bool = False, residual: torch.Tensor | None = None,
                    algo: int = TBN_CONV_AUTO, out: torch.Tensor | None = None, stream=None,
-                   pool: int = 0):
+                   pool: int = 0, in_chw=None):
     """Two-bit convolution, Eq. 1.  x is [N,C,H,W] (NCHW, NCHW_NHWC) or
     [N,H,W,C] (NHWC); y is NCHW for NCHW, else NHWC.
-    pool=2 fuses a 2x2 / stride-2 max pool (after ReLU) into the epilogue."""
+    pool=2 fuses a 2x2 / stride-2 max pool (after ReLU) into the epilogue.
+    With layout TBN_S2D_NHWC, x is the output of tbn_space_to_depth for this
+    convolution and in_chw = (C, H, W) gives the original input's size."""
     _cuda(x, "x"), _cuda(codes, "codes"), _cuda(alpha, "alpha")
-    if layout == TBN_NHWC:
+    if layout == TBN_S2D_NHWC:
+        if in_chw is None:
+            raise ValueError("layout TBN_S2D_NHWC needs in_chw = (C, H, W)")
+        N = x.shape[0]
+        C, H, W = in_chw
+        if tuple(x.shape) != space_to_depth_shape(N, C, H, W, R, S, stride, pad):
+            raise ValueError("x is not the space-to-depth form of this convolution's input")
+    elif layout == TBN_NHWC:
         N, H, W, C = x.shape
     else:
         N, C, H, W = x.shape
@@ -274,6 +286,41 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
         x.data_ptr(), _dt(x), layout, N, C, H, W, codes.data_ptr(), alpha.data_ptr(), K, R, S,
         stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,
         ctypes.byref(e) if e is not None else None, algo, _stream(stream)), "tbn_conv2d_fwd")
+    return out
+
+
+def space_to_depth_shape(N: int, C: int, H: int, W: int, R: int, S: int, stride=(4, 4),
+                         pad=(0, 0)):
+    """Shape [N, Hs, Ws, 64] of tbn_space_to_depth's output for this
+    convolution (Hs = P + ceil(R / s) - 1, Ws = Q + ceil(S / s) - 1)."""
+    n = lib().tbn_space_to_depth_elems(N, C, H, W, R, S, stride[0], stride[1], pad[0], pad[1])
+    if n < 0:
+        raise ValueError("no space-to-depth form for this convolution (needs equal strides "
+                         ">= 2 and stride^2 * C <= 64)")
+    P, Q = conv_out_hw(H, W, R, S, stride, pad)
+    s = stride[0]
+    return (N, P + (R + s - 1) // s - 1, Q + (S + s - 1) // s - 1, 64)
+
+
+def tbn_space_to_depth(x: torch.Tensor, R: int, S: int, stride=(4, 4), pad=(0, 0),
+                       layout: int = TBN_NCHW, out: torch.Tensor | None = None,
+                       stream=None) -> torch.Tensor:
+    """Space-to-depth form [N, Hs, Ws, 64] bf16 of the bf16 input x (NCHW or
+    NHWC) of an R x S convolution with this stride and padding, for
+    tbn_conv2d_fwd(..., layout=TBN_S2D_NHWC, in_chw=(C, H, W))."""
+    _cuda(x, "x")
+    if layout == TBN_NHWC:
+        N, H, W, C = x.shape
+    else:
+        N, C, H, W = x.shape
+    shape = space_to_depth_shape(N, C, H, W, R, S, stride, pad)
+    if out is None:
+        out = torch.empty(shape, dtype=torch.bfloat16, device=x.device)
+    elif tuple(out.shape) != shape or out.dtype != torch.bfloat16:
+        raise ValueError("out has the wrong shape or dtype")
+    _check(lib().tbn_space_to_depth(x.data_ptr(), _dt(x), layout, N, C, H, W, R, S, stride[0],
+                                    stride[1], pad[0], pad[1], out.data_ptr(), _stream(stream)),
+           "tbn_space_to_depth")
     return out
 
 

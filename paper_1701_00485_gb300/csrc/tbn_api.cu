@@ -126,7 +126,8 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
   if (!x || !codes || !alpha || !y) return fail(TBN_ERR_INVALID_ARG, "conv: null pointer");
   if (xdt != TBN_F32 && xdt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad x dtype");
   if (ydt != TBN_F32 && ydt != TBN_BF16) return fail(TBN_ERR_INVALID_ARG, "conv: bad y dtype");
-  if (layout != TBN_NCHW && layout != TBN_NHWC && layout != TBN_NCHW_NHWC)
+  if (layout != TBN_NCHW && layout != TBN_NHWC && layout != TBN_NCHW_NHWC &&
+      layout != TBN_S2D_NHWC)
     return fail(TBN_ERR_INVALID_ARG, "conv: bad layout");
   if (N < 1 || C < 1 || H < 1 || W < 1 || K < 1 || R < 1 || S < 1)
     return fail(TBN_ERR_INVALID_ARG, "conv: sizes must be >= 1");
@@ -172,6 +173,7 @@ tbn_status validate_conv(const void* x, tbn_dtype xdt, tbn_layout layout, int64_
 // small-tap kernel for short filters, else the implicit GEMM with gathered
 // activations, else the CUDA-core direct kernel.
 tbn_conv_algo pick_algo(const ConvProblem& p) {
+  if (p.layout == TBN_S2D_NHWC) return TBN_CONV_IMPLICIT_GEMM;   // its only kernel
   const bool igemm = conv_igemm_unsupported_reason(p)[0] == '\0';
   if (igemm && conv_igemm_uses_tma(p)) return TBN_CONV_IMPLICIT_GEMM;
   if (conv_smalltap_unsupported_reason(p)[0] == '\0') return TBN_CONV_SMALL_TAPS;
@@ -181,6 +183,11 @@ tbn_conv_algo pick_algo(const ConvProblem& p) {
 
 tbn_status run_conv(const ConvProblem& p, tbn_conv_algo algo, cudaStream_t s) {
   if (algo == TBN_CONV_AUTO) algo = pick_algo(p);
+  if (p.layout == TBN_S2D_NHWC && algo != TBN_CONV_IMPLICIT_GEMM) {
+    if (algo != TBN_CONV_SMALL_TAPS && algo != TBN_CONV_DIRECT)
+      return fail(TBN_ERR_INVALID_ARG, "conv: bad algorithm %d", (int)algo);
+    return fail(TBN_ERR_UNSUPPORTED, "conv: space-to-depth input runs on the implicit GEMM only");
+  }
   if (algo == TBN_CONV_SMALL_TAPS) {
     const char* why = conv_smalltap_unsupported_reason(p);
     if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
@@ -193,6 +200,29 @@ tbn_status run_conv(const ConvProblem& p, tbn_conv_algo algo, cudaStream_t s) {
   }
   if (algo == TBN_CONV_DIRECT) return launch_conv_direct(p, s);
   return fail(TBN_ERR_INVALID_ARG, "conv: bad algorithm %d", (int)algo);
+}
+
+// Geometry checks of the space-to-depth layout change (shared by the size
+// query and the call).
+tbn_status validate_s2d(int64_t N, int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
+                        int64_t sh, int64_t sw, int64_t ph, int64_t pw, S2dGeom* g) {
+  if (N < 1 || C < 1 || H < 1 || W < 1 || R < 1 || S < 1 || ph < 0 || pw < 0)
+    return fail(TBN_ERR_INVALID_ARG, "space_to_depth: bad sizes");
+  if (sh != sw || sh < 2)
+    return fail(TBN_ERR_UNSUPPORTED, "space_to_depth: needs equal strides >= 2");
+  if (sh > 8 || sh * sh * C > kS2dChannels)
+    return fail(TBN_ERR_UNSUPPORTED, "space_to_depth: needs stride^2 * C <= 64");
+  const int64_t lim = int64_t(1) << 31;
+  if (H >= lim || W >= lim || R > 0xFFFF || S > 0xFFFF || ph > 0xFFFF || pw > 0xFFFF)
+    return fail(TBN_ERR_UNSUPPORTED, "space_to_depth: a size is too large");
+  if (H + 2 * ph < R || W + 2 * pw < S)
+    return fail(TBN_ERR_INVALID_ARG, "space_to_depth: kernel larger than padded input");
+  const int64_t P = (H + 2 * ph - R) / sh + 1, Q = (W + 2 * pw - S) / sw + 1;
+  *g = s2d_geom(R, S, sh, P, Q);
+  if (N > 65535 || g->Hs > 65535 || !mul_ok(N, g->Hs * g->Ws, int64_t(1) << 40) ||
+      !mul_ok(N, H * W * C, int64_t(1) << 46))
+    return fail(TBN_ERR_UNSUPPORTED, "space_to_depth: tensor too large");
+  return TBN_OK;
 }
 
 }  // namespace
@@ -307,6 +337,35 @@ tbn_status tbn_conv2d_fwd(const void* x, tbn_dtype xdt, tbn_layout layout, int64
                           const tbn_epilogue* epi, tbn_stream stream) {
   return tbn_conv2d_fwd_algo(x, xdt, layout, N, C, H, W, codes, alpha, K, R, S, stride_h,
                              stride_w, pad_h, pad_w, y, ydt, epi, TBN_CONV_AUTO, stream);
+}
+
+int64_t tbn_space_to_depth_elems(int64_t N, int64_t C, int64_t H, int64_t W, int64_t R,
+                                 int64_t S, int64_t stride_h, int64_t stride_w, int64_t pad_h,
+                                 int64_t pad_w) {
+  S2dGeom g{};
+  if (validate_s2d(N, C, H, W, R, S, stride_h, stride_w, pad_h, pad_w, &g) != TBN_OK) return -1;
+  return N * g.Hs * g.Ws * kS2dChannels;
+}
+
+tbn_status tbn_space_to_depth(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                              int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
+                              int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
+                              void* out, tbn_stream stream) {
+  if (!x || !out) return fail(TBN_ERR_INVALID_ARG, "space_to_depth: null pointer");
+  if (xdt != TBN_BF16) return fail(TBN_ERR_UNSUPPORTED, "space_to_depth: x must be bf16");
+  if (layout != TBN_NCHW && layout != TBN_NHWC)
+    return fail(TBN_ERR_INVALID_ARG, "space_to_depth: x must be NCHW or NHWC");
+  S2dGeom g{};
+  const tbn_status st = validate_s2d(N, C, H, W, R, S, stride_h, stride_w, pad_h, pad_w, &g);
+  if (st != TBN_OK) return st;
+  if (!is_aligned(x, 2) || !is_aligned(out, 16))
+    return fail(TBN_ERR_MISALIGNED, "space_to_depth: x needs 2-byte, out 16-byte alignment");
+  const int64_t bytes = N * g.Hs * g.Ws * kS2dChannels * 2;
+  const int64_t xbytes = N * C * H * W * 2;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(x), b = reinterpret_cast<uintptr_t>(out);
+  if (a < b + static_cast<uintptr_t>(bytes) && b < a + static_cast<uintptr_t>(xbytes))
+    return fail(TBN_ERR_INVALID_ARG, "space_to_depth: x and out overlap");
+  return launch_space_to_depth(x, layout, N, C, H, W, g, pad_h, pad_w, out, as_stream(stream));
 }
 
 tbn_conv_algo tbn_conv2d_select_algo(tbn_dtype xdt, tbn_layout layout, int64_t N, int64_t C,
@@ -596,6 +655,8 @@ tbn_status tbn_dense_conv2d_fwd(const void* x, tbn_dtype xdt, tbn_layout layout,
                                 int64_t pad_h, int64_t pad_w, void* y, tbn_dtype ydt, int relu,
                                 tbn_stream stream) {
   if (!w) return fail(TBN_ERR_INVALID_ARG, "dense conv: null pointer");
+  if (layout == TBN_S2D_NHWC)
+    return fail(TBN_ERR_UNSUPPORTED, "dense conv: no space-to-depth input");
   // the shape, dtype, layout and alignment checks of the two-bit convolution;
   // the weights stand in for its codes and alpha (both only checked for
   // being non-null and 4-byte aligned)

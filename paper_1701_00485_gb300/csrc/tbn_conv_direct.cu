@@ -418,6 +418,156 @@ int64_t grid_for(int64_t total) {
   return std::max<int64_t>(1, std::min<int64_t>((total + 255) / 256, cap));
 }
 
+// Space-to-depth layout change (see S2dGeom): block (xc, Y, n) writes
+// space-to-depth pixels X in [pix xc, pix xc + pix) of row Y, pix = 256 / s.
+// The s input rows s Y + dy - ph, columns [pix s xc - pw, + pix s), all C
+// channels, are first staged in shared memory as [dy][column][c] (zero
+// outside the image): a warp copies one input row segment at a time
+// (NCHW: a channel's row; NHWC: all channels of a row, one contiguous
+// range of x).  In that layout the s C channels of dy-row dy of pixel X are
+// one run of the tile, so when s C % 4 == 0 a 16-byte output chunk is two
+// aligned 8-byte shared loads; otherwise it is gathered 2 bytes at a time
+// through a 64-entry offset table.  kNchw: x is [N][C][H][W], else
+// [N][H][W][C].
+constexpr int kS2dThreads = 256;
+
+template <bool kNchw>
+__global__ void __launch_bounds__(kS2dThreads) space_to_depth_kernel(
+    const uint16_t* __restrict__ x, int C, int H, int W, int s, int ph, int pw, int Hs, int Ws,
+    uint4* __restrict__ out) {
+  extern __shared__ __align__(16) uint16_t s2d_tile[];   // [s][pix s][C]
+  __shared__ int s2d_off[64];              // channel j -> tile offset of pixel 0, or -1
+  const int xc = blockIdx.x, Y = blockIdx.y, n = blockIdx.z;
+  const int pix = kS2dThreads / s;
+  const int cols = pix * s;                // <= 256
+  const int w0 = xc * cols - pw;
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int sc = s * C;                    // channels of one dy-row of a pixel
+  const bool runs = (sc & 3) == 0;
+  if (!runs && t < 64) {
+    int o = -1;
+    if (t < s * sc) {
+      const int dy = t / sc, dx = (t / C) % s, c = t % C;
+      o = (dy * cols + dx) * C + c;
+    }
+    s2d_off[t] = o;
+  }
+  // stage: segment rows, 4 loads per lane in flight before their stores
+  const int nrows = kNchw ? C * s : s;
+  const int len = kNchw ? cols : cols * C;      // elements per segment row
+  for (int r = warp; r < nrows; r += kS2dThreads / 32) {
+    const int c = kNchw ? r / s : 0, dy = kNchw ? r - c * s : r;
+    const int h = s * Y + dy - ph;
+    const bool hin = h >= 0 && h < H;
+    const uint16_t* xr =
+        kNchw ? x + ((static_cast<int64_t>(n) * C + c) * H + (hin ? h : 0)) * W + w0
+              : x + ((static_cast<int64_t>(n) * H + (hin ? h : 0)) * W + w0) * static_cast<int64_t>(C);
+    // in-image elements of the segment row: [lo, hi)
+    const int lo = max(0, -w0) * (kNchw ? 1 : C);
+    const int hi = max(lo, min(cols, W - w0) * (kNchw ? 1 : C));
+    uint16_t* tr = s2d_tile + dy * cols * C + c;
+    const int tstride = kNchw ? C : 1;
+    for (int e0 = 0; e0 < len; e0 += 128) {
+      uint16_t v[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int e = e0 + lane + 32 * i;
+        v[i] = (hin && e >= lo && e < hi) ? xr[e] : static_cast<uint16_t>(0);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int e = e0 + lane + 32 * i;
+        if (e < len) tr[e * tstride] = v[i];
+      }
+    }
+  }
+  __syncthreads();
+  const int npix = min(pix, Ws - xc * pix);
+  const int q = t & 7;   // this thread's 16-byte chunk: channels 8 q .. 8 q + 7
+  uint4* orow = out + ((static_cast<int64_t>(n) * Hs + Y) * Ws + xc * pix) * 8;
+  if (runs) {
+    // channels 4 p .. 4 p + 3 (p = 2 q, 2 q + 1): dy = 4 p / sc, at element
+    // offset 4 p % sc of dy-row dy's run, which starts at (dy cols + s X) C
+    int po[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int j = 4 * (2 * q + u);
+      po[u] = j < s * sc ? (j / sc) * cols * C + j % sc : -1;
+    }
+    const uint2* tile8 = reinterpret_cast<const uint2*>(s2d_tile);
+    for (int xi = t >> 3; xi < npix; xi += kS2dThreads / 8) {
+      uint2 a = make_uint2(0u, 0u), b = make_uint2(0u, 0u);
+      if (po[0] >= 0) a = tile8[(po[0] + xi * sc) >> 2];
+      if (po[1] >= 0) b = tile8[(po[1] + xi * sc) >> 2];
+      orow[xi * 8 + q] = make_uint4(a.x, a.y, b.x, b.y);
+    }
+  } else {
+    int off[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) off[i] = s2d_off[8 * q + i];
+    for (int xi = t >> 3; xi < npix; xi += kS2dThreads / 8) {
+      uint32_t hv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) hv[i] = off[i] >= 0 ? s2d_tile[off[i] + xi * sc] : 0u;
+      orow[xi * 8 + q] = make_uint4(hv[0] | (hv[1] << 16), hv[2] | (hv[3] << 16),
+                                    hv[4] | (hv[5] << 16), hv[6] | (hv[7] << 16));
+    }
+  }
+}
+
+// The same layout change specialized for NCHW x with stride kS and kC
+// channels, kS kC % 4 == 0 (AlexNet's first layer: 4, 3): block (Y, n)
+// writes all Ws pixels of row Y (Ws <= 256 / kS, checked by the caller).
+// Thread t owns input column t - pw of the kC kS rows and issues all its
+// loads before its stores; the tile offsets are compile-time constants.
+template <int kS, int kC>
+__global__ void __launch_bounds__(kS2dThreads) space_to_depth_nchw_kernel(
+    const uint16_t* __restrict__ x, int H, int W, int ph, int pw, int Hs, int Ws,
+    uint4* __restrict__ out) {
+  constexpr int kCols = (kS2dThreads / kS) * kS;
+  constexpr int kSc = kS * kC;
+  static_assert(kSc % 4 == 0 && kS * kSc <= 64, "specialization");
+  __shared__ __align__(16) uint16_t tile[kS * kCols * kC];   // [dy][column][c]
+  const int Y = blockIdx.x, n = blockIdx.y;
+  const int t = threadIdx.x;
+  if (t < kCols) {
+    const int w = t - pw;
+    const bool win = w >= 0 && w < W;
+    const int64_t HW = static_cast<int64_t>(H) * W;
+    const uint16_t* xc = x + static_cast<int64_t>(n) * kC * HW + w;
+    const int hb = kS * Y - ph;
+    uint16_t v[kC][kS];
+#pragma unroll
+    for (int dy = 0; dy < kS; ++dy) {
+      const int h = hb + dy;
+      const bool ok = win && h >= 0 && h < H;
+#pragma unroll
+      for (int c = 0; c < kC; ++c)
+        v[c][dy] = ok ? xc[c * HW + static_cast<int64_t>(h) * W] : static_cast<uint16_t>(0);
+    }
+#pragma unroll
+    for (int dy = 0; dy < kS; ++dy)
+#pragma unroll
+      for (int c = 0; c < kC; ++c) tile[(dy * kCols + t) * kC + c] = v[c][dy];
+  }
+  __syncthreads();
+  const int q = t & 7;
+  int po[2];
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int j = 4 * (2 * q + u);
+    po[u] = j < kS * kSc ? (j / kSc) * kCols * kC + j % kSc : -1;
+  }
+  const uint2* tile8 = reinterpret_cast<const uint2*>(tile);
+  uint4* orow = out + (static_cast<int64_t>(n) * Hs + Y) * Ws * 8;
+  for (int xi = t >> 3; xi < Ws; xi += kS2dThreads / 8) {
+    uint2 a = make_uint2(0u, 0u), b = make_uint2(0u, 0u);
+    if (po[0] >= 0) a = tile8[(po[0] + xi * kSc) >> 2];
+    if (po[1] >= 0) b = tile8[(po[1] + xi * kSc) >> 2];
+    orow[xi * 8 + q] = make_uint4(a.x, a.y, b.x, b.y);
+  }
+}
+
 }  // namespace
 
 tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s) {
@@ -534,6 +684,31 @@ tbn_status launch_nchw_to_nhwc(const void* x, tbn_dtype dt, int64_t N, int64_t C
     nchw_to_nhwc_kernel<float><<<grid, 256, 0, s>>>(
         static_cast<const float*>(x), (int)C, (int)(H * W), (int)C_pad, static_cast<float*>(y));
   return check_launch("nchw_to_nhwc_kernel");
+}
+
+tbn_status launch_space_to_depth(const void* x, tbn_layout layout, int64_t N, int64_t C,
+                                 int64_t H, int64_t W, const S2dGeom& g, int64_t ph, int64_t pw,
+                                 void* out, cudaStream_t s) {
+  const int64_t pix = kS2dThreads / g.s;
+  if (layout == TBN_NCHW && g.s == 4 && C == 3 && g.Ws <= pix) {
+    space_to_depth_nchw_kernel<4, 3><<<dim3(static_cast<unsigned>(g.Hs), static_cast<unsigned>(N)),
+                                       kS2dThreads, 0, s>>>(
+        static_cast<const uint16_t*>(x), (int)H, (int)W, (int)ph, (int)pw, (int)g.Hs, (int)g.Ws,
+        static_cast<uint4*>(out));
+    return check_launch("space_to_depth_nchw_kernel");
+  }
+  const dim3 grid(static_cast<unsigned>((g.Ws + pix - 1) / pix), static_cast<unsigned>(g.Hs),
+                  static_cast<unsigned>(N));
+  const size_t smem = static_cast<size_t>(g.s * pix * g.s * C) * 2;   // <= 512 s C <= 16 KiB
+  if (layout == TBN_NCHW)
+    space_to_depth_kernel<true><<<grid, kS2dThreads, smem, s>>>(
+        static_cast<const uint16_t*>(x), (int)C, (int)H, (int)W, (int)g.s, (int)ph, (int)pw,
+        (int)g.Hs, (int)g.Ws, static_cast<uint4*>(out));
+  else
+    space_to_depth_kernel<false><<<grid, kS2dThreads, smem, s>>>(
+        static_cast<const uint16_t*>(x), (int)C, (int)H, (int)W, (int)g.s, (int)ph, (int)pw,
+        (int)g.Hs, (int)g.Ws, static_cast<uint4*>(out));
+  return check_launch("space_to_depth_kernel");
 }
 
 }  // namespace tbn

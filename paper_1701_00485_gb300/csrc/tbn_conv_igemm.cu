@@ -110,8 +110,13 @@ constexpr int kModeTma32 = 1;   // two 32-channel TMA boxes per K block (C % 32 
 constexpr int kModeGather = 2;  // threads gather each code's activation from global memory
 constexpr int kModePatch = 3;   // the tile's input rows are staged in shared memory (bulk
                                 // copy, double-buffered) and threads build the rows from there
+constexpr int kModeS2d = 4;     // space-to-depth input: 64-channel TMA boxes, and the
+                                // filter's K blocks decoded once per CTA into tensor memory
+constexpr int kMaxResidentKB = 15;   // resident K blocks: 32 columns each beside the accumulator
 
-__host__ __device__ constexpr bool mode_gathers(int mode) { return mode >= kModeGather; }
+__host__ __device__ constexpr bool mode_gathers(int mode) {
+  return mode == kModeGather || mode == kModePatch;
+}
 // the patch buffers take the room of two ring stages
 __host__ __device__ constexpr int stages_for(int mode) { return mode == kModePatch ? kStages - 2 : kStages; }
 
@@ -151,6 +156,9 @@ struct IgArgs {
   // [ksplit][N][P][Q][K] and a second kernel adds them in split order
   int ksplit, kb_per, base_tiles;
   float* partial;
+  // space-to-depth mode: the convolution in original coordinates (stride
+  // s2d_s, C0 channels, R0 x S0 filter, codes in (r, s, c) order)
+  int s2d_s, s2d_C, s2d_R, s2d_S;
 };
 
 struct SmemCtl {
@@ -168,6 +176,7 @@ struct SmemCtl {
   int gtab_off[2][kBK];    // gather: element offset of each code of the K block
   int gtab_rs[2][kBK];     // gather: (r << 16 | s), or -1 beyond the filter
   uint64_t patch_full[2];  // patch mode: a buffer's bulk copy has landed
+  uint64_t wready[kMaxResidentKB];   // space-to-depth mode: resident K block decoded
 };
 
 constexpr int kSmemLimit = 232448;
@@ -244,6 +253,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
   constexpr bool kGather = mode_gathers(kMode);
   constexpr bool kCh32 = kMode == kModeTma32;
   constexpr bool kPatch = kMode == kModePatch;
+  constexpr bool kS2d = kMode == kModeS2d;
   constexpr int kSt = stages_for(kMode);   // ring stages
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte aligned by pointer arithmetic on the shared array, so that the
@@ -262,7 +272,9 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kSt; ++i) {
-      mbar_init(&ctl->full[i], 32 * kExpWarps + (kGather ? 32 * producer_warps(kMode) : 1));
+      // space-to-depth mode: the weights are resident, only the activation box fills a stage
+      mbar_init(&ctl->full[i], (kS2d ? 0 : 32 * kExpWarps) +
+                                   (kGather ? 32 * producer_warps(kMode) : 1));
       mbar_init(&ctl->empty[i], 1);
     }
     mbar_init(&ctl->patch_full[0], 1);
@@ -271,6 +283,8 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     mbar_init(&ctl->acc_empty, 32 * kEpiWarps);
     mbar_init(&ctl->res_full, 1);
     mbar_init(&ctl->mma_drain, 1);
+    if (kS2d)
+      for (int i = 0; i < KB && i < kMaxResidentKB; ++i) mbar_init(&ctl->wready[i], 32 * kExpWarps);
     ctl->abort = 0;
     fence_mbar_init();
     if (!kGather) prefetch_tmap(&tmap_x);
@@ -279,6 +293,30 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
   if (warp == 1) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
     tmem_relinquish();
+  }
+  if (kS2d) {
+    // gather table of the resident K blocks: column j of K block kb (tap
+    // (kb / S', kb % S') of the space-to-depth grid, channel j = (dy s + dx)
+    // C0 + c) holds original code l = ((s r' + dy) S0 + s s' + dx) C0 + c as
+    // (l / 16) | (its magnitude bit) << 16, or ~0 where the s x s block
+    // reaches past the filter.  It lives in the output staging tile, which
+    // the epilogue first writes after the first tile's MMAs, i.e. after the
+    // decode.
+    uint32_t* tab = reinterpret_cast<uint32_t*>(out_stage);
+    const int ss = a.s2d_s, C0 = a.s2d_C;
+    for (int e = threadIdx.x; e < KB * kBK; e += blockDim.x) {
+      const int kb = e / kBK, j = e - (e / kBK) * kBK;
+      uint32_t v = 0xFFFFFFFFu;
+      if (j < ss * ss * C0) {
+        const int dy = j / (ss * C0), dx = (j / C0) % ss, c = j % C0;
+        const int r = ss * (kb / a.S) + dy, q = ss * (kb % a.S) + dx;
+        if (r < a.s2d_R && q < a.s2d_S) {
+          const int l = (r * a.s2d_S + q) * C0 + c;
+          v = static_cast<uint32_t>(l >> 4) | (static_cast<uint32_t>(code_mag_bit(l & 15)) << 16);
+        }
+      }
+      tab[e] = v;
+    }
   }
   tc_fence_before_sync();
   __syncthreads();
@@ -682,9 +720,13 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         const int st = g % kSt;
         ok = mbar_wait(&ctl->full[st], static_cast<uint32_t>(g / kSt) & 1u, abort_flag, a.err,
                        kWaitLimitNs);
+        if (kS2d && tiles_done == 0 && ok)   // first use of a resident K block
+          ok = mbar_wait(&ctl->wready[kb], 0u, abort_flag, a.err, kWaitLimitNs);
         if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
         tc_fence_after_sync();
-        const uint32_t a_col = a_tmem0 + static_cast<uint32_t>(st * kAColsPerStage);
+        const uint32_t a_col =
+            kS2d ? static_cast<uint32_t>(kTmemCols - 32 * KB + 32 * kb)
+                 : a_tmem0 + static_cast<uint32_t>(st * kAColsPerStage);
         if (elect_one()) {
           if constexpr (kCh32) {
             // two halves of 32 codes, 64-byte rows with the 64-byte swizzle
@@ -726,6 +768,33 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     const int half = (warp - kFirstExpWarp) >> 2;     // which 32 codes of a K block
     const int m = sub * 32 + lane;                    // filter row within the tile
     const uint32_t lane_off = static_cast<uint32_t>(sub * 32) << 16;
+    if constexpr (kS2d) {
+      // Decode every K block of the filter once into its resident columns
+      // [512 - 32 KB + 32 kb, + 32) (this warp: codes [32 half, + 32) of
+      // each, i.e. 16 columns).  Filter rows past K hold zeros.
+      const uint32_t* tab = reinterpret_cast<const uint32_t*>(out_stage);
+      const uint32_t* crow = m < a.K ? a.codes + static_cast<size_t>(m) * a.wpf : nullptr;
+      const uint32_t res0 = static_cast<uint32_t>(kTmemCols - 32 * KB);
+      for (int kb = 0; kb < KB; ++kb) {
+        uint32_t v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const uint32_t e0 = tab[kb * kBK + 32 * half + 2 * i];
+          const uint32_t e1 = tab[kb * kBK + 32 * half + 2 * i + 1];
+          uint32_t lo = 0u, hi = 0u;
+          // W~/2 in bf16: 0x3F00 (0.5) | m << 7 (1.0) | s << 15
+          if (crow != nullptr && e0 != 0xFFFFFFFFu)
+            lo = ((__ldg(crow + (e0 & 0xFFFFu)) >> (e0 >> 16)) & 0x101u) * 128u + 0x3F00u;
+          if (crow != nullptr && e1 != 0xFFFFFFFFu)
+            hi = ((__ldg(crow + (e1 & 0xFFFFu)) >> (e1 >> 16)) & 0x101u) * 128u + 0x3F00u;
+          v[i] = lo | (hi << 16);
+        }
+        tmem_st_32x32b_x16(tmem + lane_off + res0 + static_cast<uint32_t>(32 * kb + 16 * half), v);
+        tmem_wait_st();
+        tc_fence_before_sync();
+        mbar_arrive(&ctl->wready[kb]);
+      }
+    } else {
     const bool pair_ok = ((a.wpf & 1) == 0) && ((reinterpret_cast<uintptr_t>(a.codes) & 7) == 0);
     // this CTA's K blocks, all tiles in sequence (g = tile_index * KB + kb)
     int total = 0;   // K blocks of all this CTA's tiles
@@ -795,6 +864,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
       tc_fence_before_sync();
       mbar_arrive(&ctl->full[s0]);
       if (two) mbar_arrive(&ctl->full[s1]);
+    }
     }
   } else if (warp >= kFirstEpiWarp && warp < kFirstEpiWarp + kEpiWarps) {
     // ================= epilogue =================
@@ -1268,10 +1338,11 @@ int patch_cap_bytes(const ConvProblem& p, const TilePlan& t) {
 bool conv_igemm_uses_tma(const ConvProblem& p) { return use_tma(p); }
 
 // Split K when the output tiles fill fewer than half the SMs and the filter
-// has at least 8 K blocks: every MMA instruction costs about as much at 64
-// pixels as at 256 (measured: the per-K-block time of one CTA barely moves
-// between 32 and 256 pixels), so idle SMs are filled with K ranges of
-// full-width tiles rather than with narrower tiles.
+// has at least 8 K blocks.  The tensor core's time per K block is
+// proportional to the tile's pixels, but a CTA's time per K block is not
+// (measured: it barely moves between 32 and 256 pixels; the operand supply
+// sets it), so idle SMs are filled with K ranges of full-width tiles rather
+// than with narrower tiles.
 int conv_igemm_splitk(const ConvProblem& p, size_t* workspace_bytes) {
   *workspace_bytes = 0;
   // fully-connected shapes only (a 1x1 convolution over a 1x1 image): a
@@ -1292,7 +1363,42 @@ int conv_igemm_splitk(const ConvProblem& p, size_t* workspace_bytes) {
   return static_cast<int>(S);
 }
 
+// The stride-1 convolution over the space-to-depth input that a
+// TBN_S2D_NHWC problem runs as.
+ConvProblem s2d_problem(const ConvProblem& p) {
+  const S2dGeom g = s2d_geom(p.R, p.S, p.sh, p.P, p.Q);
+  ConvProblem q = p;
+  q.layout = TBN_NHWC;
+  q.C = kS2dChannels;
+  q.H = g.Hs;
+  q.W = g.Ws;
+  q.R = g.Rp;
+  q.S = g.Sp;
+  q.sh = q.sw = 1;
+  q.ph = q.pw = 0;
+  return q;
+}
+
+const char* s2d_unsupported_reason(const ConvProblem& p) {
+  if (p.xdt != TBN_BF16) return "space-to-depth input must be bf16";
+  if (p.sh != p.sw || p.sh < 2) return "space-to-depth needs equal strides >= 2";
+  if (p.sh * p.sh * p.C > kS2dChannels) return "space-to-depth needs stride^2 * C <= 64";
+  if (p.K > kBM) return "space-to-depth keeps one filter block (K <= 128) resident";
+  if (p.pool || p.residual) return "space-to-depth takes no pool and no residual";
+  if (p.ksplit > 1) return "space-to-depth takes no split K";
+  const ConvProblem q = s2d_problem(p);
+  const int64_t kb = q.R * q.S;
+  if (kb > kMaxResidentKB || plan_tiles(q).tile_n + 32 * kb > kTmemCols)
+    return "space-to-depth: the filter's K blocks do not fit in tensor memory beside the tile";
+  return "";
+}
+
 const char* conv_igemm_unsupported_reason(const ConvProblem& p) {
+  if (p.layout == TBN_S2D_NHWC) {
+    const char* r = s2d_unsupported_reason(p);
+    if (*r) return r;
+    return conv_igemm_unsupported_reason(s2d_problem(p));
+  }
   if (p.layout != TBN_NHWC) return "implicit GEMM needs NHWC";
   if (p.xdt != TBN_BF16) return "implicit GEMM needs bf16 activations";
   if (!is_aligned(p.x, 16)) return "implicit GEMM needs 16-byte aligned x";
@@ -1315,7 +1421,9 @@ const char* conv_igemm_unsupported_reason(const ConvProblem& p) {
   return "";
 }
 
-tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
+tbn_status launch_conv_igemm(const ConvProblem& p0, cudaStream_t s) {
+  const bool s2d = p0.layout == TBN_S2D_NHWC;
+  const ConvProblem p = s2d ? s2d_problem(p0) : p0;
   const TilePlan t = plan_tiles(p);
   IgArgs a{};
   a.N = (int)p.N; a.C = (int)p.C; a.H = (int)p.H; a.W = (int)p.W; a.K = (int)p.K;
@@ -1338,6 +1446,17 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
   a.tiles = static_cast<int>(tiles * a.ksplit);
   a.partial = split ? p.partial : nullptr;
   a.wpf = (a.ncodes + 15) / 16;
+  if (s2d) {
+    // codes of the original (r, s, c) filter
+    a.wpf = static_cast<int>((p0.C * p0.R * p0.S + 15) / 16);
+    a.s2d_s = static_cast<int>(p0.sh);
+    a.s2d_C = static_cast<int>(p0.C);
+    a.s2d_R = static_cast<int>(p0.R);
+    a.s2d_S = static_cast<int>(p0.S);
+    if (split || a.tiles_k != 1 || a.kblocks > kMaxResidentKB ||
+        t.tile_n + 32 * a.kblocks > kTmemCols || p.pool || p.residual)
+      return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: space-to-depth problem out of range");
+  }
   a.x = static_cast<const __nv_bfloat16*>(p.x);
   a.codes = p.codes; a.alpha = p.alpha; a.y = p.y; a.residual = p.residual;
   a.relu = p.relu; a.y_bf16 = p.ydt == TBN_BF16 ? 1 : 0;
@@ -1362,6 +1481,9 @@ tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s) {
           p.partial, a.ksplit, mk, (int)p.K, p.alpha, p.residual, p.relu, p.y,
           p.ydt == TBN_BF16 ? 1 : 0);
     return check_launch("splitk_reduce_kernel");
+  }
+  if (s2d) {
+    return tst ? launch_t<kModeS2d, 0, true>(p, t, a, s) : launch_t<kModeS2d, 0, false>(p, t, a, s);
   }
   if (use_tma(p) && use_ch32(p)) {
     return tst ? launch_pool<kModeTma32, true>(p, t, a, pw, s)

@@ -64,6 +64,28 @@ struct ConvProblem {
   int ksplit;
 };
 
+// Space-to-depth form of a strided convolution with few input channels
+// (layout TBN_S2D_NHWC): with s = stride, R' = ceil(R / s), S' = ceil(S / s),
+// the input becomes xs [N][Hs][Ws][64] bf16, Hs = P + R' - 1, Ws = Q + S' - 1,
+//   xs[n][Y][X][(dy s + dx) C + c] = x[n][c][s Y + dy - ph][s X + dx - pw]
+// (zero outside the image and for channels >= s^2 C), and the convolution
+// becomes a stride-1 R' x S' convolution of xs whose weight for s2d channel
+// (dy, dx, c) of tap (r', s') is W~[k][s r' + dy][s s' + dx][c] (zero where
+// that reaches past the filter).
+struct S2dGeom {
+  int64_t s, Rp, Sp, Hs, Ws;
+};
+constexpr int64_t kS2dChannels = 64;
+inline S2dGeom s2d_geom(int64_t R, int64_t S, int64_t stride, int64_t P, int64_t Q) {
+  S2dGeom g;
+  g.s = stride;
+  g.Rp = (R + stride - 1) / stride;
+  g.Sp = (S + stride - 1) / stride;
+  g.Hs = P + g.Rp - 1;
+  g.Ws = Q + g.Sp - 1;
+  return g;
+}
+
 // The shape of one convolution for its backward pass (NHWC bf16).
 struct BwdConvShape {
   int64_t N, C, H, W, K, R, S, sh, sw, ph, pw, P, Q;
@@ -82,6 +104,11 @@ tbn_status launch_conv_direct(const ConvProblem& p, cudaStream_t s);
 // Empty string when the implicit-GEMM kernel can run `p`, else the reason.
 const char* conv_igemm_unsupported_reason(const ConvProblem& p);
 tbn_status launch_conv_igemm(const ConvProblem& p, cudaStream_t s);
+// Space-to-depth layout change of a bf16 NCHW or NHWC input for the
+// convolution geometry (C, H, W, R, S, stride, pad) (see S2dGeom).
+tbn_status launch_space_to_depth(const void* x, tbn_layout layout, int64_t N, int64_t C,
+                                 int64_t H, int64_t W, const S2dGeom& g, int64_t ph, int64_t pw,
+                                 void* out, cudaStream_t s);
 // Split-K plan of the implicit GEMM for `p` (a layer whose output tiles
 // leave most SMs idle, e.g. a fully-connected layer at batch 256): the number
 // of K ranges (1 = no split) and the fp32 workspace bytes it needs.

@@ -10,7 +10,9 @@ tbn_quantize_pack_group launch for all layers; ``requantize=False`` runs the
 inference form (codes + alpha only, Section 3).
 
 Activations are NHWC bf16 between layers; the input batch arrives NCHW and
-is converted by tbn_nchw_to_nhwc.  Weights of an NHWC layer are packed in
+is converted by tbn_nchw_to_nhwc, or, for a strided first layer over few
+channels (AlexNet's 11x11/4), by tbn_space_to_depth into the input of that
+layer's space-to-depth convolution.  Weights of an NHWC layer are packed in
 (r, s, c) order: the fp32 [K, C, R, S] weights are permuted once at build
 time (quantization is elementwise and alpha is order-independent).
 """
@@ -20,7 +22,8 @@ from dataclasses import dataclass
 
 import torch
 
-from . import (TBN_NHWC, TBN_NCHW_NHWC, tbn_conv2d_fwd, tbn_linear_fwd_ws,
+from . import (TBN_NCHW, TBN_NHWC, TBN_NCHW_NHWC, TBN_S2D_NHWC, tbn_conv2d_fwd,
+               tbn_space_to_depth, space_to_depth_shape, tbn_linear_fwd_ws,
                tbn_linear_workspace_bytes, tbn_maxpool2d_nhwc,
                tbn_nchw_to_nhwc, tbn_quantize_pack_group, tbn_dense_conv2d_fwd,
                tbn_avgpool2d_global_nhwc, tbn_dense_linear_fwd, packed_words, conv_out_hw)
@@ -53,7 +56,20 @@ class ConvStack:
         N, C, H, W = x_nchw.shape
         self.N = N
         self.x_in = x_nchw.to(self.device).contiguous()
-        self.x_nhwc = torch.empty((N, H, W, C), dtype=torch.bfloat16, device=self.device)
+        self.in_chw = (C, H, W)
+        s0 = specs[0]
+        # a strided first layer over few channels runs on its space-to-depth
+        # input (the implicit GEMM with the filter resident in tensor memory)
+        # instead of an NHWC copy of the input
+        self.s2d = (self.x_in.dtype == torch.bfloat16 and s0.stride >= 2 and
+                    s0.stride * s0.stride * C <= 64 and s0.K <= 128 and s0.pool != (2, 2) and
+                    -(-s0.R // s0.stride) * -(-s0.S // s0.stride) <= 9)
+        if self.s2d:
+            self.x_s2d = torch.empty(space_to_depth_shape(N, C, H, W, s0.R, s0.S,
+                                                          (s0.stride,) * 2, (s0.pad,) * 2),
+                                     dtype=torch.bfloat16, device=self.device)
+        else:
+            self.x_nhwc = torch.empty((N, H, W, C), dtype=torch.bfloat16, device=self.device)
         self.layers = []
         hw = (H, W)
         for spec, Wt in zip(specs, weights):
@@ -102,15 +118,23 @@ class ConvStack:
             self.quantize()
         if conv_hook:
             conv_hook(-1, None, "quantized")
-        tbn_nchw_to_nhwc(self.x_in, out=self.x_nhwc)
-        h = self.x_nhwc
+        if self.s2d:
+            s0 = self.layers[0].spec
+            tbn_space_to_depth(self.x_in, s0.R, s0.S, (s0.stride,) * 2, (s0.pad,) * 2,
+                               layout=TBN_NCHW, out=self.x_s2d)
+            h = self.x_s2d
+        else:
+            tbn_nchw_to_nhwc(self.x_in, out=self.x_nhwc)
+            h = self.x_nhwc
         for i, l in enumerate(self.layers):
             s = l.spec
             if conv_hook:
                 conv_hook(i, l, "before")
+            s2d = i == 0 and self.s2d
             tbn_conv2d_fwd(h, l.codes, l.alpha, s.K, s.R, s.S, (s.stride, s.stride),
-                           (s.pad, s.pad), layout=TBN_NHWC, relu=s.relu, out=l.y,
-                           pool=2 if s.pool == (2, 2) else 0)
+                           (s.pad, s.pad), layout=TBN_S2D_NHWC if s2d else TBN_NHWC,
+                           relu=s.relu, out=l.y, pool=2 if s.pool == (2, 2) else 0,
+                           in_chw=self.in_chw if s2d else None)
             if conv_hook:
                 conv_hook(i, l, "after")
             h = l.y
@@ -121,7 +145,7 @@ class ConvStack:
         return h
 
     def launches_per_forward(self, requantize: bool = True) -> int:
-        # NCHW->NHWC, one launch per conv, one per pool that is not fused
+        # the input layout change, one launch per conv, one per pool that is not fused
         n = 1 + len(self.layers) + sum(1 for l in self.layers if l.pooled is not None)
         if requantize:
             n += (len(self.layers) + 15) // 16

@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 6
+    assert L.tbn_abi_version() == 7
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -81,7 +81,7 @@ def test_conv_rejects_bad_arguments(L):
     assert _conv(L, N=0) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, xdt=5) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, layout=9) == tbn.TBN_ERR_INVALID_ARG
-    assert _conv(L, layout=3) == tbn.TBN_ERR_INVALID_ARG
+    assert _conv(L, layout=4) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, sh=0) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, ph=-1) == tbn.TBN_ERR_INVALID_ARG
     assert _conv(L, H=2, W=2, ph=0, pw=0) == tbn.TBN_ERR_INVALID_ARG   # kernel > input
@@ -94,6 +94,34 @@ def test_conv_rejects_bad_arguments(L):
     assert _conv(L, C=1 << 40, R=1 << 30) == tbn.TBN_ERR_UNSUPPORTED
     assert _conv(L, N=1 << 20, H=8, W=8, C=1, ph=0xFFFF, pw=0xFFFF) == \
         tbn.TBN_ERR_UNSUPPORTED                                      # N P Q above 2^46
+
+
+def test_space_to_depth_host_rules(L):
+    # out [N][Hs][Ws][64], Hs = P + ceil(R/s) - 1, Ws = Q + ceil(S/s) - 1
+    assert L.tbn_space_to_depth_elems(256, 3, 227, 227, 11, 11, 4, 4, 0, 0) == 256 * 57 * 57 * 64
+    assert L.tbn_space_to_depth_elems(2, 16, 17, 19, 5, 5, 2, 2, 2, 2) == 2 * 11 * 12 * 64
+    assert L.tbn_space_to_depth_elems(1, 3, 227, 227, 11, 11, 1, 1, 0, 0) == -1   # stride 1
+    assert L.tbn_space_to_depth_elems(1, 5, 227, 227, 11, 11, 4, 4, 0, 0) == -1   # 80 channels
+    assert L.tbn_space_to_depth_elems(1, 3, 227, 227, 11, 11, 4, 2, 0, 0) == -1   # unequal
+    assert L.tbn_space_to_depth_elems(1, 3, 5, 5, 11, 11, 4, 4, 0, 0) == -1       # kernel > input
+    assert L.tbn_space_to_depth_elems(0, 3, 227, 227, 11, 11, 4, 4, 0, 0) == -1
+    d, o = ctypes.c_void_p(256), ctypes.c_void_p(1 << 40)
+    args = [1, 3, 227, 227, 11, 11, 4, 4, 0, 0]
+    assert L.tbn_space_to_depth(None, 1, 0, *args, o, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_space_to_depth(d, 0, 0, *args, o, None) == tbn.TBN_ERR_UNSUPPORTED     # fp32
+    assert L.tbn_space_to_depth(d, 1, 2, *args, o, None) == tbn.TBN_ERR_INVALID_ARG     # layout
+    assert L.tbn_space_to_depth(d, 1, 0, *args, ctypes.c_void_p((1 << 40) + 8), None) == \
+        tbn.TBN_ERR_MISALIGNED
+    assert L.tbn_space_to_depth(d, 1, 0, *args, ctypes.c_void_p(512), None) == \
+        tbn.TBN_ERR_INVALID_ARG                                                    # overlap
+    # the convolution over it: the implicit GEMM only, bf16, equal strides
+    s2d = dict(layout=3, C=3, H=227, W=227, K=96, R=11, S=11, sh=4, sw=4, ph=0, pw=0)
+    assert _conv(L, algo=1, **s2d) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, algo=3, **s2d) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, xdt=0, **s2d) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, **dict(s2d, K=129)) == tbn.TBN_ERR_UNSUPPORTED
+    assert _conv(L, **dict(s2d, sw=2)) == tbn.TBN_ERR_UNSUPPORTED
+    assert b"space-to-depth" in L.tbn_last_error()
 
 
 def test_select_algo_host_rules(L):
