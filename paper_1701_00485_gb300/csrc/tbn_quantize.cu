@@ -273,36 +273,74 @@ __device__ __forceinline__ void reduce_rows(const QJob& jb, int64_t k0, int nrow
   }
 }
 
+// A streamed task's weights: nrows whole filters from filter k0 of job jb,
+// `words` packed words (64 bytes of fp32 weights each), in `nch` chunks.
+struct StreamTask {
+  const QJob* jb;
+  int64_t k0;
+  int nrows;
+  int words;
+  int nch;
+  const uint8_t* src;
+};
+
+__device__ __forceinline__ StreamTask stream_task(const QJob& jb, int64_t k0, int nrows) {
+  StreamTask t;
+  t.jb = &jb;
+  t.k0 = k0;
+  t.nrows = nrows;
+  t.words = nrows * jb.wpf;
+  t.nch = (t.words + kChunkWords - 1) / kChunkWords;
+  t.src = reinterpret_cast<const uint8_t*>(jb.W + k0 * static_cast<int64_t>(jb.n));
+  return t;
+}
+
+// Thread 0: bulk copy of chunk i of task t into ring slot g % kStages.
+__device__ __forceinline__ void issue_chunk(const StreamTask& t, int i, uint32_t g, uint8_t* ring,
+                                            uint64_t* full) {
+  const uint32_t bytes = static_cast<uint32_t>(t.words) * 64u;
+  const uint32_t off = static_cast<uint32_t>(i) * kChunkBytes;
+  const uint32_t len = bytes - off < static_cast<uint32_t>(kChunkBytes) ? bytes - off
+                                                                        : static_cast<uint32_t>(kChunkBytes);
+  mbar_arrive_expect_tx(&full[g % kStages], len);
+  bulk_load_1d(ring + (g % kStages) * kChunkBytes, t.src + off, len, &full[g % kStages]);
+}
+
 // Streamed task: nrows whole filters (n % 16 == 0, 16-byte aligned rows,
 // nrows * wpf <= kItemWords words) flow through the ring of kStages 32 KB
-// chunks; thread 0 keeps up to kStages bulk copies in flight.  `seq` counts
-// the chunks this CTA has pushed through the ring (slot and phase).
-// Returns false if a wait timed out (after draining its copies).
-__device__ bool task_stream(const QJob& jb, int64_t k0, int nrows, QShared& sh, uint8_t* ring,
-                            uint64_t* full, uint32_t& seq, uint32_t* err) {
-  const int words = nrows * jb.wpf;
-  const float* base = jb.W + k0 * static_cast<int64_t>(jb.n);
-  const uint8_t* src = reinterpret_cast<const uint8_t*>(base);
-  uint32_t* out = jb.codes + k0 * static_cast<int64_t>(jb.wpf);
-  const uint32_t bytes = static_cast<uint32_t>(words) * 64u;
-  const int nch = (words + kChunkWords - 1) / kChunkWords;
-  auto issue = [&](int i) {
-    const uint32_t g = seq + static_cast<uint32_t>(i);
-    const uint32_t off = static_cast<uint32_t>(i) * kChunkBytes;
-    const uint32_t len = bytes - off < static_cast<uint32_t>(kChunkBytes) ? bytes - off
-                                                                          : static_cast<uint32_t>(kChunkBytes);
-    mbar_arrive_expect_tx(&full[g % kStages], len);
-    bulk_load_1d(ring + (g % kStages) * kChunkBytes, src + off, len, &full[g % kStages]);
+// chunks; thread 0 keeps up to kStages bulk copies in flight.  The chunks of
+// all this CTA's consecutive streamed tasks form one sequence: `seq` counts
+// the chunks consumed so far (every thread), `issued` those whose copy was
+// issued (thread 0, which issues them).  Once a task has issued its last
+// chunk, the freed slots take the first chunks of the next task (`nxt`, if
+// it streams too), so the ring does not drain at task boundaries.  Returns false if a wait timed
+// out (after draining every copy in flight).
+__device__ bool task_stream(const StreamTask& t, const StreamTask* nxt, QShared& sh, uint8_t* ring,
+                            uint64_t* full, uint32_t& seq, uint32_t& issued, uint32_t* err) {
+  const QJob& jb = *t.jb;
+  uint32_t* out = jb.codes + t.k0 * static_cast<int64_t>(jb.wpf);
+  const uint32_t end = seq + static_cast<uint32_t>(t.nch);   // this task's chunks: [seq, end)
+  // issue (thread 0) every chunk of the sequence up to `upto`
+  auto top_up = [&](uint32_t upto) {
+    while (issued < upto) {
+      if (issued < end) {
+        issue_chunk(t, static_cast<int>(issued - seq), issued, ring, full);
+      } else if (nxt != nullptr && issued < end + static_cast<uint32_t>(nxt->nch)) {
+        issue_chunk(*nxt, static_cast<int>(issued - end), issued, ring, full);
+      } else {
+        break;
+      }
+      ++issued;
+    }
   };
-  if (threadIdx.x == 0)
-    for (int i = 0; i < nch && i < kStages; ++i) issue(i);
-  for (int i = 0; i < nch; ++i) {
+  if (threadIdx.x == 0) top_up(seq + kStages);
+  for (int i = 0; i < t.nch; ++i) {
     const uint32_t g = seq + static_cast<uint32_t>(i);
     const bool ok = mbar_wait(&full[g % kStages], (g / kStages) & 1u, nullptr, err, kWaitLimitNs);
     if (ok) {
       const float* chunk = reinterpret_cast<const float*>(ring + (g % kStages) * kChunkBytes);
       const int w0 = i * kChunkWords;
-      const int wn = words - w0 < kChunkWords ? words - w0 : kChunkWords;
+      const int wn = t.words - w0 < kChunkWords ? t.words - w0 : kChunkWords;
 #pragma unroll
       for (int u = 0; u < kChunkWords / kThreads; ++u) {
         const int w = threadIdx.x + u * kThreads;
@@ -329,18 +367,16 @@ __device__ bool task_stream(const QJob& jb, int64_t k0, int nrows, QShared& sh, 
     // everyone is done with this slot (or something timed out)
     if (__syncthreads_or(!ok)) {
       if (threadIdx.x == 0) {
-        // copies issued but not consumed: chunks i .. min(nch, i + kStages) - 1
-        for (int j = i; j < nch && j < i + kStages; ++j) {
-          const uint32_t gj = seq + static_cast<uint32_t>(j);
+        // copies issued but not consumed: g .. issued - 1
+        for (uint32_t gj = g; gj != issued; ++gj)
           mbar_wait(&full[gj % kStages], (gj / kStages) & 1u, nullptr, err, kWaitLimitNs);
-        }
       }
       return false;
     }
-    if (threadIdx.x == 0 && i + kStages < nch) issue(i + kStages);
+    if (threadIdx.x == 0) top_up(g + 1 + kStages);
   }
-  seq += static_cast<uint32_t>(nch);
-  reduce_rows(jb, k0, nrows, base, sh);
+  seq = end;
+  reduce_rows(jb, t.k0, t.nrows, reinterpret_cast<const float*>(t.src), sh);
   __syncthreads();   // sums consumed before the next task overwrites them
   return true;
 }
@@ -400,6 +436,15 @@ __device__ void task_long(const QJob& jb, int64_t k, QShared& sh) {
   __syncthreads();
 }
 
+// The job a task belongs to.
+__device__ __forceinline__ int job_of(const QParams& prm, int64_t task) {
+  int ji = 0;
+#pragma unroll 1
+  for (int i = 1; i < prm.njobs; ++i)
+    if (task >= prm.job[i].first_task) ji = i;
+  return ji;
+}
+
 // Persistent: CTA b takes tasks b, b + grid, ...; a task is a run of whole
 // filters of one job (sized so that tasks carry about equal bytes).
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) quantize_pack_kernel(const __grid_constant__ QParams prm,
@@ -412,13 +457,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) quantize_pack_kernel(con
     fence_mbar_init();
   }
   __syncthreads();
-  uint32_t seq = 0;
+  uint32_t seq = 0, issued = 0;   // streamed chunks consumed (all threads) / issued (thread 0)
   for (int64_t task = blockIdx.x; task < ntasks; task += gridDim.x) {
-    int ji = 0;
-#pragma unroll 1
-    for (int i = 1; i < prm.njobs; ++i)
-      if (task >= prm.job[i].first_task) ji = i;
-    const QJob& jb = prm.job[ji];
+    const QJob& jb = prm.job[job_of(prm, task)];
     const int64_t local = task - jb.first_task;
     if (jb.mode == kModeLong) {
       task_long(jb, local, sh);
@@ -426,7 +467,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) quantize_pack_kernel(con
       const int64_t k0 = local * jb.rows;
       const int nrows = static_cast<int>(jb.K - k0 < jb.rows ? jb.K - k0 : jb.rows);
       if (jb.mode == kModeStream) {
-        if (!task_stream(jb, k0, nrows, sh, q_ring, full, seq, prm.err)) return;
+        // the CTA's next task, when it streams too, is prefetched into the ring
+        StreamTask nt{};
+        const StreamTask* nxt = nullptr;
+        const int64_t task2 = task + gridDim.x;
+        if (task2 < ntasks) {
+          const QJob& jb2 = prm.job[job_of(prm, task2)];
+          if (jb2.mode == kModeStream) {
+            const int64_t k2 = (task2 - jb2.first_task) * jb2.rows;
+            nt = stream_task(jb2, k2, static_cast<int>(jb2.K - k2 < jb2.rows ? jb2.K - k2 : jb2.rows));
+            nxt = &nt;
+          }
+        }
+        if (!task_stream(stream_task(jb, k0, nrows), nxt, sh, q_ring, full, seq, issued, prm.err))
+          return;
       } else {
         task_regs(jb, k0, nrows, sh);
       }
