@@ -538,6 +538,9 @@ def run_gemv(args, rank, world, local_rank, sizes=None, batches=None, reps=None)
         code_bytes = codes.numel() * 4
         copies = max(2, int(np.ceil(3 * l2 / code_bytes)))
         bufs = [codes] + [codes.clone() for _ in range(copies - 1)]
+        # the fp8 tensor-core path reads its own prepared copy of the codes
+        f8 = tbn.tbn_linear_f8_prepared_words(K, K) > 0
+        pbufs = [tbn.tbn_linear_prepare_f8(c, K) for c in bufs] if f8 else []
         for B in batches:
             gx = torch.Generator(device=dev)
             gx.manual_seed(1000 * K + B)
@@ -548,10 +551,19 @@ def run_gemv(args, rank, world, local_rank, sizes=None, batches=None, reps=None)
             x32 = x.float()
             reps = max(copies, 64)
             # "mma": bf16 activations (tensor-core GEMV); "table-f32": fp32
-            # activations on the batch-1 table-lookup GEMV (tbn_linear_fwd_ws)
+            # activations on the batch-1 table-lookup GEMV (tbn_linear_fwd_ws);
+            # "tcgen05-f8": batch 1 on the fp8 tensor-core path
             paths = ["mma", "table-f32"] if ws_bytes > 0 else ["mma"]
+            f8_ws = tbn.tbn_linear_f8_workspace_bytes(B, K, K) if f8 else 0
+            if f8_ws > 0:
+                paths.append("tcgen05-f8")
+                wsf = torch.empty(f8_ws, dtype=torch.uint8, device=dev)
             for path in paths:
-                if path == "table-f32":
+                if path == "tcgen05-f8":
+                    fns = [(lambda c=pbufs[r % copies]:
+                            tbn.tbn_linear_fwd_f8(x, c, alpha, K, wsf, out=y))
+                           for r in range(reps)]
+                elif path == "table-f32":
                     fns = [(lambda c=bufs[r % copies]:
                             tbn.tbn_linear_fwd_ws(x32, c, alpha, K, ws, out=y))
                            for r in range(reps)]
@@ -578,7 +590,7 @@ def run_gemv(args, rank, world, local_rank, sizes=None, batches=None, reps=None)
                               "frac_hbm": round(byts / t / 1e9 / hbm, 4),
                               "tflops": round(2 * B * K * K / t / 1e12, 3)})
                 del g
-        del bufs
+        del bufs, pbufs
         torch.cuda.empty_cache()
     clocks = sampler.stop(t0, time.time())
     head = ([s for s in sweep if s["K"] == 16384 and s["B"] == 1 and s["path"] == "mma"] or

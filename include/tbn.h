@@ -84,7 +84,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 7
+#define TBN_ABI_VERSION 8
 
 typedef enum {
   TBN_OK = 0,
@@ -214,6 +214,42 @@ tbn_status tbn_quantize_pack_group(const tbn_quant_job *jobs, int njobs, tbn_str
  * Padding fields are ignored. */
 tbn_status tbn_unpack(const uint32_t *codes, const float *alpha, int64_t K, int64_t n,
                       void *out, tbn_unpack_format fmt, tbn_stream stream);
+
+/* Batch-1 two-bit linear layer on fp8 tensor cores (Section 3: y[k] =
+ * alpha[k] sum_j x[j] W~[k, j]).  W~/2 in {+-0.5, +-1} is exact in e4m3; x
+ * (bf16) is split exactly into three e4m3 terms under one power-of-two
+ * scale, x 2^E = t1 + t2/16 + t3/256 + r with |r| <= 2^-25 max|x| per
+ * element, so the result stays within 2e-3 alpha sum|x| for K_in <= 16384;
+ * accumulation is fp32, and the partial sums of a row are added in a fixed
+ * order (bitwise reproducible).
+ *
+ * tbn_linear_prepare_f8 rewrites codes [K_out][tbn_packed_words(K_in)]
+ * (the byte-planar layout; K_in a multiple of 512) into this path's
+ * prepared layout, once per weight matrix: "e4m3-planar" words (the 16
+ * codes of a word, code 4j + b at bits 8b + j (m) and 8b + 4 + j (s)),
+ * blocked by 128 rows x 512 codes (16 KiB contiguous per block, the 16-byte
+ * chunks of a row permuted by the row's low 3 bits), rows past K_out zero.
+ * prepared holds tbn_linear_f8_prepared_words(K_out, K_in) words (-1: the
+ * shape is not taken), 16-byte aligned, not overlapping codes.
+ *
+ * tbn_linear_fwd_f8 runs it: x bf16 [1][K_in], K_in a multiple of 512 and at
+ * most 16384, x 16-byte aligned, prepared codes of the same K_out and K_in, alpha fp32 [K_out], y [1][K_out]
+ * bf16 or fp32, optional epilogue (ReLU, residual; no pool), and a caller
+ * workspace (256-byte aligned, contents on entry irrelevant, at least
+ * tbn_linear_f8_workspace_bytes) that calls which may run concurrently must
+ * not share.  One launch when the 128-row tiles fill most SMs (each CTA
+ * owns whole tiles), else two (the rows' K ranges are spread over CTAs and
+ * a second kernel adds their partial sums in a fixed order).
+ * tbn_linear_f8_workspace_bytes returns 0 for shapes this path does not
+ * take (then tbn_linear_fwd_f8 returns TBN_ERR_UNSUPPORTED). */
+int64_t tbn_linear_f8_prepared_words(int64_t K_out, int64_t K_in);
+tbn_status tbn_linear_prepare_f8(const uint32_t *codes, int64_t K_out, int64_t K_in,
+                                 uint32_t *prepared, tbn_stream stream);
+size_t tbn_linear_f8_workspace_bytes(int64_t B, int64_t K_in, int64_t K_out);
+tbn_status tbn_linear_fwd_f8(const void *x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                             const uint32_t *prepared, const float *alpha, int64_t K_out, void *y,
+                             tbn_dtype ydt, const tbn_epilogue *epi, void *workspace,
+                             size_t workspace_bytes, tbn_stream stream);
 
 /* Canonical ("sequential") two-bit layout, the interchange format for codes
  * exchanged with other software: the same field f = m + 2 s per code (Section

@@ -31,6 +31,8 @@ __all__ = [
     "tbn_selftest_wait_timeout", "tbn_repack", "TBN_REPACK_CANONICAL_TO_PLANAR",
     "TBN_REPACK_PLANAR_TO_CANONICAL", "tbn_dense_conv2d_fwd", "tbn_avgpool2d_global_nhwc",
     "tbn_dense_linear_fwd", "tbn_space_to_depth", "space_to_depth_shape", "TBN_S2D_NHWC",
+    "tbn_linear_prepare_f8", "tbn_linear_f8_workspace_bytes", "tbn_linear_fwd_f8",
+    "tbn_linear_f8_prepared_words",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -56,7 +58,8 @@ EXPORTED = [
     "tbn_conv2d_bwd_data", "tbn_conv2d_bwd_filter_workspace_bytes", "tbn_conv2d_bwd_filter",
     "tbn_selftest_wait_timeout", "tbn_repack", "tbn_dense_conv2d_fwd",
     "tbn_avgpool2d_global_nhwc", "tbn_dense_linear_fwd", "tbn_space_to_depth_elems",
-    "tbn_space_to_depth",
+    "tbn_space_to_depth", "tbn_linear_prepare_f8", "tbn_linear_f8_workspace_bytes",
+    "tbn_linear_fwd_f8", "tbn_linear_f8_prepared_words",
 ]
 
 
@@ -80,7 +83,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 7  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 8  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -136,6 +139,11 @@ def lib():
             "tbn_nchw_to_nhwc": ([P, I32, I64, I64, I64, I64, I64, P, P], I32),
             "tbn_space_to_depth_elems": ([I64] * 10, I64),
             "tbn_space_to_depth": ([P, I32, I32] + [I64] * 10 + [P, P], I32),
+            "tbn_linear_prepare_f8": ([U32P, I64, I64, U32P, P], I32),
+            "tbn_linear_f8_workspace_bytes": ([I64, I64, I64], ctypes.c_size_t),
+            "tbn_linear_f8_prepared_words": ([I64, I64], I64),
+            "tbn_linear_fwd_f8": ([P, I32, I64, I64, U32P, P, I64, P, I32,
+                                   ctypes.POINTER(Epilogue), P, ctypes.c_size_t, P], I32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(L, name)
@@ -421,6 +429,54 @@ def tbn_linear_fwd_ws(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor,
                                    ctypes.byref(e) if e is not None else None, ws_ptr, ws_bytes,
                                    _stream(stream)),
            "tbn_linear_fwd_ws")
+    return out
+
+
+def tbn_linear_f8_prepared_words(K_out: int, K_in: int) -> int:
+    return int(lib().tbn_linear_f8_prepared_words(K_out, K_in))
+
+
+def tbn_linear_prepare_f8(codes: torch.Tensor, K_in: int, out: torch.Tensor | None = None,
+                          stream=None) -> torch.Tensor:
+    """The codes [K_out, packed_words(K_in)] rewritten in the fp8 GEMV's
+    prepared layout (once per weight matrix): a flat int32 tensor of
+    tbn_linear_f8_prepared_words(K_out, K_in) words."""
+    _cuda(codes, "codes")
+    K_out = codes.shape[0]
+    n = tbn_linear_f8_prepared_words(K_out, K_in)
+    if n < 0:
+        raise ValueError("no fp8 GEMV layout for K_in = %d (a multiple of 512 is needed)" % K_in)
+    if out is None:
+        out = torch.empty((n,), dtype=torch.int32, device=codes.device)
+    elif out.numel() != n:
+        raise ValueError("out must hold tbn_linear_f8_prepared_words(K_out, K_in) words")
+    _check(lib().tbn_linear_prepare_f8(codes.data_ptr(), K_out, K_in, out.data_ptr(),
+                                       _stream(stream)), "tbn_linear_prepare_f8")
+    return out
+
+
+def tbn_linear_f8_workspace_bytes(B: int, K_in: int, K_out: int) -> int:
+    return int(lib().tbn_linear_f8_workspace_bytes(B, K_in, K_out))
+
+
+def tbn_linear_fwd_f8(x: torch.Tensor, prepared: torch.Tensor, alpha: torch.Tensor, K_out: int,
+                      workspace: torch.Tensor, out_dtype=None, relu: bool = False,
+                      residual: torch.Tensor | None = None, out: torch.Tensor | None = None,
+                      stream=None):
+    """Batch-1 fp8 tensor-core linear layer on codes from tbn_linear_prepare_f8
+    (x bf16 [1, K_in]; workspace of at least tbn_linear_f8_workspace_bytes)."""
+    _cuda(x, "x"), _cuda(prepared, "prepared"), _cuda(alpha, "alpha"), _cuda(workspace, "workspace")
+    B, K_in = x.shape
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    if out is None:
+        out = torch.empty((B, K_out), dtype=_torch_dt(ydt), device=x.device)
+    e = _epi(relu, residual)
+    _check(lib().tbn_linear_fwd_f8(x.data_ptr(), _dt(x), B, K_in, prepared.data_ptr(),
+                                   alpha.data_ptr(), K_out, out.data_ptr(), ydt,
+                                   ctypes.byref(e) if e is not None else None,
+                                   workspace.data_ptr(),
+                                   workspace.numel() * workspace.element_size(), _stream(stream)),
+           "tbn_linear_fwd_f8")
     return out
 
 

@@ -429,6 +429,52 @@ tbn_status tbn_linear_fwd(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
   return tbn_linear_fwd_ws(x, xdt, B, K_in, codes, alpha, K_out, y, ydt, epi, nullptr, 0, stream);
 }
 
+int64_t tbn_linear_f8_prepared_words(int64_t K_out, int64_t K_in) {
+  if (K_out < 1 || K_in < 1 || K_in % 512 != 0 || K_in > (int64_t(1) << 30) ||
+      K_out >= (int64_t(1) << 24))
+    return -1;
+  return gemv_f8_prepared_words(K_out, K_in);
+}
+
+tbn_status tbn_linear_prepare_f8(const uint32_t* codes, int64_t K_out, int64_t K_in,
+                                 uint32_t* prepared, tbn_stream stream) {
+  if (!codes || !prepared) return fail(TBN_ERR_INVALID_ARG, "prepare_f8: null pointer");
+  if (K_out < 1 || K_in < 1) return fail(TBN_ERR_INVALID_ARG, "prepare_f8: sizes must be >= 1");
+  const int64_t words = tbn_linear_f8_prepared_words(K_out, K_in);
+  if (words < 0) return fail(TBN_ERR_UNSUPPORTED, "prepare_f8: K_in must be a multiple of 512");
+  if (!is_aligned(codes, 4) || !is_aligned(prepared, 16))
+    return fail(TBN_ERR_MISALIGNED, "prepare_f8: codes need 4-byte, prepared 16-byte alignment");
+  const uintptr_t a = reinterpret_cast<uintptr_t>(codes), b = reinterpret_cast<uintptr_t>(prepared);
+  const uintptr_t na = static_cast<uintptr_t>(K_out * (K_in / 16)) * 4;
+  const uintptr_t nb = static_cast<uintptr_t>(words) * 4;
+  if (a < b + nb && b < a + na) return fail(TBN_ERR_INVALID_ARG, "prepare_f8: codes and prepared overlap");
+  return launch_prepare_f8(codes, K_out, K_in, prepared, as_stream(stream));
+}
+
+size_t tbn_linear_f8_workspace_bytes(int64_t B, int64_t K_in, int64_t K_out) {
+  if (B != 1 || K_in < 1 || K_out < 1 || K_out >= (int64_t(1) << 24)) return 0;
+  return gemv_f8_workspace_bytes(K_in, K_out);
+}
+
+tbn_status tbn_linear_fwd_f8(const void* x, tbn_dtype xdt, int64_t B, int64_t K_in,
+                             const uint32_t* prepared, const float* alpha, int64_t K_out, void* y,
+                             tbn_dtype ydt, const tbn_epilogue* epi, void* workspace,
+                             size_t workspace_bytes, tbn_stream stream) {
+  const tbn_status st = validate_linear(x, xdt, B, K_in, prepared, alpha, K_out, y, ydt, epi);
+  if (st != TBN_OK) return st;
+  if (xdt != TBN_BF16) return fail(TBN_ERR_UNSUPPORTED, "fp8 GEMV: x must be bf16");
+  const char* why = gemv_f8_unsupported_reason(B, K_in, K_out);
+  if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
+  if (!workspace) return fail(TBN_ERR_INVALID_ARG, "fp8 GEMV: null workspace");
+  if (!is_aligned(x, 16) || !is_aligned(prepared, 16) || !is_aligned(workspace, 256))
+    return fail(TBN_ERR_MISALIGNED,
+                "fp8 GEMV: x and the codes need 16-byte, the workspace 256-byte alignment");
+  if (workspace_bytes < gemv_f8_workspace_bytes(K_in, K_out))
+    return fail(TBN_ERR_INVALID_ARG, "fp8 GEMV: workspace smaller than tbn_linear_f8_workspace_bytes");
+  return launch_gemv_f8(x, K_in, prepared, alpha, K_out, y, ydt, epi ? epi->residual : nullptr,
+                        epi ? epi->relu : 0, workspace, workspace_bytes, as_stream(stream));
+}
+
 size_t tbn_linear_workspace_bytes(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out) {
   if ((xdt != TBN_F32 && xdt != TBN_BF16) || B < 1 || K_in < 1 || K_out < 1) return 0;
   if (gemv_lut_shape_reason(xdt, B, K_in, K_out)[0] == '\0')

@@ -130,6 +130,16 @@ const char* gemv_lut_shape_reason(tbn_dtype xdt, int64_t B, int64_t K_in, int64_
 const char* gemv_lut_unsupported_reason(tbn_dtype xdt, int64_t B, int64_t K_in, int64_t K_out,
                                         const uint32_t* codes);
 size_t gemv_lut_workspace_bytes(int64_t K_in, int64_t K_out);
+// batch-1 fp8 tensor-core GEMV (csrc/tbn_gemv_f8.cu) on codes in the
+// e4m3-planar layout written by launch_prepare_f8
+const char* gemv_f8_unsupported_reason(int64_t B, int64_t K_in, int64_t K_out);
+size_t gemv_f8_workspace_bytes(int64_t K_in, int64_t K_out);
+int64_t gemv_f8_prepared_words(int64_t K_out, int64_t K_in);
+tbn_status launch_prepare_f8(const uint32_t* codes, int64_t K_out, int64_t K_in, uint32_t* out,
+                             cudaStream_t s);
+tbn_status launch_gemv_f8(const void* x, int64_t K_in, const uint32_t* prepared, const float* alpha,
+                          int64_t K_out, void* y, tbn_dtype ydt, const void* residual, int relu,
+                          void* workspace, size_t workspace_bytes, cudaStream_t s);
 tbn_status launch_gemv_lut(const void* x, int64_t K_in, const uint32_t* codes,
                            const float* alpha, int64_t K_out, void* y, tbn_dtype ydt, int relu,
                            const void* residual, void* workspace, size_t workspace_bytes,

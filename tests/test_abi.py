@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 7
+    assert L.tbn_abi_version() == 8
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -122,6 +122,33 @@ def test_space_to_depth_host_rules(L):
     assert _conv(L, **dict(s2d, K=129)) == tbn.TBN_ERR_UNSUPPORTED
     assert _conv(L, **dict(s2d, sw=2)) == tbn.TBN_ERR_UNSUPPORTED
     assert b"space-to-depth" in L.tbn_last_error()
+
+
+def test_f8_linear_host_rules(L):
+    # prepared layout: ceil(K_out / 128) * 128 rows x K_in / 16 words; K_in % 512 == 0
+    assert L.tbn_linear_f8_prepared_words(1000, 16384) == 1024 * 1024
+    assert L.tbn_linear_f8_prepared_words(128, 512) == 128 * 32
+    assert L.tbn_linear_f8_prepared_words(128, 500) == -1
+    assert L.tbn_linear_f8_prepared_words(0, 512) == -1
+    assert L.tbn_linear_f8_workspace_bytes(1, 4096, 4096) >= 256
+    assert L.tbn_linear_f8_workspace_bytes(2, 4096, 4096) == 0      # batch 1 only
+    assert L.tbn_linear_f8_workspace_bytes(1, 32768, 64) == 0       # K_in <= 16384
+    assert L.tbn_linear_f8_workspace_bytes(1, 1000, 64) == 0        # K_in % 512
+    d = ctypes.c_void_p(256)
+    assert L.tbn_linear_prepare_f8(None, 4, 512, d, None) == tbn.TBN_ERR_INVALID_ARG
+    assert L.tbn_linear_prepare_f8(d, 4, 500, ctypes.c_void_p(1 << 40), None) == tbn.TBN_ERR_UNSUPPORTED
+    assert L.tbn_linear_prepare_f8(d, 4, 512, ctypes.c_void_p((1 << 40) + 4), None) == \
+        tbn.TBN_ERR_MISALIGNED
+    assert L.tbn_linear_prepare_f8(d, 4, 512, ctypes.c_void_p(512), None) == \
+        tbn.TBN_ERR_INVALID_ARG                                                  # overlap
+    ws = ctypes.c_void_p(1 << 20)
+    args = [d, 1, 1, 4096, d, d, 64, d, 1, None]
+    assert L.tbn_linear_fwd_f8(*args[:1], 0, *args[2:], ws, 1 << 20, None) == \
+        tbn.TBN_ERR_UNSUPPORTED                                                  # fp32 x
+    assert L.tbn_linear_fwd_f8(d, 1, 2, 4096, d, d, 64, d, 1, None, ws, 1 << 20, None) == \
+        tbn.TBN_ERR_UNSUPPORTED                                                  # B = 2
+    assert L.tbn_linear_fwd_f8(d, 1, 1, 4096, d, d, 64, d, 1, None, None, 0, None) == \
+        tbn.TBN_ERR_INVALID_ARG                                                  # no workspace
 
 
 def test_select_algo_host_rules(L):
