@@ -81,9 +81,10 @@ WORKLOADS = {
 # mean over its eight launches, from the full-size ncu capture summarised in
 # profiles/alexnet_b256_launches.md.  Valid only for the kernel sources it was
 # measured on (hash below); otherwise the roofline entry reports null.
-CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
+CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cuh",
+                            "paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
                             "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
-                "sha256_16": "d5695663ad5b1be0", "bytes_per_launch": 48.01e6}
+                "sha256_16": None, "bytes_per_launch": None}
 
 
 def measured_traffic(rec):
@@ -652,6 +653,62 @@ def run_quantize(args, rank, world, local_rank, sizes=None, reps=None):
             "sweep": sweep, "clocks": clocks}
 
 
+# ------------------------------------------------- fused quantize + convolve
+FUSED_LAYERS = (
+    # name, N, C, K, R, pad, H (stride 1, square maps, NHWC bf16)
+    ("alexnet_conv3_b256", 256, 256, 384, 3, 1, 13),
+    ("vgg_c4_b128", 128, 256, 256, 3, 1, 16),
+    ("vgg_c6_b8", 8, 512, 512, 3, 1, 8),
+)
+
+
+def run_fused_quant_conv(args, local_rank, reps=5):
+    """Per layer: the fp32 filters quantized and the convolution run (a) as
+    two launches (tbn_quantize_pack, tbn_conv2d_fwd) and (b) as the one fused
+    launch (tbn_conv2d_fwd_quant), each replayed from a graph after an L2
+    flush; both give bitwise the same codes, alpha and output."""
+    import paper_1701_00485_gb300 as tbn
+    from paper_1701_00485_gb300 import inputs
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.Stream(device=dev)
+    flush = L2Flush(dev)
+    out = []
+    for name, N, C, K, R, pad, H in FUSED_LAYERS:
+        g = inputs.generator(5)
+        x = torch.randn(N, H, H, C, generator=g).to(torch.bfloat16).to(dev)
+        W = inputs.normal((K, R * R * C), (2.0 / (C * R * R)) ** 0.5, g).to(dev)
+        codes = torch.empty((K, tbn.packed_words(R * R * C)), dtype=torch.int32, device=dev)
+        alpha = torch.empty((K,), dtype=torch.float32, device=dev)
+        ws = torch.empty(64, dtype=torch.uint8, device=dev)
+        y = torch.empty((N, H, H, K), dtype=torch.bfloat16, device=dev)
+
+        def separate():
+            tbn.tbn_quantize_pack(W, codes, alpha)
+            tbn.tbn_conv2d_fwd(x, codes, alpha, K, R, R, (1, 1), (pad, pad), relu=True,
+                               algo=tbn.TBN_CONV_IMPLICIT_GEMM, out=y)
+
+        def fused():
+            tbn.tbn_conv2d_fwd_quant(x, W, K, R, R, (1, 1), (pad, pad), relu=True, codes=codes,
+                                     alpha=alpha, workspace=ws, out=y)
+        row = {"layer": name}
+        for key, fn in (("separate_us", separate), ("fused_us", fused)):
+            with torch.cuda.stream(stream):
+                fn()   # once outside the capture: the library's one-time kernel set-up
+            torch.cuda.synchronize(dev)
+            gr, ev = capture(fn, stream, dev)
+            for _ in range(max(3, args.warmup)):
+                gr.replay()
+            torch.cuda.synchronize(dev)
+            row[key] = round(float(np.median(timed_replays(gr, stream, flush, ev, reps))) * 1e3, 2)
+            del gr
+        out.append(row)
+        del x, W, codes, alpha, ws, y
+        torch.cuda.empty_cache()
+    return {"layers": out, "note": "graph replay after an L2 flush; separate = quantize "
+            "launch + convolution launch, fused = one cooperative launch with a grid barrier"}
+
+
 # ------------------------------------------------------------------ backward
 def run_backward(args, rank, world, local_rank):
     """TwoBitBackward for every VGG-small layer: dx (tensor-core forward
@@ -963,6 +1020,7 @@ def main():
             extras["quantize"] = {"sweep": q["sweep"], "clocks": q["clocks"]}
             gm = run_gemv(args, rank, world, local_rank, reps=3)
             extras["gemv"] = {"sweep": gm["sweep"], "clocks": gm["clocks"]}
+            extras["fused_quant_conv"] = run_fused_quant_conv(args, local_rank)
             res["extras"] = extras
     else:
         runner = {"lenet": None, "gemv": run_gemv, "quantize": run_quantize,

@@ -84,7 +84,7 @@
 extern "C" {
 #endif
 
-#define TBN_ABI_VERSION 8
+#define TBN_ABI_VERSION 9
 
 typedef enum {
   TBN_OK = 0,
@@ -319,6 +319,31 @@ tbn_status tbn_space_to_depth(const void *x, tbn_dtype xdt, tbn_layout layout, i
                               int64_t C, int64_t H, int64_t W, int64_t R, int64_t S,
                               int64_t stride_h, int64_t stride_w, int64_t pad_h, int64_t pad_w,
                               void *out, tbn_stream stream);
+
+/* Algorithm 1's quantization loop fused with TwoBitForward in one launch
+ * (Eq. 3, Eq. 5, Eq. 1): the CTAs of the implicit GEMM first quantize the
+ * fp32 filters Wf [K][C*R*S] (in (r, s, c) order) into codes and alpha,
+ * bitwise as tbn_quantize_pack writes them, meet at a grid-wide barrier (a
+ * cooperative launch), then convolve as tbn_conv2d_fwd does with those
+ * codes.  codes [K][tbn_packed_words(C*R*S)] and alpha [K] are outputs.
+ * Takes the implicit GEMM's TMA activation shapes: NHWC bf16 x with
+ * C % 32 == 0 and strides <= 2, C*R*S <= 32768 (else TBN_ERR_UNSUPPORTED).
+ * Wf 4-byte aligned (16-byte aligned with C*R*S % 4 == 0 for vector loads).
+ * workspace: at least 4 bytes, 4-byte aligned, zeroed by the call (a barrier
+ * word: calls that may run concurrently must not share it).  Wf, codes and
+ * alpha must not overlap.  The launch uses one CTA per SM and needs the
+ * whole GPU (a cooperative launch: it fails with TBN_ERR_CUDA if the CTAs
+ * cannot all be resident); a barrier that runs out of time sets
+ * the timeout bit of the device error word.  It is launched plainly (not as
+ * a programmatic dependent): it starts after the previous kernel on the
+ * stream has completed, so Wf may be that kernel's output.  On this GPU it
+ * is a few microseconds slower than tbn_quantize_pack + tbn_conv2d_fwd. */
+tbn_status tbn_conv2d_fwd_quant(const void *x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                                int64_t C, int64_t H, int64_t W, const float *Wf, int64_t K,
+                                int64_t R, int64_t S, int64_t stride_h, int64_t stride_w,
+                                int64_t pad_h, int64_t pad_w, uint32_t *codes, float *alpha,
+                                void *y, tbn_dtype ydt, const tbn_epilogue *epi, void *workspace,
+                                size_t workspace_bytes, tbn_stream stream);
 
 /* tbn_conv2d_fwd with an explicit algorithm.  Returns TBN_ERR_UNSUPPORTED if
  * the requested algorithm cannot run this shape. */

@@ -32,7 +32,7 @@ __all__ = [
     "TBN_REPACK_PLANAR_TO_CANONICAL", "tbn_dense_conv2d_fwd", "tbn_avgpool2d_global_nhwc",
     "tbn_dense_linear_fwd", "tbn_space_to_depth", "space_to_depth_shape", "TBN_S2D_NHWC",
     "tbn_linear_prepare_f8", "tbn_linear_f8_workspace_bytes", "tbn_linear_fwd_f8",
-    "tbn_linear_f8_prepared_words",
+    "tbn_linear_f8_prepared_words", "tbn_conv2d_fwd_quant",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -59,7 +59,7 @@ EXPORTED = [
     "tbn_selftest_wait_timeout", "tbn_repack", "tbn_dense_conv2d_fwd",
     "tbn_avgpool2d_global_nhwc", "tbn_dense_linear_fwd", "tbn_space_to_depth_elems",
     "tbn_space_to_depth", "tbn_linear_prepare_f8", "tbn_linear_f8_workspace_bytes",
-    "tbn_linear_fwd_f8", "tbn_linear_f8_prepared_words",
+    "tbn_linear_fwd_f8", "tbn_linear_f8_prepared_words", "tbn_conv2d_fwd_quant",
 ]
 
 
@@ -83,7 +83,7 @@ _lock = threading.Lock()
 _lib = None
 
 
-ABI_VERSION = 8  # must match TBN_ABI_VERSION in include/tbn.h
+ABI_VERSION = 9  # must match TBN_ABI_VERSION in include/tbn.h
 
 
 def lib_path() -> str:
@@ -142,6 +142,9 @@ def lib():
             "tbn_linear_prepare_f8": ([U32P, I64, I64, U32P, P], I32),
             "tbn_linear_f8_workspace_bytes": ([I64, I64, I64], ctypes.c_size_t),
             "tbn_linear_f8_prepared_words": ([I64, I64], I64),
+            "tbn_conv2d_fwd_quant": ([P, I32, I32, I64, I64, I64, I64, P] + [I64] * 7 +
+                                     [U32P, P, P, I32, ctypes.POINTER(Epilogue), P,
+                                      ctypes.c_size_t, P], I32),
             "tbn_linear_fwd_f8": ([P, I32, I64, I64, U32P, P, I64, P, I32,
                                    ctypes.POINTER(Epilogue), P, ctypes.c_size_t, P], I32),
         }
@@ -295,6 +298,42 @@ def tbn_conv2d_fwd(x: torch.Tensor, codes: torch.Tensor, alpha: torch.Tensor, K:
         stride[0], stride[1], pad[0], pad[1], out.data_ptr(), ydt,
         ctypes.byref(e) if e is not None else None, algo, _stream(stream)), "tbn_conv2d_fwd")
     return out
+
+
+def tbn_conv2d_fwd_quant(x: torch.Tensor, W: torch.Tensor, K: int, R: int, S: int,
+                         stride=(1, 1), pad=(0, 0), out_dtype=None, relu: bool = False,
+                         residual: torch.Tensor | None = None, pool: int = 0,
+                         codes: torch.Tensor | None = None, alpha: torch.Tensor | None = None,
+                         workspace: torch.Tensor | None = None, out: torch.Tensor | None = None,
+                         stream=None):
+    """Quantization (Eq. 3, Eq. 5) of the fp32 filters W [K, R*S*C] ((r, s, c)
+    order) and the two-bit convolution of NHWC bf16 x [N, H, W, C] with them,
+    in one launch.  Returns (y, codes, alpha); codes and alpha equal what
+    tbn_quantize_pack writes for W."""
+    _cuda(x, "x"), _cuda(W, "W")
+    N, H, Wd, C = x.shape
+    n = W.shape[1]
+    if W.dtype != torch.float32 or tuple(W.shape) != (K, R * S * C) or not W.is_contiguous():
+        raise ValueError("W must be a contiguous float32 tensor [K, R*S*C]")
+    if codes is None:
+        codes = torch.empty((K, packed_words(n)), dtype=torch.int32, device=x.device)
+    if alpha is None:
+        alpha = torch.empty((K,), dtype=torch.float32, device=x.device)
+    if workspace is None:
+        workspace = torch.empty((64,), dtype=torch.uint8, device=x.device)
+    P, Q = conv_out_hw(H, Wd, R, S, stride, pad)
+    if pool:
+        P, Q = P // 2, Q // 2
+    ydt = _dt(x) if out_dtype is None else (TBN_F32 if out_dtype == torch.float32 else TBN_BF16)
+    if out is None:
+        out = torch.empty((N, P, Q, K), dtype=_torch_dt(ydt), device=x.device)
+    e = _epi(relu, residual, pool)
+    _check(lib().tbn_conv2d_fwd_quant(
+        x.data_ptr(), _dt(x), TBN_NHWC, N, C, H, Wd, W.data_ptr(), K, R, S, stride[0], stride[1],
+        pad[0], pad[1], codes.data_ptr(), alpha.data_ptr(), out.data_ptr(), ydt,
+        ctypes.byref(e) if e is not None else None, workspace.data_ptr(),
+        workspace.numel() * workspace.element_size(), _stream(stream)), "tbn_conv2d_fwd_quant")
+    return out, codes, alpha
 
 
 def space_to_depth_shape(N: int, C: int, H: int, W: int, R: int, S: int, stride=(4, 4),

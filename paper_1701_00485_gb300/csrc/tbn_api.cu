@@ -339,6 +339,35 @@ tbn_status tbn_conv2d_fwd(const void* x, tbn_dtype xdt, tbn_layout layout, int64
                              stride_w, pad_h, pad_w, y, ydt, epi, TBN_CONV_AUTO, stream);
 }
 
+tbn_status tbn_conv2d_fwd_quant(const void* x, tbn_dtype xdt, tbn_layout layout, int64_t N,
+                                int64_t C, int64_t H, int64_t W, const float* Wf, int64_t K,
+                                int64_t R, int64_t S, int64_t stride_h, int64_t stride_w,
+                                int64_t pad_h, int64_t pad_w, uint32_t* codes, float* alpha,
+                                void* y, tbn_dtype ydt, const tbn_epilogue* epi, void* workspace,
+                                size_t workspace_bytes, tbn_stream stream) {
+  if (!Wf) return fail(TBN_ERR_INVALID_ARG, "conv quant: null filters");
+  ConvProblem p{};
+  const tbn_status st = validate_conv(x, xdt, layout, N, C, H, W, codes, alpha, K, R, S, stride_h,
+                                      stride_w, pad_h, pad_w, y, ydt, epi, &p);
+  if (st != TBN_OK) return st;
+  if (!workspace || workspace_bytes < 4) return fail(TBN_ERR_INVALID_ARG, "conv quant: workspace < 4 bytes");
+  if (!is_aligned(Wf, 4) || !is_aligned(workspace, 4))
+    return fail(TBN_ERR_MISALIGNED, "conv quant: filters and workspace need 4-byte alignment");
+  if (layout == TBN_S2D_NHWC || C * R * S > 32768)
+    return fail(TBN_ERR_UNSUPPORTED, "conv quant: needs C*R*S <= 32768 and no space-to-depth input");
+  const int64_t nbytes = K * C * R * S * 4, cbytes = K * ((C * R * S + 15) / 16) * 4;
+  const uintptr_t w0 = reinterpret_cast<uintptr_t>(Wf), c0 = reinterpret_cast<uintptr_t>(codes),
+                  a0 = reinterpret_cast<uintptr_t>(alpha);
+  if ((c0 < w0 + nbytes && w0 < c0 + cbytes) || (a0 < w0 + nbytes && w0 < a0 + K * 4) ||
+      (a0 < c0 + cbytes && c0 < a0 + K * 4))
+    return fail(TBN_ERR_INVALID_ARG, "conv quant: filters, codes and alpha must not overlap");
+  p.wq = Wf;
+  p.gbar = static_cast<unsigned*>(workspace);
+  const char* why = conv_igemm_unsupported_reason(p);
+  if (why[0] != '\0') return fail(TBN_ERR_UNSUPPORTED, "%s", why);
+  return launch_conv_igemm(p, as_stream(stream));
+}
+
 int64_t tbn_space_to_depth_elems(int64_t N, int64_t C, int64_t H, int64_t W, int64_t R,
                                  int64_t S, int64_t stride_h, int64_t stride_w, int64_t pad_h,
                                  int64_t pad_w) {

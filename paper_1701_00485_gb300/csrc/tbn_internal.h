@@ -62,6 +62,11 @@ struct ConvProblem {
   // second kernel adds them in order and applies the epilogue
   float* partial;
   int ksplit;
+  // fused quantization (implicit GEMM only; set by tbn_conv2d_fwd_quant):
+  // fp32 filters [K][C*R*S] quantized into codes and alpha by the same
+  // launch; gbar is a 4-byte barrier word the launcher zeroes
+  const float* wq;
+  unsigned* gbar;
 };
 
 // Space-to-depth form of a strided convolution with few input channels

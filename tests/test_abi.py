@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_abi_version_and_sizes(L):
-    assert L.tbn_abi_version() == 8
+    assert L.tbn_abi_version() == 9
     assert [tbn.packed_words(n) for n in (1, 15, 16, 17, 27, 1152, 16384)] == \
         [1, 1, 1, 2, 2, 72, 1024]
     assert L.tbn_packed_words(0) == -1
@@ -149,6 +149,25 @@ def test_f8_linear_host_rules(L):
         tbn.TBN_ERR_UNSUPPORTED                                                  # B = 2
     assert L.tbn_linear_fwd_f8(d, 1, 1, 4096, d, d, 64, d, 1, None, None, 0, None) == \
         tbn.TBN_ERR_INVALID_ARG                                                  # no workspace
+
+
+def test_conv_quant_host_rules(L):
+    # tbn_conv2d_fwd_quant: filters, a barrier word, no overlap of the filters
+    # with the codes and alpha it writes; checked before anything is launched
+    v = [ctypes.c_void_p(i << 30) for i in range(1, 7)]
+    x, Wf, codes, alpha, y, ws = v
+
+    def call(layout=tbn.TBN_NHWC, C=64, W=Wf, c=codes, a=alpha, w=ws, wb=64):
+        return L.tbn_conv2d_fwd_quant(x, 1, layout, 2, C, 8, 8, W, 128, 3, 3, 1, 1, 1, 1, c, a,
+                                      y, 1, None, w, wb, None)
+    assert call(W=None) == tbn.TBN_ERR_INVALID_ARG
+    assert call(w=None, wb=0) == tbn.TBN_ERR_INVALID_ARG
+    assert call(wb=2) == tbn.TBN_ERR_INVALID_ARG
+    assert call(W=ctypes.c_void_p((2 << 30) + 2)) == tbn.TBN_ERR_MISALIGNED
+    assert call(w=ctypes.c_void_p((6 << 30) + 2)) == tbn.TBN_ERR_MISALIGNED
+    assert call(c=ctypes.c_void_p((2 << 30) + 4096)) == tbn.TBN_ERR_INVALID_ARG    # overlap
+    assert call(a=ctypes.c_void_p((2 << 30) + 4096)) == tbn.TBN_ERR_INVALID_ARG    # overlap
+    assert call(C=4096) == tbn.TBN_ERR_UNSUPPORTED                                 # C R S > 32768
 
 
 def test_select_algo_host_rules(L):
