@@ -192,6 +192,10 @@ tbn_status launch_conv_igemm(const ConvProblem& p0, cudaStream_t s) {
         t.tile_n + 32 * a.kblocks > kTmemCols || p.pool || p.residual)
       return fail(TBN_ERR_UNSUPPORTED, "implicit GEMM: space-to-depth problem out of range");
   }
+  // tiles of at most 176 pixels: two accumulators, so each tile's MMAs
+  // overlap the previous tile's epilogue (space-to-depth mode keeps its
+  // resident K blocks where the second accumulator would be)
+  a.acc2 = (!s2d && t.tile_n <= kAcc2Cols) ? 1 : 0;
   a.x = static_cast<const __nv_bfloat16*>(p.x);
   a.codes = p.codes; a.alpha = p.alpha; a.y = p.y; a.residual = p.residual;
   if (p0.wq != nullptr) {

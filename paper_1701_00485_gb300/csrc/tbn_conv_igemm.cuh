@@ -113,6 +113,10 @@ struct IgArgs {
   // tile t % base_tiles; the fp32 partial sums go to `partial`
   // [ksplit][N][P][Q][K] and a second kernel adds them in split order
   int ksplit, kb_per, base_tiles;
+  // two accumulators (tile_n <= 176): tile i accumulates into columns
+  // [176 (i % 2), + 176), so its MMAs need not wait for the epilogue of
+  // tile i - 1; the weight ring then starts at column 352
+  int acc2;
   float* partial;
   // space-to-depth mode: the convolution in original coordinates (stride
   // s2d_s, C0 channels, R0 x S0 filter, codes in (r, s, c) order)
@@ -142,6 +146,7 @@ constexpr int kStages = 5;          // pipeline depth: activation ring (shared
                                     // memory) and weight ring (tensor memory)
 constexpr int kAColsPerStage = kBK / 2;   // 64 bf16 = 32 columns of 32 bits
 constexpr int kAccCols = kMaxTileN;       // the accumulator
+constexpr int kAcc2Cols = 176;            // each of two accumulators (tiles of <= 176 pixels)
 constexpr int kTmemCols = 512;      // accumulator [0,256) + weight ring [256,416)
 constexpr int kExpWarps = 8;
 constexpr int kEpiWarps = 8;
@@ -157,6 +162,7 @@ constexpr int kOutStageBytes = kMaxTileN * kBM * 2;  // 64 KiB bf16 output box
 constexpr uint64_t kWaitLimitNs = 1000000000ull;    // 1 s
 
 static_assert(kAccCols + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
+static_assert(2 * kAcc2Cols + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
 // How the activation operand reaches the stage ring.
 constexpr int kModeTma64 = 0;   // one 64-channel TMA box per K block (C % 64 == 0)
@@ -192,8 +198,8 @@ struct SmemCtl {
   // written; empty: the MMAs that read them have completed.
   uint64_t full[kStages];
   uint64_t empty[kStages];
-  uint64_t acc_full;
-  uint64_t acc_empty;
+  uint64_t acc_full[2];     // accumulator b holds a finished tile
+  uint64_t acc_empty[2];    // accumulator b has been read by the epilogue
   uint64_t res_full;
   uint64_t mma_drain;      // used only to drain in-flight MMAs after an abort
   uint32_t tmem_base;
@@ -415,8 +421,10 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     }
     mbar_init(&ctl->patch_full[0], 1);
     mbar_init(&ctl->patch_full[1], 1);
-    mbar_init(&ctl->acc_full, 1);
-    mbar_init(&ctl->acc_empty, 32 * kEpiWarps);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&ctl->acc_full[b], 1);
+      mbar_init(&ctl->acc_empty[b], 32 * kEpiWarps);
+    }
     mbar_init(&ctl->res_full, 1);
     mbar_init(&ctl->mma_drain, 1);
     if (kS2d)
@@ -476,8 +484,8 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     if (warp == 1) tmem_dealloc(ctl->tmem_base, kTmemCols);
     return;
   }
-  const uint32_t acc_tmem = tmem;               // columns [0, 256)
-  const uint32_t a_tmem0 = tmem + kAccCols;     // weight ring
+  const uint32_t acc_tmem = tmem;               // columns [0, 256), or two of 176
+  const uint32_t a_tmem0 = tmem + (a.acc2 ? 2u * kAcc2Cols : static_cast<uint32_t>(kAccCols));   // weight ring
 
   if (!kGather && (warp == 0 || warp >= kFirstGatherWarp)) {
     // ================= TMA producers =================
@@ -852,8 +860,11 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     bool ok = true;
     for (int t = blockIdx.x; t < a.tiles && ok; t += gridDim.x, ++tiles_done) {
       const TileCoord tc = tile_coord(a, t);
-      // the epilogue must have drained the previous tile's accumulator
-      ok = mbar_wait(&ctl->acc_empty, (tiles_done & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
+      // the epilogue must have drained this accumulator's previous tile
+      const uint32_t ab = a.acc2 ? (tiles_done & 1u) : 0u;
+      const uint32_t use = a.acc2 ? (tiles_done >> 1) : tiles_done;   // uses of accumulator ab
+      const uint32_t acc_t = acc_tmem + ab * kAcc2Cols;
+      ok = mbar_wait(&ctl->acc_empty[ab], (use & 1u) ^ 1u, abort_flag, a.err, kWaitLimitNs);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after_sync();
       for (int kb = tc.kb0; kb < tc.kb1; ++kb, ++g) {
@@ -874,7 +885,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
             for (int kk = 0; kk < kBK / 16; ++kk) {
               const uint64_t bdesc = smem_desc_sw64_kmajor(
                   smem_addr(ring + st * kStageBytes + (kk >> 1) * (kStageBytes / 2)));
-              tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * (kk & 1)),
+              tc_mma_ts(acc_t, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * (kk & 1)),
                         idesc, ((kb - tc.kb0) | kk) != 0 ? 1u : 0u);
             }
           } else {
@@ -882,7 +893,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
               // K step kk: 16 codes = 8 TMEM columns of A, 32 bytes of B rows
-              tc_mma_ts(acc_tmem, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
+              tc_mma_ts(acc_t, a_col + 8u * kk, bdesc + static_cast<uint64_t>(2 * kk), idesc,
                         ((kb - tc.kb0) | kk) != 0 ? 1u : 0u);
             }
           }
@@ -892,7 +903,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         ++issued;
       }
       if (ok) {
-        if (elect_one()) tc_commit(&ctl->acc_full);
+        if (elect_one()) tc_commit(&ctl->acc_full[ab]);
         __syncwarp();
       }
     }
@@ -1034,8 +1045,11 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
     // keep walking the tile loop (reaching every barrier) without working.
     for (int t = blockIdx.x; t < a.tiles; t += gridDim.x, ++tiles_done) {
       const TileCoord tc = tile_coord(a, t);
-      const uint32_t par = tiles_done & 1u;
-      const uint32_t acc = acc_tmem + lane_off;
+      const uint32_t par = tiles_done & 1u;   // the residual box
+      const uint32_t ab = a.acc2 ? (tiles_done & 1u) : 0u;
+      const uint32_t apar = (a.acc2 ? (tiles_done >> 1) : tiles_done) & 1u;
+      const uint32_t acc_b = acc_tmem + ab * kAcc2Cols;
+      const uint32_t acc = acc_b + lane_off;
       const int k = tc.ktile * kBM + m;
       const bool kvalid = k < a.K;
       const float a2 = kvalid ? 2.0f * (kFuse ? __ldca(a.alpha + k) : __ldg(a.alpha + k)) : 0.0f;
@@ -1054,8 +1068,8 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         }
       }
       if (ok)
-        ok = kPatch ? mbar_wait_sleep(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs)
-                    : mbar_wait(&ctl->acc_full, par, abort_flag, a.err, kWaitLimitNs);
+        ok = kPatch ? mbar_wait_sleep(&ctl->acc_full[ab], apar, abort_flag, a.err, kWaitLimitNs)
+                    : mbar_wait(&ctl->acc_full[ab], apar, abort_flag, a.err, kWaitLimitNs);
       if (kTmaStore && a.residual && ok)
         ok = mbar_wait(&ctl->res_full, par, abort_flag, a.err, kWaitLimitNs);
       ok = __all_sync(0xffffffffu, ok);
@@ -1087,13 +1101,13 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
           uint32_t v[2][16];
 #pragma unroll
           for (int lg = 0; lg < 2; ++lg)
-            tmem_ld_16x256b_x4(acc_tmem + (static_cast<uint32_t>(sub * 32 + lg * 16) << 16) +
+            tmem_ld_16x256b_x4(acc_b + (static_cast<uint32_t>(sub * 32 + lg * 16) << 16) +
                                    static_cast<uint32_t>(32 * j),
                                v[lg]);
           tmem_wait_ld();
           if (j == c_end - 1) {
             tc_fence_before_sync();
-            mbar_arrive(&ctl->acc_empty);
+            mbar_arrive(&ctl->acc_empty[ab]);
           }
 #pragma unroll
           for (int lg = 0; lg < 2; ++lg) {
@@ -1127,7 +1141,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         }
         if (c_begin >= c_end) {
           tc_fence_before_sync();
-          mbar_arrive(&ctl->acc_empty);
+          mbar_arrive(&ctl->acc_empty[ab]);
         }
       } else if constexpr (kPoolBW == 0) {
         const int T = a.bw * a.bh * a.bn;
@@ -1144,7 +1158,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
           if (j == c_end - 1) {
             // this warp has read its part of the accumulator
             tc_fence_before_sync();
-            mbar_arrive(&ctl->acc_empty);
+            mbar_arrive(&ctl->acc_empty[ab]);
           }
           if (!kTmaStore && a.partial != nullptr) {
             // split K (1x1 image): pixel px is image n0 + px; the raw sum of
@@ -1183,7 +1197,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         }
         if (c_begin >= c_end) {
           tc_fence_before_sync();
-          mbar_arrive(&ctl->acc_empty);
+          mbar_arrive(&ctl->acc_empty[ab]);
         }
       } else {
         // fused 2x2 max pool: tiles hold whole rows of width kPoolBW (q0 = 0)
@@ -1206,7 +1220,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
           tmem_wait_ld();
           if (j == l_end - 1) {
             tc_fence_before_sync();
-            mbar_arrive(&ctl->acc_empty);
+            mbar_arrive(&ctl->acc_empty[ab]);
           }
 #pragma unroll
           for (int pp = 0; pp < kPairs; ++pp) {
@@ -1236,7 +1250,7 @@ __global__ void __launch_bounds__(threads_for<kMode>(), 1)
         }
         if (l_begin >= l_end) {
           tc_fence_before_sync();
-          mbar_arrive(&ctl->acc_empty);
+          mbar_arrive(&ctl->acc_empty[ab]);
         }
       }
       if (kTmaStore) {
