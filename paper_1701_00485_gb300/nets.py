@@ -358,10 +358,15 @@ class ResNet18:
         tbn_dense_linear_fwd(self.feat, self.fc_w, out=self.logits)
         return self.logits
 
-    def forward(self, requantize: bool = False):
+    def forward(self, requantize: bool = False, conv_hook=None):
+        """conv_hook(0, None, "before") is called once, after the stem has
+        read the input (the benchmark copies the next batch from then on)."""
         if requantize:
             self.quantize()
-        return self.head(self.body(self.stem()))
+        h = self.stem()
+        if conv_hook:
+            conv_hook(0, None, "before")
+        return self.head(self.body(h))
 
     def launches_per_forward(self, requantize: bool = False) -> int:
         n = 2 + len(self.convs) + 2
