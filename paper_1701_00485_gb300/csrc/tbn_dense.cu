@@ -49,6 +49,8 @@ struct DenseConvArgs {
   const float* w;    // [K][C][R][S]
   void* y;
   int relu;
+  int stage_out;     // bf16 NHWC output, K % 8 == 0, y 16-byte aligned: the tile's
+                     // outputs go through shared memory and leave as 16-byte stores
 };
 
 // kXNhwc: x is [N][H][W][C] (else [N][C][H][W]); kYNhwc: y is [N][P][Q][K]
@@ -63,6 +65,11 @@ __global__ void __launch_bounds__(kDcThreads) dense_conv_kernel(const DenseConvA
   const int RS = a.R * a.S;
   float* s_w = dsm;                                   // [cc * R * S][64]
   float* s_x = dsm + static_cast<size_t>(a.cc) * RS * kDcFilt;   // [cc][prows][pcols]
+  // staged outputs [4 rows x 32 columns][64 filters] bf16, 128 bytes per
+  // pixel with its 16-byte filter chunks permuted by the pixel's low 3 bits
+  // (after the weights and the patch, rounded up to 128 bytes)
+  uint8_t* s_o = reinterpret_cast<uint8_t*>(
+      dsm + ((static_cast<size_t>(a.cc) * (RS * kDcFilt + a.prows * a.pcols) + 31) & ~size_t(31)));
   const TX* __restrict__ x = static_cast<const TX*>(a.x);
 
   const int k0 = blockIdx.y * kDcFilt;
@@ -155,6 +162,40 @@ __global__ void __launch_bounds__(kDcThreads) dense_conv_kernel(const DenseConvA
       }
     }
 
+    if constexpr (kYNhwc && sizeof(TY) == 2) {
+      if (a.stage_out) {
+        // lane = output column, this warp's 8 filters = one 16-byte chunk
+        const uint32_t o_base = smem_addr(s_o);
+#pragma unroll
+        for (int i = 0; i < kDcRows; ++i) {
+          float v[8];
+#pragma unroll
+          for (int f = 0; f < 8; ++f) v[f] = a.relu ? fmaxf(acc[i][f], 0.0f) : acc[i][f];
+          const int px = i * kDcCols + lane;
+          const uint32_t addr = o_base + static_cast<uint32_t>(px * 128 + ((warp ^ (lane & 7)) << 4));
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+                       "r"(pack_bf16x2(v[0], v[1])), "r"(pack_bf16x2(v[2], v[3])),
+                       "r"(pack_bf16x2(v[4], v[5])), "r"(pack_bf16x2(v[6], v[7]))
+                       : "memory");
+        }
+        __syncthreads();
+        // 4 x 32 pixels x 8 chunks of 8 filters: consecutive threads take a
+        // pixel's chunks, so a warp writes four whole 128-byte pixel rows
+        for (int c = threadIdx.x; c < kDcRows * kDcCols * 8; c += kDcThreads) {
+          const int px = c >> 3, ch = c & 7;
+          const int col = px % kDcCols, p = p0 + px / kDcCols, q = q0 + col;
+          const int k = k0 + ch * 8;
+          if (p >= a.P || q >= a.Q || k >= a.K) continue;
+          uint4 v;
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                       : "r"(o_base + static_cast<uint32_t>(px * 128 + ((ch ^ (col & 7)) << 4)))
+                       : "memory");
+          *reinterpret_cast<uint4*>(y + ((static_cast<int64_t>(b) * a.P + p) * a.Q + q) * a.K + k) = v;
+        }
+        continue;
+      }
+    }
     const int q = q0 + lane;
     if (q >= a.Q) continue;
 #pragma unroll
@@ -309,9 +350,14 @@ tbn_status launch_dense_conv(const ConvProblem& p, const float* w, cudaStream_t 
   a.cc = static_cast<int>(cc);
   a.tiles_q = static_cast<int>((p.Q + kDcCols - 1) / kDcCols);
   a.tiles_p = static_cast<int>((p.P + kDcRows - 1) / kDcRows);
-  const size_t smem = static_cast<size_t>(cc * per_c) * 4;
   const bool xn = p.layout == TBN_NHWC, yn = p.layout != TBN_NCHW;
   const bool xb = p.xdt == TBN_BF16, yb = p.ydt == TBN_BF16;
+  constexpr size_t kStageOutBytes = kDcRows * kDcCols * kDcFilt * 2;
+  const size_t in_bytes = ((static_cast<size_t>(cc * per_c) + 31) & ~size_t(31)) * 4;
+  a.stage_out = (yn && yb && p.K % 8 == 0 && is_aligned(p.y, 16) &&
+                 in_bytes + kStageOutBytes <= static_cast<size_t>(kDcSmemMax))
+                    ? 1 : 0;
+  const size_t smem = a.stage_out ? in_bytes + kStageOutBytes : static_cast<size_t>(cc * per_c) * 4;
   using bf = __nv_bfloat16;
   if (xb && yb) return launch_dense_conv_l<bf, bf>(a, smem, xn, yn, s);
   if (xb && !yb) return launch_dense_conv_l<bf, float>(a, smem, xn, yn, s);
