@@ -143,3 +143,59 @@ def test_bwd_stays_inside_its_workspace(case):
     assert_guards(wb, "bwd filter workspace %s" % (case,))
     assert torch.equal(dx, dx_ref) and torch.equal(dw, dw_ref)
     assert tbn.tbn_device_error() == 0
+
+
+DENSE = [
+    # N, C, H, W, K, R, S, stride, pad, layout, out dtype
+    (2, 3, 37, 45, 64, 7, 7, (2, 2), (3, 3), tbn.TBN_NCHW_NHWC, torch.bfloat16),   # stem, staged
+    (1, 5, 13, 70, 72, 3, 3, (1, 1), (1, 1), tbn.TBN_NCHW_NHWC, torch.bfloat16),   # two filter blocks
+    (2, 3, 19, 21, 20, 5, 5, (2, 2), (2, 2), tbn.TBN_NCHW_NHWC, torch.float32),    # direct stores
+    (1, 4, 9, 11, 12, 3, 3, (1, 1), (0, 0), tbn.TBN_NHWC, torch.bfloat16),         # K % 8 != 0
+]
+
+
+@pytest.mark.parametrize("case", DENSE)
+def test_dense_conv_stays_inside_its_output(case):
+    N, C, H, W, K, R, S, st, pd, layout, ydt = case
+    g = inputs.generator(sum(case[:7]) + 3)
+    x = torch.randn(N, C, H, W, generator=g).to(torch.bfloat16)
+    if layout == tbn.TBN_NHWC:
+        x = x.permute(0, 2, 3, 1).contiguous()
+    x = x.cuda()
+    w = inputs.normal((K, C, R, S), 0.2, g).cuda()
+    ref = tbn.tbn_dense_conv2d_fwd(x, w, st, pd, layout=layout, out_dtype=ydt, relu=True)
+    yb, y = guarded(tuple(ref.shape), ydt)
+    tbn.tbn_dense_conv2d_fwd(x, w, st, pd, layout=layout, out_dtype=ydt, relu=True, out=y)
+    torch.cuda.synchronize()
+    assert_guards(yb, "dense conv %s" % (case[:9],))
+    assert torch.equal(y, ref)
+
+
+def test_fused_quant_conv_stays_inside_its_outputs():
+    # codes, alpha and y of the fused quantize-and-convolve launch
+    N, C, H, W, K = 2, 96, 9, 11, 200
+    g = inputs.generator(91)
+    x = torch.randn(N, H, W, C, generator=g).to(torch.bfloat16).cuda()
+    Wl = inputs.normal((K, 9 * C), 1.2, g).cuda()
+    y_ref, c_ref, a_ref = tbn.tbn_conv2d_fwd_quant(x, Wl, K, 3, 3, (1, 1), (1, 1), relu=True)
+    cb, codes = guarded(tuple(c_ref.shape), torch.int32)
+    ab, alpha = guarded((K,), torch.float32)
+    yb, y = guarded(tuple(y_ref.shape), torch.bfloat16)
+    tbn.tbn_conv2d_fwd_quant(x, Wl, K, 3, 3, (1, 1), (1, 1), relu=True, codes=codes, alpha=alpha,
+                             out=y)
+    torch.cuda.synchronize()
+    for buf, what in ((cb, "codes"), (ab, "alpha"), (yb, "y")):
+        assert_guards(buf, "fused quant conv " + what)
+    assert torch.equal(codes, c_ref) and torch.equal(alpha, a_ref) and torch.equal(y, y_ref)
+    assert tbn.tbn_device_error() == 0
+
+
+def test_space_to_depth_stays_inside_its_output():
+    N, C, H, W = 2, 3, 45, 51
+    x = torch.randn(N, C, H, W, generator=inputs.generator(92)).to(torch.bfloat16).cuda()
+    ref = tbn.tbn_space_to_depth(x, 11, 11, (4, 4), (0, 0), layout=tbn.TBN_NCHW)
+    ob, out = guarded(tuple(ref.shape), torch.bfloat16)
+    tbn.tbn_space_to_depth(x, 11, 11, (4, 4), (0, 0), layout=tbn.TBN_NCHW, out=out)
+    torch.cuda.synchronize()
+    assert_guards(ob, "space to depth")
+    assert torch.equal(out, ref)

@@ -73,6 +73,9 @@ S2D_CONV = [
     (2, 16, 17, 19, 40, 5, 5, 2, (2, 2)),      # 64 s2d channels, ragged K
     (2, 5, 20, 14, 8, 7, 5, 3, (1, 2)),        # 45 channels, R != S
     (4, 4, 16, 16, 64, 3, 3, 2, (1, 1)),       # 2x2 resident K blocks
+    (1, 5, 60, 44, 8, 7, 5, 3, (1, 2)),        # R' != S', ragged last tile
+    (2, 3, 63, 63, 96, 11, 11, 4, (0, 0)),     # one tile per image
+    (1, 12, 64, 64, 32, 3, 3, 2, (1, 1)),      # 3x3 / 2 over 12 channels
 ]
 
 
