@@ -27,12 +27,15 @@ nvidia-smi samples the SM clock through the timed regions.  The roofline
 entry is the tcgen05 implicit-GEMM kernel: its launches of one step (the
 five convolutions and the three FC layers) replayed back to back in a graph
 of their own after an L2 flush, algorithmic flops over that time.  The e2e
-figure replays a graph that adds, each step, the copy of the input batch
-from pinned host memory and of the logits back to pinned host memory.
+figure replays a graph that adds, each step, the copy of a whole input
+batch from pinned host memory and of the logits back to pinned host memory;
+the copy of the next batch runs on a second stream once the step's layout
+change has consumed the current one, so it overlaps the convolutions.
 
 Extra keys of the default run (each its own small timed region): VGG-small
 b128 and ResNet-18 b128 forward TFLOP/s and images/s, the LeNet-like layer's
-quantize + conv latency, the quantizer's and the GEMV's HBM GB/s.
+quantize + conv latency, the quantizer's and the GEMV's HBM GB/s, and the
+fused quantize-and-convolve launch against the two-launch path.
 
 Under torchrun (N > 1) every rank runs its own batch on its own GPU (data
 parallel replicas, no collective on the data path): value = the work of all
