@@ -215,6 +215,9 @@ class AlexNet:
         self.classifier = FCStack(_inputs.ALEXNET["fcs"], Wfc, self.N, device)
         self.x_in = self.features.x_in
         self.out = self.classifier.layers[-1][4]
+        # re-quantization runs beside the input's layout change (both read
+        # HBM, neither fills it; only the first convolution needs both)
+        self.quant_stream = torch.cuda.Stream(device=self.features.device)
 
     @property
     def conv_flops(self) -> int:
@@ -234,9 +237,26 @@ class AlexNet:
                       [(W, c, a) for (W, c, a, _, _) in self.classifier.layers])
 
     def forward(self, requantize: bool = False, conv_hook=None):
+        """One forward pass on the current stream.  With requantize, the
+        grouped quantizer runs on a second stream while the input's layout
+        change runs on this one; the streams join before the first
+        convolution (every launch keeps its order and inputs)."""
+        hook = conv_hook
         if requantize:
-            self.quantize()
-        h = self.features.forward(requantize=False, conv_hook=conv_hook)
+            cur = torch.cuda.current_stream(self.features.device)
+            qs = self.quant_stream
+            qs.wait_stream(cur)
+            with torch.cuda.stream(qs):
+                self.quantize()
+            joined = [False]
+
+            def hook(i, layer, when):
+                if not joined[0] and i == 0 and when == "before":
+                    cur.wait_stream(qs)   # codes and alpha of every layer are ready
+                    joined[0] = True
+                if conv_hook:
+                    conv_hook(i, layer, when)
+        h = self.features.forward(requantize=False, conv_hook=hook)
         return self.classifier.forward(h.reshape(self.N, -1))
 
     def launches_per_forward(self, requantize: bool = False) -> int:
