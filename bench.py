@@ -87,7 +87,7 @@ WORKLOADS = {
 CONV_TRAFFIC = {"sources": ["paper_1701_00485_gb300/csrc/tbn_conv_igemm.cuh",
                             "paper_1701_00485_gb300/csrc/tbn_conv_igemm.cu",
                             "paper_1701_00485_gb300/csrc/tbn_device.cuh"],
-                "sha256_16": "a5dcd95824c85e7d", "bytes_per_launch": 48.08e6}
+                "sha256_16": "2edd57ba5c2ffeed", "bytes_per_launch": 48.08e6}
 
 
 def measured_traffic(rec):

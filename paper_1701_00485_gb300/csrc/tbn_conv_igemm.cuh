@@ -279,7 +279,7 @@ __device__ __forceinline__ void store_out(const IgArgs& a, size_t o, float v) {
 // with `scratch` (the stage ring, not yet in use) holding a chunk of rows'
 // per-word sums and counts; then all CTAs meet at a grid-wide barrier on
 // a.gbar (bounded: on expiry the device error word records a timeout and
-// false is returned).
+// the CTA's abort flag is set, so it does no convolution work).
 __device__ void quantize_prologue(const IgArgs& a, uint8_t* scratch, int scratch_words,
                                   volatile int* abort_flag) {
   // every thread has read the abort flag before anyone can set it below
